@@ -1,0 +1,6 @@
+"""fp64 CPU oracle (test infrastructure only; see pad_oracle.py)."""
+from .pad_oracle import (bf16_to_f64, event_mask, video_attention, decode_step, event_rows,
+                         lse_merge, simulate_append, OK, OUT_OF_PAGES, INVALID)
+
+__all__ = ["bf16_to_f64", "event_mask", "video_attention", "decode_step", "event_rows",
+           "lse_merge", "simulate_append", "OK", "OUT_OF_PAGES", "INVALID"]

@@ -1,0 +1,293 @@
+"""Pins for the fp64 oracle: checks against what the paper and the mathematics fix.
+
+None of these re-types the oracle's formula: they compare it with a library
+routine (torch SDPA), a scalar brute force written separately, closed forms,
+invariances that Eq. 3 implies, and hand-worked fixtures in tests/golden/.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle
+from paper_2607_02963_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rand_video(rng, E, S, L, H_q=4, H_kv=2, D=16):
+    q = rng.standard_normal((E, H_q, D))
+    kp = rng.standard_normal((S, H_kv, D))
+    vp = rng.standard_normal((S, H_kv, D))
+    kb = [rng.standard_normal((n, H_kv, D)) for n in L]
+    vb = [rng.standard_normal((n, H_kv, D)) for n in L]
+    return q, kp, vp, kb, vb
+
+
+def _sdpa_single(q_row, K, V, scale):
+    """Library decode attention: one query [H_q, D] over keys K, V [n, H_kv, D] (GQA expanded
+    with the contiguous mapping q-head j -> kv-head j // G)."""
+    H_q = q_row.shape[0]
+    H_kv = K.shape[1]
+    G = H_q // H_kv
+    qt = torch.from_numpy(q_row)[:, None, :]                                 # [H_q, 1, D]
+    kt = torch.from_numpy(K).permute(1, 0, 2).repeat_interleave(G, dim=0)   # [H_q, n, D]
+    vt = torch.from_numpy(V).permute(1, 0, 2).repeat_interleave(G, dim=0)
+    out = F.scaled_dot_product_attention(qt, kt, vt, scale=scale)
+    return out[:, 0, :].numpy()
+
+
+# (i) E = 1 reduces to ordinary causal decode attention (Eq. 1).
+@pytest.mark.parametrize("L", [0, 1, 7, 33])
+def test_single_event_is_plain_decode(L):
+    rng = np.random.default_rng(10 + L)
+    q, kp, vp, kb, vb = _rand_video(rng, 1, 37, [L + 1])
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.25)
+    ref = _sdpa_single(q[0], np.concatenate([kp, kb[0]]), np.concatenate([vp, vb[0]]), 0.25)
+    np.testing.assert_allclose(o[0], ref, rtol=1e-12, atol=1e-13)
+
+
+# (ii) every event equals plain decode over concat(prefix, own branch) alone.
+def test_each_event_is_decode_over_prefix_and_own_branch():
+    rng = np.random.default_rng(3)
+    L = [1, 4, 17, 9, 2]
+    q, kp, vp, kb, vb = _rand_video(rng, len(L), 50, L, H_q=6, H_kv=2, D=8)
+    o, _, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.3)
+    for e in range(len(L)):
+        ref = _sdpa_single(q[e], np.concatenate([kp, kb[e]]), np.concatenate([vp, vb[e]]), 0.3)
+        np.testing.assert_allclose(o[e], ref, rtol=1e-12, atol=1e-13)
+
+
+# (iii) permuting the events permutes the outputs.
+def test_permutation_equivariance():
+    rng = np.random.default_rng(4)
+    L = [3, 1, 6, 2]
+    q, kp, vp, kb, vb = _rand_video(rng, 4, 21, L)
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.5)
+    perm = [2, 0, 3, 1]
+    o2, lse2, _ = oracle.video_attention(q[perm], kp, vp, [kb[i] for i in perm],
+                                         [vb[i] for i in perm], 0.5)
+    np.testing.assert_allclose(o2, o[perm], rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(lse2, lse[perm], rtol=1e-13, atol=1e-14)
+
+
+# (iv) an event's output ignores every other event's KV.
+def test_other_events_kv_do_not_matter():
+    rng = np.random.default_rng(5)
+    L = [4, 2, 7]
+    q, kp, vp, kb, vb = _rand_video(rng, 3, 19, L)
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.5)
+    kb2 = [kb[0]] + [100.0 * rng.standard_normal(x.shape) for x in kb[1:]]
+    vb2 = [vb[0]] + [100.0 * rng.standard_normal(x.shape) for x in vb[1:]]
+    o2, lse2, _ = oracle.video_attention(q, kp, vp, kb2, vb2, 0.5)
+    assert np.array_equal(o2[0], o[0]) and np.array_equal(lse2[0], lse[0])
+    # other branches of different length: same result up to summation order
+    kb3 = [kb[0], rng.standard_normal((11, 2, 16)), rng.standard_normal((1, 2, 16))]
+    vb3 = [vb[0], rng.standard_normal((11, 2, 16)), rng.standard_normal((1, 2, 16))]
+    o3, _, _ = oracle.video_attention(q, kp, vp, kb3, vb3, 0.5)
+    np.testing.assert_allclose(o3[0], o[0], rtol=1e-12, atol=1e-14)
+
+
+# (v) softmax rows sum to one and put no weight on masked keys.
+def test_rows_sum_to_one_and_mask_is_respected():
+    rng = np.random.default_rng(6)
+    L = [2, 5, 1]
+    q, kp, vp, kb, vb = _rand_video(rng, 3, 13, L)
+    _, _, p = oracle.video_attention(q, kp, vp, kb, vb, 1.0, return_p=True)
+    np.testing.assert_allclose(p.sum(axis=-1), 1.0, rtol=0, atol=1e-12)
+    starts = np.cumsum([13] + L)
+    for e in range(3):
+        for f in range(3):
+            blk = p[e, :, starts[f]:starts[f] + L[f]]
+            if f != e:
+                assert np.all(blk == 0.0)
+            else:
+                assert np.all(blk > 0.0)
+
+
+# (vi) a scalar brute force, written separately, agrees on tiny shapes.
+def _brute(q, kp, vp, kb, vb, scale):
+    E, H_q, D = q.shape
+    H_kv = kp.shape[1]
+    G = H_q // H_kv
+    o = np.zeros_like(q)
+    lse = np.zeros((E, H_q))
+    for e in range(E):
+        keys = [kp[t] for t in range(kp.shape[0])] + [kb[e][t] for t in range(kb[e].shape[0])]
+        vals = [vp[t] for t in range(vp.shape[0])] + [vb[e][t] for t in range(vb[e].shape[0])]
+        for j in range(H_q):
+            h = j // G
+            sc = []
+            for key in keys:
+                acc = 0.0
+                for d in range(D):
+                    acc += q[e, j, d] * key[h, d]
+                sc.append(acc * scale)
+            mx = max(sc)
+            ws = [math.exp(x - mx) for x in sc]
+            tot = sum(ws)
+            for d in range(D):
+                o[e, j, d] = sum(w * val[h, d] for w, val in zip(ws, vals)) / tot
+            lse[e, j] = mx + math.log(tot)
+    return o, lse
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_brute_force_tiny(seed):
+    rng = np.random.default_rng(100 + seed)
+    E = int(rng.integers(1, 4))
+    L = [int(x) for x in rng.integers(1, 5, size=E)]
+    S = int(rng.integers(0, 6))
+    q, kp, vp, kb, vb = _rand_video(rng, E, S, L, H_q=4, H_kv=2, D=3)
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.7)
+    ob, lb = _brute(q, kp, vp, kb, vb, 0.7)
+    np.testing.assert_allclose(o, ob, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(lse, lb, rtol=1e-12, atol=1e-13)
+
+
+# (vii) identical keys: uniform weights -> mean of the visible values; lse = s + ln(n).
+def test_identical_keys_give_mean_of_visible_values():
+    rng = np.random.default_rng(7)
+    L = [3, 5]
+    S = 9
+    q, kp, vp, kb, vb = _rand_video(rng, 2, S, L, H_q=2, H_kv=1, D=4)
+    key = rng.standard_normal(4)
+    kp[:] = key
+    for x in kb:
+        x[:] = key
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.5)
+    for e in range(2):
+        visible = np.concatenate([vp, vb[e]])[:, 0, :]
+        np.testing.assert_allclose(o[e, 0], visible.mean(axis=0), rtol=1e-12, atol=1e-13)
+        s = 0.5 * float(q[e, 0] @ key)
+        np.testing.assert_allclose(lse[e, 0], s + math.log(S + L[e]), rtol=1e-12)
+
+
+# (viii) constant values: the output is that constant whatever the weights.
+def test_constant_values():
+    rng = np.random.default_rng(8)
+    L = [2, 6, 1]
+    q, kp, vp, kb, vb = _rand_video(rng, 3, 11, L)
+    c = rng.standard_normal(16)
+    vp[:] = c
+    for x in vb:
+        x[:] = c
+    o, _, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.8)
+    np.testing.assert_allclose(o, np.broadcast_to(c, o.shape), rtol=1e-12, atol=1e-13)
+
+
+# lse pinned through a library routine: a zero key scores exactly 0, so its weight is
+# exp(-lse); reading that weight out of SDPA with a one-hot value column gives -ln p_0.
+def test_lse_against_sdpa_weight_of_zero_key():
+    rng = np.random.default_rng(9)
+    q, kp, vp, kb, vb = _rand_video(rng, 1, 12, [4], H_q=2, H_kv=1, D=6)
+    kp[0] = 0.0
+    vp[:, :, 0] = 0.0
+    kb[0][:, :, 0] = 0.0
+    vb[0][:, :, 0] = 0.0
+    vp[0, :, 0] = 1.0
+    _, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.6)
+    ref = _sdpa_single(q[0], np.concatenate([kp, kb[0]]), np.concatenate([vp, vb[0]]), 0.6)
+    np.testing.assert_allclose(lse[0], -np.log(ref[:, 0]), rtol=1e-12)
+
+
+# (ix) the log-sum-exp merge of prefix-only and branch-only results equals the full result.
+def test_lse_merge_identity():
+    rng = np.random.default_rng(11)
+    L = [5, 3]
+    q, kp, vp, kb, vb = _rand_video(rng, 2, 30, L)
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, 0.4)
+    empty = np.zeros((0, 2, 16))
+    op, lp, _ = oracle.video_attention(q, kp, vp, [empty, empty], [empty, empty], 0.4)
+    ob, lb, _ = oracle.video_attention(q, kp[:0], vp[:0], kb, vb, 0.4)
+    # split the prefix further into three chunks
+    parts = [(ob, lb)]
+    for a, b in [(0, 7), (7, 19), (19, 30)]:
+        parts.append(oracle.video_attention(q, kp[a:b], vp[a:b], [empty, empty], [empty, empty], 0.4)[:2])
+    om, lm = oracle.lse_merge(parts)
+    np.testing.assert_allclose(om, o, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(lm, lse, rtol=1e-12, atol=1e-13)
+    om2, lm2 = oracle.lse_merge([(op, lp), (ob, lb)])
+    np.testing.assert_allclose(om2, o, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(lm2, lse, rtol=1e-12, atol=1e-13)
+
+
+def test_hand_worked_two_events():
+    g = json.load(open(os.path.join(GOLDEN, "hand_two_events.json")))
+    q = np.array(g["q"])
+    kp = np.array(g["k_prefix"])
+    vp = np.array(g["v_prefix"])
+    kb = [np.array(x) for x in g["k_branches"]]
+    vb = [np.array(x) for x in g["v_branches"]]
+    o, lse, _ = oracle.video_attention(q, kp, vp, kb, vb, g["scale"])
+    np.testing.assert_allclose(o, np.array(g["expect_o"]), rtol=1e-14)
+    np.testing.assert_allclose(lse, np.array(g["expect_lse"]), rtol=1e-14)
+    assert oracle.event_mask(2, [1, 1]).tolist() == g["expect_mask"]
+
+
+def test_hand_worked_page_append():
+    g = json.load(open(os.path.join(GOLDEN, "hand_page_append.json")))
+    st, pt, free, slots = oracle.simulate_append(np.array(g["page_table"]), g["free_pages"],
+                                                 g["event_len"], g["page_size"])
+    assert st == oracle.OK
+    assert pt.tolist() == g["expect_page_table"]
+    assert free.tolist() == g["expect_free_pages"]
+    assert slots.tolist() == g["expect_slots"]
+    st, pt2, free2, slots = oracle.simulate_append(np.array(g["page_table"]),
+                                                   g["out_of_pages_case"]["free_pages"],
+                                                   g["event_len"], g["page_size"])
+    assert st == g["out_of_pages_case"]["expect_status"] and slots is None
+    assert pt2.tolist() == g["page_table"] and free2.tolist() == [0, 3]
+
+
+def test_append_simulation_invariants():
+    rng = np.random.default_rng(12)
+    for trial in range(20):
+        E = int(rng.integers(1, 12))
+        ps = int(rng.choice([4, 16]))
+        L = rng.integers(0, 50, size=E)
+        maxp = int(L.max()) // ps + 2
+        n_pages = 80
+        perm = rng.permutation(n_pages)
+        pt = np.full((E, maxp), -1, dtype=np.int32)
+        cur = 0
+        for e in range(E):
+            for p in range((int(L[e]) + ps - 1) // ps):
+                pt[e, p] = perm[cur]
+                cur += 1
+        free = np.sort(perm[cur:])
+        st, pt2, free2, slots = oracle.simulate_append(pt, free, L, ps)
+        assert st == oracle.OK
+        need = [e for e in range(E) if L[e] % ps == 0]
+        new = [int(pt2[e, L[e] // ps]) for e in need]
+        assert new == sorted(new) and new == [int(x) for x in free[:len(need)]]
+        assert sorted(free2.tolist() + new) == sorted(free.tolist())
+        for e in range(E):
+            assert slots[e, 0] == pt2[e, L[e] // ps] and slots[e, 1] == L[e] % ps
+
+
+def test_decode_step_on_tiny_workload_matches_sdpa():
+    """The whole-batch oracle on the tiny workload (bf16 inputs widened exactly) against SDPA."""
+    w = synth.tiny()
+    o, lse = oracle.decode_step(w)
+    for e in range(w.n_events):
+        K = np.concatenate([oracle.bf16_to_f64(w.prefix_k(0)), oracle.bf16_to_f64(w.priv_k(e)),
+                            oracle.bf16_to_f64(w.k_new[e:e + 1])])
+        V = np.concatenate([oracle.bf16_to_f64(w.prefix_v(0)), oracle.bf16_to_f64(w.priv_v(e)),
+                            oracle.bf16_to_f64(w.v_new[e:e + 1])])
+        ref = _sdpa_single(oracle.bf16_to_f64(w.q[e]), K, V, w.scale)
+        np.testing.assert_allclose(o[e], ref, rtol=1e-11, atol=1e-12)
+
+
+def test_bf16_widening_is_exact():
+    x = np.array([1.0, -2.5, 3.140625, 0.0, -0.0], dtype=np.float32)
+    bits = synth.f32_to_bf16_bits(x)
+    np.testing.assert_array_equal(oracle.bf16_to_f64(bits), x.astype(np.float64))
+    # round to nearest even at a tie: 1 + 2^-8 lies halfway between 1 and 1 + 2^-7
+    tie = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8], dtype=np.float32)
+    np.testing.assert_array_equal(oracle.bf16_to_f64(synth.f32_to_bf16_bits(tie)),
+                                  [1.0, 1.0 + 2.0 ** -6])
