@@ -1,0 +1,212 @@
+/*
+ * libpad — event-factorized parallel decode attention on GB300 (sm_103a).
+ *
+ * One decode step of one attention layer under the event-factorized
+ * dependency structure of Sec. 3.4 (Eq. 3 and the restructured causal mask of
+ * Fig. 3): every active event branch contributes one query token; the query of
+ * branch e attends to the shared prefix of its video (the multimodal prefix P
+ * followed by the planning tokens G^1..G^K, S of Sec. 3.3) and to its own
+ * branch's private tokens (anchor, L^e_<j and the token appended at this
+ * step), never to another branch's tokens.
+ *
+ * A step is three calls, all stream-ordered and asynchronous:
+ *   pad_plan              host: validate, allocate pages, build the work list,
+ *                         upload it into the caller's device workspace;
+ *   pad_kv_append         device: write each branch's new K/V into its page;
+ *   pad_event_decode_attn device: shared-prefix split-KV pass, private-suffix
+ *                         pass and log-sum-exp merge; writes O and LSE.
+ *
+ * Ownership: the caller owns every device buffer (prefix KV, page pools, page
+ * table, Q, outputs, workspace); the library never allocates device memory.
+ * A pad_plan_t holds host metadata only, plus offsets into the workspace; it
+ * stays valid until pad_plan_destroy and is tied to the workspace it was built
+ * on (a later pad_plan on the same workspace overwrites it in stream order).
+ *
+ * Errors: every call validates its arguments on the host and returns a
+ * pad_status before launching anything; pad_last_error() gives a message
+ * (thread-local).  Errors found by a kernel (a page id outside the pool) set a
+ * status word in the workspace, which pad_device_status() reads.
+ *
+ * Layouts (row-major, element type bf16 unless stated):
+ *   q          [n_events, h_q, head_dim]
+ *   k_prefix   [T_total, h_kv, head_dim]   (video b's prefix starts at token
+ *   v_prefix   [T_total, h_kv, head_dim]    prefix_offset[b] and has prefix_len[b] tokens)
+ *   k_pool     [n_pages, h_kv, page_size, head_dim]
+ *   v_pool     [n_pages, h_kv, page_size, head_dim]
+ *   k_new      [n_events, h_kv, head_dim]
+ *   v_new      [n_events, h_kv, head_dim]
+ *   page_table [n_events, max_pages] int32 (row e belongs to event e of this step)
+ *   out        [n_events, h_q, head_dim]   fp32 (out_dtype 0) or bf16 (out_dtype 1)
+ *   lse        [n_events, h_q] fp32, natural log
+ * q-head j reads kv-head floor(j / G) with G = h_q / h_kv.
+ */
+#ifndef PAD_H
+#define PAD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream handle (the same object as cudaStream_t); NULL = legacy default stream. */
+typedef struct CUstream_st* pad_stream_t;
+
+typedef enum {
+  PAD_OK = 0,
+  PAD_ERR_INVALID_ARG = 1,         /* a pointer, size, layout or length is not acceptable */
+  PAD_ERR_UNSUPPORTED = 2,         /* a valid shape this build does not implement */
+  PAD_ERR_OUT_OF_PAGES = 3,        /* the free pages do not cover this step's new pages */
+  PAD_ERR_WORKSPACE_TOO_SMALL = 4, /* workspace_bytes < pad_workspace_size(...) */
+  PAD_ERR_CUDA = 5,                /* a CUDA runtime call failed (message has the reason) */
+  PAD_ERR_DEVICE_TIMEOUT = 6,      /* a bounded device-side wait gave up */
+  PAD_ERR_DEVICE_BOUNDS = 7        /* a kernel met a page id outside the pool and skipped it */
+} pad_status;
+
+/* Shape of one attention layer.
+ *   h_q, h_kv   query and key/value heads, h_q % h_kv == 0, G = h_q / h_kv in [1, 16]
+ *   head_dim    64 or 128
+ *   page_size   tokens per page of the private KV pool: 4, 8, 16, 32 or 64
+ *   scale       softmax scale applied to q.k (1/sqrt(head_dim) in the paper's model)
+ *   out_dtype   0 = fp32 output, 1 = bf16 output
+ *   num_sms     SM count used to size the split-KV grid; 0 = query the current device
+ *   flags       PAD_FLAG_* below; 0 = automatic choice of the prefix kernel */
+typedef struct {
+  int32_t h_q;
+  int32_t h_kv;
+  int32_t head_dim;
+  int32_t page_size;
+  float scale;
+  int32_t out_dtype;
+  int32_t num_sms;
+  int32_t flags;
+} pad_problem;
+
+/* Force one implementation of the shared-prefix pass (tests and benchmarks). */
+#define PAD_FLAG_PREFIX_SIMT 0x1   /* CUDA-core path */
+#define PAD_FLAG_PREFIX_MMA 0x2    /* warp-level mma.sync path */
+#define PAD_FLAG_PREFIX_TC 0x4     /* tcgen05 / TMEM / TMA path */
+
+/* ---------------------------------------------------------------------------
+ * Page pool bookkeeping (host).  Tracks which pages of the private KV pool are
+ * in use.  The new token of a branch whose pre-step length is a multiple of
+ * page_size starts a page: pad_plan gives it the lowest-numbered free page,
+ * walking events in ascending order (one new token per branch per step, Eq. 3;
+ * a branch that emitted EOS simply leaves the event list, Sec. 3.4).
+ * ------------------------------------------------------------------------- */
+typedef struct pad_cache_state pad_cache_state;
+
+/* Create a pool of n_pages (>= 0) pages, all free.  *out receives the handle. */
+pad_status pad_cache_state_create(int32_t n_pages, pad_cache_state** out);
+void pad_cache_state_destroy(pad_cache_state* cache);
+/* Mark pages [n] as in use (a cache built before the library took over).
+ * Fails with PAD_ERR_INVALID_ARG, changing nothing, if a page is out of range or already used. */
+pad_status pad_cache_state_mark_used(pad_cache_state* cache, const int32_t* pages, int32_t n);
+/* Return pages [n] to the free set (pages of branches that terminated).
+ * Fails with PAD_ERR_INVALID_ARG, changing nothing, if a page is out of range or already free. */
+pad_status pad_cache_state_release(pad_cache_state* cache, const int32_t* pages, int32_t n);
+int32_t pad_cache_state_num_pages(const pad_cache_state* cache);
+int32_t pad_cache_state_free_count(const pad_cache_state* cache);
+/* Checkpoint: used[p] = 1 if page p is in use, else 0; used has num_pages entries (host). */
+pad_status pad_cache_state_export(const pad_cache_state* cache, uint8_t* used);
+/* Restore a checkpoint written by pad_cache_state_export (n_pages entries, host). */
+pad_status pad_cache_state_import(pad_cache_state* cache, const uint8_t* used, int32_t n_pages);
+
+/* ---------------------------------------------------------------------------
+ * Planning (a1 of the step; the paper gives no kernel, so the work split is
+ * this library's design: split-KV over each video's shared prefix).
+ * ------------------------------------------------------------------------- */
+typedef struct pad_plan_t pad_plan_t;
+
+/* Bytes of device workspace pad_plan needs for this batch (host arrays, same
+ * meaning as in pad_plan).  Returns 0 on invalid arguments. */
+size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32_t* prefix_len,
+                          int32_t n_events, const int32_t* event_video);
+
+/* Plan one decode step.
+ *   prob           layer shape (see pad_problem)
+ *   cache          page bookkeeping; pages for this step's new page starts are taken from it
+ *   n_videos       videos in the batch (>= 0)
+ *   prefix_len     [n_videos] host: shared-prefix tokens of each video (>= 0)
+ *   prefix_offset  [n_videos] host: first token of each prefix in k_prefix/v_prefix,
+ *                  or NULL for packed prefixes (exclusive prefix sum of prefix_len)
+ *   n_events       active event branches this step (>= 0); 0 gives a plan that launches nothing
+ *   event_video    [n_events] host: video of each event, non-decreasing, in [0, n_videos)
+ *   event_len      [n_events] host: private tokens of each branch BEFORE this step's append;
+ *                  branch e attends to event_len[e] + 1 private keys after the append
+ *   page_table     [n_events * max_pages] device: row e lists branch e's pages; the
+ *                  new-page entries are written by pad_kv_append
+ *   max_pages      columns of page_table; event_len[e] / page_size must be < max_pages
+ *   workspace      device, 256-byte aligned, at least pad_workspace_size(...) bytes;
+ *                  NULL plans on the host only (no upload; the plan cannot be launched)
+ *   stream         stream the plan upload (one cudaMemcpyAsync) is ordered on
+ *   plan_out       receives the new plan (free with pad_plan_destroy)
+ * On any error nothing changes: no page is taken and nothing is uploaded. */
+pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
+                    const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
+                    const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
+                    int32_t max_pages, void* workspace, size_t workspace_bytes,
+                    pad_stream_t stream, pad_plan_t** plan_out);
+
+/* Page given to each event this step: new_page[e] = page id, or -1 if branch e
+ * keeps writing into its current page.  new_page has n_events entries (host). */
+pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page);
+
+/* Summary of a plan (host): the split-KV decomposition chosen for the prefix pass. */
+typedef struct {
+  int32_t n_videos;
+  int32_t n_events;
+  int32_t n_work_items;     /* (video, kv-head, split) items of the prefix pass */
+  int32_t split_len;        /* prefix tokens per split (last split of a video may be shorter) */
+  int32_t prefix_kernel;    /* PAD_FLAG_PREFIX_* of the implementation that will run */
+  int32_t n_new_pages;
+  int64_t partial_rows;     /* rows of (m, l, O) partial softmax states in the workspace */
+  int64_t workspace_bytes;  /* bytes of workspace this plan uses */
+} pad_plan_info;
+pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info);
+pad_status pad_plan_destroy(pad_plan_t* plan);
+
+/* ---------------------------------------------------------------------------
+ * Device work.
+ * ------------------------------------------------------------------------- */
+
+/* a2: write k_new[e] / v_new[e] (bf16 [n_events, h_kv, head_dim], 16-byte aligned) into
+ * slot event_len[e] of branch e (page page_table[e][event_len[e] / page_size], offset
+ * event_len[e] % page_size) of k_pool / v_pool, and write the new page-table entries.
+ * One new token per branch per step (Eq. 3). */
+pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new,
+                         void* k_pool, void* v_pool, pad_stream_t stream);
+
+/* a3-a5: decode attention of every active branch's query under the event-factorized
+ * mask (Sec. 3.4): the shared prefix of its video plus its own event_len[e] + 1 private
+ * keys (read through page_table, so pad_kv_append must precede this call on the stream).
+ * All pointers device, 16-byte aligned; lse may be NULL. */
+pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
+                                 const void* v_prefix, const void* k_pool, const void* v_pool,
+                                 void* out, float* lse, pad_stream_t stream);
+
+/* Synchronise the stream and read the plan's device status word:
+ * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */
+pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream);
+
+/* Message for the last error on this thread ("" if none). */
+const char* pad_last_error(void);
+const char* pad_status_string(pad_status status);
+
+/* ---------------------------------------------------------------------------
+ * Measurement aid: CUDA-event timing of the dominant kernel (the shared-prefix
+ * pass).  After pad_timing_enable(n), the next n pad_event_decode_attn calls
+ * record an event pair around that kernel on the call's stream;
+ * pad_timing_read synchronises those events and returns the summed time in ms
+ * and the number of launches timed, then disables timing.  Process-global; not
+ * for concurrent use from several threads.
+ * ------------------------------------------------------------------------- */
+pad_status pad_timing_enable(int32_t max_launches);
+pad_status pad_timing_read(float* total_ms, int32_t* n_launches);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PAD_H */

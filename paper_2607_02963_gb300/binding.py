@@ -1,0 +1,265 @@
+"""ctypes binding of libpad (include/pad.h): argument marshalling only.
+
+Every step of the decode path runs in the CUDA library; this module converts
+torch tensors to device pointers, numpy arrays to host pointers, and status
+codes to exceptions.  It fails loudly when libpad.so has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int32, c_int64, c_size_t, c_uint8, c_void_p
+
+import numpy as np
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libpad.so")
+_lib = None
+
+PAD_OK = 0
+STATUS_NAMES = {
+    0: "PAD_OK", 1: "PAD_ERR_INVALID_ARG", 2: "PAD_ERR_UNSUPPORTED", 3: "PAD_ERR_OUT_OF_PAGES",
+    4: "PAD_ERR_WORKSPACE_TOO_SMALL", 5: "PAD_ERR_CUDA", 6: "PAD_ERR_DEVICE_TIMEOUT",
+    7: "PAD_ERR_DEVICE_BOUNDS",
+}
+FLAG_PREFIX_SIMT = 0x1
+FLAG_PREFIX_MMA = 0x2
+FLAG_PREFIX_TC = 0x4
+
+
+class PadError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class Problem(ctypes.Structure):
+    _fields_ = [("h_q", c_int32), ("h_kv", c_int32), ("head_dim", c_int32),
+                ("page_size", c_int32), ("scale", c_float), ("out_dtype", c_int32),
+                ("num_sms", c_int32), ("flags", c_int32)]
+
+
+class PlanInfo(ctypes.Structure):
+    _fields_ = [("n_videos", c_int32), ("n_events", c_int32), ("n_work_items", c_int32),
+                ("split_len", c_int32), ("prefix_kernel", c_int32), ("n_new_pages", c_int32),
+                ("partial_rows", c_int64), ("workspace_bytes", c_int64)]
+
+
+_I32P = POINTER(c_int32)
+_I64P = POINTER(c_int64)
+
+# name -> (restype, argtypes); mirrors include/pad.h
+_SIGNATURES = {
+    "pad_cache_state_create": (c_int32, [c_int32, POINTER(c_void_p)]),
+    "pad_cache_state_destroy": (None, [c_void_p]),
+    "pad_cache_state_mark_used": (c_int32, [c_void_p, _I32P, c_int32]),
+    "pad_cache_state_release": (c_int32, [c_void_p, _I32P, c_int32]),
+    "pad_cache_state_num_pages": (c_int32, [c_void_p]),
+    "pad_cache_state_free_count": (c_int32, [c_void_p]),
+    "pad_cache_state_export": (c_int32, [c_void_p, POINTER(c_uint8)]),
+    "pad_cache_state_import": (c_int32, [c_void_p, POINTER(c_uint8), c_int32]),
+    "pad_workspace_size": (c_size_t, [POINTER(Problem), c_int32, _I32P, c_int32, _I32P]),
+    "pad_plan": (c_int32, [POINTER(Problem), c_void_p, c_int32, _I32P, _I64P, c_int32, _I32P,
+                           _I32P, c_void_p, c_int32, c_void_p, c_size_t, c_void_p,
+                           POINTER(c_void_p)]),
+    "pad_plan_new_pages": (c_int32, [c_void_p, _I32P]),
+    "pad_plan_get_info": (c_int32, [c_void_p, POINTER(PlanInfo)]),
+    "pad_plan_destroy": (c_int32, [c_void_p]),
+    "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "pad_event_decode_attn": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                        c_void_p, c_void_p, c_void_p, c_void_p]),
+    "pad_device_status": (c_int32, [c_void_p, c_void_p]),
+    "pad_last_error": (ctypes.c_char_p, []),
+    "pad_status_string": (ctypes.c_char_p, [c_int32]),
+    "pad_timing_enable": (c_int32, [c_int32]),
+    "pad_timing_read": (c_int32, [POINTER(c_float), _I32P]),
+}
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """Load libpad.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"libpad.so is not built ({_LIB_PATH}); run "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(_LIB_PATH)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(status: int):
+    if status != PAD_OK:
+        msg = lib().pad_last_error().decode(errors="replace")
+        raise PadError(status, msg)
+
+
+def _i32(a):
+    a = np.ascontiguousarray(a, dtype=np.int32)
+    return a, a.ctypes.data_as(_I32P)
+
+
+def _ptr(t):
+    """Device pointer of a tensor (None -> NULL)."""
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libpad must be contiguous")
+    return c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return c_void_p(stream)
+    return c_void_p(stream.cuda_stream)
+
+
+def make_problem(h_q, h_kv, head_dim, page_size=16, scale=None, out_dtype=0, num_sms=0, flags=0):
+    if scale is None:
+        scale = 1.0 / float(head_dim) ** 0.5
+    return Problem(h_q, h_kv, head_dim, page_size, scale, out_dtype, num_sms, flags)
+
+
+class CacheState:
+    """Host bookkeeping of the private-KV page pool (pad_cache_state)."""
+
+    def __init__(self, n_pages: int, used_pages=None):
+        h = c_void_p()
+        _check(lib().pad_cache_state_create(int(n_pages), ctypes.byref(h)))
+        self._h = h
+        if used_pages is not None and len(used_pages):
+            self.mark_used(used_pages)
+
+    @property
+    def handle(self):
+        return self._h
+
+    def mark_used(self, pages):
+        a, p = _i32(pages)
+        _check(lib().pad_cache_state_mark_used(self._h, p, int(a.size)))
+
+    def release(self, pages):
+        a, p = _i32(pages)
+        _check(lib().pad_cache_state_release(self._h, p, int(a.size)))
+
+    @property
+    def n_pages(self) -> int:
+        return int(lib().pad_cache_state_num_pages(self._h))
+
+    @property
+    def free_count(self) -> int:
+        return int(lib().pad_cache_state_free_count(self._h))
+
+    def export(self) -> np.ndarray:
+        out = np.zeros(self.n_pages, dtype=np.uint8)
+        _check(lib().pad_cache_state_export(self._h, out.ctypes.data_as(POINTER(c_uint8))))
+        return out
+
+    def import_(self, used: np.ndarray):
+        u = np.ascontiguousarray(used, dtype=np.uint8)
+        _check(lib().pad_cache_state_import(self._h, u.ctypes.data_as(POINTER(c_uint8)), int(u.size)))
+
+    def free_pages(self) -> np.ndarray:
+        return np.nonzero(self.export() == 0)[0].astype(np.int32)
+
+    def __del__(self):
+        if getattr(self, "_h", None) is not None and _lib is not None:
+            _lib.pad_cache_state_destroy(self._h)
+            self._h = None
+
+
+class Plan:
+    """A planned decode step (pad_plan_t)."""
+
+    def __init__(self, handle, n_events):
+        self._h = handle
+        self.n_events = n_events
+
+    @property
+    def handle(self):
+        return self._h
+
+    def new_pages(self) -> np.ndarray:
+        out = np.full(self.n_events, -1, dtype=np.int32)
+        _check(lib().pad_plan_new_pages(self._h, out.ctypes.data_as(_I32P)))
+        return out
+
+    def info(self) -> dict:
+        i = PlanInfo()
+        _check(lib().pad_plan_get_info(self._h, ctypes.byref(i)))
+        return {f: getattr(i, f) for f, _ in PlanInfo._fields_}
+
+    def destroy(self):
+        if self._h is not None and _lib is not None:
+            _lib.pad_plan_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        self.destroy()
+
+
+def pad_workspace_size(problem: Problem, prefix_len, event_video) -> int:
+    pl, plp = _i32(prefix_len)
+    ev, evp = _i32(event_video)
+    return int(lib().pad_workspace_size(ctypes.byref(problem), int(pl.size), plp, int(ev.size), evp))
+
+
+def pad_plan(problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
+             page_table=None, max_pages: int = 0, workspace=None, prefix_offset=None,
+             stream=None) -> Plan:
+    """Plan one decode step (host).  page_table / workspace are device tensors
+    (int32 [E, max_pages] / uint8 [bytes]); workspace=None plans on the host only."""
+    pl, plp = _i32(prefix_len)
+    ev, evp = _i32(event_video)
+    el, elp = _i32(event_len)
+    po = None
+    if prefix_offset is not None:
+        po_arr = np.ascontiguousarray(prefix_offset, dtype=np.int64)
+        po = po_arr.ctypes.data_as(_I64P)
+    if page_table is not None and max_pages == 0:
+        max_pages = int(page_table.shape[-1])
+    ws_ptr = _ptr(workspace)
+    ws_bytes = int(workspace.numel() * workspace.element_size()) if workspace is not None else 0
+    strm = _stream(stream) if workspace is not None else c_void_p(0)
+    h = c_void_p()
+    _check(lib().pad_plan(ctypes.byref(problem), cache.handle, int(pl.size), plp, po, int(ev.size),
+                          evp, elp, _ptr(page_table), int(max_pages), ws_ptr, ws_bytes, strm,
+                          ctypes.byref(h)))
+    return Plan(h, int(el.size))
+
+
+def pad_kv_append(plan: Plan, k_new, v_new, k_pool, v_pool, stream=None):
+    _check(lib().pad_kv_append(plan.handle, _ptr(k_new), _ptr(v_new), _ptr(k_pool), _ptr(v_pool),
+                               _stream(stream)))
+
+
+def pad_event_decode_attn(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,
+                          stream=None):
+    _check(lib().pad_event_decode_attn(plan.handle, _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
+                                       _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
+                                       _stream(stream)))
+
+
+def pad_device_status(plan: Plan, stream=None):
+    _check(lib().pad_device_status(plan.handle, _stream(stream)))
+
+
+def pad_timing_enable(max_launches: int):
+    _check(lib().pad_timing_enable(int(max_launches)))
+
+
+def pad_timing_read():
+    ms = c_float()
+    n = c_int32()
+    _check(lib().pad_timing_read(ctypes.byref(ms), ctypes.byref(n)))
+    return float(ms.value), int(n.value)

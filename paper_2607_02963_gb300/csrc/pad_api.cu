@@ -1,0 +1,603 @@
+// C ABI of libpad: argument validation, page-pool bookkeeping, the split-KV
+// planner, workspace layout, and the launch sequence of one decode step.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "pad_internal.h"
+
+using namespace pad;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+pad_status fail(pad_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+pad_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(PAD_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int kDefaultSms = 152;
+
+int query_num_sms() {
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return kDefaultSms;
+  }
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = kDefaultSms;
+    }
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+pad_status check_problem(const pad_problem* prob) {
+  if (!prob) return fail(PAD_ERR_INVALID_ARG, "problem is NULL");
+  if (prob->h_q <= 0 || prob->h_kv <= 0 || prob->h_q % prob->h_kv != 0)
+    return fail(PAD_ERR_INVALID_ARG, "h_q=%d must be a positive multiple of h_kv=%d", prob->h_q,
+                prob->h_kv);
+  const int G = prob->h_q / prob->h_kv;
+  if (G > kMaxGroup)
+    return fail(PAD_ERR_UNSUPPORTED, "group size h_q/h_kv=%d exceeds %d", G, kMaxGroup);
+  if (prob->head_dim != 64 && prob->head_dim != 128)
+    return fail(PAD_ERR_UNSUPPORTED, "head_dim=%d (supported: 64, 128)", prob->head_dim);
+  const int ps = prob->page_size;
+  if (ps != 4 && ps != 8 && ps != 16 && ps != 32 && ps != 64)
+    return fail(PAD_ERR_UNSUPPORTED, "page_size=%d (supported: 4, 8, 16, 32, 64)", ps);
+  if (!(prob->scale > 0.f) || !std::isfinite(prob->scale))
+    return fail(PAD_ERR_INVALID_ARG, "scale must be finite and > 0");
+  if (prob->out_dtype != 0 && prob->out_dtype != 1)
+    return fail(PAD_ERR_INVALID_ARG, "out_dtype=%d (0 = fp32, 1 = bf16)", prob->out_dtype);
+  if (prob->num_sms < 0) return fail(PAD_ERR_INVALID_ARG, "num_sms < 0");
+  const int known = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC;
+  if (prob->flags & ~known) return fail(PAD_ERR_INVALID_ARG, "unknown flags 0x%x", prob->flags);
+  const int f = prob->flags & known;
+  if (f && (f & (f - 1))) return fail(PAD_ERR_INVALID_ARG, "at most one PAD_FLAG_PREFIX_* flag");
+  return PAD_OK;
+}
+
+// Split-KV decomposition and workspace layout of a batch.
+struct Layout {
+  int group = 1;
+  int n_sms = kDefaultSms;
+  int split_len = kSplitGranule;
+  int max_rows = 0;
+  int prefix_kernel = 0;
+  std::vector<int32_t> ev_first, ev_count, n_splits, part_base;
+  int64_t n_items = 0;
+  int64_t partial_rows = 0;
+  size_t off_videos = 0, off_events = 0, off_items = 0, upload_bytes = 0;
+  size_t off_ml = 0, off_o = 0, total_bytes = 0;
+};
+
+pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32_t* prefix_len,
+                          int32_t n_events, const int32_t* event_video, int n_sms, Layout* L) {
+  if (n_videos < 0 || n_events < 0) return fail(PAD_ERR_INVALID_ARG, "negative batch size");
+  if (n_videos > 0 && !prefix_len) return fail(PAD_ERR_INVALID_ARG, "prefix_len is NULL");
+  if (n_events > 0 && !event_video) return fail(PAD_ERR_INVALID_ARG, "event_video is NULL");
+  if (n_events > 0 && n_videos == 0) return fail(PAD_ERR_INVALID_ARG, "events without videos");
+  L->group = prob->h_q / prob->h_kv;
+  L->n_sms = n_sms;
+  L->ev_first.assign(n_videos, 0);
+  L->ev_count.assign(n_videos, 0);
+  L->n_splits.assign(n_videos, 0);
+  L->part_base.assign(n_videos, 0);
+  for (int b = 0; b < n_videos; ++b)
+    if (prefix_len[b] < 0) return fail(PAD_ERR_INVALID_ARG, "prefix_len[%d]=%d < 0", b, prefix_len[b]);
+  int prev = 0;
+  for (int e = 0; e < n_events; ++e) {
+    const int v = event_video[e];
+    if (v < 0 || v >= n_videos)
+      return fail(PAD_ERR_INVALID_ARG, "event_video[%d]=%d outside [0, %d)", e, v, n_videos);
+    if (v < prev) return fail(PAD_ERR_INVALID_ARG, "event_video must be non-decreasing (event %d)", e);
+    if (L->ev_count[v] == 0) L->ev_first[v] = e;
+    L->ev_count[v]++;
+    prev = v;
+  }
+  int64_t work = 0;
+  int max_rows = 0;
+  for (int b = 0; b < n_videos; ++b) {
+    if (L->ev_count[b] > 0) {
+      work += (int64_t)prefix_len[b] * prob->h_kv;
+      max_rows = std::max(max_rows, L->ev_count[b] * L->group);
+    }
+  }
+  L->max_rows = max_rows;
+  const int64_t target = std::max(1, n_sms);
+  int64_t chunk = (work + target - 1) / target;
+  chunk = std::max<int64_t>(kSplitGranule, (chunk + kSplitGranule - 1) / kSplitGranule * kSplitGranule);
+  if (chunk > (int64_t)1 << 30) return fail(PAD_ERR_UNSUPPORTED, "prefix too long");
+  L->split_len = (int)chunk;
+  int64_t items = 0, rows = 0;
+  for (int b = 0; b < n_videos; ++b) {
+    if (L->ev_count[b] == 0 || prefix_len[b] == 0) continue;
+    const int ns = (int)((prefix_len[b] + chunk - 1) / chunk);
+    if (ns > 32767) return fail(PAD_ERR_UNSUPPORTED, "too many splits for video %d", b);
+    L->n_splits[b] = ns;
+    if (rows > INT32_MAX) return fail(PAD_ERR_UNSUPPORTED, "partial rows exceed int32");
+    L->part_base[b] = (int32_t)rows;
+    items += (int64_t)ns * prob->h_kv;
+    rows += (int64_t)prob->h_kv * ns * L->ev_count[b] * L->group;
+  }
+  if (rows > INT32_MAX || items > INT32_MAX) return fail(PAD_ERR_UNSUPPORTED, "batch too large");
+  L->n_items = items;
+  L->partial_rows = rows;
+
+  int kern = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
+  if (kern == 0) kern = (max_rows <= 8) ? PAD_FLAG_PREFIX_SIMT : PAD_FLAG_PREFIX_MMA;
+  if (kern == PAD_FLAG_PREFIX_SIMT && max_rows > 16)
+    return fail(PAD_ERR_UNSUPPORTED, "SIMT prefix path takes at most 16 rows per (video, kv-head); got %d",
+                max_rows);
+  if (kern == PAD_FLAG_PREFIX_TC)
+    return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path is not built into this library");
+  L->prefix_kernel = kern;
+
+  size_t off = sizeof(PadDevHeader);
+  L->off_videos = off;
+  off = align_up(off + (size_t)n_videos * sizeof(PadVideoDesc), 256);
+  L->off_events = off;
+  off = align_up(off + (size_t)n_events * sizeof(PadEventDesc), 256);
+  L->off_items = off;
+  off = off + (size_t)items * sizeof(PadWorkItem);
+  L->upload_bytes = off;
+  off = align_up(off, 256);
+  L->off_ml = off;
+  off = align_up(off + (size_t)rows * sizeof(float2), 256);
+  L->off_o = off;
+  off = align_up(off + (size_t)rows * prob->head_dim * sizeof(float), 256);
+  L->total_bytes = off;
+  return PAD_OK;
+}
+
+// Timing of the dominant kernel (process-global measurement aid).
+struct Timing {
+  bool on = false;
+  int max = 0;
+  int n = 0;
+  std::vector<cudaEvent_t> ev;
+};
+Timing g_timing;
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Page pool bookkeeping
+// ---------------------------------------------------------------------------
+struct pad_cache_state {
+  int32_t n_pages = 0;
+  int32_t free_count = 0;
+  std::vector<uint64_t> used;  // bit p set = page p in use
+
+  bool is_used(int p) const { return (used[p >> 6] >> (p & 63)) & 1u; }
+  void set(int p, bool u) {
+    if (u)
+      used[p >> 6] |= (uint64_t)1 << (p & 63);
+    else
+      used[p >> 6] &= ~((uint64_t)1 << (p & 63));
+  }
+  // Lowest-numbered free page >= from, or -1.
+  int next_free(int from) const {
+    if (from >= n_pages) return -1;
+    size_t w = (size_t)from >> 6;
+    uint64_t bits = ~used[w] & (~(uint64_t)0 << (from & 63));
+    while (true) {
+      if (bits) {
+        int p = (int)(w * 64 + __builtin_ctzll(bits));
+        return p < n_pages ? p : -1;
+      }
+      if (++w >= used.size()) return -1;
+      bits = ~used[w];
+    }
+  }
+};
+
+struct pad_plan_t {
+  pad_problem prob{};
+  Layout lay;
+  int32_t n_videos = 0, n_events = 0;
+  int32_t max_pages = 0, n_pages = 0;
+  int32_t* page_table = nullptr;
+  void* workspace = nullptr;
+  int64_t total_prefix_tokens = 0;
+  int32_t n_new_pages = 0;
+  std::vector<int32_t> new_pages;
+  std::vector<uint8_t> host_image;  // header + videos + events + items, as uploaded
+};
+
+extern "C" {
+
+const char* pad_last_error(void) { return g_last_error.c_str(); }
+
+const char* pad_status_string(pad_status s) {
+  switch (s) {
+    case PAD_OK: return "PAD_OK";
+    case PAD_ERR_INVALID_ARG: return "PAD_ERR_INVALID_ARG";
+    case PAD_ERR_UNSUPPORTED: return "PAD_ERR_UNSUPPORTED";
+    case PAD_ERR_OUT_OF_PAGES: return "PAD_ERR_OUT_OF_PAGES";
+    case PAD_ERR_WORKSPACE_TOO_SMALL: return "PAD_ERR_WORKSPACE_TOO_SMALL";
+    case PAD_ERR_CUDA: return "PAD_ERR_CUDA";
+    case PAD_ERR_DEVICE_TIMEOUT: return "PAD_ERR_DEVICE_TIMEOUT";
+    case PAD_ERR_DEVICE_BOUNDS: return "PAD_ERR_DEVICE_BOUNDS";
+  }
+  return "PAD_ERR_UNKNOWN";
+}
+
+pad_status pad_cache_state_create(int32_t n_pages, pad_cache_state** out) {
+  if (!out) return fail(PAD_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (n_pages < 0) return fail(PAD_ERR_INVALID_ARG, "n_pages=%d < 0", n_pages);
+  auto* c = new pad_cache_state();
+  c->n_pages = n_pages;
+  c->free_count = n_pages;
+  c->used.assign(((size_t)n_pages + 63) / 64 + 1, 0);
+  *out = c;
+  return PAD_OK;
+}
+
+void pad_cache_state_destroy(pad_cache_state* cache) { delete cache; }
+
+int32_t pad_cache_state_num_pages(const pad_cache_state* c) { return c ? c->n_pages : -1; }
+int32_t pad_cache_state_free_count(const pad_cache_state* c) { return c ? c->free_count : -1; }
+
+static pad_status set_pages(pad_cache_state* c, const int32_t* pages, int32_t n, bool to_used) {
+  if (!c) return fail(PAD_ERR_INVALID_ARG, "cache is NULL");
+  if (n < 0 || (n > 0 && !pages)) return fail(PAD_ERR_INVALID_ARG, "bad page list");
+  std::vector<int32_t> seen(pages, pages + n);
+  std::sort(seen.begin(), seen.end());
+  for (int i = 0; i < n; ++i) {
+    const int p = seen[i];
+    if (p < 0 || p >= c->n_pages) return fail(PAD_ERR_INVALID_ARG, "page %d outside [0, %d)", p, c->n_pages);
+    if (i > 0 && seen[i - 1] == p) return fail(PAD_ERR_INVALID_ARG, "page %d listed twice", p);
+    if (c->is_used(p) == to_used)
+      return fail(PAD_ERR_INVALID_ARG, "page %d is already %s", p, to_used ? "in use" : "free");
+  }
+  for (int i = 0; i < n; ++i) c->set(pages[i], to_used);
+  c->free_count += to_used ? -n : n;
+  return PAD_OK;
+}
+
+pad_status pad_cache_state_mark_used(pad_cache_state* c, const int32_t* pages, int32_t n) {
+  return set_pages(c, pages, n, true);
+}
+
+pad_status pad_cache_state_release(pad_cache_state* c, const int32_t* pages, int32_t n) {
+  return set_pages(c, pages, n, false);
+}
+
+pad_status pad_cache_state_export(const pad_cache_state* c, uint8_t* used) {
+  if (!c || (!used && c->n_pages > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  for (int p = 0; p < c->n_pages; ++p) used[p] = c->is_used(p) ? 1 : 0;
+  return PAD_OK;
+}
+
+pad_status pad_cache_state_import(pad_cache_state* c, const uint8_t* used, int32_t n_pages) {
+  if (!c || (!used && n_pages > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  if (n_pages != c->n_pages)
+    return fail(PAD_ERR_INVALID_ARG, "checkpoint has %d pages, pool has %d", n_pages, c->n_pages);
+  int fc = 0;
+  for (int p = 0; p < n_pages; ++p) {
+    if (used[p] > 1) return fail(PAD_ERR_INVALID_ARG, "used[%d]=%d is not 0/1", p, used[p]);
+  }
+  for (int p = 0; p < n_pages; ++p) {
+    c->set(p, used[p] != 0);
+    fc += used[p] == 0;
+  }
+  c->free_count = fc;
+  return PAD_OK;
+}
+
+size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32_t* prefix_len,
+                          int32_t n_events, const int32_t* event_video) {
+  if (check_problem(prob) != PAD_OK) return 0;
+  Layout L;
+  const int sms = prob->num_sms > 0 ? prob->num_sms : query_num_sms();
+  if (compute_layout(prob, n_videos, prefix_len, n_events, event_video, sms, &L) != PAD_OK) return 0;
+  return L.total_bytes;
+}
+
+pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
+                    const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
+                    const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
+                    int32_t max_pages, void* workspace, size_t workspace_bytes,
+                    pad_stream_t stream, pad_plan_t** plan_out) {
+  if (!plan_out) return fail(PAD_ERR_INVALID_ARG, "plan_out is NULL");
+  *plan_out = nullptr;
+  pad_status st = check_problem(prob);
+  if (st != PAD_OK) return st;
+  if (!cache) return fail(PAD_ERR_INVALID_ARG, "cache is NULL");
+  if (n_events > 0 && !event_len) return fail(PAD_ERR_INVALID_ARG, "event_len is NULL");
+  if (max_pages <= 0 && n_events > 0) return fail(PAD_ERR_INVALID_ARG, "max_pages must be > 0");
+  if (workspace && (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return fail(PAD_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (workspace && n_events > 0 && !page_table)
+    return fail(PAD_ERR_INVALID_ARG, "page_table is NULL");
+
+  const int sms = prob->num_sms > 0 ? prob->num_sms : (workspace ? query_num_sms() : kDefaultSms);
+  auto* plan = new pad_plan_t();
+  Layout& L = plan->lay;
+  st = compute_layout(prob, n_videos, prefix_len, n_events, event_video, sms, &L);
+  if (st != PAD_OK) {
+    delete plan;
+    return st;
+  }
+  if (workspace && workspace_bytes < L.total_bytes) {
+    delete plan;
+    return fail(PAD_ERR_WORKSPACE_TOO_SMALL, "workspace has %zu bytes, plan needs %zu",
+                workspace_bytes, L.total_bytes);
+  }
+  const int ps = prob->page_size;
+  int need = 0;
+  for (int e = 0; e < n_events; ++e) {
+    const int len = event_len[e];
+    if (len < 0) {
+      delete plan;
+      return fail(PAD_ERR_INVALID_ARG, "event_len[%d]=%d < 0", e, len);
+    }
+    if (len / ps >= max_pages) {
+      delete plan;
+      return fail(PAD_ERR_INVALID_ARG, "event %d: length %d needs page index %d >= max_pages=%d", e,
+                  len, len / ps, max_pages);
+    }
+    need += (len % ps) == 0;
+  }
+  if (need > cache->free_count) {
+    delete plan;
+    return fail(PAD_ERR_OUT_OF_PAGES, "step needs %d new pages, %d free", need, cache->free_count);
+  }
+
+  // Host image of the device plan.
+  std::vector<PadVideoDesc> vids(n_videos);
+  int64_t packed = 0, total_tokens = 0;
+  for (int b = 0; b < n_videos; ++b) {
+    int64_t off = prefix_offset ? prefix_offset[b] : packed;
+    if (off < 0) {
+      delete plan;
+      return fail(PAD_ERR_INVALID_ARG, "prefix_offset[%d] < 0", b);
+    }
+    packed += prefix_len[b];
+    total_tokens = std::max(total_tokens, off + prefix_len[b]);
+    PadVideoDesc& v = vids[b];
+    v.prefix_off = off;
+    v.prefix_len = prefix_len[b];
+    v.first_event = L.ev_first[b];
+    v.n_events = L.ev_count[b];
+    v.n_splits = L.n_splits[b];
+    v.part_base = L.part_base[b];
+    v.pad = 0;
+  }
+  std::vector<PadWorkItem> items;
+  items.reserve(L.n_items);
+  for (int b = 0; b < n_videos; ++b) {
+    for (int h = 0; h < prob->h_kv; ++h) {
+      for (int s = 0; s < L.n_splits[b]; ++s) {
+        PadWorkItem it;
+        it.video = b;
+        it.kvh = (int16_t)h;
+        it.split = (int16_t)s;
+        it.tok_begin = s * L.split_len;
+        it.tok_end = std::min(prefix_len[b], (s + 1) * L.split_len);
+        items.push_back(it);
+      }
+    }
+  }
+
+  // Page allocation: ascending events, lowest free page first.
+  std::vector<PadEventDesc> evs(n_events);
+  plan->new_pages.assign(n_events, -1);
+  int cursor = 0;
+  for (int e = 0; e < n_events; ++e) {
+    PadEventDesc& d = evs[e];
+    d.video = event_video[e];
+    d.len = event_len[e];
+    d.local = e - L.ev_first[d.video];
+    d.new_page = -1;
+    if (event_len[e] % ps == 0) {
+      const int pg = cache->next_free(cursor);
+      // need <= free_count guarantees a page exists
+      d.new_page = pg;
+      plan->new_pages[e] = pg;
+      cache->set(pg, true);
+      cursor = pg + 1;
+    }
+  }
+  cache->free_count -= need;
+
+  PadDevHeader hdr;
+  std::memset(&hdr, 0, sizeof(hdr));
+  plan->host_image.assign(L.upload_bytes, 0);
+  std::memcpy(plan->host_image.data(), &hdr, sizeof(hdr));
+  if (n_videos) std::memcpy(plan->host_image.data() + L.off_videos, vids.data(), vids.size() * sizeof(PadVideoDesc));
+  if (n_events) std::memcpy(plan->host_image.data() + L.off_events, evs.data(), evs.size() * sizeof(PadEventDesc));
+  if (!items.empty())
+    std::memcpy(plan->host_image.data() + L.off_items, items.data(), items.size() * sizeof(PadWorkItem));
+
+  if (workspace) {
+    cudaError_t ce = cudaMemcpyAsync(workspace, plan->host_image.data(), L.upload_bytes,
+                                     cudaMemcpyHostToDevice, reinterpret_cast<cudaStream_t>(stream));
+    if (ce != cudaSuccess) {
+      for (int e = 0; e < n_events; ++e)
+        if (plan->new_pages[e] >= 0) cache->set(plan->new_pages[e], false);
+      cache->free_count += need;
+      delete plan;
+      return cuda_fail(ce, "plan upload");
+    }
+  }
+  plan->prob = *prob;
+  plan->n_videos = n_videos;
+  plan->n_events = n_events;
+  plan->max_pages = max_pages;
+  plan->n_pages = cache->n_pages;
+  plan->page_table = page_table;
+  plan->workspace = workspace;
+  plan->total_prefix_tokens = total_tokens;
+  plan->n_new_pages = need;
+  *plan_out = plan;
+  return PAD_OK;
+}
+
+pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page) {
+  if (!plan || (!new_page && plan->n_events > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  std::copy(plan->new_pages.begin(), plan->new_pages.end(), new_page);
+  return PAD_OK;
+}
+
+pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
+  if (!plan || !info) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  info->n_videos = plan->n_videos;
+  info->n_events = plan->n_events;
+  info->n_work_items = (int32_t)plan->lay.n_items;
+  info->split_len = plan->lay.split_len;
+  info->prefix_kernel = plan->lay.prefix_kernel;
+  info->n_new_pages = plan->n_new_pages;
+  info->partial_rows = plan->lay.partial_rows;
+  info->workspace_bytes = (int64_t)plan->lay.total_bytes;
+  return PAD_OK;
+}
+
+pad_status pad_plan_destroy(pad_plan_t* plan) {
+  delete plan;
+  return PAD_OK;
+}
+
+static KParams make_params(const pad_plan_t* plan) {
+  KParams p;
+  const pad_problem& pr = plan->prob;
+  p.h_q = pr.h_q;
+  p.h_kv = pr.h_kv;
+  p.group = pr.h_q / pr.h_kv;
+  p.head_dim = pr.head_dim;
+  p.page_size = pr.page_size;
+  p.max_pages = plan->max_pages;
+  p.n_pages = plan->n_pages;
+  p.n_videos = plan->n_videos;
+  p.n_events = plan->n_events;
+  p.n_items = (int32_t)plan->lay.n_items;
+  p.out_bf16 = pr.out_dtype == 1;
+  p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
+  auto* ws = static_cast<uint8_t*>(plan->workspace);
+  p.header = reinterpret_cast<PadDevHeader*>(ws);
+  p.videos = reinterpret_cast<const PadVideoDesc*>(ws + plan->lay.off_videos);
+  p.events = reinterpret_cast<const PadEventDesc*>(ws + plan->lay.off_events);
+  p.items = reinterpret_cast<const PadWorkItem*>(ws + plan->lay.off_items);
+  p.part_ml = reinterpret_cast<float2*>(ws + plan->lay.off_ml);
+  p.part_o = reinterpret_cast<float*>(ws + plan->lay.off_o);
+  p.page_table = plan->page_table;
+  return p;
+}
+
+pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new,
+                         void* k_pool, void* v_pool, pad_stream_t stream) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (plan->n_events == 0) return PAD_OK;
+  if (!plan->workspace) return fail(PAD_ERR_INVALID_ARG, "plan was built without a workspace");
+  if (!k_new || !v_new || !k_pool || !v_pool) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_pool) || !aligned16(v_pool))
+    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaError_t e = launch_append(make_params(plan), k_new, v_new, k_pool, v_pool,
+                                reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  return PAD_OK;
+}
+
+pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
+                                 const void* v_prefix, const void* k_pool, const void* v_pool,
+                                 void* out, float* lse, pad_stream_t stream) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (plan->n_events == 0) return PAD_OK;
+  if (!plan->workspace) return fail(PAD_ERR_INVALID_ARG, "plan was built without a workspace");
+  if (!q || !k_pool || !v_pool || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (plan->lay.n_items > 0 && (!k_prefix || !v_prefix))
+    return fail(PAD_ERR_INVALID_ARG, "k_prefix / v_prefix is NULL");
+  if (!aligned16(q) || !aligned16(k_prefix) || !aligned16(v_prefix) || !aligned16(k_pool) ||
+      !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const KParams p = make_params(plan);
+  const bool timed = g_timing.on && g_timing.n < g_timing.max;
+  if (timed) cudaEventRecord(g_timing.ev[2 * g_timing.n], s);
+  cudaError_t e = cudaSuccess;
+  switch (plan->lay.prefix_kernel) {
+    case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
+    case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
+    default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "prefix launch");
+  if (timed) {
+    cudaEventRecord(g_timing.ev[2 * g_timing.n + 1], s);
+    g_timing.n++;
+  }
+  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, s);
+  if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
+  return PAD_OK;
+}
+
+pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (!plan->workspace) return PAD_OK;
+  PadDevHeader h;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(&h, plan->workspace, sizeof(h), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "reading device status");
+  if (h.status != PAD_OK)
+    return fail((pad_status)h.status, "device reported %s (detail %d %d %d)",
+                pad_status_string((pad_status)h.status), h.info[0], h.info[1], h.info[2]);
+  return PAD_OK;
+}
+
+pad_status pad_timing_enable(int32_t max_launches) {
+  if (max_launches <= 0) return fail(PAD_ERR_INVALID_ARG, "max_launches must be > 0");
+  while ((int)g_timing.ev.size() < 2 * max_launches) {
+    cudaEvent_t ev;
+    cudaError_t e = cudaEventCreate(&ev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+    g_timing.ev.push_back(ev);
+  }
+  g_timing.on = true;
+  g_timing.max = max_launches;
+  g_timing.n = 0;
+  return PAD_OK;
+}
+
+pad_status pad_timing_read(float* total_ms, int32_t* n_launches) {
+  if (!total_ms || !n_launches) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  float tot = 0.f;
+  for (int i = 0; i < g_timing.n; ++i) {
+    cudaError_t e = cudaEventSynchronize(g_timing.ev[2 * i + 1]);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+    float ms = 0.f;
+    e = cudaEventElapsedTime(&ms, g_timing.ev[2 * i], g_timing.ev[2 * i + 1]);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+    tot += ms;
+  }
+  *total_ms = tot;
+  *n_launches = g_timing.n;
+  g_timing.on = false;
+  g_timing.n = 0;
+  return PAD_OK;
+}
+
+}  // extern "C"

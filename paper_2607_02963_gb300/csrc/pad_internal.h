@@ -1,0 +1,89 @@
+// Internal declarations shared by the host planner (pad_api.cu) and the kernels.
+// The device-side plan is a flat block at the start of the caller's workspace:
+//
+//   [0, 256)            PadDevHeader (status word; reset by every plan upload)
+//   videos              PadVideoDesc[n_videos]
+//   events              PadEventDesc[n_events]
+//   items               PadWorkItem[n_work_items]       (prefix split-KV work list)
+//   -- end of the uploaded part --
+//   part_ml             float2[partial_rows]            (m in log2 units, l)
+//   part_o              float[partial_rows * head_dim]  (unnormalised O)
+//
+// Partial row of (video b, kv-head h, split s, row r) with r = e_local * G + g:
+//   part_base[b] + (h * n_splits[b] + s) * R_b + r,   R_b = n_events[b] * G.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/pad.h"
+
+namespace pad {
+
+constexpr int kSplitGranule = 128;   // prefix splits are multiples of this many tokens
+constexpr int kMaxGroup = 16;        // G = h_q / h_kv supported by the kernels
+
+struct PadDevHeader {
+  int32_t status;      // pad_status written by kernels (first error wins)
+  int32_t info[3];     // kernel-specific detail of the first error (e.g. event, page)
+  int32_t pad[60];
+};
+static_assert(sizeof(PadDevHeader) == 256, "header is 256 bytes");
+
+struct PadVideoDesc {
+  int64_t prefix_off;   // first token of the prefix in k_prefix / v_prefix
+  int32_t prefix_len;
+  int32_t first_event;
+  int32_t n_events;
+  int32_t n_splits;     // prefix splits per kv-head (0 if prefix_len == 0 or no events)
+  int32_t part_base;    // first partial row of this video
+  int32_t pad;
+};
+static_assert(sizeof(PadVideoDesc) == 32, "video desc is 32 bytes");
+
+struct PadEventDesc {
+  int32_t video;
+  int32_t len;          // private length before this step
+  int32_t new_page;     // page taken this step, or -1
+  int32_t local;        // index of the event within its video
+};
+static_assert(sizeof(PadEventDesc) == 16, "event desc is 16 bytes");
+
+struct PadWorkItem {
+  int32_t video;
+  int16_t kvh;
+  int16_t split;
+  int32_t tok_begin;    // [tok_begin, tok_end) relative to the video's prefix start
+  int32_t tok_end;
+};
+static_assert(sizeof(PadWorkItem) == 16, "work item is 16 bytes");
+
+// Everything a kernel needs, passed by value.
+struct KParams {
+  int32_t h_q, h_kv, group, head_dim, page_size, max_pages, n_pages;
+  int32_t n_videos, n_events, n_items;
+  int32_t out_bf16;
+  float scale_log2;               // scale * log2(e)
+  PadDevHeader* header;
+  const PadVideoDesc* videos;
+  const PadEventDesc* events;
+  const PadWorkItem* items;
+  float2* part_ml;
+  float* part_o;
+  int32_t* page_table;
+};
+
+// Launchers (pad_kernels.cu, pad_prefix_tc.cu).  Return the launch error.
+cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,
+                          void* v_pool, cudaStream_t s);
+cudaError_t launch_prefix_simt(const KParams& p, int max_rows, const void* q, const void* kp,
+                               const void* vp, cudaStream_t s);
+cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, const void* kp,
+                              const void* vp, cudaStream_t s);
+cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
+                             const void* vp, int64_t total_prefix_tokens, cudaStream_t s);
+cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
+                                const void* v_pool, void* out, float* lse, cudaStream_t s);
+
+}  // namespace pad

@@ -1,0 +1,701 @@
+// Kernels of one event-factorized decode step (Sec. 3.4, Eq. 3):
+//   append_kernel        a2: scatter each branch's new K/V into its page, write new page-table entries
+//   prefix_simt_kernel   a3 for few rows (R = E_b * G <= 16): warp-shuffle split-KV flash-decode
+//   prefix_mma_kernel    a3 with warp-level mma.sync (m16n8k16, bf16 in, fp32 accumulate)
+//   branch_merge_kernel  a4 + a5: each branch's private-suffix pass, then the log-sum-exp merge
+//                        of its prefix partials (the mask of Fig. 3: own branch only)
+//
+// Partial softmax states (m, l, O) keep m in log2 units of the scaled score:
+// m = max_k s_k * scale * log2(e), l = sum_k 2^(s_k*scale*log2(e) - m), O = sum_k 2^(...) v_k.
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "pad_internal.h"
+
+namespace pad {
+
+namespace {
+
+constexpr float kNegInf = -__builtin_huge_valf();
+
+__device__ __forceinline__ void set_error(PadDevHeader* h, int code, int a, int b, int c) {
+  if (atomicCAS(&h->status, 0, code) == 0) {
+    h->info[0] = a;
+    h->info[1] = b;
+    h->info[2] = c;
+  }
+}
+
+// Hardware base-2 exponential (MUFU.EX2); exp2(-inf) = 0.
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ void unpack8(const uint4& r, float* f) {
+  f[0] = bf16_lo(r.x); f[1] = bf16_hi(r.x);
+  f[2] = bf16_lo(r.y); f[3] = bf16_hi(r.y);
+  f[4] = bf16_lo(r.z); f[5] = bf16_hi(r.z);
+  f[6] = bf16_lo(r.w); f[7] = bf16_hi(r.w);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, bool pred) {
+  unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+  int n = pred ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3,
+                                        const void* p) {
+  unsigned a = static_cast<unsigned>(__cvta_generic_to_shared(p));
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(a));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3,
+                                          const void* p) {
+  unsigned a = static_cast<unsigned>(__cvta_generic_to_shared(p));
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(a));
+}
+
+__device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Query row r of (video, kv-head): event e_local = r / G, head kvh*G + r % G.
+__device__ __forceinline__ const __nv_bfloat16* q_row(const KParams& p, const PadVideoDesc& vd,
+                                                      const __nv_bfloat16* q, int kvh, int r) {
+  int el = r / p.group;
+  int gh = r - el * p.group;
+  return q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * p.head_dim;
+}
+
+__device__ __forceinline__ int64_t part_row(const PadVideoDesc& vd, int kvh, int split, int R, int r) {
+  return (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + split) * R + r;
+}
+
+// ---------------------------------------------------------------------------
+// a2: fused append.  One thread per 16-byte chunk of one (event, kv-head) row.
+// ---------------------------------------------------------------------------
+__global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
+                              const uint4* __restrict__ v_new, uint4* __restrict__ k_pool,
+                              uint4* __restrict__ v_pool) {
+  const int chunks = p.head_dim / 8;
+  const int per_event = p.h_kv * chunks;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= p.n_events * per_event) return;
+  const int e = idx / per_event;
+  const int rem = idx - e * per_event;
+  const int h = rem / chunks;
+  const int c = rem - h * chunks;
+  const PadEventDesc ev = p.events[e];
+  const int pidx = ev.len / p.page_size;
+  const int slot = ev.len - pidx * p.page_size;
+  int page;
+  if (ev.new_page >= 0) {
+    page = ev.new_page;
+    if (rem == 0) p.page_table[(size_t)e * p.max_pages + pidx] = page;
+  } else {
+    page = p.page_table[(size_t)e * p.max_pages + pidx];
+  }
+  if (page < 0 || page >= p.n_pages) {
+    set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pidx, page);
+    return;
+  }
+  const size_t dst = (((size_t)page * p.h_kv + h) * p.page_size + slot) * chunks + c;
+  const size_t src = ((size_t)e * p.h_kv + h) * chunks + c;
+  k_pool[dst] = k_new[src];
+  v_pool[dst] = v_new[src];
+}
+
+// ---------------------------------------------------------------------------
+// a3, few rows: warp-shuffle split-KV flash-decode.  One CTA (8 warps) per work
+// item; warp w takes 32-token chunks w, w+8, ...; lane = token for q.k, lane =
+// head_dim slice for p.v; the 8 warps' states are merged through shared memory.
+// ---------------------------------------------------------------------------
+template <int D, int MAXR>
+__global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
+                                                          const __nv_bfloat16* __restrict__ q,
+                                                          const __nv_bfloat16* __restrict__ kp,
+                                                          const __nv_bfloat16* __restrict__ vp) {
+  constexpr int NW = 8;
+  constexpr int VPL = D / 32;  // head_dim elements per lane in p.v
+  __shared__ float sq[MAXR][D];
+  __shared__ float sp[NW][MAXR][32];
+  __shared__ float sm[NW][MAXR];
+  __shared__ float sl[NW][MAXR];
+  __shared__ float so[MAXR][D];
+
+  const PadWorkItem it = p.items[blockIdx.x];
+  const PadVideoDesc vd = p.videos[it.video];
+  const int R = vd.n_events * p.group;
+  const int kvh = it.kvh;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  for (int i = threadIdx.x; i < MAXR * D; i += blockDim.x) {
+    int r = i / D, d = i - r * D;
+    float v = 0.f;
+    if (r < R) v = __bfloat162float(q_row(p, vd, q, kvh, r)[d]);
+    sq[r][d] = v;
+    so[r][d] = 0.f;
+  }
+  __syncthreads();
+
+  float o[MAXR][VPL];
+  float m[MAXR], l[MAXR];
+#pragma unroll
+  for (int r = 0; r < MAXR; ++r) {
+    m[r] = kNegInf;
+    l[r] = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) o[r][i] = 0.f;
+  }
+
+  const int ntok = it.tok_end - it.tok_begin;
+  const size_t row_stride = (size_t)p.h_kv * D;
+  const __nv_bfloat16* kbase = kp + ((size_t)vd.prefix_off + it.tok_begin) * row_stride + (size_t)kvh * D;
+  const __nv_bfloat16* vbase = vp + ((size_t)vd.prefix_off + it.tok_begin) * row_stride + (size_t)kvh * D;
+
+  for (int c0 = warp * 32; c0 < ntok; c0 += NW * 32) {
+    const int t = c0 + lane;
+    const bool valid = t < ntok;
+    float s[MAXR];
+#pragma unroll
+    for (int r = 0; r < MAXR; ++r) s[r] = 0.f;
+    if (valid) {
+      const uint4* kr = reinterpret_cast<const uint4*>(kbase + (size_t)t * row_stride);
+#pragma unroll 4
+      for (int d8 = 0; d8 < D / 8; ++d8) {
+        float kf[8];
+        unpack8(__ldg(kr + d8), kf);
+#pragma unroll
+        for (int r = 0; r < MAXR; ++r) {
+          if (r < R) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) s[r] = fmaf(sq[r][d8 * 8 + j], kf[j], s[r]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < MAXR; ++r) {
+      if (r < R) {
+        float sv = valid ? s[r] * p.scale_log2 : kNegInf;
+        float mn = fmaxf(m[r], warp_max(sv));       // finite: lane 0's token is valid
+        float alpha = ex2(m[r] - mn);
+        float pr = ex2(sv - mn);
+        l[r] = l[r] * alpha + warp_sum(pr);
+        m[r] = mn;
+#pragma unroll
+        for (int i = 0; i < VPL; ++i) o[r][i] *= alpha;
+        sp[warp][r][lane] = pr;
+      }
+    }
+    __syncwarp();
+    const int nv = min(32, ntok - c0);
+    for (int j = 0; j < nv; ++j) {
+      const __nv_bfloat16* vr = vbase + (size_t)(c0 + j) * row_stride + lane * VPL;
+      float vf[VPL];
+      if constexpr (VPL == 4) {
+        uint2 raw = __ldg(reinterpret_cast<const uint2*>(vr));
+        vf[0] = bf16_lo(raw.x); vf[1] = bf16_hi(raw.x); vf[2] = bf16_lo(raw.y); vf[3] = bf16_hi(raw.y);
+      } else {
+        uint32_t raw = __ldg(reinterpret_cast<const unsigned int*>(vr));
+        vf[0] = bf16_lo(raw); vf[1] = bf16_hi(raw);
+      }
+#pragma unroll
+      for (int r = 0; r < MAXR; ++r) {
+        if (r < R) {
+          float pj = sp[warp][r][j];
+#pragma unroll
+          for (int i = 0; i < VPL; ++i) o[r][i] = fmaf(pj, vf[i], o[r][i]);
+        }
+      }
+    }
+    __syncwarp();
+  }
+
+  if (lane == 0) {
+#pragma unroll
+    for (int r = 0; r < MAXR; ++r) {
+      sm[warp][r] = m[r];
+      sl[warp][r] = l[r];
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < MAXR; ++r) {
+    if (r < R) {
+      float M = kNegInf;
+#pragma unroll
+      for (int w = 0; w < NW; ++w) M = fmaxf(M, sm[w][r]);
+      float f = (m[r] == kNegInf) ? 0.f : ex2(m[r] - M);
+#pragma unroll
+      for (int i = 0; i < VPL; ++i) atomicAdd(&so[r][lane * VPL + i], o[r][i] * f);
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < R * D; i += blockDim.x) {
+    int r = i / D, d = i - r * D;
+    float M = kNegInf;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, sm[w][r]);
+    int64_t pr = part_row(vd, kvh, it.split, R, r);
+    if (d == 0) {
+      float L = 0.f;
+#pragma unroll
+      for (int w = 0; w < NW; ++w)
+        if (sm[w][r] != kNegInf) L += sl[w][r] * ex2(sm[w][r] - M);
+      p.part_ml[pr] = make_float2(M, L);
+    }
+    p.part_o[pr * D + d] = so[r][d];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// a3, tensor path on the warp-level MMA: one CTA per (work item, 64-row block);
+// 4 warps x 16 query rows; 64-token K/V tiles double-buffered with cp.async.
+// ---------------------------------------------------------------------------
+template <int D>
+__global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
+                                                         const __nv_bfloat16* __restrict__ q,
+                                                         const __nv_bfloat16* __restrict__ kp,
+                                                         const __nv_bfloat16* __restrict__ vp) {
+  constexpr int TN = 64;
+  constexpr int LDS = D + 8;  // padded row: ldmatrix rows land in distinct banks
+  constexpr int KSTEPS = D / 16;
+  constexpr int DBLK = D / 8;
+  constexpr int CH = D / 8;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw);
+  __nv_bfloat16* sV = sK + 2 * TN * LDS;
+
+  const PadWorkItem it = p.items[blockIdx.x];
+  const PadVideoDesc vd = p.videos[it.video];
+  const int R = vd.n_events * p.group;
+  const int row0 = blockIdx.y * 64;
+  if (row0 >= R) return;
+  const int kvh = it.kvh;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t4 = lane & 3;
+
+  const int rlo = row0 + warp * 16 + g, rhi = rlo + 8;
+  uint32_t qa[KSTEPS][4];
+  {
+    const __nv_bfloat16* ql = rlo < R ? q_row(p, vd, q, kvh, rlo) : nullptr;
+    const __nv_bfloat16* qh = rhi < R ? q_row(p, vd, q, kvh, rhi) : nullptr;
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk) {
+      const int c = kk * 16 + 2 * t4;
+      qa[kk][0] = ql ? *reinterpret_cast<const uint32_t*>(ql + c) : 0u;
+      qa[kk][1] = qh ? *reinterpret_cast<const uint32_t*>(qh + c) : 0u;
+      qa[kk][2] = ql ? *reinterpret_cast<const uint32_t*>(ql + c + 8) : 0u;
+      qa[kk][3] = qh ? *reinterpret_cast<const uint32_t*>(qh + c + 8) : 0u;
+    }
+  }
+
+  const size_t row_stride = (size_t)p.h_kv * D;
+  const __nv_bfloat16* kbase = kp + (size_t)vd.prefix_off * row_stride + (size_t)kvh * D;
+  const __nv_bfloat16* vbase = vp + (size_t)vd.prefix_off * row_stride + (size_t)kvh * D;
+  const int ntiles = (it.tok_end - it.tok_begin + TN - 1) / TN;
+
+  auto load_tile = [&](int tile, int stage) {
+    const int base = it.tok_begin + tile * TN;
+    for (int i = threadIdx.x; i < TN * CH; i += 128) {
+      const int r = i / CH, c = i - (i / CH) * CH;
+      const int tok = base + r;
+      const bool ok = tok < it.tok_end;
+      const size_t go = (size_t)(ok ? tok : it.tok_begin) * row_stride + c * 8;
+      cp_async16(sK + (stage * TN + r) * LDS + c * 8, kbase + go, ok);
+      cp_async16(sV + (stage * TN + r) * LDS + c * 8, vbase + go, ok);
+    }
+    cp_async_commit();
+  };
+
+  float o[DBLK][4];
+#pragma unroll
+  for (int i = 0; i < DBLK; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m_lo = kNegInf, m_hi = kNegInf, l_lo = 0.f, l_hi = 0.f;
+
+  load_tile(0, 0);
+  for (int tile = 0; tile < ntiles; ++tile) {
+    if (tile + 1 < ntiles) {
+      load_tile(tile + 1, (tile + 1) & 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const __nv_bfloat16* tK = sK + (tile & 1) * TN * LDS;
+    const __nv_bfloat16* tV = sV + (tile & 1) * TN * LDS;
+
+    float s[TN / 8][4];
+#pragma unroll
+    for (int i = 0; i < TN / 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
+#pragma unroll
+    for (int nb2 = 0; nb2 < TN / 16; ++nb2) {
+#pragma unroll
+      for (int kk = 0; kk < KSTEPS; ++kk) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(b0, b1, b2, b3,
+                tK + (nb2 * 16 + (lane >> 4) * 8 + (lane & 7)) * LDS + kk * 16 + ((lane >> 3) & 1) * 8);
+        mma_bf16(s[2 * nb2], qa[kk], b0, b1);
+        mma_bf16(s[2 * nb2 + 1], qa[kk], b2, b3);
+      }
+    }
+
+    const int valid = it.tok_end - (it.tok_begin + tile * TN);
+    float mx_lo = kNegInf, mx_hi = kNegInf;
+#pragma unroll
+    for (int nb = 0; nb < TN / 8; ++nb) {
+      const int c0 = nb * 8 + 2 * t4;
+      s[nb][0] = c0 < valid ? s[nb][0] * p.scale_log2 : kNegInf;
+      s[nb][1] = c0 + 1 < valid ? s[nb][1] * p.scale_log2 : kNegInf;
+      s[nb][2] = c0 < valid ? s[nb][2] * p.scale_log2 : kNegInf;
+      s[nb][3] = c0 + 1 < valid ? s[nb][3] * p.scale_log2 : kNegInf;
+      mx_lo = fmaxf(mx_lo, fmaxf(s[nb][0], s[nb][1]));
+      mx_hi = fmaxf(mx_hi, fmaxf(s[nb][2], s[nb][3]));
+    }
+    mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, 1));
+    mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, 2));
+    mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 1));
+    mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 2));
+    const float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);  // finite (valid >= 1)
+    const float a_lo = ex2(m_lo - mn_lo), a_hi = ex2(m_hi - mn_hi);
+    m_lo = mn_lo;
+    m_hi = mn_hi;
+    float rs_lo = 0.f, rs_hi = 0.f;
+#pragma unroll
+    for (int nb = 0; nb < TN / 8; ++nb) {
+      s[nb][0] = ex2(s[nb][0] - mn_lo);
+      s[nb][1] = ex2(s[nb][1] - mn_lo);
+      s[nb][2] = ex2(s[nb][2] - mn_hi);
+      s[nb][3] = ex2(s[nb][3] - mn_hi);
+      rs_lo += s[nb][0] + s[nb][1];
+      rs_hi += s[nb][2] + s[nb][3];
+    }
+    l_lo = l_lo * a_lo + rs_lo;
+    l_hi = l_hi * a_hi + rs_hi;
+#pragma unroll
+    for (int db = 0; db < DBLK; ++db) {
+      o[db][0] *= a_lo;
+      o[db][1] *= a_lo;
+      o[db][2] *= a_hi;
+      o[db][3] *= a_hi;
+    }
+
+#pragma unroll
+    for (int ks = 0; ks < TN / 16; ++ks) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(s[2 * ks][0], s[2 * ks][1]);
+      pa[1] = pack_bf16(s[2 * ks][2], s[2 * ks][3]);
+      pa[2] = pack_bf16(s[2 * ks + 1][0], s[2 * ks + 1][1]);
+      pa[3] = pack_bf16(s[2 * ks + 1][2], s[2 * ks + 1][3]);
+#pragma unroll
+      for (int db2 = 0; db2 < DBLK / 2; ++db2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(b0, b1, b2, b3,
+                  tV + (ks * 16 + ((lane >> 3) & 1) * 8 + (lane & 7)) * LDS + (2 * db2 + (lane >> 4)) * 8);
+        mma_bf16(o[2 * db2], pa, b0, b1);
+        mma_bf16(o[2 * db2 + 1], pa, b2, b3);
+      }
+    }
+    __syncthreads();
+  }
+
+  l_lo += __shfl_xor_sync(0xffffffffu, l_lo, 1);
+  l_lo += __shfl_xor_sync(0xffffffffu, l_lo, 2);
+  l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 1);
+  l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 2);
+  if (rlo < R) {
+    const int64_t pr = part_row(vd, kvh, it.split, R, rlo);
+    if (t4 == 0) p.part_ml[pr] = make_float2(m_lo, l_lo);
+    float* dst = p.part_o + pr * D;
+#pragma unroll
+    for (int db = 0; db < DBLK; ++db)
+      *reinterpret_cast<float2*>(dst + db * 8 + 2 * t4) = make_float2(o[db][0], o[db][1]);
+  }
+  if (rhi < R) {
+    const int64_t pr = part_row(vd, kvh, it.split, R, rhi);
+    if (t4 == 0) p.part_ml[pr] = make_float2(m_hi, l_hi);
+    float* dst = p.part_o + pr * D;
+#pragma unroll
+    for (int db = 0; db < DBLK; ++db)
+      *reinterpret_cast<float2*>(dst + db * 8 + 2 * t4) = make_float2(o[db][2], o[db][3]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// a4 + a5: one CTA (128 threads) per (event, kv-head).  Private-suffix pass over
+// the branch's len+1 paged keys (thread = key for q.k, thread = head_dim element
+// for p.v), then the log-sum-exp merge with the prefix partials of its G rows.
+// ---------------------------------------------------------------------------
+template <int D, int MAXG>
+__global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
+                                                           const __nv_bfloat16* __restrict__ q,
+                                                           const __nv_bfloat16* __restrict__ kpool,
+                                                           const __nv_bfloat16* __restrict__ vpool,
+                                                           void* __restrict__ out,
+                                                           float* __restrict__ lse) {
+  constexpr int NT = 128;
+  __shared__ float sq[MAXG][D];
+  __shared__ float sp[MAXG][NT];
+  __shared__ int spage[NT];
+  __shared__ float sred[NT / 32][MAXG];
+  __shared__ float s_m[MAXG], s_l[MAXG], s_a[MAXG];
+
+  const int e = blockIdx.x / p.h_kv;
+  const int kvh = blockIdx.x - e * p.h_kv;
+  const int G = p.group;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const PadEventDesc ev = p.events[e];
+  const PadVideoDesc vd = p.videos[ev.video];
+
+  for (int i = tid; i < MAXG * D; i += NT) {
+    int g = i / D, d = i - g * D;
+    sq[g][d] = g < G ? __bfloat162float(q[((size_t)e * p.h_q + kvh * G + g) * D + d]) : 0.f;
+  }
+  if (tid < MAXG) {
+    s_m[tid] = kNegInf;
+    s_l[tid] = 0.f;
+  }
+  __syncthreads();
+
+  float acc[MAXG];
+#pragma unroll
+  for (int g = 0; g < MAXG; ++g) acc[g] = 0.f;
+  const int nk = ev.len + 1;
+  const int ps = p.page_size;
+
+  for (int c0 = 0; c0 < nk; c0 += NT) {
+    const int k = c0 + tid;
+    bool valid = k < nk;
+    int page = -1;
+    if (valid) {
+      const int pi = k / ps;
+      page = p.page_table[(size_t)e * p.max_pages + pi];
+      if (page < 0 || page >= p.n_pages) {
+        set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
+        valid = false;
+        page = -1;
+      }
+    }
+    spage[tid] = page;
+    float s[MAXG];
+#pragma unroll
+    for (int g = 0; g < MAXG; ++g) s[g] = 0.f;
+    if (valid) {
+      const uint4* kr = reinterpret_cast<const uint4*>(
+          kpool + (((size_t)page * p.h_kv + kvh) * ps + (k - (k / ps) * ps)) * D);
+#pragma unroll 4
+      for (int d8 = 0; d8 < D / 8; ++d8) {
+        float kf[8];
+        unpack8(__ldg(kr + d8), kf);
+#pragma unroll
+        for (int g = 0; g < MAXG; ++g) {
+          if (g < G) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) s[g] = fmaf(sq[g][d8 * 8 + j], kf[j], s[g]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < MAXG; ++g) {
+      s[g] = valid ? s[g] * p.scale_log2 : kNegInf;
+      float wm = warp_max(s[g]);
+      if (lane == 0) sred[warp][g] = wm;
+    }
+    __syncthreads();
+    if (tid < G) {
+      float cm = kNegInf;
+#pragma unroll
+      for (int w = 0; w < NT / 32; ++w) cm = fmaxf(cm, sred[w][tid]);
+      const float mo = s_m[tid];
+      float mn = fmaxf(mo, cm);
+      if (mn == kNegInf) mn = 0.f;  // only if every key so far failed its bounds check
+      s_a[tid] = ex2(mo - mn);
+      s_m[tid] = mn;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int g = 0; g < MAXG; ++g) {
+      float pr = 0.f;
+      if (g < G) pr = ex2(s[g] - s_m[g]);
+      sp[g][tid] = pr;
+      float ws = warp_sum(pr);
+      if (lane == 0) sred[warp][g] = ws;
+    }
+    __syncthreads();
+    if (tid < G) {
+      float cs = 0.f;
+#pragma unroll
+      for (int w = 0; w < NT / 32; ++w) cs += sred[w][tid];
+      s_l[tid] = s_l[tid] * s_a[tid] + cs;
+    }
+    if (tid < D) {
+      const int d = tid;
+#pragma unroll
+      for (int g = 0; g < MAXG; ++g) acc[g] *= s_a[g];
+      const int nv = min(NT, nk - c0);
+      for (int j = 0; j < nv; ++j) {
+        const int pg = spage[j];
+        if (pg < 0) continue;
+        const int kk = c0 + j;
+        const float v = __bfloat162float(
+            vpool[(((size_t)pg * p.h_kv + kvh) * ps + (kk - (kk / ps) * ps)) * D + d]);
+#pragma unroll
+        for (int g = 0; g < MAXG; ++g) acc[g] = fmaf(sp[g][j], v, acc[g]);
+      }
+    }
+    __syncthreads();
+  }
+
+  // a5: merge the branch state with the prefix partials of the same rows.
+  if (tid < D) {
+    const int d = tid;
+    const int R = vd.n_events * G;
+    const int ns = vd.n_splits;
+#pragma unroll
+    for (int g = 0; g < MAXG; ++g) {
+      if (g >= G) break;
+      const int r = ev.local * G + g;
+      float M = s_m[g];
+      for (int sidx = 0; sidx < ns; ++sidx) M = fmaxf(M, p.part_ml[part_row(vd, kvh, sidx, R, r)].x);
+      const float wb = ex2(s_m[g] - M);
+      float L = s_l[g] * wb;
+      float O = acc[g] * wb;
+      for (int sidx = 0; sidx < ns; ++sidx) {
+        const int64_t pr = part_row(vd, kvh, sidx, R, r);
+        const float2 ml = p.part_ml[pr];
+        const float w = ex2(ml.x - M);
+        L = fmaf(ml.y, w, L);
+        O = fmaf(p.part_o[pr * D + d], w, O);
+      }
+      const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
+      const float res = O / L;
+      if (p.out_bf16)
+        reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
+      else
+        reinterpret_cast<float*>(out)[oi] = res;
+      if (lse != nullptr && d == 0)
+        lse[(size_t)e * p.h_q + kvh * G + g] = (M + log2f(L)) * 0.69314718055994531f;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,
+                          void* v_pool, cudaStream_t s) {
+  const int total = p.n_events * p.h_kv * (p.head_dim / 8);
+  if (total == 0) return cudaSuccess;
+  const int bs = 256;
+  append_kernel<<<(total + bs - 1) / bs, bs, 0, s>>>(
+      p, static_cast<const uint4*>(k_new), static_cast<const uint4*>(v_new),
+      static_cast<uint4*>(k_pool), static_cast<uint4*>(v_pool));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefix_simt(const KParams& p, int max_rows, const void* q, const void* kp,
+                               const void* vp, cudaStream_t s) {
+  if (p.n_items == 0) return cudaSuccess;
+  auto Q = static_cast<const __nv_bfloat16*>(q);
+  auto K = static_cast<const __nv_bfloat16*>(kp);
+  auto V = static_cast<const __nv_bfloat16*>(vp);
+  dim3 grid(p.n_items);
+  if (p.head_dim == 128) {
+    if (max_rows <= 8)
+      prefix_simt_kernel<128, 8><<<grid, 256, 0, s>>>(p, Q, K, V);
+    else
+      prefix_simt_kernel<128, 16><<<grid, 256, 0, s>>>(p, Q, K, V);
+  } else {
+    if (max_rows <= 8)
+      prefix_simt_kernel<64, 8><<<grid, 256, 0, s>>>(p, Q, K, V);
+    else
+      prefix_simt_kernel<64, 16><<<grid, 256, 0, s>>>(p, Q, K, V);
+  }
+  return cudaGetLastError();
+}
+
+template <int D>
+static cudaError_t launch_mma_d(const KParams& p, int max_rows, const void* q, const void* kp,
+                                const void* vp, cudaStream_t s) {
+  constexpr int TN = 64, LDS = D + 8;
+  const size_t smem = 2ull * 2 * TN * LDS * sizeof(__nv_bfloat16);
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(prefix_mma_kernel<D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  dim3 grid(p.n_items, (max_rows + 63) / 64);
+  prefix_mma_kernel<D><<<grid, 128, smem, s>>>(p, static_cast<const __nv_bfloat16*>(q),
+                                               static_cast<const __nv_bfloat16*>(kp),
+                                               static_cast<const __nv_bfloat16*>(vp));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, const void* kp,
+                              const void* vp, cudaStream_t s) {
+  if (p.n_items == 0) return cudaSuccess;
+  if (p.head_dim == 128) return launch_mma_d<128>(p, max_rows, q, kp, vp, s);
+  return launch_mma_d<64>(p, max_rows, q, kp, vp, s);
+}
+
+cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
+                                const void* v_pool, void* out, float* lse, cudaStream_t s) {
+  if (p.n_events == 0) return cudaSuccess;
+  dim3 grid(p.n_events * p.h_kv);
+  auto Q = static_cast<const __nv_bfloat16*>(q);
+  auto K = static_cast<const __nv_bfloat16*>(k_pool);
+  auto V = static_cast<const __nv_bfloat16*>(v_pool);
+  if (p.head_dim == 128) {
+    if (p.group <= 8)
+      branch_merge_kernel<128, 8><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+    else
+      branch_merge_kernel<128, 16><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+  } else {
+    if (p.group <= 8)
+      branch_merge_kernel<64, 8><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+    else
+      branch_merge_kernel<64, 16><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace pad

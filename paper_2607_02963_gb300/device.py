@@ -1,0 +1,87 @@
+"""Device-resident decode batch: uploads a workload's tensors and runs the
+three C-ABI calls of one step (pad_plan -> pad_kv_append -> pad_event_decode_attn).
+
+PyTorch is used only for device memory and streams; every step of the path
+runs in libpad's kernels.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import binding as B
+
+
+def bits_to_bf16(a: np.ndarray, device) -> torch.Tensor:
+    """uint16 bf16 bit patterns -> torch.bfloat16 tensor on ``device`` (exact)."""
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.uint16).view(np.int16))
+    return t.view(torch.bfloat16).to(device)
+
+
+class DeviceBatch:
+    """All device state of one decode step for a ``synth.Workload``-like object."""
+
+    def __init__(self, w, device="cuda", fill_nan: bool = True, flags: int = 0,
+                 out_dtype: int = 0, num_sms: int = 0):
+        self.w = w
+        self.device = torch.device(device)
+        self.problem = B.make_problem(w.h_q, w.h_kv, w.head_dim, w.page_size, w.scale,
+                                      out_dtype=out_dtype, num_sms=num_sms, flags=flags)
+        kp, vp = w.build_pools(fill_nan=fill_nan)
+        self.k_pool = bits_to_bf16(kp, self.device)
+        self.v_pool = bits_to_bf16(vp, self.device)
+        self.k_prefix = bits_to_bf16(w.k_prefix, self.device)
+        self.v_prefix = bits_to_bf16(w.v_prefix, self.device)
+        self.q = bits_to_bf16(w.q, self.device)
+        self.k_new = bits_to_bf16(w.k_new, self.device)
+        self.v_new = bits_to_bf16(w.v_new, self.device)
+        self.page_table = torch.from_numpy(w.page_table.copy()).to(self.device)
+        used = w.page_table[w.page_table >= 0]
+        self.cache = B.CacheState(w.n_pages, used_pages=used)
+        ws = B.pad_workspace_size(self.problem, w.prefix_len, w.event_video)
+        if ws == 0:
+            raise B.PadError(1, B.lib().pad_last_error().decode())
+        self.workspace = torch.empty(ws, dtype=torch.uint8, device=self.device)
+        odt = torch.float32 if out_dtype == 0 else torch.bfloat16
+        self.out = torch.empty((w.n_events, w.h_q, w.head_dim), dtype=odt, device=self.device)
+        self.lse = torch.empty((w.n_events, w.h_q), dtype=torch.float32, device=self.device)
+        self.plan = None
+
+    def plan_step(self, stream=None):
+        w = self.w
+        if self.plan is not None:
+            self.plan.destroy()
+        self.plan = B.pad_plan(self.problem, self.cache, w.prefix_len, w.event_video, w.event_len,
+                               page_table=self.page_table, max_pages=w.max_pages,
+                               workspace=self.workspace, prefix_offset=w.prefix_offset,
+                               stream=stream)
+        return self.plan
+
+    def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None):
+        """plan + append + attention; returns the plan (its new pages stay allocated)."""
+        plan = self.plan_step(stream)
+        B.pad_kv_append(plan, self.k_new if k_new is None else k_new,
+                        self.v_new if v_new is None else v_new, self.k_pool, self.v_pool, stream)
+        B.pad_event_decode_attn(plan, self.q if q is None else q, self.k_prefix, self.v_prefix,
+                                self.k_pool, self.v_pool, self.out if out is None else out,
+                                self.lse if lse is None else lse, stream)
+        return plan
+
+    def release_new_pages(self, plan=None):
+        """Return the pages the last plan took (keeps repeated steps idempotent)."""
+        plan = plan or self.plan
+        np_ = plan.new_pages()
+        np_ = np_[np_ >= 0]
+        if np_.size:
+            self.cache.release(np_)
+
+    def gather_branch(self, e: int, n_tokens: int):
+        """Read branch e's first n_tokens K/V rows back through the device page table."""
+        pt = self.page_table[e].cpu().numpy()
+        ps = self.w.page_size
+        ks, vs = [], []
+        for t in range(n_tokens):
+            pg = int(pt[t // ps])
+            ks.append(self.k_pool[pg, :, t % ps, :])
+            vs.append(self.v_pool[pg, :, t % ps, :])
+        return torch.stack(ks), torch.stack(vs)

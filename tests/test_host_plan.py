@@ -1,0 +1,169 @@
+"""Host logic of the C ABI (no GPU): page bookkeeping of pad_plan against the oracle's
+simulation (bit-exact), the split-KV work list, and argument validation."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_02963_gb300 import binding as B
+from paper_2607_02963_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _dry_plan(prob, cache, w_like):
+    return B.pad_plan(prob, cache, w_like["prefix_len"], w_like["event_video"], w_like["event_len"],
+                      page_table=None, max_pages=w_like["max_pages"], workspace=None)
+
+
+def test_hand_worked_page_append(padlib):
+    g = json.load(open(os.path.join(GOLDEN, "hand_page_append.json")))
+    pt = np.array(g["page_table"], dtype=np.int32)
+    n_pages = 10
+    used = pt[pt >= 0]
+    cache = B.CacheState(n_pages, used_pages=used)
+    assert sorted(cache.free_pages().tolist()) == g["free_pages"]
+    prob = B.make_problem(4, 2, 64, page_size=g["page_size"], num_sms=8)
+    E = len(g["event_len"])
+    plan = _dry_plan(prob, cache, dict(prefix_len=[8], event_video=[0] * E,
+                                       event_len=g["event_len"], max_pages=pt.shape[1]))
+    new = plan.new_pages()
+    expect = np.array(g["expect_page_table"])
+    for e, L in enumerate(g["event_len"]):
+        if L % g["page_size"] == 0:
+            assert new[e] == expect[e, L // g["page_size"]]
+        else:
+            assert new[e] == -1
+    assert cache.free_pages().tolist() == g["expect_free_pages"]
+    # out of pages: nothing changes
+    cache2 = B.CacheState(n_pages, used_pages=[p for p in range(n_pages) if p not in (0, 3)])
+    before = cache2.export().copy()
+    with pytest.raises(B.PadError) as ei:
+        _dry_plan(prob, cache2, dict(prefix_len=[8], event_video=[0] * E, event_len=g["event_len"],
+                                     max_pages=pt.shape[1]))
+    assert ei.value.status == 3
+    assert np.array_equal(cache2.export(), before)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_page_allocation_matches_oracle_simulation(padlib, seed):
+    w = synth.random_small(seed, max_events=9, max_len=70, max_prefix=300)
+    cache = B.CacheState(w.n_pages, used_pages=w.page_table[w.page_table >= 0])
+    prob = B.make_problem(w.h_q, w.h_kv, w.head_dim, w.page_size, num_sms=16)
+    plan = _dry_plan(prob, cache, dict(prefix_len=w.prefix_len, event_video=w.event_video,
+                                       event_len=w.event_len, max_pages=w.max_pages))
+    st, pt, free, slots = oracle.simulate_append(w.page_table, w.free_pages, w.event_len, w.page_size)
+    assert st == oracle.OK
+    new = plan.new_pages()
+    for e in range(w.n_events):
+        L = int(w.event_len[e])
+        if L % w.page_size == 0:
+            assert new[e] == pt[e, L // w.page_size]
+        else:
+            assert new[e] == -1
+    assert np.array_equal(cache.free_pages(), free)
+    assert plan.info()["n_new_pages"] == int(np.sum(w.event_len % w.page_size == 0))
+
+
+def test_split_work_list_covers_each_prefix_once(padlib):
+    w = synth.ragged_serving.__wrapped__ if hasattr(synth.ragged_serving, "__wrapped__") else None
+    rng = np.random.default_rng(0)
+    P = rng.integers(1, 5000, size=7).astype(np.int32)
+    Ev = rng.integers(0, 5, size=7)
+    P[3] = 0
+    ev_video = np.repeat(np.arange(7, dtype=np.int32), Ev)
+    L = np.zeros(ev_video.size, dtype=np.int32) + 3
+    cache = B.CacheState(64)
+    prob = B.make_problem(28, 4, 128, num_sms=152)
+    plan = B.pad_plan(prob, cache, P, ev_video, L, max_pages=2, workspace=None)
+    info = plan.info()
+    sl = info["split_len"]
+    assert sl % 128 == 0
+    expect_items = sum(4 * -(-int(P[b]) // sl) for b in range(7) if Ev[b] > 0 and P[b] > 0)
+    assert info["n_work_items"] == expect_items
+    expect_rows = sum(4 * -(-int(P[b]) // sl) * int(Ev[b]) * 7 for b in range(7) if P[b] > 0)
+    assert info["partial_rows"] == expect_rows
+    ws = B.pad_workspace_size(prob, P, ev_video)
+    assert ws == info["workspace_bytes"] and ws % 256 == 0
+
+
+def test_workload_sizes_and_kernel_choice(padlib):
+    prob = B.make_problem(28, 4, 128, num_sms=152)
+    cache = B.CacheState(1000)
+    # 32k prefix, 32 events: R = 224 rows -> tensor path
+    plan = B.pad_plan(prob, cache, [32768], [0] * 32, [1] * 32, max_pages=4, workspace=None)
+    info = plan.info()
+    assert info["prefix_kernel"] in (B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC)
+    assert info["n_work_items"] >= 140
+    # one event (R = 7 rows): warp-shuffle path
+    plan = B.pad_plan(prob, cache, [16384], [0], [1], max_pages=4, workspace=None)
+    assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_SIMT
+
+
+@pytest.mark.parametrize("case,status", [
+    (dict(event_video=[1, 0]), 1),                       # not sorted by video
+    (dict(event_video=[0, 2]), 1),                       # video out of range
+    (dict(event_len=[-1, 0]), 1),                        # negative length
+    (dict(event_len=[64, 0]), 1),                        # page index beyond max_pages
+    (dict(head_dim=96), 2),                              # unsupported head_dim
+    (dict(h_q=6, h_kv=4), 1),                            # h_q not a multiple of h_kv
+    (dict(page_size=12), 2),                             # unsupported page size
+    (dict(h_q=34, h_kv=2), 2),                           # group 17 > 16
+    (dict(prefix_len=[-3, 4]), 1),                       # negative prefix
+])
+def test_invalid_arguments_change_nothing(padlib, case, status):
+    args = dict(event_video=[0, 1], event_len=[3, 0], prefix_len=[100, 50], h_q=8, h_kv=2,
+                head_dim=64, page_size=16, max_pages=4)
+    args.update(case)
+    prob = B.make_problem(args["h_q"], args["h_kv"], args["head_dim"], args["page_size"])
+    cache = B.CacheState(16)
+    before = cache.export().copy()
+    with pytest.raises(B.PadError) as ei:
+        B.pad_plan(prob, cache, args["prefix_len"], args["event_video"], args["event_len"],
+                   max_pages=args["max_pages"], workspace=None)
+    assert ei.value.status == status
+    assert np.array_equal(cache.export(), before)
+
+
+def test_empty_step(padlib):
+    prob = B.make_problem(8, 2, 64)
+    cache = B.CacheState(4)
+    plan = B.pad_plan(prob, cache, [10], [], [], max_pages=1, workspace=None)
+    info = plan.info()
+    assert info["n_events"] == 0 and info["n_work_items"] == 0 and info["n_new_pages"] == 0
+    plan = B.pad_plan(prob, cache, [], [], [], max_pages=1, workspace=None)
+    assert plan.info()["n_work_items"] == 0
+
+
+def test_cache_state_checkpoint_and_errors(padlib):
+    c = B.CacheState(10, used_pages=[1, 4, 5])
+    assert c.free_count == 7
+    snap = c.export()
+    with pytest.raises(B.PadError):
+        c.mark_used([4])          # already used
+    with pytest.raises(B.PadError):
+        c.release([2])            # already free
+    with pytest.raises(B.PadError):
+        c.mark_used([10])         # out of range
+    with pytest.raises(B.PadError):
+        c.mark_used([2, 2])       # listed twice
+    assert np.array_equal(c.export(), snap)
+    c.release([1, 4])
+    assert c.free_count == 9
+    c2 = B.CacheState(10)
+    c2.import_(snap)
+    assert c2.free_count == 7 and np.array_equal(c2.export(), snap)
+    with pytest.raises(B.PadError):
+        c2.import_(np.zeros(9, dtype=np.uint8))
+
+
+def test_launch_calls_reject_plans_without_workspace(padlib):
+    prob = B.make_problem(8, 2, 64)
+    cache = B.CacheState(4)
+    plan = B.pad_plan(prob, cache, [10], [0], [0], max_pages=1, workspace=None)
+    with pytest.raises(B.PadError) as ei:
+        B.lib().pad_kv_append(plan.handle, None, None, None, None, None) and None
+        B._check(B.lib().pad_kv_append(plan.handle, None, None, None, None, None))
+    assert ei.value.status == 1
