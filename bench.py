@@ -1,0 +1,550 @@
+#!/usr/bin/env python3
+"""Throughput of one event-factorized parallel decode step (one attention layer) on GB300.
+
+A step is the whole hot path: pad_plan (host work list + page allocation, uploaded
+asynchronously), pad_kv_append (each branch's new K/V into its page) and
+pad_event_decode_attn (shared-prefix split-KV pass, private-suffix pass and
+log-sum-exp merge).  The default workload is the long-video case: batch 1,
+H_q=28, H_kv=4, head_dim 128, shared prefix 32768 tokens, 32 events with private
+lengths uniform in [0, 128], K with per-channel LogNormal(0, 0.5) scale.
+
+Timing: W warm-up steps, then exactly K steps between CUDA events on the
+launching stream; every step uses the next of several cold replicas of the whole
+device state (their total exceeds 3x the L2 size), so each step reads from HBM.
+The JSON line also carries:
+  roofline      the shared-prefix kernel: algorithmic bytes (prefix K+V read once)
+                per launch / its event-timed duration, against the measured HBM peak;
+  e2e           the same metric through the C ABI with host buffers: H2D of the
+                step's inputs (q, k_new, v_new) from pinned memory and D2H of the
+                outputs (O, LSE) inside the timed region, synchronised every step;
+  cpu_baseline  the fp64 oracle on this host's cores over a bounded sample;
+  clocks        NVML SM clock and clock-event reasons sampled during the timed loop.
+
+Multi-GPU: the path does not shard (one GPU, no collectives); with N ranks every
+rank runs an independent replica of the step ("replicas only"), and value is
+the events of all ranks divided by the slowest rank's time.
+
+--impl reference times the fp64 oracle (the only other implementation) on the
+host cores with the same metric; each step is a bounded sample of the workload.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "event-tokens/s per decode step per layer; achieved HBM GB/s vs ~8 TB/s roofline"
+UNIT = "event-tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+
+WORKLOADS = {
+    "long_32k": "batch 1, H_q 28, H_kv 4, D 128, prefix 32768 (32736 audio-visual + 32 planning), "
+                "E 32, private lengths uniform [0,128], K per-channel LogNormal(0,0.5) scale",
+    "gqa_8k": "batch 1, H_q 28, H_kv 4, D 128, prefix 8192, E 8, private lengths uniform [0,64]",
+    "ragged": "16 videos, H_q 28, H_kv 4, D 128, prefix uniform [4096,16384]+16, "
+              "E per video uniform [4,24], private lengths uniform [0,96]",
+    "tiny": "batch 1, H_q 4, H_kv 1, D 64, prefix 512, E 4, private lengths {0,5,11,16}",
+}
+for _E in (1, 2, 4, 8, 16, 32, 64):
+    WORKLOADS[f"sweep_e{_E}"] = f"batch 1, H_q 28, H_kv 4, D 128, prefix 16384, E {_E}, private length 48"
+
+
+def make_workload(name):
+    from paper_2607_02963_gb300 import synth
+    if name == "long_32k":
+        return synth.long_32k()
+    if name == "gqa_8k":
+        return synth.gqa_8k()
+    if name == "ragged":
+        return synth.ragged_serving()
+    if name == "tiny":
+        return synth.tiny()
+    if name.startswith("sweep_e"):
+        return synth.event_sweep(int(name[len("sweep_e"):]))
+    raise SystemExit(f"unknown workload {name}")
+
+
+# ---------------------------------------------------------------------------
+# Distributed helpers (replicas only: a barrier and max/sum reductions)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), \
+        int(os.environ.get("LOCAL_RANK", 0))
+
+
+def init_dist(backend):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return rank, world
+
+
+def barrier(device=None):
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        if device is not None and device.type == "cuda":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+def aggregate(units: float, ms: float, device=None):
+    """(sum of units over ranks, max of ms over ranks)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return units, ms
+    dev = device if device is not None else torch.device("cpu")
+    u = torch.tensor([units], dtype=torch.float64, device=dev)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(u.item()), float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling through NVML (read-only)
+# ---------------------------------------------------------------------------
+
+_REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+            0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+            0x100: "display_clock_setting"}
+
+
+class ClockSampler:
+    def __init__(self, torch_index=0, period_s=0.005):
+        self.period = period_s
+        self.samples = []
+        self.max_mhz = None
+        self.ok = False
+        self._stop = threading.Event()
+        self._thread = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            found = False
+            try:
+                import torch
+                uuid = str(torch.cuda.get_device_properties(torch_index).uuid)
+                if not uuid.startswith("GPU-"):
+                    uuid = "GPU-" + uuid
+                found = nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) == 0
+            except Exception:
+                found = False
+            if not found and nv.nvmlDeviceGetHandleByIndex_v2(torch_index, ctypes.byref(h)) != 0:
+                return
+            self.nv, self.h = nv, h
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = int(mx.value)
+            fn = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None)
+            self._reasons_fn = fn or getattr(nv, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            self.ok = True
+        except Exception:
+            self.ok = False
+
+    def _loop(self):
+        c = ctypes.c_uint()
+        r = ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            if self.nv.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(c)) == 0:
+                rv = int(r.value) if self._reasons_fn(self.h, ctypes.byref(r)) == 0 else 0
+                self.samples.append((int(c.value), rv))
+            time.sleep(self.period)
+
+    def start(self):
+        if self.ok:
+            self._stop.clear()
+            self._thread = threading.Thread(target=self._loop, daemon=True)
+            self._thread.start()
+
+    def stop(self):
+        if self._thread is not None:
+            self._stop.set()
+            self._thread.join()
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [], "samples": 0,
+                    "source": "nvml" if self.ok else "unavailable"}
+        mhz = [s[0] for s in self.samples]
+        bits = 0
+        for _, rv in self.samples:
+            bits |= rv
+        reasons = [n for b, n in _REASONS.items() if bits & b]
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": self.max_mhz,
+                "sm_mhz_min": min(mhz), "reasons": reasons, "samples": len(mhz), "source": "nvml"}
+
+
+# ---------------------------------------------------------------------------
+# Peaks and ncu-derived traffic
+# ---------------------------------------------------------------------------
+
+def hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as fh:
+            d = json.load(fh)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_02963_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".h")):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload, kernel):
+    """dram read+write bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources for this workload; else None."""
+    p = os.path.join(ROOT, "profiles", "prefix_traffic.txt")
+    if not os.path.exists(p):
+        return None
+    want = kernel_source_hash()
+    for line in open(p):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        kv = dict(x.split("=", 1) for x in line.split() if "=" in x)
+        if kv.get("workload") == workload and kv.get("kernel") == kernel and kv.get("src") == want:
+            return int(float(kv["dram_bytes_per_launch"]))
+    return None
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the fp64 oracle on a bounded sample
+# ---------------------------------------------------------------------------
+
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    env = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS")
+    return int(env) if env else os.cpu_count()
+
+
+class OracleSample:
+    """The fp64 oracle, as it stands, on (event, q-heads) samples of a workload.  The bf16
+    inputs are widened to fp64 once, outside any timed region (the GPU arm likewise
+    starts with its inputs resident)."""
+
+    def __init__(self, w):
+        import oracle
+        self.oracle = oracle
+        self.w = w
+        f = oracle.bf16_to_f64
+        self.kp = [f(w.prefix_k(b)) for b in range(w.n_videos)]
+        self.vp = [f(w.prefix_v(b)) for b in range(w.n_videos)]
+        self.q = f(w.q)
+        self.kb = [np.concatenate([f(w.priv_k(e)), f(w.k_new[e:e + 1])]) for e in range(w.n_events)]
+        self.vb = [np.concatenate([f(w.priv_v(e)), f(w.v_new[e:e + 1])]) for e in range(w.n_events)]
+
+    def run(self, e, heads=None):
+        """Oracle for event e (all heads, or the listed q-heads); returns event-tokens done."""
+        b = int(self.w.event_video[e])
+        self.oracle.video_attention(self.q[e:e + 1], self.kp[b], self.vp[b], [self.kb[e]],
+                                    [self.vb[e]], self.w.scale, heads=heads)
+        return 1.0 if heads is None else len(heads) / self.w.h_q
+
+
+def cpu_baseline(w, budget_s=10.0):
+    """Oracle, as it stands, on whole events of the workload until ~budget_s of CPU work."""
+    smp = OracleSample(w)
+    t0 = time.perf_counter()
+    n = 0
+    while n < w.n_events:
+        smp.run(n)
+        n += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": f"{n} of {w.n_events} events of the workload (all {w.h_q} q-heads each; "
+                      f"numpy fp64 with the explicit event mask; inputs widened to fp64 before "
+                      f"timing), {dt:.1f} s"}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    init_dist("nccl")
+
+    from paper_2607_02963_gb300 import binding as B
+    from paper_2607_02963_gb300 import build as pad_build
+    from paper_2607_02963_gb300.device import DeviceBatch, bits_to_bf16
+
+    if rank == 0 or world == 1:
+        pad_build.build()
+    barrier(device)
+    B.lib()
+
+    w = make_workload(args.workload)
+    byt = w.bytes_algorithmic()
+    l2 = int(getattr(torch.cuda.get_device_properties(device), "L2_cache_size", 0) or (126 << 20))
+    stream = torch.cuda.current_stream(device)
+
+    first = DeviceBatch(w, device=device, fill_nan=False)
+    per_rep = sum(t.numel() * t.element_size() for t in
+                  (first.k_prefix, first.v_prefix, first.k_pool, first.v_pool, first.q, first.k_new,
+                   first.v_new, first.out, first.lse, first.workspace, first.page_table))
+    n_rep = args.replicas or max(2, -(-3 * l2 // per_rep))
+    reps = [first] + [DeviceBatch(w, device=device, fill_nan=False) for _ in range(n_rep - 1)]
+
+    def launcher(db, **kw):
+        return B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                              db.page_table, w.max_pages, db.workspace, w.prefix_offset,
+                              kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
+                              db.k_pool, db.v_pool, db.out, db.lse, stream)
+
+    steps = [launcher(db) for db in reps]
+    info = reps[0].plan_step(stream).info()
+    reps[0].release_new_pages()
+    torch.cuda.synchronize()
+
+    W, K = max(3, args.warmup), args.steps
+    for i in range(W):
+        steps[i % n_rep]()
+    torch.cuda.synchronize()
+    barrier(device)
+
+    sampler = ClockSampler(local)
+    B.pad_timing_enable(K)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    sampler.start()
+    h0 = time.perf_counter()
+    ev0.record(stream)
+    for i in range(K):
+        steps[(W + i) % n_rep]()
+    ev1.record(stream)
+    h1 = time.perf_counter()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1)
+    pre_ms, pre_n = B.pad_timing_read()
+    for db in reps:
+        B.pad_device_status(db.plan_step(stream))
+        db.release_new_pages()
+
+    units, ms_max = aggregate(float(w.n_events * K), ms, device)
+    value = units / (ms_max * 1e-3)
+
+    # e2e through the C ABI with host buffers: H2D inputs, step, D2H outputs, sync.
+    Ke = max(3, min(K, args.e2e_steps))
+    hq = torch.empty(reps[0].q.shape, dtype=torch.bfloat16, pin_memory=True)
+    hkn = torch.empty(reps[0].k_new.shape, dtype=torch.bfloat16, pin_memory=True)
+    hvn = torch.empty(reps[0].v_new.shape, dtype=torch.bfloat16, pin_memory=True)
+    hq.copy_(bits_to_bf16(w.q, "cpu"))
+    hkn.copy_(bits_to_bf16(w.k_new, "cpu"))
+    hvn.copy_(bits_to_bf16(w.v_new, "cpu"))
+    hout = torch.empty(reps[0].out.shape, dtype=reps[0].out.dtype, pin_memory=True)
+    hlse = torch.empty(reps[0].lse.shape, dtype=torch.float32, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for t in (hq, hkn, hvn))
+    d2h = sum(t.numel() * t.element_size() for t in (hout, hlse))
+
+    def e2e_step(i):
+        db = reps[i % n_rep]
+        db.q.copy_(hq, non_blocking=True)
+        db.k_new.copy_(hkn, non_blocking=True)
+        db.v_new.copy_(hvn, non_blocking=True)
+        steps[i % n_rep]()
+        hout.copy_(db.out, non_blocking=True)
+        hlse.copy_(db.lse, non_blocking=True)
+        stream.synchronize()
+
+    for i in range(3):
+        e2e_step(i)
+    barrier(device)
+    t0 = time.perf_counter()
+    for i in range(Ke):
+        e2e_step(i)
+    e2e_ms = (time.perf_counter() - t0) * 1e3
+    e_units, e_ms = aggregate(float(w.n_events * Ke), e2e_ms, device)
+    e2e = {"value": e_units / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "steps": Ke,
+           "path": "pinned H2D of q/k_new/v_new, pad_plan + pad_kv_append + pad_event_decode_attn "
+                   "through the C ABI, D2H of O and LSE, stream sync every step"}
+
+    if rank != 0:
+        return
+    peak, peak_kind = hbm_peak()
+    kern_name = {1: "prefix_simt_kernel", 2: "prefix_mma_kernel", 4: "prefix_tc_kernel"}[
+        info["prefix_kernel"]]
+    prefix_ms_per_launch = pre_ms / max(1, pre_n)
+    achieved = byt["prefix"] / (prefix_ms_per_launch * 1e-3) / 1e9
+    step_ms = ms / K
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": ms_max / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic: seeded N(0,1) bf16 Q/K/V shaped like the paper's long omni-modal "
+                "videos (no dataset or weights)",
+        "config": {
+            "workload": args.workload,
+            "description": WORKLOADS[args.workload],
+            "videos": w.n_videos, "events": w.n_events, "h_q": w.h_q, "h_kv": w.h_kv,
+            "head_dim": w.head_dim, "page_size": w.page_size,
+            "prefix_tokens": int(w.prefix_len.sum()),
+            "private_tokens_after_append": int((w.event_len + 1).sum()),
+            "prefix_kernel": kern_name, "splits": info["n_work_items"],
+            "l2": f"{n_rep} rotating cold replicas of the whole device state "
+                  f"({n_rep * per_rep / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
+            "parallelism": "replicas" if world > 1 else "single GPU",
+        },
+        "clocks": clocks,
+        "gpu_launches": K * (1 + (info["n_work_items"] > 0) + 1),
+        "roofline": {
+            "bound": "hbm",
+            "kernel": kern_name,
+            "achieved": achieved,
+            "peak": peak,
+            "unit": "GB/s",
+            "frac": achieved / peak,
+            "peak_kind": peak_kind,
+            "traffic": recorded_traffic(args.workload, kern_name),
+            "algorithmic_bytes_per_launch": byt["prefix"],
+            "launch_us": prefix_ms_per_launch * 1e3,
+            "launches_timed": pre_n,
+        },
+        "step": {
+            "us": step_ms * 1e3,
+            "algorithmic_bytes": byt["total"],
+            "achieved_gbs": byt["total"] / (step_ms * 1e-3) / 1e9,
+            "frac_of_measured_hbm": byt["total"] / (step_ms * 1e-3) / 1e9 / peak,
+            "frac_of_nominal_8tbs": byt["total"] / (step_ms * 1e-3) / 1e9 / 8000.0,
+            "host_us_per_step": (h1 - h0) * 1e6 / K,
+        },
+        "e2e": e2e,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_budget)
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# Reference arm: the fp64 oracle on the host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    w = make_workload(args.workload)
+    H = w.h_q
+    smp = OracleSample(w)
+    # size each step's sample (q-head rows of one event) so the run stays within ~120 s
+    t0 = time.perf_counter()
+    smp.run(0, [0])
+    t_row = max(time.perf_counter() - t0, 1e-4)
+    total = args.steps + max(3, args.warmup)
+    rows_per_step = int(max(1, min(H, 120.0 / (total * t_row))))
+
+    def step(i):
+        e = i % w.n_events
+        h0 = (i * rows_per_step) % H
+        return smp.run(e, [(h0 + j) % H for j in range(rows_per_step)])
+
+    W, K = max(3, args.warmup), args.steps
+    for i in range(W):
+        step(i)
+    t0 = time.perf_counter()
+    done = 0.0
+    for i in range(K):
+        done += step(W + i)
+    dt = time.perf_counter() - t0
+    value = done / dt
+    line = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": dt * 1e3 / K,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic: seeded N(0,1) bf16 Q/K/V widened exactly to fp64",
+        "config": {"workload": args.workload, "description": WORKLOADS[args.workload],
+                   "videos": w.n_videos, "events": w.n_events, "h_q": w.h_q, "h_kv": w.h_kv,
+                   "head_dim": w.head_dim, "prefix_tokens": int(w.prefix_len.sum()),
+                   "parallelism": "host cores"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                         "sample": f"{rows_per_step} q-head row(s) of one event of the workload per step "
+                                   f"(numpy fp64, explicit event mask, inputs widened to fp64 "
+                                   f"before timing)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="long_32k")
+    ap.add_argument("--replicas", type=int, default=0, help="cold replicas (0 = enough for 3x L2)")
+    ap.add_argument("--e2e-steps", type=int, default=500)
+    ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+    try:
+        import torch.distributed as dist
+        if dist.is_initialized():
+            dist.destroy_process_group()
+    except Exception:
+        pass
+
+
+if __name__ == "__main__":
+    main()

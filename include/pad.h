@@ -140,7 +140,10 @@ size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32
  *   max_pages      columns of page_table; event_len[e] / page_size must be < max_pages
  *   workspace      device, 256-byte aligned, at least pad_workspace_size(...) bytes;
  *                  NULL plans on the host only (no upload; the plan cannot be launched)
- *   stream         stream the plan upload (one cudaMemcpyAsync) is ordered on
+ *   stream         stream the plan upload (one cudaMemcpyAsync) is ordered on; the copy is
+ *                  made from library-owned page-locked staging memory (eight slots per
+ *                  device, allocated on first use and kept until exit), so pad_plan does
+ *                  not wait for work already queued on the stream
  *   plan_out       receives the new plan (free with pad_plan_destroy)
  * On any error nothing changes: no page is taken and nothing is uploaded. */
 pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,

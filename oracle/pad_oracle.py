@@ -71,7 +71,8 @@ def event_mask(prefix_len: int, branch_lens) -> np.ndarray:
 # Masked softmax attention for one video (all its events at once)
 # ---------------------------------------------------------------------------
 
-def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return_p=False):
+def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return_p=False,
+                    heads=None):
     """Decode attention of one video's events under the event-factorized mask.
 
     q:          [E_b, H_q, D] float64, one query token per event branch
@@ -81,6 +82,7 @@ def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return
     v_branches: list of E_b arrays [n_e, H_kv, D]
     Returns o [E_b, H_q, D], lse [E_b, H_q] (natural log) and, when asked,
     the probabilities p [E_b, H_q, n_keys] over the full key sequence.
+    ``heads`` restricts the work to those q-heads (the others are left at 0).
     """
     E_b, H_q, D = q.shape
     S, H_kv, _ = k_prefix.shape
@@ -92,7 +94,7 @@ def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return
     o = np.zeros((E_b, H_q, D), dtype=np.float64)
     lse = np.zeros((E_b, H_q), dtype=np.float64)
     p_all = np.zeros((E_b, H_q, n_keys), dtype=np.float64) if return_p else None
-    for j in range(H_q):
+    for j in (range(H_q) if heads is None else heads):
         h = j // G                                   # contiguous GQA head mapping
         s = scale * (q[:, j, :] @ K_all[:, h, :].T)  # [E_b, n_keys]
         s = np.where(M, s, -np.inf)
@@ -145,7 +147,7 @@ def event_rows(w, e, heads=None):
     vp = bf16_to_f64(w.prefix_v(b))
     kb = np.concatenate([bf16_to_f64(w.priv_k(e)), bf16_to_f64(w.k_new[e:e + 1])])
     vb = np.concatenate([bf16_to_f64(w.priv_v(e)), bf16_to_f64(w.v_new[e:e + 1])])
-    o, lse, _ = video_attention(qb, kp, vp, [kb], [vb], w.scale)
+    o, lse, _ = video_attention(qb, kp, vp, [kb], [vb], w.scale, heads=heads)
     if heads is not None:
         return o[0, heads], lse[0, heads]
     return o[0], lse[0]

@@ -263,3 +263,63 @@ def pad_timing_read():
     n = c_int32()
     _check(lib().pad_timing_read(ctypes.byref(ms), ctypes.byref(n)))
     return float(ms.value), int(n.value)
+
+
+class StepLauncher:
+    """One decode step (pad_plan -> pad_kv_append -> pad_event_decode_attn) with every
+    argument converted to ctypes once, so a repeated step costs only the C calls.
+
+    ``release_pages``: return the pages the step took after launching it (keeps a
+    repeated identical step idempotent, as when re-running one step for timing)."""
+
+    def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
+                 page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
+                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True):
+        self.L = lib()
+        self.problem = problem
+        self.cache = cache
+        self._keep = []
+        pl, self.plp = _i32(prefix_len)
+        ev, self.evp = _i32(event_video)
+        el, self.elp = _i32(event_len)
+        self._keep += [pl, ev, el]
+        self.nv, self.ne = int(pl.size), int(ev.size)
+        if prefix_offset is not None:
+            po = np.ascontiguousarray(prefix_offset, dtype=np.int64)
+            self._keep.append(po)
+            self.pop = po.ctypes.data_as(_I64P)
+        else:
+            self.pop = None
+        self.pt = _ptr(page_table)
+        self.maxp = int(max_pages)
+        self.ws = _ptr(workspace)
+        self.wsb = int(workspace.numel())
+        self.stream = _stream(stream)
+        self.args_append = [_ptr(k_new), _ptr(v_new), _ptr(k_pool), _ptr(v_pool), self.stream]
+        self.args_attn = [_ptr(q), _ptr(k_prefix), _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool),
+                          _ptr(out), _ptr(lse), self.stream]
+        self.newp = np.full(self.ne, -1, dtype=np.int32)
+        self.newpp = self.newp.ctypes.data_as(_I32P)
+        self.release = release_pages
+        self.h = c_void_p()
+        self.ph = ctypes.byref(self.h)
+        self.pprob = ctypes.byref(problem)
+
+    def __call__(self):
+        L = self.L
+        _check(L.pad_plan(self.pprob, self.cache.handle, self.nv, self.plp, self.pop, self.ne,
+                          self.evp, self.elp, self.pt, self.maxp, self.ws, self.wsb, self.stream,
+                          self.ph))
+        h = self.h
+        try:
+            _check(L.pad_kv_append(h, *self.args_append))
+            _check(L.pad_event_decode_attn(h, *self.args_attn))
+            if self.release:
+                L.pad_plan_new_pages(h, self.newpp)
+                sel = self.newp[self.newp >= 0]
+                if sel.size:
+                    _check(L.pad_cache_state_release(self.cache.handle,
+                                                     np.ascontiguousarray(sel).ctypes.data_as(_I32P),
+                                                     int(sel.size)))
+        finally:
+            L.pad_plan_destroy(h)

@@ -5,6 +5,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -170,6 +171,61 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   off = align_up(off + (size_t)rows * prob->head_dim * sizeof(float), 256);
   L->total_bytes = off;
   return PAD_OK;
+}
+
+// Pinned staging for the plan upload.  A pageable cudaMemcpyAsync may wait for
+// the stream, which would stall the host behind the previous step; copying
+// from page-locked memory keeps pad_plan asynchronous.  Eight slots per device
+// are reused round-robin; a slot is rewritten only after the event recorded
+// behind its last copy has completed.  Slots are allocated on first use (and
+// grown when a larger plan arrives) and kept until the process exits.
+struct StagingSlot {
+  void* host = nullptr;
+  size_t cap = 0;
+  cudaEvent_t done = nullptr;
+  bool pending = false;
+};
+struct StagingRing {
+  std::mutex mu;
+  StagingSlot slot[8];
+  int next = 0;
+};
+StagingRing g_staging[64];
+
+cudaError_t upload_plan(void* dst, const void* src, size_t n, cudaStream_t s) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  StagingRing& ring = g_staging[dev];
+  std::lock_guard<std::mutex> lk(ring.mu);
+  StagingSlot& sl = ring.slot[ring.next];
+  ring.next = (ring.next + 1) % 8;
+  if (sl.pending) {
+    e = cudaEventSynchronize(sl.done);
+    if (e != cudaSuccess) return e;
+    sl.pending = false;
+  }
+  if (sl.cap < n) {
+    if (sl.host) cudaFreeHost(sl.host);
+    sl.host = nullptr;
+    sl.cap = 0;
+    const size_t cap = std::max<size_t>(n, 64 * 1024);
+    e = cudaHostAlloc(&sl.host, cap, cudaHostAllocDefault);
+    if (e != cudaSuccess) return e;
+    sl.cap = cap;
+  }
+  if (!sl.done) {
+    e = cudaEventCreateWithFlags(&sl.done, cudaEventDisableTiming);
+    if (e != cudaSuccess) return e;
+  }
+  std::memcpy(sl.host, src, n);
+  e = cudaMemcpyAsync(dst, sl.host, n, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return e;
+  e = cudaEventRecord(sl.done, s);
+  if (e != cudaSuccess) return e;
+  sl.pending = true;
+  return cudaSuccess;
 }
 
 // Timing of the dominant kernel (process-global measurement aid).
@@ -435,8 +491,8 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
     std::memcpy(plan->host_image.data() + L.off_items, items.data(), items.size() * sizeof(PadWorkItem));
 
   if (workspace) {
-    cudaError_t ce = cudaMemcpyAsync(workspace, plan->host_image.data(), L.upload_bytes,
-                                     cudaMemcpyHostToDevice, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t ce = upload_plan(workspace, plan->host_image.data(), L.upload_bytes,
+                                 reinterpret_cast<cudaStream_t>(stream));
     if (ce != cudaSuccess) {
       for (int e = 0; e < n_events; ++e)
         if (plan->new_pages[e] >= 0) cache->set(plan->new_pages[e], false);

@@ -195,9 +195,22 @@ def test_sixty_four_events():
 
 
 def test_bf16_output():
+    """bf16 output = round-to-nearest-even of the fp32 output of the same plan (bit-exact);
+    against the oracle the bound grows by the rounding itself: |RNE(x) - x| <= 2^-9 |x|,
+    so rel-L2 <= 2e-3 + 2^-9."""
     w = synth.random_small(3, h_q=8, h_kv=2, max_prefix=900, max_events=6)
-    db, _ = run_full(w, flags=B.FLAG_PREFIX_MMA, out_dtype=1)
-    assert db.out.dtype == torch.bfloat16
+    db32 = DeviceBatch(w, flags=B.FLAG_PREFIX_MMA, out_dtype=0)
+    db32.run_step()
+    db16 = DeviceBatch(w, flags=B.FLAG_PREFIX_MMA, out_dtype=1)
+    plan = db16.run_step()
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    assert db16.out.dtype == torch.bfloat16
+    assert torch.equal(db16.out, db32.out.to(torch.bfloat16))
+    ref_o, _ = oracle.decode_step(w)
+    got = db16.out.double().cpu().numpy()
+    assert np.abs(got - ref_o).max() <= MAX_ABS
+    assert np.linalg.norm(got - ref_o) / np.linalg.norm(ref_o) <= REL_L2 + 2.0 ** -9
 
 
 def test_empty_step_launches_nothing():
