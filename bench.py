@@ -317,12 +317,15 @@ def run_ours(args):
     l2 = int(getattr(torch.cuda.get_device_properties(device), "L2_cache_size", 0) or (126 << 20))
     stream = torch.cuda.current_stream(device)
 
-    first = DeviceBatch(w, device=device, fill_nan=False)
+    flags = {"auto": 0, "simt": B.FLAG_PREFIX_SIMT, "mma": B.FLAG_PREFIX_MMA,
+             "tc": B.FLAG_PREFIX_TC}[args.prefix]
+    first = DeviceBatch(w, device=device, fill_nan=False, flags=flags)
     per_rep = sum(t.numel() * t.element_size() for t in
                   (first.k_prefix, first.v_prefix, first.k_pool, first.v_pool, first.q, first.k_new,
                    first.v_new, first.out, first.lse, first.workspace, first.page_table))
     n_rep = args.replicas or max(2, -(-3 * l2 // per_rep))
-    reps = [first] + [DeviceBatch(w, device=device, fill_nan=False) for _ in range(n_rep - 1)]
+    reps = [first] + [DeviceBatch(w, device=device, fill_nan=False, flags=flags)
+                      for _ in range(n_rep - 1)]
 
     def launcher(db, **kw):
         return B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
@@ -530,6 +533,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="long_32k")
     ap.add_argument("--replicas", type=int, default=0, help="cold replicas (0 = enough for 3x L2)")
+    ap.add_argument("--prefix", choices=["auto", "simt", "mma", "tc"], default="auto",
+                    help="shared-prefix kernel (auto = the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -152,8 +152,8 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   if (kern == PAD_FLAG_PREFIX_SIMT && max_rows > 16)
     return fail(PAD_ERR_UNSUPPORTED, "SIMT prefix path takes at most 16 rows per (video, kv-head); got %d",
                 max_rows);
-  if (kern == PAD_FLAG_PREFIX_TC)
-    return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path is not built into this library");
+  if (kern == PAD_FLAG_PREFIX_TC && prob->head_dim != 128)
+    return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path takes head_dim 128; got %d", prob->head_dim);
   L->prefix_kernel = kern;
 
   size_t off = sizeof(PadDevHeader);
@@ -598,6 +598,9 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
   switch (plan->lay.prefix_kernel) {
     case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
+    case PAD_FLAG_PREFIX_TC:
+      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, s);
+      break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }
   if (e != cudaSuccess) return cuda_fail(e, "prefix launch");

@@ -457,23 +457,33 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
 }
 
 // ---------------------------------------------------------------------------
-// a4 + a5: one CTA (128 threads) per (event, kv-head).  Private-suffix pass over
-// the branch's len+1 paged keys (thread = key for q.k, thread = head_dim element
-// for p.v), then the log-sum-exp merge with the prefix partials of its G rows.
+// a4 + a5: one CTA (256 threads) per (event, kv-head).
+//   a4, private-suffix pass over the branch's len+1 paged keys: thread = key for
+//   q.k; in p.v each warp takes every 8th key and each lane a head_dim slice, so
+//   the V loads of a warp are independent and 8-16 bytes wide.
+//   a5, log-sum-exp merge with the prefix partials of the branch's G rows: the
+//   row maxima and sums are reduced over splits in parallel, the split weights
+//   are staged in shared memory, and each thread accumulates O for (row, d)
+//   outputs over a chunk of splits with independent loads.
 // ---------------------------------------------------------------------------
 template <int D, int MAXG>
-__global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
+__global__ void __launch_bounds__(256) branch_merge_kernel(KParams p,
                                                            const __nv_bfloat16* __restrict__ q,
                                                            const __nv_bfloat16* __restrict__ kpool,
                                                            const __nv_bfloat16* __restrict__ vpool,
                                                            void* __restrict__ out,
                                                            float* __restrict__ lse) {
-  constexpr int NT = 128;
+  constexpr int NT = 256, NW = NT / 32;
+  constexpr int VPL = D / 32;     // head_dim elements per lane in p.v
+  constexpr int SCH = 64;         // splits per merge chunk
   __shared__ float sq[MAXG][D];
   __shared__ float sp[MAXG][NT];
   __shared__ int spage[NT];
-  __shared__ float sred[NT / 32][MAXG];
+  __shared__ float sred[NW][MAXG];
   __shared__ float s_m[MAXG], s_l[MAXG], s_a[MAXG];
+  __shared__ float so[MAXG][D];
+  __shared__ float sM[MAXG], sL[MAXG];
+  __shared__ float sw[MAXG][SCH];
 
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
@@ -485,6 +495,7 @@ __global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
   for (int i = tid; i < MAXG * D; i += NT) {
     int g = i / D, d = i - g * D;
     sq[g][d] = g < G ? __bfloat162float(q[((size_t)e * p.h_q + kvh * G + g) * D + d]) : 0.f;
+    so[g][d] = 0.f;
   }
   if (tid < MAXG) {
     s_m[tid] = kNegInf;
@@ -492,11 +503,15 @@ __global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
   }
   __syncthreads();
 
-  float acc[MAXG];
+  float acc[MAXG][VPL];
 #pragma unroll
-  for (int g = 0; g < MAXG; ++g) acc[g] = 0.f;
+  for (int g = 0; g < MAXG; ++g)
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) acc[g][i] = 0.f;
   const int nk = ev.len + 1;
   const int ps = p.page_size;
+  const size_t head_off = (size_t)kvh * ps * D;
+  const size_t page_stride = (size_t)p.h_kv * ps * D;
 
   for (int c0 = 0; c0 < nk; c0 += NT) {
     const int k = c0 + tid;
@@ -516,12 +531,15 @@ __global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
 #pragma unroll
     for (int g = 0; g < MAXG; ++g) s[g] = 0.f;
     if (valid) {
-      const uint4* kr = reinterpret_cast<const uint4*>(
-          kpool + (((size_t)page * p.h_kv + kvh) * ps + (k - (k / ps) * ps)) * D);
-#pragma unroll 4
+      const uint4* kr = reinterpret_cast<const uint4*>(kpool + (size_t)page * page_stride + head_off +
+                                                       (size_t)(k % ps) * D);
+      uint4 raw[D / 8];
+#pragma unroll
+      for (int d8 = 0; d8 < D / 8; ++d8) raw[d8] = __ldg(kr + d8);
+#pragma unroll
       for (int d8 = 0; d8 < D / 8; ++d8) {
         float kf[8];
-        unpack8(__ldg(kr + d8), kf);
+        unpack8(raw[d8], kf);
 #pragma unroll
         for (int g = 0; g < MAXG; ++g) {
           if (g < G) {
@@ -541,7 +559,7 @@ __global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
     if (tid < G) {
       float cm = kNegInf;
 #pragma unroll
-      for (int w = 0; w < NT / 32; ++w) cm = fmaxf(cm, sred[w][tid]);
+      for (int w = 0; w < NW; ++w) cm = fmaxf(cm, sred[w][tid]);
       const float mo = s_m[tid];
       float mn = fmaxf(mo, cm);
       if (mn == kNegInf) mn = 0.f;  // only if every key so far failed its bounds check
@@ -561,56 +579,135 @@ __global__ void __launch_bounds__(128) branch_merge_kernel(KParams p,
     if (tid < G) {
       float cs = 0.f;
 #pragma unroll
-      for (int w = 0; w < NT / 32; ++w) cs += sred[w][tid];
+      for (int w = 0; w < NW; ++w) cs += sred[w][tid];
       s_l[tid] = s_l[tid] * s_a[tid] + cs;
     }
-    if (tid < D) {
-      const int d = tid;
 #pragma unroll
-      for (int g = 0; g < MAXG; ++g) acc[g] *= s_a[g];
-      const int nv = min(NT, nk - c0);
-      for (int j = 0; j < nv; ++j) {
-        const int pg = spage[j];
-        if (pg < 0) continue;
-        const int kk = c0 + j;
-        const float v = __bfloat162float(
-            vpool[(((size_t)pg * p.h_kv + kvh) * ps + (kk - (kk / ps) * ps)) * D + d]);
+    for (int g = 0; g < MAXG; ++g) {
+      const float a = s_a[g];
 #pragma unroll
-        for (int g = 0; g < MAXG; ++g) acc[g] = fmaf(sp[g][j], v, acc[g]);
+      for (int i = 0; i < VPL; ++i) acc[g][i] *= a;
+    }
+    const int nv = min(NT, nk - c0);
+#pragma unroll 2
+    for (int j = warp; j < nv; j += NW) {
+      const int pg = spage[j];
+      if (pg < 0) continue;
+      const int kk = c0 + j;
+      const __nv_bfloat16* vr = vpool + (size_t)pg * page_stride + head_off + (size_t)(kk % ps) * D +
+                                lane * VPL;
+      float vf[VPL];
+      if constexpr (VPL == 4) {
+        uint2 raw = __ldg(reinterpret_cast<const uint2*>(vr));
+        vf[0] = bf16_lo(raw.x); vf[1] = bf16_hi(raw.x); vf[2] = bf16_lo(raw.y); vf[3] = bf16_hi(raw.y);
+      } else {
+        uint32_t raw = __ldg(reinterpret_cast<const unsigned int*>(vr));
+        vf[0] = bf16_lo(raw); vf[1] = bf16_hi(raw);
+      }
+#pragma unroll
+      for (int g = 0; g < MAXG; ++g) {
+        if (g < G) {
+          const float pj = sp[g][j];
+#pragma unroll
+          for (int i = 0; i < VPL; ++i) acc[g][i] = fmaf(pj, vf[i], acc[g][i]);
+        }
       }
     }
     __syncthreads();
   }
-
-  // a5: merge the branch state with the prefix partials of the same rows.
-  if (tid < D) {
-    const int d = tid;
-    const int R = vd.n_events * G;
-    const int ns = vd.n_splits;
 #pragma unroll
-    for (int g = 0; g < MAXG; ++g) {
-      if (g >= G) break;
-      const int r = ev.local * G + g;
-      float M = s_m[g];
-      for (int sidx = 0; sidx < ns; ++sidx) M = fmaxf(M, p.part_ml[part_row(vd, kvh, sidx, R, r)].x);
-      const float wb = ex2(s_m[g] - M);
-      float L = s_l[g] * wb;
-      float O = acc[g] * wb;
-      for (int sidx = 0; sidx < ns; ++sidx) {
-        const int64_t pr = part_row(vd, kvh, sidx, R, r);
-        const float2 ml = p.part_ml[pr];
-        const float w = ex2(ml.x - M);
-        L = fmaf(ml.y, w, L);
-        O = fmaf(p.part_o[pr * D + d], w, O);
+  for (int g = 0; g < MAXG; ++g) {
+    if (g < G) {
+#pragma unroll
+      for (int i = 0; i < VPL; ++i) atomicAdd(&so[g][lane * VPL + i], acc[g][i]);
+    }
+  }
+
+  // a5 stage 1: row maxima and sums over the branch and every prefix split.
+  const int R = vd.n_events * G;
+  const int ns = vd.n_splits;
+  const int rbase = ev.local * G;
+  {
+    const int g = tid >> 4, part = tid & 15;  // 16 threads per row
+    float mm = kNegInf;
+    if (g < G) {
+      if (part == 0) mm = s_m[g];
+      for (int sidx = part; sidx < ns; sidx += 16)
+        mm = fmaxf(mm, p.part_ml[part_row(vd, kvh, sidx, R, rbase + g)].x);
+    }
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
+    float ll = 0.f;
+    if (g < G) {
+      if (part == 0) ll = s_l[g] * ex2(s_m[g] - mm);
+      for (int sidx = part; sidx < ns; sidx += 16) {
+        const float2 ml = p.part_ml[part_row(vd, kvh, sidx, R, rbase + g)];
+        ll = fmaf(ml.y, ex2(ml.x - mm), ll);
       }
+    }
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) ll += __shfl_xor_sync(0xffffffffu, ll, o);
+    if (g < G && part == 0) {
+      sM[g] = mm;
+      sL[g] = ll;
+    }
+  }
+  __syncthreads();
+
+  // a5 stage 2: O = (w_b O_b + sum_s w_s O_s) / L, splits in chunks of SCH.
+  constexpr int OUT_PER_T = (MAXG * D + NT - 1) / NT;
+  float oacc[OUT_PER_T];
+#pragma unroll
+  for (int u = 0; u < OUT_PER_T; ++u) {
+    const int idx = tid + u * NT;
+    const int g = idx / D, d = idx - (idx / D) * D;
+    oacc[u] = (g < G) ? so[g][d] * ex2(s_m[g] - sM[g]) : 0.f;
+  }
+  for (int s0 = 0; s0 < ns; s0 += SCH) {
+    const int nch = min(SCH, ns - s0);
+    __syncthreads();
+    for (int i = tid; i < MAXG * SCH; i += NT) {
+      const int g = i / SCH, sl = i - g * SCH;
+      float wv = 0.f;
+      if (g < G && sl < nch) wv = ex2(p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)].x - sM[g]);
+      sw[g][sl] = wv;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < OUT_PER_T; ++u) {
+      const int idx = tid + u * NT;
+      const int g = idx / D, d = idx - (idx / D) * D;
+      if (g < G) {
+        const float* src = p.part_o + part_row(vd, kvh, s0, R, rbase + g) * D + d;
+        const size_t step = (size_t)R * D;
+        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+        int sl = 0;
+        for (; sl + 4 <= nch; sl += 4) {
+          const float v0 = src[(size_t)(sl + 0) * step], v1 = src[(size_t)(sl + 1) * step];
+          const float v2 = src[(size_t)(sl + 2) * step], v3 = src[(size_t)(sl + 3) * step];
+          a0 = fmaf(sw[g][sl + 0], v0, a0);
+          a1 = fmaf(sw[g][sl + 1], v1, a1);
+          a2 = fmaf(sw[g][sl + 2], v2, a2);
+          a3 = fmaf(sw[g][sl + 3], v3, a3);
+        }
+        for (; sl < nch; ++sl) a0 = fmaf(sw[g][sl], src[(size_t)sl * step], a0);
+        oacc[u] += (a0 + a1) + (a2 + a3);
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < OUT_PER_T; ++u) {
+    const int idx = tid + u * NT;
+    const int g = idx / D, d = idx - (idx / D) * D;
+    if (g < G) {
       const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
-      const float res = O / L;
+      const float res = oacc[u] / sL[g];
       if (p.out_bf16)
         reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
       else
         reinterpret_cast<float*>(out)[oi] = res;
       if (lse != nullptr && d == 0)
-        lse[(size_t)e * p.h_q + kvh * G + g] = (M + log2f(L)) * 0.69314718055994531f;
+        lse[(size_t)e * p.h_q + kvh * G + g] = (sM[g] + log2f(sL[g])) * 0.69314718055994531f;
     }
   }
 }
@@ -686,14 +783,14 @@ cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_p
   auto V = static_cast<const __nv_bfloat16*>(v_pool);
   if (p.head_dim == 128) {
     if (p.group <= 8)
-      branch_merge_kernel<128, 8><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+      branch_merge_kernel<128, 8><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
     else
-      branch_merge_kernel<128, 16><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+      branch_merge_kernel<128, 16><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
   } else {
     if (p.group <= 8)
-      branch_merge_kernel<64, 8><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+      branch_merge_kernel<64, 8><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
     else
-      branch_merge_kernel<64, 16><<<grid, 128, 0, s>>>(p, Q, K, V, out, lse);
+      branch_merge_kernel<64, 16><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
   }
   return cudaGetLastError();
 }

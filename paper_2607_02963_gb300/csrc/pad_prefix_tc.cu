@@ -1,0 +1,590 @@
+// a3 on the 5th-generation tensor cores: split-KV flash-decode over the shared
+// prefix (the part of the event-factorized mask of Sec. 3.4 that every branch
+// of a video sees: the multimodal prefix P and all planning tokens G^1..G^K, S).
+//
+// One CTA per (work item = video, kv-head, prefix split; row group of <= 256
+// query rows).  The R = E_b * G query rows of the video's events that read this
+// kv-head are the M dimension of two 128-row MMA tiles, so each K/V tile is
+// brought from HBM once and used by every event and every GQA head of the group.
+//
+//   warp 0      TMA producer: K and V tiles of 64 tokens (two 64-column halves,
+//               128-byte swizzle) into a 4-stage ring, mbarrier transaction counts
+//   warp 1      MMA issuer (one thread): S = Q K^T into TMEM (double-buffered per
+//               M-tile), then O += P V with P read back from TMEM
+//   warp 2      TMEM allocator (512 columns) and deallocator
+//   warps 4-7   softmax of M-tile 0; warps 8-11 softmax of M-tile 1: one thread
+//               per query row (its TMEM lane), online max / sum in base 2, P
+//               written as packed bf16 over its S columns, lazy rescaling of O
+//               (only when a row maximum grows by more than 2^8)
+//
+// TMEM columns: S[m][b] at 64*(2m+b) (fp32, 64 tokens), O[m] at 256+128m (fp32,
+// 128 head-dim columns).  Output: the partial softmax state (m, l, O) of every
+// row for this split, merged with the other splits and the branch by the
+// branch/merge kernel.
+//
+// Every mbarrier wait is bounded (about one second of %globaltimer); a wait
+// that runs out records PAD_ERR_DEVICE_TIMEOUT in the status word, raises a
+// CTA-wide abort flag, lets the producer and the MMA issuer drain what they
+// already started, frees TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "pad_internal.h"
+
+namespace pad {
+
+namespace {
+
+constexpr int kD = 128;
+constexpr int kBN = 64;        // prefix tokens per K/V tile
+constexpr int kStages = 4;
+constexpr int kThreads = 384;
+constexpr uint32_t kHalfBytes = kBN * 128;         // 64 tokens x 64 bf16 = 8 KB
+constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 16 KB
+constexpr uint32_t kQHalfBytes = 128 * 128;        // 128 rows x 64 bf16 = 16 KB
+constexpr uint32_t kQTileBytes = 2 * kQHalfBytes;  // one M-tile of Q: 32 KB
+constexpr uint32_t kOffQ = 0;
+constexpr uint32_t kOffK = kOffQ + 2 * kQTileBytes;
+constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
+constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;   // + slack for 1024-byte alignment
+constexpr uint32_t kTmemCols = 512;
+constexpr float kLazyRescale = 8.0f;                  // log2 units
+constexpr unsigned long long kWaitNs = 1000000000ull; // one second per wait
+
+struct TcBars {
+  uint64_t kfull[kStages];
+  uint64_t vfull[kStages];
+  uint64_t kempty[kStages];
+  uint64_t vempty[kStages];
+  uint64_t sfull[2][2];   // [M-tile][S buffer]
+  uint64_t pfull[2][2];
+  uint64_t pvdone[2];     // one completion per P.V of that M-tile
+  uint64_t drain;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+static_assert(sizeof(TcBars) <= 256, "barrier block fits its slot");
+
+// Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1), A and B
+// bf16 (bits 7-9, 10-12 = 1), K-major A (bit 15 = 0), B major-ness in bit 16,
+// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+constexpr uint32_t make_idesc(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+constexpr uint32_t kIdescS = make_idesc(128, kBN, false);   // S = Q K^T: B = K tile, K-major
+constexpr uint32_t kIdescPV = make_idesc(128, kD, true);    // O += P V: B = V tile, N(=d)-major
+
+__device__ __forceinline__ uint32_t colS(int m, int b) { return 64u * (2 * m + b); }
+__device__ __forceinline__ uint32_t colO(int m) { return 256u + 128u * m; }
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void set_error(PadDevHeader* h, int code, int a, int b, int c) {
+  if (atomicCAS(&h->status, 0, code) == 0) {
+    h->info[0] = a;
+    h->info[1] = b;
+    h->info[2] = c;
+  }
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// ---------------------------------------------------------------- mbarrier
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase of the given parity.  false = gave up (timeout or abort).
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
+                                       PadDevHeader* hdr, int where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 0) {
+      if (*reinterpret_cast<volatile int32_t*>(&bars->abort)) return false;
+      if (globaltimer() - t0 > kWaitNs) {
+        set_error(hdr, PAD_ERR_DEVICE_TIMEOUT, (int)blockIdx.x, where, (int)threadIdx.x);
+        *reinterpret_cast<volatile int32_t*>(&bars->abort) = 1;
+        return false;
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------- TMA
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
+                                            int c2, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// ---------------------------------------------------------------- tcgen05
+__device__ __forceinline__ void fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: start address, leading / stride byte offsets,
+// version 1 (bits 46-47), 128-byte swizzle (layout type 2 in bits 61-63).
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    prefix_tc_kernel(const KParams p, const __nv_bfloat16* __restrict__ q,
+                     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  TcBars* bars = reinterpret_cast<TcBars*>(smem + kOffBar);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const PadWorkItem it = p.items[blockIdx.x];
+  const PadVideoDesc vd = p.videos[it.video];
+  const int R = vd.n_events * p.group;
+  const int row0 = blockIdx.y * 256;
+  if (row0 >= R) return;  // uniform over the CTA, before any barrier or allocation
+  const int rows = min(256, R - row0);
+  const int n_mt = (rows + 127) >> 7;
+  const int ntok = it.tok_end - it.tok_begin;
+  const int n_tiles = (ntok + kBN - 1) / kBN;
+  const int kvh = it.kvh;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bars->kfull[s], 1);
+      mbar_init(&bars->vfull[s], 1);
+      mbar_init(&bars->kempty[s], 1);
+      mbar_init(&bars->vempty[s], 1);
+    }
+    for (int m = 0; m < 2; ++m) {
+      for (int b = 0; b < 2; ++b) {
+        mbar_init(&bars->sfull[m][b], 1);
+        mbar_init(&bars->pfull[m][b], 4);  // one arrival per softmax warp
+      }
+      mbar_init(&bars->pvdone[m], 1);
+    }
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 2) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&bars->tmem_base)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+
+  // Q rows of this row group into the 128-byte-swizzled K-major layout the MMA reads:
+  // M-tile m, half h (head-dim 64h..64h+63), row r, 16-byte chunk c at
+  // m*32K + h*16K + r*128 + ((c ^ (r & 7)) << 4).  Rows past R are zero.
+  for (int idx = threadIdx.x; idx < n_mt * 128 * 16; idx += kThreads) {
+    const int r = idx >> 4, c = idx & 15;
+    const int m = r >> 7, rr = r & 127, h = c >> 3, cc = c & 7;
+    const int grow = row0 + r;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (grow < R) {
+      const int el = grow / p.group;
+      const int gh = grow - el * p.group;
+      const __nv_bfloat16* src =
+          q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * kD + c * 8;
+      v = __ldg(reinterpret_cast<const uint4*>(src));
+    }
+    *reinterpret_cast<uint4*>(smem + kOffQ + m * kQTileBytes + h * kQHalfBytes + rr * 128 +
+                              ((cc ^ (rr & 7)) << 4)) = v;
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = bars->tmem_base;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+      const int tok0 = (int)(vd.prefix_off + it.tok_begin);
+      int issued = 0;
+      bool ok = true;
+      for (int j = 0; j < n_tiles && ok; ++j) {
+        const int s = j % kStages;
+        const uint32_t par = (uint32_t)((j / kStages - 1) & 1);
+        if (j >= kStages) ok = mbar_wait(&bars->kempty[s], par, bars, p.header, 1);
+        if (!ok) break;
+        mbar_expect_tx(&bars->kfull[s], kTileBytes);
+        const uint32_t kd = sbase + kOffK + s * kTileBytes;
+        tma_load_3d(kd, &tmK, 0, kvh, tok0 + j * kBN, &bars->kfull[s]);
+        tma_load_3d(kd + kHalfBytes, &tmK, 64, kvh, tok0 + j * kBN, &bars->kfull[s]);
+        if (j >= kStages) ok = mbar_wait(&bars->vempty[s], par, bars, p.header, 2);
+        if (!ok) {
+          issued = 2 * j + 1;
+          break;
+        }
+        mbar_expect_tx(&bars->vfull[s], kTileBytes);
+        const uint32_t vdst = sbase + kOffV + s * kTileBytes;
+        tma_load_3d(vdst, &tmV, 0, kvh, tok0 + j * kBN, &bars->vfull[s]);
+        tma_load_3d(vdst + kHalfBytes, &tmV, 64, kvh, tok0 + j * kBN, &bars->vfull[s]);
+        issued = 2 * (j + 1);
+      }
+      if (!ok) {
+        // drain: the last loads issued must land before the CTA leaves
+        for (int u = max(0, issued - 2 * kStages); u < issued; ++u) {
+          const int j = u >> 1;
+          const int s = j % kStages;
+          uint64_t* bar = (u & 1) ? &bars->vfull[s] : &bars->kfull[s];
+          const unsigned long long t0 = globaltimer();
+          while (!mbar_try_wait(bar, (uint32_t)((j / kStages) & 1)) && globaltimer() - t0 < kWaitNs) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      auto issue_S = [&](int m, int j) {
+        const int s = j % kStages, b = j & 1;
+        const uint32_t d = tmem + colS(m, b);
+        const uint32_t qa = sbase + kOffQ + m * kQTileBytes;
+        const uint32_t kb = sbase + kOffK + s * kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t half = kk >> 2, koff = (kk & 3) * 32;
+          mma_ss(d, sdesc(qa + half * kQHalfBytes + koff, 16, 1024),
+                 sdesc(kb + half * kHalfBytes + koff, 16, 1024), kIdescS, kk > 0 ? 1u : 0u);
+        }
+      };
+      auto issue_PV = [&](int m, int j) {
+        const int s = j % kStages, b = j & 1;
+        const uint32_t d = tmem + colO(m);
+        const uint32_t a = tmem + colS(m, b);
+        const uint32_t vb = sbase + kOffV + s * kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          // V tile, N(=head-dim)-major: 16 tokens per step (2048 bytes), the second
+          // 64-column half at +kHalfBytes (leading byte offset), 8-row groups 1024 apart.
+          mma_ts(d, a + kk * 8, sdesc(vb + kk * 2048, kHalfBytes, 1024), kIdescPV,
+                 (j > 0 || kk > 0) ? 1u : 0u);
+        }
+      };
+      bool ok = true;
+      for (int j = 0; j < min(2, n_tiles) && ok; ++j) {
+        const int s = j % kStages;
+        ok = mbar_wait(&bars->kfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 3);
+        if (!ok) break;
+        fence_after();
+        for (int m = 0; m < n_mt; ++m) {
+          issue_S(m, j);
+          mma_commit(&bars->sfull[m][j & 1]);
+        }
+        mma_commit(&bars->kempty[s]);
+      }
+      for (int j = 0; j < n_tiles && ok; ++j) {
+        const int s = j % kStages;
+        ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
+        for (int m = 0; m < n_mt && ok; ++m) {
+          ok = mbar_wait(&bars->pfull[m][j & 1], (uint32_t)((j >> 1) & 1), bars, p.header, 5);
+          if (!ok) break;
+          fence_after();
+          issue_PV(m, j);
+          mma_commit(&bars->pvdone[m]);
+        }
+        if (!ok) break;
+        mma_commit(&bars->vempty[s]);
+        const int jn = j + 2;
+        if (jn < n_tiles) {
+          const int sn = jn % kStages;
+          ok = mbar_wait(&bars->kfull[sn], (uint32_t)((jn / kStages) & 1), bars, p.header, 6);
+          if (!ok) break;
+          fence_after();
+          for (int m = 0; m < n_mt && ok; ++m) {
+            // S[m][jn & 1] still holds P of tile j until that P.V has completed
+            ok = mbar_wait(&bars->pvdone[m], (uint32_t)(j & 1), bars, p.header, 7);
+            if (!ok) break;
+            fence_after();
+            issue_S(m, jn);
+            mma_commit(&bars->sfull[m][jn & 1]);
+          }
+          if (!ok) break;
+          mma_commit(&bars->kempty[sn]);
+        }
+      }
+      // every MMA issued by this thread has completed once this commit lands
+      mma_commit(&bars->drain);
+      const unsigned long long t0 = globaltimer();
+      while (!mbar_try_wait(&bars->drain, 0u) && globaltimer() - t0 < kWaitNs) {
+      }
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ softmax
+    const int m = (warp - 4) >> 2;
+    if (m < n_mt) {
+      const int lane_base = 32 * (warp & 3);
+      const int grow = row0 + m * 128 + lane_base + lane;
+      const bool warp_active = (row0 + m * 128 + lane_base) < R;
+      const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
+      const float sl2 = p.scale_log2;
+      float m_run = -__builtin_huge_valf(), l_run = 0.f;
+      bool ok = true;
+      uint32_t r[32];
+      for (int j = 0; j < n_tiles; ++j) {
+        const int b = j & 1;
+        ok = mbar_wait(&bars->sfull[m][b], (uint32_t)((j >> 1) & 1), bars, p.header, 8);
+        ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
+        if (!ok) break;
+        fence_after();
+        if (warp_active) {
+          const int valid = min(kBN, ntok - j * kBN);
+          float mx = -__builtin_huge_valf();
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            tmem_ld32(tl + colS(m, b) + 32 * c, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
+          }
+          mx *= sl2;
+          const float m_new = fmaxf(m_run, mx);
+          const bool need = m_new > m_run + kLazyRescale;
+          if (__any_sync(0xffffffffu, need && j > 0)) {
+            // O[m] must hold P.V of tile j-1 before it is rescaled
+            ok = mbar_wait(&bars->pvdone[m], (uint32_t)((j - 1) & 1), bars, p.header, 9);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            fence_after();
+            const float alpha = need ? ex2(m_run - m_new) : 1.f;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+              tmem_ld32(tl + colO(m) + 32 * c, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+              tmem_st32(tl + colO(m) + 32 * c, r);
+            }
+            tmem_wait_st();
+            if (need) l_run *= alpha;
+          }
+          if (need) m_run = m_new;
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            tmem_ld32(tl + colS(m, b) + 32 * c, r);
+            tmem_wait_ld();
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const int col = 32 * c + 2 * i;
+              const float p0 = col < valid ? ex2(fmaf(__uint_as_float(r[2 * i]), sl2, -m_run)) : 0.f;
+              const float p1 =
+                  col + 1 < valid ? ex2(fmaf(__uint_as_float(r[2 * i + 1]), sl2, -m_run)) : 0.f;
+              l_run += p0 + p1;
+              pk[i] = pack_bf16(p0, p1);
+            }
+            tmem_st16(tl + colS(m, b) + 16 * c, pk);
+          }
+          tmem_wait_st();
+        }
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->pfull[m][b]);
+      }
+      // the issuer commits `drain` after its last MMA: O[m] is final once it lands
+      if (ok) ok = mbar_wait(&bars->drain, 0u, bars, p.header, 10);
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok && warp_active) {
+        fence_after();
+        const int64_t pr = (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + it.split) * R + grow;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          tmem_ld32(tl + colO(m) + 32 * c, r);
+          tmem_wait_ld();
+          if (grow < R) {
+            float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                   __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+          }
+        }
+        if (grow < R) p.part_ml[pr] = make_float2(m_run, l_run);
+      }
+    }
+  }
+
+  __syncwarp();
+  fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &qres) == cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// Token-major [T, h_kv, 128] bf16 prefix as a 3-D tensor (d, head, token); one box is
+// 64 head-dim columns x 1 head x 64 tokens with the 128-byte swizzle.
+bool make_map(CUtensorMap* map, const void* base, int h_kv, int64_t tokens) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)h_kv, (cuuint64_t)tokens};
+  cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)h_kv * kD * 2};
+  cuuint32_t box[3] = {64, 1, (cuuint32_t)kBN};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
+                             const void* vp, int64_t total_prefix_tokens, cudaStream_t s) {
+  if (p.n_items == 0) return cudaSuccess;
+  if (p.head_dim != kD || total_prefix_tokens <= 0 || total_prefix_tokens > (int64_t)INT32_MAX)
+    return cudaErrorInvalidValue;
+  CUtensorMap mk, mv;
+  if (!make_map(&mk, kp, p.h_kv, total_prefix_tokens) || !make_map(&mv, vp, p.h_kv, total_prefix_tokens))
+    return cudaErrorInvalidValue;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(prefix_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  dim3 grid(p.n_items, (max_rows + 255) / 256);
+  prefix_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, static_cast<const __nv_bfloat16*>(q), mk, mv);
+  return cudaGetLastError();
+}
+
+}  // namespace pad

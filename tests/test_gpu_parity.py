@@ -107,31 +107,35 @@ def test_tiny_full(flags):
     run_full(synth.tiny(), flags=flags)
 
 
-def test_gqa_8k_full():
-    run_full(synth.gqa_8k())
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+def test_gqa_8k_full(flags):
+    run_full(synth.gqa_8k(), flags=flags)
 
 
-def test_long_32k_sampled():
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
+def test_long_32k_sampled(flags):
     w = synth.long_32k()
     rng = np.random.default_rng(0)
     ev = sorted(set([0, w.n_events - 1] + list(rng.choice(w.n_events, 4, replace=False))))
-    run_sampled(w, ev)
+    run_sampled(w, ev, flags=flags)
 
 
-def test_ragged_serving_sampled():
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
+def test_ragged_serving_sampled(flags):
     w = synth.ragged_serving()
     ev = []
     for b in range(w.n_videos):
         idx = w.events_of_video(b)
         ev += [int(idx[0]), int(idx[-1])] if b % 3 == 0 else [int(idx[len(idx) // 2])]
-    run_sampled(w, sorted(set(ev)))
+    run_sampled(w, sorted(set(ev)), flags=flags)
 
 
 @pytest.mark.parametrize("E", synth.SWEEP_E)
-def test_event_sweep_sampled(E):
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
+def test_event_sweep_sampled(E, flags):
     w = synth.event_sweep(E)
     ev = sorted(set([0, E - 1, E // 2]))
-    run_sampled(w, ev)
+    run_sampled(w, ev, flags=flags)
 
 
 # ---------------------------------------------------------------------------
@@ -142,6 +146,12 @@ def test_event_sweep_sampled(E):
 def test_random_small_mma(seed):
     run_full(synth.random_small(seed, h_q=8, h_kv=2, max_prefix=900, max_events=7),
              flags=B.FLAG_PREFIX_MMA)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_small_tc(seed):
+    run_full(synth.random_small(seed, h_q=8, h_kv=2, max_prefix=900, max_events=7),
+             flags=B.FLAG_PREFIX_TC)
 
 
 @pytest.mark.parametrize("seed", range(6))
@@ -157,9 +167,10 @@ def test_random_small_head_dim_64(seed):
     run_full(w, flags=B.FLAG_PREFIX_SIMT)
 
 
-def test_large_group_and_outlier_channels():
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+def test_large_group_and_outlier_channels(flags):
     w = synth.random_small(60, h_q=32, h_kv=2, max_prefix=700, max_events=3, k_scale_sigma=0.5)
-    run_full(w, flags=B.FLAG_PREFIX_MMA)
+    run_full(w, flags=flags)
 
 
 # ---------------------------------------------------------------------------
@@ -172,7 +183,7 @@ def _w(prefix, epv, lens, seed=7, h_q=28, h_kv=4, D=128, sigma=None):
                                k_scale_sigma=sigma)
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_SIMT, B.FLAG_PREFIX_MMA])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_SIMT, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
 def test_single_event_empty_branch(flags):
     run_full(_w([300], [1], [0]), flags=flags)          # query sees the prefix and itself
 
@@ -182,16 +193,32 @@ def test_page_boundaries(lens):
     run_full(_w([257], [len(lens)], lens))
 
 
-def test_prefix_not_multiple_of_tile_and_tiny_prefix():
-    run_full(_w([1, 129, 65], [2, 3, 2], [3, 0, 9, 16, 2, 5, 7]))
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+def test_prefix_not_multiple_of_tile_and_tiny_prefix(flags):
+    run_full(_w([1, 129, 65], [2, 3, 2], [3, 0, 9, 16, 2, 5, 7]), flags=flags)
 
 
-def test_video_with_empty_prefix_and_video_without_events():
-    run_full(_w([0, 500, 200], [2, 0, 3], [4, 1, 0, 16, 2]))
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+def test_video_with_empty_prefix_and_video_without_events(flags):
+    run_full(_w([0, 500, 200], [2, 0, 3], [4, 1, 0, 16, 2]), flags=flags)
 
 
-def test_sixty_four_events():
-    run_full(_w([700], [64], list(np.arange(64) % 40)))
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+def test_sixty_four_events(flags):
+    run_full(_w([700], [64], list(np.arange(64) % 40)), flags=flags)
+
+
+def test_long_split_many_tiles_tc():
+    """Few SMs -> long splits: many 64-token tiles per CTA (the 4-stage ring wraps several
+    times, both S buffers alternate, lazy rescaling meets growing maxima)."""
+    w = _w([5000, 3001], [5, 9], list(range(0, 70, 5)), sigma=0.5)
+    db = DeviceBatch(w, flags=B.FLAG_PREFIX_TC, num_sms=4)
+    plan = db.run_step()
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    assert plan.info()["split_len"] >= 2048
+    ref_o, ref_lse = oracle.decode_step(w)
+    check_outputs(db.out.cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, "long splits")
 
 
 def test_bf16_output():
