@@ -118,18 +118,50 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
     L->ev_count[v]++;
     prev = v;
   }
-  int64_t work = 0;
   int max_rows = 0;
-  for (int b = 0; b < n_videos; ++b) {
-    if (L->ev_count[b] > 0) {
-      work += (int64_t)prefix_len[b] * prob->h_kv;
-      max_rows = std::max(max_rows, L->ev_count[b] * L->group);
-    }
-  }
+  for (int b = 0; b < n_videos; ++b)
+    if (L->ev_count[b] > 0) max_rows = std::max(max_rows, L->ev_count[b] * L->group);
   L->max_rows = max_rows;
+
+  // Prefix kernel: forced by a flag, else the tensor-core path for head_dim 128 and the
+  // warp-level paths for head_dim 64 (mma.sync above 8 rows, warp-shuffle below).
+  int kern = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
+  if (kern == 0) {
+    if (prob->head_dim == 128)
+      kern = PAD_FLAG_PREFIX_TC;
+    else
+      kern = (max_rows <= 8) ? PAD_FLAG_PREFIX_SIMT : PAD_FLAG_PREFIX_MMA;
+  }
+  if (kern == PAD_FLAG_PREFIX_SIMT && max_rows > 16)
+    return fail(PAD_ERR_UNSUPPORTED, "SIMT prefix path takes at most 16 rows per (video, kv-head); got %d",
+                max_rows);
+  if (kern == PAD_FLAG_PREFIX_TC && prob->head_dim != 128)
+    return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path takes head_dim 128; got %d", prob->head_dim);
+  L->prefix_kernel = kern;
+
+  // Split length: a multiple of kSplitGranule tokens sized so that the prefix work
+  // (token-heads, times the 128-row groups each item occupies on the tensor-core path)
+  // spreads over one wave of SMs.  The tensor-core kernel runs one CTA per SM, so its
+  // split is grown until items x row groups fit in a single wave.
+  const int groups = (kern == PAD_FLAG_PREFIX_TC) ? std::max(1, (max_rows + 127) / 128) : 1;
+  int64_t work = 0;
+  for (int b = 0; b < n_videos; ++b)
+    if (L->ev_count[b] > 0) work += (int64_t)prefix_len[b] * prob->h_kv * groups;
   const int64_t target = std::max(1, n_sms);
   int64_t chunk = (work + target - 1) / target;
   chunk = std::max<int64_t>(kSplitGranule, (chunk + kSplitGranule - 1) / kSplitGranule * kSplitGranule);
+  auto ctas_for = [&](int64_t c) {
+    int64_t n = 0;
+    for (int b = 0; b < n_videos; ++b)
+      if (L->ev_count[b] > 0 && prefix_len[b] > 0) n += (int64_t)prob->h_kv * ((prefix_len[b] + c - 1) / c);
+    return n * groups;
+  };
+  if (kern == PAD_FLAG_PREFIX_TC) {
+    int64_t max_prefix = 0;
+    for (int b = 0; b < n_videos; ++b)
+      if (L->ev_count[b] > 0) max_prefix = std::max<int64_t>(max_prefix, prefix_len[b]);
+    while (ctas_for(chunk) > target && chunk < max_prefix) chunk += kSplitGranule;
+  }
   if (chunk > (int64_t)1 << 30) return fail(PAD_ERR_UNSUPPORTED, "prefix too long");
   L->split_len = (int)chunk;
   int64_t items = 0, rows = 0;
@@ -146,15 +178,6 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   if (rows > INT32_MAX || items > INT32_MAX) return fail(PAD_ERR_UNSUPPORTED, "batch too large");
   L->n_items = items;
   L->partial_rows = rows;
-
-  int kern = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
-  if (kern == 0) kern = (max_rows <= 8) ? PAD_FLAG_PREFIX_SIMT : PAD_FLAG_PREFIX_MMA;
-  if (kern == PAD_FLAG_PREFIX_SIMT && max_rows > 16)
-    return fail(PAD_ERR_UNSUPPORTED, "SIMT prefix path takes at most 16 rows per (video, kv-head); got %d",
-                max_rows);
-  if (kern == PAD_FLAG_PREFIX_TC && prob->head_dim != 128)
-    return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path takes head_dim 128; got %d", prob->head_dim);
-  L->prefix_kernel = kern;
 
   size_t off = sizeof(PadDevHeader);
   L->off_videos = off;

@@ -254,18 +254,23 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
     }
   }
   __syncthreads();
+  // deterministic combination of the warps' states (fixed order: warp 0, 1, ...)
+  for (int w = 0; w < NW; ++w) {
+    if (warp == w) {
 #pragma unroll
-  for (int r = 0; r < MAXR; ++r) {
-    if (r < R) {
-      float M = kNegInf;
+      for (int r = 0; r < MAXR; ++r) {
+        if (r < R) {
+          float M = kNegInf;
 #pragma unroll
-      for (int w = 0; w < NW; ++w) M = fmaxf(M, sm[w][r]);
-      float f = (m[r] == kNegInf) ? 0.f : ex2(m[r] - M);
+          for (int u = 0; u < NW; ++u) M = fmaxf(M, sm[u][r]);
+          const float f = (m[r] == kNegInf) ? 0.f : ex2(m[r] - M);
 #pragma unroll
-      for (int i = 0; i < VPL; ++i) atomicAdd(&so[r][lane * VPL + i], o[r][i] * f);
+          for (int i = 0; i < VPL; ++i) so[r][lane * VPL + i] += o[r][i] * f;
+        }
+      }
     }
+    __syncthreads();
   }
-  __syncthreads();
   for (int i = threadIdx.x; i < R * D; i += blockDim.x) {
     int r = i / D, d = i - r * D;
     float M = kNegInf;
@@ -615,12 +620,18 @@ __global__ void __launch_bounds__(256) branch_merge_kernel(KParams p,
     }
     __syncthreads();
   }
+  // deterministic reduction of the warps' p.v partial sums (fixed order: warp 0, 1, ...)
+  for (int w = 0; w < NW; ++w) {
+    if (warp == w) {
 #pragma unroll
-  for (int g = 0; g < MAXG; ++g) {
-    if (g < G) {
+      for (int g = 0; g < MAXG; ++g) {
+        if (g < G) {
 #pragma unroll
-      for (int i = 0; i < VPL; ++i) atomicAdd(&so[g][lane * VPL + i], acc[g][i]);
+          for (int i = 0; i < VPL; ++i) so[g][lane * VPL + i] += acc[g][i];
+        }
+      }
     }
+    __syncthreads();
   }
 
   // a5 stage 1: row maxima and sums over the branch and every prefix split.

@@ -2,29 +2,33 @@
 // prefix (the part of the event-factorized mask of Sec. 3.4 that every branch
 // of a video sees: the multimodal prefix P and all planning tokens G^1..G^K, S).
 //
-// One CTA per (work item = video, kv-head, prefix split; row group of <= 256
-// query rows).  The R = E_b * G query rows of the video's events that read this
-// kv-head are the M dimension of two 128-row MMA tiles, so each K/V tile is
-// brought from HBM once and used by every event and every GQA head of the group.
+// One CTA per (work item = video, kv-head, prefix split; group of <= 128 query
+// rows).  The R = E_b * G query rows of the video's events that read this
+// kv-head form the M dimension of the MMA, so each K/V tile brought from HBM
+// serves every event and every GQA head of the group at once; the row groups of
+// one item are adjacent CTAs that run together and share the tiles through L2.
 //
-//   warp 0      TMA producer: K and V tiles of 64 tokens (two 64-column halves,
-//               128-byte swizzle) into a 4-stage ring, mbarrier transaction counts
-//   warp 1      MMA issuer (one thread): S = Q K^T into TMEM (double-buffered per
-//               M-tile), then O += P V with P read back from TMEM
+//   warp 0      TMA producer of K tiles (128 tokens: two 64-column halves, 128-byte
+//               swizzle) into a 3-stage ring; a stage is refilled once the S of
+//               the tile it held has completed
+//   warp 1      MMA issuer (one thread): S = Q K^T into one of three TMEM S
+//               buffers, O += P V with P read back from TMEM; it runs up to two
+//               tiles ahead of the softmax
 //   warp 2      TMEM allocator (512 columns) and deallocator
-//   warps 4-7   softmax of M-tile 0; warps 8-11 softmax of M-tile 1: one thread
-//               per query row (its TMEM lane), online max / sum in base 2, P
-//               written as packed bf16 over its S columns, lazy rescaling of O
-//               (only when a row maximum grows by more than 2^8)
+//   warp 3      TMA producer of V tiles (refilled once the P.V of the tile completed)
+//   warps 4-7   softmax: one thread per query row (its TMEM lane), online max and
+//               sum in base 2, P written as packed bf16 over its S columns, lazy
+//               rescaling of O (only when a row maximum grows by more than 2^8)
 //
-// TMEM columns: S[m][b] at 64*(2m+b) (fp32, 64 tokens), O[m] at 256+128m (fp32,
-// 128 head-dim columns).  Output: the partial softmax state (m, l, O) of every
-// row for this split, merged with the other splits and the branch by the
-// branch/merge kernel.
+// Every MMA has N = 128 (S: 128 tokens; P.V: 128 head-dim columns), the size at
+// which one tcgen05.mma carries as much tensor work as it costs to issue.
+// TMEM columns: S[b] at 128*b (b = 0, 1, 2), O at 384.  Output: the partial
+// softmax state (m, l, O) of every row for this split, merged with the other
+// splits and the branch by the branch/merge kernel.
 //
 // Every mbarrier wait is bounded (about one second of %globaltimer); a wait
 // that runs out records PAD_ERR_DEVICE_TIMEOUT in the status word, raises a
-// CTA-wide abort flag, lets the producer and the MMA issuer drain what they
+// CTA-wide abort flag, lets the producers and the MMA issuer drain what they
 // already started, frees TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -38,30 +42,32 @@ namespace pad {
 namespace {
 
 constexpr int kD = 128;
-constexpr int kBN = 64;        // prefix tokens per K/V tile
-constexpr int kStages = 4;
-constexpr int kThreads = 384;
-constexpr uint32_t kHalfBytes = kBN * 128;         // 64 tokens x 64 bf16 = 8 KB
-constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 16 KB
+constexpr int kBN = 128;       // prefix tokens per K/V tile
+constexpr int kStages = 3;
+constexpr int kSBuf = 3;       // S buffers in TMEM
+constexpr int kThreads = 256;
+constexpr uint32_t kHalfBytes = kBN * 128;         // 128 tokens x 64 bf16 = 16 KB
+constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 32 KB
 constexpr uint32_t kQHalfBytes = 128 * 128;        // 128 rows x 64 bf16 = 16 KB
-constexpr uint32_t kQTileBytes = 2 * kQHalfBytes;  // one M-tile of Q: 32 KB
+constexpr uint32_t kQTileBytes = 2 * kQHalfBytes;  // Q of one 128-row group: 32 KB
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + 2 * kQTileBytes;
+constexpr uint32_t kOffK = kOffQ + kQTileBytes;
 constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;   // + slack for 1024-byte alignment
 constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColO = 384;
 constexpr float kLazyRescale = 8.0f;                  // log2 units
 constexpr unsigned long long kWaitNs = 1000000000ull; // one second per wait
+static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 
 struct TcBars {
   uint64_t kfull[kStages];
   uint64_t vfull[kStages];
-  uint64_t kempty[kStages];
-  uint64_t vempty[kStages];
-  uint64_t sfull[2][2];   // [M-tile][S buffer]
-  uint64_t pfull[2][2];
-  uint64_t pvdone[2];     // one completion per P.V of that M-tile
+  uint64_t vempty[kStages];   // P.V of the tile in this V stage has completed
+  uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
+  uint64_t pfull;             // softmax of the current tile done (4 warp arrivals per tile)
+  uint64_t pvdone;            // one completion per P.V, in tile order
   uint64_t drain;
   uint32_t tmem_base;
   int32_t abort;
@@ -77,9 +83,6 @@ constexpr uint32_t make_idesc(int M, int N, bool b_mn_major) {
 }
 constexpr uint32_t kIdescS = make_idesc(128, kBN, false);   // S = Q K^T: B = K tile, K-major
 constexpr uint32_t kIdescPV = make_idesc(128, kD, true);    // O += P V: B = V tile, N(=d)-major
-
-__device__ __forceinline__ uint32_t colS(int m, int b) { return 64u * (2 * m + b); }
-__device__ __forceinline__ uint32_t colO(int m) { return 256u + 128u * m; }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -134,9 +137,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase of the given parity.  false = gave up (timeout or abort).
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
-                                       PadDevHeader* hdr, int where) {
-  if (mbar_try_wait(bar, parity)) return true;
+__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, TcBars* bars,
+                                            PadDevHeader* hdr, int where) {
   const unsigned long long t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -149,6 +151,11 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* b
       }
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
+                                          PadDevHeader* hdr, int where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, bars, hdr, where);
 }
 
 // ---------------------------------------------------------------- TMA
@@ -242,8 +249,14 @@ __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const unsigned long long t0 = globaltimer();
+  while (!mbar_try_wait(bar, parity) && globaltimer() - t0 < kWaitNs) {
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    prefix_tc_kernel(const KParams p, const __nv_bfloat16* __restrict__ q,
+    prefix_tc_kernel(const KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -252,13 +265,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   TcBars* bars = reinterpret_cast<TcBars*>(smem + kOffBar);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  const PadWorkItem it = p.items[blockIdx.x];
+  const int item = blockIdx.x / n_groups;
+  const int group = blockIdx.x - item * n_groups;
+  const PadWorkItem it = p.items[item];
   const PadVideoDesc vd = p.videos[it.video];
   const int R = vd.n_events * p.group;
-  const int row0 = blockIdx.y * 256;
+  const int row0 = group * 128;
   if (row0 >= R) return;  // uniform over the CTA, before any barrier or allocation
-  const int rows = min(256, R - row0);
-  const int n_mt = (rows + 127) >> 7;
   const int ntok = it.tok_end - it.tok_begin;
   const int n_tiles = (ntok + kBN - 1) / kBN;
   const int kvh = it.kvh;
@@ -267,16 +280,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bars->kfull[s], 1);
       mbar_init(&bars->vfull[s], 1);
-      mbar_init(&bars->kempty[s], 1);
       mbar_init(&bars->vempty[s], 1);
     }
-    for (int m = 0; m < 2; ++m) {
-      for (int b = 0; b < 2; ++b) {
-        mbar_init(&bars->sfull[m][b], 1);
-        mbar_init(&bars->pfull[m][b], 4);  // one arrival per softmax warp
-      }
-      mbar_init(&bars->pvdone[m], 1);
-    }
+    for (int b = 0; b < kSBuf; ++b) mbar_init(&bars->sfull[b], 1);
+    mbar_init(&bars->pfull, 4);  // one arrival per softmax warp
+    mbar_init(&bars->pvdone, 1);
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -289,12 +297,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
 
-  // Q rows of this row group into the 128-byte-swizzled K-major layout the MMA reads:
-  // M-tile m, half h (head-dim 64h..64h+63), row r, 16-byte chunk c at
-  // m*32K + h*16K + r*128 + ((c ^ (r & 7)) << 4).  Rows past R are zero.
-  for (int idx = threadIdx.x; idx < n_mt * 128 * 16; idx += kThreads) {
+  // Q rows of this group into the 128-byte-swizzled K-major layout the MMA reads:
+  // half h (head-dim 64h..64h+63), row r, 16-byte chunk c at
+  // h*16K + r*128 + ((c ^ (r & 7)) << 4).  Rows past R are zero.
+  for (int idx = threadIdx.x; idx < 128 * 16; idx += kThreads) {
     const int r = idx >> 4, c = idx & 15;
-    const int m = r >> 7, rr = r & 127, h = c >> 3, cc = c & 7;
+    const int h = c >> 3, cc = c & 7;
     const int grow = row0 + r;
     uint4 v = make_uint4(0u, 0u, 0u, 0u);
     if (grow < R) {
@@ -304,224 +312,202 @@ __global__ void __launch_bounds__(kThreads, 1)
           q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * kD + c * 8;
       v = __ldg(reinterpret_cast<const uint4*>(src));
     }
-    *reinterpret_cast<uint4*>(smem + kOffQ + m * kQTileBytes + h * kQHalfBytes + rr * 128 +
-                              ((cc ^ (rr & 7)) << 4)) = v;
+    *reinterpret_cast<uint4*>(smem + kOffQ + h * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = v;
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   fence_before();
   __syncthreads();
   fence_after();
   const uint32_t tmem = bars->tmem_base;
+  const int tok0 = (int)(vd.prefix_off + it.tok_begin);
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+  if (warp == 0 || warp == 3) {
+    // ------------------------------------------------------------ TMA producers
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
-      const int tok0 = (int)(vd.prefix_off + it.tok_begin);
+      const bool isK = warp == 0;
+      const CUtensorMap* map = isK ? &tmK : &tmV;
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
       int issued = 0;
       bool ok = true;
-      for (int j = 0; j < n_tiles && ok; ++j) {
-        const int s = j % kStages;
-        const uint32_t par = (uint32_t)((j / kStages - 1) & 1);
-        if (j >= kStages) ok = mbar_wait(&bars->kempty[s], par, bars, p.header, 1);
-        if (!ok) break;
-        mbar_expect_tx(&bars->kfull[s], kTileBytes);
-        const uint32_t kd = sbase + kOffK + s * kTileBytes;
-        tma_load_3d(kd, &tmK, 0, kvh, tok0 + j * kBN, &bars->kfull[s]);
-        tma_load_3d(kd + kHalfBytes, &tmK, 64, kvh, tok0 + j * kBN, &bars->kfull[s]);
-        if (j >= kStages) ok = mbar_wait(&bars->vempty[s], par, bars, p.header, 2);
-        if (!ok) {
-          issued = 2 * j + 1;
-          break;
+      for (int t = 0; t < n_tiles && ok; ++t) {
+        const int s = t % kStages;
+        if (t >= kStages) {
+          // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
+          uint64_t* freed = isK ? &bars->sfull[s] : &bars->vempty[s];
+          ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
+          if (!ok) break;
         }
-        mbar_expect_tx(&bars->vfull[s], kTileBytes);
-        const uint32_t vdst = sbase + kOffV + s * kTileBytes;
-        tma_load_3d(vdst, &tmV, 0, kvh, tok0 + j * kBN, &bars->vfull[s]);
-        tma_load_3d(vdst + kHalfBytes, &tmV, 64, kvh, tok0 + j * kBN, &bars->vfull[s]);
-        issued = 2 * (j + 1);
+        uint64_t* full = isK ? &bars->kfull[s] : &bars->vfull[s];
+        mbar_expect_tx(full, kTileBytes);
+        const uint32_t dst = sbase + (isK ? kOffK : kOffV) + s * kTileBytes;
+        tma_load_3d(dst, map, 0, kvh, tok0 + t * kBN, full);
+        tma_load_3d(dst + kHalfBytes, map, 64, kvh, tok0 + t * kBN, full);
+        issued = t + 1;
       }
       if (!ok) {
-        // drain: the last loads issued must land before the CTA leaves
-        for (int u = max(0, issued - 2 * kStages); u < issued; ++u) {
-          const int j = u >> 1;
-          const int s = j % kStages;
-          uint64_t* bar = (u & 1) ? &bars->vfull[s] : &bars->kfull[s];
-          const unsigned long long t0 = globaltimer();
-          while (!mbar_try_wait(bar, (uint32_t)((j / kStages) & 1)) && globaltimer() - t0 < kWaitNs) {
-          }
+        // the loads already issued must land before the CTA leaves
+        for (int t = max(0, issued - kStages); t < issued; ++t) {
+          uint64_t* full = isK ? &bars->kfull[t % kStages] : &bars->vfull[t % kStages];
+          drain_wait(full, (uint32_t)((t / kStages) & 1));
         }
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      auto issue_S = [&](int m, int j) {
-        const int s = j % kStages, b = j & 1;
-        const uint32_t d = tmem + colS(m, b);
-        const uint32_t qa = sbase + kOffQ + m * kQTileBytes;
-        const uint32_t kb = sbase + kOffK + s * kTileBytes;
+      // Descriptors are built once; a K-step moves the start address, i.e. adds
+      // (byte offset >> 4) to the low field (no carry: addresses stay below 256 KB).
+      const uint64_t dQ = sdesc(sbase + kOffQ, 16, 1024);
+      const uint64_t dK = sdesc(sbase + kOffK, 16, 1024);
+      // V tile, N(=head-dim)-major: 16 tokens per step (2048 bytes), the second
+      // 64-column half at +kHalfBytes (leading byte offset), 8-row groups 1024 apart.
+      const uint64_t dV = sdesc(sbase + kOffV, kHalfBytes, 1024);
+      auto issue_S = [&](int t) {
+        const uint32_t s = (uint32_t)(t % kStages), b = (uint32_t)(t % kSBuf);
+        const uint32_t d = tmem + 128u * b;
+        const uint64_t kb = dK + (s * kTileBytes >> 4);
 #pragma unroll
         for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t half = kk >> 2, koff = (kk & 3) * 32;
-          mma_ss(d, sdesc(qa + half * kQHalfBytes + koff, 16, 1024),
-                 sdesc(kb + half * kHalfBytes + koff, 16, 1024), kIdescS, kk > 0 ? 1u : 0u);
+          const uint32_t off = (uint32_t)(kk >> 2) * kQHalfBytes + (uint32_t)(kk & 3) * 32;
+          mma_ss(d, dQ + (off >> 4), kb + (off >> 4), kIdescS, kk > 0 ? 1u : 0u);
         }
       };
-      auto issue_PV = [&](int m, int j) {
-        const int s = j % kStages, b = j & 1;
-        const uint32_t d = tmem + colO(m);
-        const uint32_t a = tmem + colS(m, b);
-        const uint32_t vb = sbase + kOffV + s * kTileBytes;
+      auto issue_PV = [&](int t) {
+        const uint32_t s = (uint32_t)(t % kStages), b = (uint32_t)(t % kSBuf);
+        const uint32_t a = tmem + 128u * b;
+        const uint64_t vb = dV + (s * kTileBytes >> 4);
+        const uint32_t acc0 = t > 0 ? 1u : 0u;
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          // V tile, N(=head-dim)-major: 16 tokens per step (2048 bytes), the second
-          // 64-column half at +kHalfBytes (leading byte offset), 8-row groups 1024 apart.
-          mma_ts(d, a + kk * 8, sdesc(vb + kk * 2048, kHalfBytes, 1024), kIdescPV,
-                 (j > 0 || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < kBN / 16; ++kk)
+          mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
+                 kk > 0 ? 1u : acc0);
       };
       bool ok = true;
-      for (int j = 0; j < min(2, n_tiles) && ok; ++j) {
-        const int s = j % kStages;
-        ok = mbar_wait(&bars->kfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 3);
+      for (int t = 0; t < min(2, n_tiles) && ok; ++t) {
+        ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
         if (!ok) break;
         fence_after();
-        for (int m = 0; m < n_mt; ++m) {
-          issue_S(m, j);
-          mma_commit(&bars->sfull[m][j & 1]);
-        }
-        mma_commit(&bars->kempty[s]);
+        issue_S(t);
+        mma_commit(&bars->sfull[t % kSBuf]);
       }
       for (int j = 0; j < n_tiles && ok; ++j) {
         const int s = j % kStages;
         ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
-        for (int m = 0; m < n_mt && ok; ++m) {
-          ok = mbar_wait(&bars->pfull[m][j & 1], (uint32_t)((j >> 1) & 1), bars, p.header, 5);
-          if (!ok) break;
-          fence_after();
-          issue_PV(m, j);
-          mma_commit(&bars->pvdone[m]);
-        }
         if (!ok) break;
+        ok = mbar_wait(&bars->pfull, (uint32_t)(j & 1), bars, p.header, 5);
+        if (!ok) break;
+        fence_after();
+        issue_PV(j);
+        mma_commit(&bars->pvdone);
         mma_commit(&bars->vempty[s]);
-        const int jn = j + 2;
-        if (jn < n_tiles) {
-          const int sn = jn % kStages;
-          ok = mbar_wait(&bars->kfull[sn], (uint32_t)((jn / kStages) & 1), bars, p.header, 6);
+        const int t = j + 2;
+        if (t < n_tiles) {
+          ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 6);
+          if (!ok) break;
+          // S buffer t % 3 == (j - 1) % 3 holds P of tile j - 1 until that P.V completes
+          if (j >= 1) ok = mbar_wait(&bars->pvdone, (uint32_t)((j - 1) & 1), bars, p.header, 7);
           if (!ok) break;
           fence_after();
-          for (int m = 0; m < n_mt && ok; ++m) {
-            // S[m][jn & 1] still holds P of tile j until that P.V has completed
-            ok = mbar_wait(&bars->pvdone[m], (uint32_t)(j & 1), bars, p.header, 7);
-            if (!ok) break;
-            fence_after();
-            issue_S(m, jn);
-            mma_commit(&bars->sfull[m][jn & 1]);
-          }
-          if (!ok) break;
-          mma_commit(&bars->kempty[sn]);
+          issue_S(t);
+          mma_commit(&bars->sfull[t % kSBuf]);
         }
       }
       // every MMA issued by this thread has completed once this commit lands
       mma_commit(&bars->drain);
-      const unsigned long long t0 = globaltimer();
-      while (!mbar_try_wait(&bars->drain, 0u) && globaltimer() - t0 < kWaitNs) {
-      }
+      drain_wait(&bars->drain, 0u);
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax
-    const int m = (warp - 4) >> 2;
-    if (m < n_mt) {
-      const int lane_base = 32 * (warp & 3);
-      const int grow = row0 + m * 128 + lane_base + lane;
-      const bool warp_active = (row0 + m * 128 + lane_base) < R;
-      const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
-      const float sl2 = p.scale_log2;
-      float m_run = -__builtin_huge_valf(), l_run = 0.f;
-      bool ok = true;
-      uint32_t r[32];
-      for (int j = 0; j < n_tiles; ++j) {
-        const int b = j & 1;
-        ok = mbar_wait(&bars->sfull[m][b], (uint32_t)((j >> 1) & 1), bars, p.header, 8);
-        ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
-        if (!ok) break;
-        fence_after();
-        if (warp_active) {
-          const int valid = min(kBN, ntok - j * kBN);
-          float mx = -__builtin_huge_valf();
+    const int lane_base = 32 * (warp & 3);
+    const int grow = row0 + lane_base + lane;
+    const bool warp_active = (row0 + lane_base) < R;
+    const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
+    const float sl2 = p.scale_log2;
+    float m_run = -__builtin_huge_valf(), l_run = 0.f;
+    bool ok = true;
+    uint32_t r[32];
+    for (int j = 0; j < n_tiles; ++j) {
+      const uint32_t cS = 128u * (uint32_t)(j % kSBuf);
+      ok = mbar_wait(&bars->sfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 8);
+      ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
+      if (!ok) break;
+      fence_after();
+      if (warp_active) {
+        const int valid = min(kBN, ntok - j * kBN);
+        float mx = -__builtin_huge_valf();
 #pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            tmem_ld32(tl + colS(m, b) + 32 * c, r);
+        for (int c = 0; c < kBN / 32; ++c) {
+          tmem_ld32(tl + cS + 32 * c, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
+        }
+        mx *= sl2;
+        const float m_new = fmaxf(m_run, mx);
+        const bool need = m_new > m_run + kLazyRescale;
+        if (__any_sync(0xffffffffu, need && j > 0)) {
+          // O must hold P.V of tile j-1 before it is rescaled
+          ok = mbar_wait(&bars->pvdone, (uint32_t)((j - 1) & 1), bars, p.header, 9);
+          ok = __all_sync(0xffffffffu, ok);
+          if (!ok) break;
+          fence_after();
+          const float alpha = need ? ex2(m_run - m_new) : 1.f;
+#pragma unroll
+          for (int c = 0; c < kD / 32; ++c) {
+            tmem_ld32(tl + kColO + 32 * c, r);
             tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
-          }
-          mx *= sl2;
-          const float m_new = fmaxf(m_run, mx);
-          const bool need = m_new > m_run + kLazyRescale;
-          if (__any_sync(0xffffffffu, need && j > 0)) {
-            // O[m] must hold P.V of tile j-1 before it is rescaled
-            ok = mbar_wait(&bars->pvdone[m], (uint32_t)((j - 1) & 1), bars, p.header, 9);
-            ok = __all_sync(0xffffffffu, ok);
-            if (!ok) break;
-            fence_after();
-            const float alpha = need ? ex2(m_run - m_new) : 1.f;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-              tmem_ld32(tl + colO(m) + 32 * c, r);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-              tmem_st32(tl + colO(m) + 32 * c, r);
-            }
-            tmem_wait_st();
-            if (need) l_run *= alpha;
-          }
-          if (need) m_run = m_new;
-#pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            tmem_ld32(tl + colS(m, b) + 32 * c, r);
-            tmem_wait_ld();
-            uint32_t pk[16];
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int col = 32 * c + 2 * i;
-              const float p0 = col < valid ? ex2(fmaf(__uint_as_float(r[2 * i]), sl2, -m_run)) : 0.f;
-              const float p1 =
-                  col + 1 < valid ? ex2(fmaf(__uint_as_float(r[2 * i + 1]), sl2, -m_run)) : 0.f;
-              l_run += p0 + p1;
-              pk[i] = pack_bf16(p0, p1);
-            }
-            tmem_st16(tl + colS(m, b) + 16 * c, pk);
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+            tmem_st32(tl + kColO + 32 * c, r);
           }
           tmem_wait_st();
+          if (need) l_run *= alpha;
         }
-        fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->pfull[m][b]);
-      }
-      // the issuer commits `drain` after its last MMA: O[m] is final once it lands
-      if (ok) ok = mbar_wait(&bars->drain, 0u, bars, p.header, 10);
-      ok = __all_sync(0xffffffffu, ok);
-      if (ok && warp_active) {
-        fence_after();
-        const int64_t pr = (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + it.split) * R + grow;
+        if (need) m_run = m_new;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          tmem_ld32(tl + colO(m) + 32 * c, r);
+        for (int c = 0; c < kBN / 32; ++c) {
+          tmem_ld32(tl + cS + 32 * c, r);
           tmem_wait_ld();
-          if (grow < R) {
-            float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c);
+          uint32_t pk[16];
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-              dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
-                                   __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+          for (int i = 0; i < 16; ++i) {
+            const int col = 32 * c + 2 * i;
+            const float p0 = col < valid ? ex2(fmaf(__uint_as_float(r[2 * i]), sl2, -m_run)) : 0.f;
+            const float p1 =
+                col + 1 < valid ? ex2(fmaf(__uint_as_float(r[2 * i + 1]), sl2, -m_run)) : 0.f;
+            l_run += p0 + p1;
+            pk[i] = pack_bf16(p0, p1);
           }
+          // P over the first half of this S buffer; S chunk c sits at columns 32c..32c+31,
+          // so P chunk c (columns 16c..16c+15) only overwrites S values already read.
+          tmem_st16(tl + cS + 16 * c, pk);
         }
-        if (grow < R) p.part_ml[pr] = make_float2(m_run, l_run);
+        tmem_wait_st();
       }
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->pfull);
+    }
+    // the issuer commits `drain` after its last MMA: O is final once it lands
+    if (ok) ok = mbar_wait(&bars->drain, 0u, bars, p.header, 10);
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok && warp_active) {
+      fence_after();
+      const int64_t pr = (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + it.split) * R + grow;
+#pragma unroll
+      for (int c = 0; c < kD / 32; ++c) {
+        tmem_ld32(tl + kColO + 32 * c, r);
+        tmem_wait_ld();
+        if (grow < R) {
+          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                 __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+        }
+      }
+      if (grow < R) p.part_ml[pr] = make_float2(m_run, l_run);
     }
   }
 
@@ -549,7 +535,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 }
 
 // Token-major [T, h_kv, 128] bf16 prefix as a 3-D tensor (d, head, token); one box is
-// 64 head-dim columns x 1 head x 64 tokens with the 128-byte swizzle.
+// 64 head-dim columns x 1 head x 128 tokens with the 128-byte swizzle.
 bool make_map(CUtensorMap* map, const void* base, int h_kv, int64_t tokens) {
   auto enc = get_encode();
   if (!enc) return false;
@@ -582,8 +568,10 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  dim3 grid(p.n_items, (max_rows + 255) / 256);
-  prefix_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, static_cast<const __nv_bfloat16*>(q), mk, mv);
+  const int n_groups = (max_rows + 127) / 128;
+  dim3 grid(p.n_items * n_groups);
+  prefix_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, static_cast<const __nv_bfloat16*>(q),
+                                                      n_groups, mk, mv);
   return cudaGetLastError();
 }
 

@@ -90,16 +90,43 @@ def test_split_work_list_covers_each_prefix_once(padlib):
 
 
 def test_workload_sizes_and_kernel_choice(padlib):
-    prob = B.make_problem(28, 4, 128, num_sms=152)
+    prob = B.make_problem(28, 4, 128, num_sms=148)
     cache = B.CacheState(1000)
-    # 32k prefix, 32 events: R = 224 rows -> tensor path
+    # head_dim 128: tensor-core path; 32 events -> R = 224 rows = two 128-row groups per
+    # item, and items x groups fill one wave of SMs without exceeding it
     plan = B.pad_plan(prob, cache, [32768], [0] * 32, [1] * 32, max_pages=4, workspace=None)
     info = plan.info()
-    assert info["prefix_kernel"] in (B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC)
-    assert info["n_work_items"] >= 140
-    # one event (R = 7 rows): warp-shuffle path
+    assert info["prefix_kernel"] == B.FLAG_PREFIX_TC
+    assert 120 <= 2 * info["n_work_items"] <= 148
     plan = B.pad_plan(prob, cache, [16384], [0], [1], max_pages=4, workspace=None)
+    assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_TC
+    assert plan.info()["n_work_items"] <= 148
+    # head_dim 64: warp-level paths, warp-shuffle for <= 8 rows
+    prob64 = B.make_problem(16, 4, 64, num_sms=148)
+    plan = B.pad_plan(prob64, cache, [4096], [0, 0], [1, 1], max_pages=4, workspace=None)
     assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_SIMT
+    plan = B.pad_plan(prob64, cache, [4096], [0, 0, 0], [1, 1, 1], max_pages=4, workspace=None)
+    assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_MMA
+
+
+def test_tc_split_fits_one_wave(padlib):
+    rng = np.random.default_rng(5)
+    for trial in range(50):
+        B_ = int(rng.integers(1, 17))
+        P = rng.integers(1, 40000, size=B_).astype(np.int32)
+        Ev = rng.integers(1, 40, size=B_)
+        ev_video = np.repeat(np.arange(B_, dtype=np.int32), Ev)
+        L = np.zeros(ev_video.size, dtype=np.int32)
+        sms = int(rng.integers(8, 160))
+        prob = B.make_problem(28, 4, 128, num_sms=sms)
+        plan = B.pad_plan(prob, B.CacheState(4096), P, ev_video, L, max_pages=2, workspace=None)
+        info = plan.info()
+        groups = -(-int(Ev.max()) * 7 // 128)
+        sl = info["split_len"]
+        assert sl % 128 == 0
+        # one wave unless a single split per (video, kv-head) is already too many
+        if sl < int(P.max()):
+            assert info["n_work_items"] * groups <= sms
 
 
 @pytest.mark.parametrize("case,status", [
