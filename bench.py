@@ -342,6 +342,9 @@ def run_ours(args):
     for i in range(W):
         steps[i % n_rep]()
     torch.cuda.synchronize()
+    for db in reps:  # a kernel-side error (e.g. a bounded wait that gave up) stops the run here
+        B.pad_device_status(db.plan_step(stream))
+        db.release_new_pages()
     barrier(device)
 
     sampler = ClockSampler(local)

@@ -26,6 +26,11 @@
 // softmax state (m, l, O) of every row for this split, merged with the other
 // splits and the branch by the branch/merge kernel.
 //
+// Barrier phases: a thread waits for completion #c of a barrier by its parity, which is
+// only sound while completion #c+1 cannot yet have happened.  Every barrier here is
+// therefore per slot (stage, S buffer, or tile parity) so that its next completion
+// depends on progress of the waiting thread itself.
+//
 // Every mbarrier wait is bounded (about one second of %globaltimer); a wait
 // that runs out records PAD_ERR_DEVICE_TIMEOUT in the status word, raises a
 // CTA-wide abort flag, lets the producers and the MMA issuer drain what they
@@ -66,8 +71,8 @@ struct TcBars {
   uint64_t vfull[kStages];
   uint64_t vempty[kStages];   // P.V of the tile in this V stage has completed
   uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
-  uint64_t pfull;             // softmax of the current tile done (4 warp arrivals per tile)
-  uint64_t pvdone;            // one completion per P.V, in tile order
+  uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (4 warp arrivals)
+  uint64_t pvdone[2];         // P.V of tile j completes pvdone[j & 1]
   uint64_t drain;
   uint32_t tmem_base;
   int32_t abort;
@@ -282,9 +287,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->vfull[s], 1);
       mbar_init(&bars->vempty[s], 1);
     }
-    for (int b = 0; b < kSBuf; ++b) mbar_init(&bars->sfull[b], 1);
-    mbar_init(&bars->pfull, 4);  // one arrival per softmax warp
-    mbar_init(&bars->pvdone, 1);
+    for (int b = 0; b < kSBuf; ++b) {
+      mbar_init(&bars->sfull[b], 1);
+      mbar_init(&bars->pfull[b], 4);  // one arrival per softmax warp
+    }
+    mbar_init(&bars->pvdone[0], 1);
+    mbar_init(&bars->pvdone[1], 1);
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -394,18 +402,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = j % kStages;
         ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
         if (!ok) break;
-        ok = mbar_wait(&bars->pfull, (uint32_t)(j & 1), bars, p.header, 5);
+        ok = mbar_wait(&bars->pfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
         if (!ok) break;
         fence_after();
         issue_PV(j);
-        mma_commit(&bars->pvdone);
+        mma_commit(&bars->pvdone[j & 1]);
         mma_commit(&bars->vempty[s]);
         const int t = j + 2;
         if (t < n_tiles) {
           ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 6);
           if (!ok) break;
           // S buffer t % 3 == (j - 1) % 3 holds P of tile j - 1 until that P.V completes
-          if (j >= 1) ok = mbar_wait(&bars->pvdone, (uint32_t)((j - 1) & 1), bars, p.header, 7);
+          if (j >= 1)
+            ok = mbar_wait(&bars->pvdone[(j - 1) & 1], (uint32_t)(((j - 1) >> 1) & 1), bars, p.header, 7);
           if (!ok) break;
           fence_after();
           issue_S(t);
@@ -448,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool need = m_new > m_run + kLazyRescale;
         if (__any_sync(0xffffffffu, need && j > 0)) {
           // O must hold P.V of tile j-1 before it is rescaled
-          ok = mbar_wait(&bars->pvdone, (uint32_t)((j - 1) & 1), bars, p.header, 9);
+          ok = mbar_wait(&bars->pvdone[(j - 1) & 1], (uint32_t)(((j - 1) >> 1) & 1), bars, p.header, 9);
           ok = __all_sync(0xffffffffu, ok);
           if (!ok) break;
           fence_after();
@@ -487,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->pfull);
+      if (lane == 0) mbar_arrive(&bars->pfull[j % kSBuf]);
     }
     // the issuer commits `drain` after its last MMA: O is final once it lands
     if (ok) ok = mbar_wait(&bars->drain, 0u, bars, p.header, 10);
