@@ -575,6 +575,9 @@ static KParams make_params(const pad_plan_t* plan) {
   p.n_events = plan->n_events;
   p.n_items = (int32_t)plan->lay.n_items;
   p.out_bf16 = pr.out_dtype == 1;
+  p.n_sms = plan->lay.n_sms;
+  p.max_splits = 0;
+  for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   auto* ws = static_cast<uint8_t*>(plan->workspace);
   p.header = reinterpret_cast<PadDevHeader*>(ws);
@@ -622,7 +625,11 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
     case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_TC:
-      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, s);
+      // programmatic dependent launch: the prefix pass overlaps the append kernel and the
+      // branch/merge pass's prologue overlaps the prefix pass (not while timing events
+      // are recorded between the kernels)
+      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens,
+                           !timed, s);
       break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }
@@ -631,7 +638,8 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
     cudaEventRecord(g_timing.ev[2 * g_timing.n + 1], s);
     g_timing.n++;
   }
-  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, s);
+  const bool pdl = !timed && plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC;
+  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, pdl, s);
   if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
   return PAD_OK;
 }

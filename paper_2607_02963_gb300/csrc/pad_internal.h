@@ -64,6 +64,8 @@ struct KParams {
   int32_t h_q, h_kv, group, head_dim, page_size, max_pages, n_pages;
   int32_t n_videos, n_events, n_items;
   int32_t out_bf16;
+  int32_t n_sms;                  // SMs the grid sizes were planned for
+  int32_t max_splits;             // largest per-video prefix split count of the batch
   float scale_log2;               // scale * log2(e)
   PadDevHeader* header;
   const PadVideoDesc* videos;
@@ -82,8 +84,10 @@ cudaError_t launch_prefix_simt(const KParams& p, int max_rows, const void* q, co
 cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, const void* kp,
                               const void* vp, cudaStream_t s);
 cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
-                             const void* vp, int64_t total_prefix_tokens, cudaStream_t s);
+                             const void* vp, int64_t total_prefix_tokens, bool pdl, cudaStream_t s);
+// pdl: launch with programmatic stream serialization (the kernel waits for its
+// predecessor with griddepcontrol.wait before it reads anything the predecessor wrote).
 cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
-                                const void* v_pool, void* out, float* lse, cudaStream_t s);
+                                const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 
 }  // namespace pad

@@ -111,6 +111,8 @@ __device__ __forceinline__ int64_t part_row(const PadVideoDesc& vd, int kvh, int
 __global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
                               const uint4* __restrict__ v_new, uint4* __restrict__ k_pool,
                               uint4* __restrict__ v_pool) {
+  // the shared-prefix pass launched after this kernel reads nothing it writes
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int chunks = p.head_dim / 8;
   const int per_event = p.h_kv * chunks;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -462,264 +464,280 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
 }
 
 // ---------------------------------------------------------------------------
-// a4 + a5: one CTA (256 threads) per (event, kv-head).
-//   a4, private-suffix pass over the branch's len+1 paged keys: thread = key for
-//   q.k; in p.v each warp takes every 8th key and each lane a head_dim slice, so
-//   the V loads of a warp are independent and 8-16 bytes wide.
-//   a5, log-sum-exp merge with the prefix partials of the branch's G rows: the
-//   row maxima and sums are reduced over splits in parallel, the split weights
-//   are staged in shared memory, and each thread accumulates O for (row, d)
-//   outputs over a chunk of splits with independent loads.
+// a4 + a5: one CTA (256 threads, 8 warps) per (event, kv-head).
+//   At entry the prefix partials (m, l, O of the branch's G rows for up to `sch`
+//   splits) start streaming into shared memory with cp.async, so they land while
+//   the branch is computed.
+//   a4, the own-branch part of the mask of Sec. 3.4: the branch's len+1 keys, in
+//   chunks of 128, are staged (K and V rows through the page table, cp.async) and
+//   processed as a small flash-attention on the warp-level MMA: the G <= 16 query
+//   rows form one m16 tile; S = Q K^T (warps split the keys), a row softmax (one
+//   warp per row), O += P V (warps split the head dimension).
+//   a5: the log-sum-exp merge of the branch state with the staged partials.
 // ---------------------------------------------------------------------------
-template <int D, int MAXG>
-__global__ void __launch_bounds__(256) branch_merge_kernel(KParams p,
-                                                           const __nv_bfloat16* __restrict__ q,
-                                                           const __nv_bfloat16* __restrict__ kpool,
-                                                           const __nv_bfloat16* __restrict__ vpool,
-                                                           void* __restrict__ out,
-                                                           float* __restrict__ lse) {
-  constexpr int NT = 256, NW = NT / 32;
-  constexpr int VPL = D / 32;     // head_dim elements per lane in p.v
-  constexpr int SCH = 64;         // splits per merge chunk
-  __shared__ float sq[MAXG][D];
-  __shared__ float sp[MAXG][NT];
-  __shared__ int spage[NT];
-  __shared__ float sred[NW][MAXG];
-  __shared__ float s_m[MAXG], s_l[MAXG], s_a[MAXG];
-  __shared__ float so[MAXG][D];
-  __shared__ float sM[MAXG], sL[MAXG];
-  __shared__ float sw[MAXG][SCH];
+constexpr int kBmThreads = 256;
+constexpr int kBmKeys = 64;                   // branch keys per chunk
+
+__host__ __device__ constexpr size_t bm_align16(size_t x) { return (x + 15) / 16 * 16; }
+
+template <int D>
+struct BmSmem {
+  static constexpr int LD = D + 8;            // padded bf16 row: ldmatrix rows in distinct banks
+  __nv_bfloat16 q[16][LD];
+  __nv_bfloat16 k[kBmKeys][LD];
+  __nv_bfloat16 v[kBmKeys][LD];
+  __nv_bfloat16 pb[16][kBmKeys + 8];          // P of the chunk (bf16, A operand of P.V)
+  float sc[16][kBmKeys];                      // scaled scores of the chunk
+  float ob[16][D];                            // branch O, then the merged numerator
+  int page[kBmKeys];
+  float m[16], l[16], a[16];
+  float M[16], L[16];
+};
+
+template <int D>
+__global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
+                                                                  const __nv_bfloat16* __restrict__ q,
+                                                                  const __nv_bfloat16* __restrict__ kpool,
+                                                                  const __nv_bfloat16* __restrict__ vpool,
+                                                                  void* __restrict__ out,
+                                                                  float* __restrict__ lse,
+                                                                  int sch) {
+  constexpr int NT = kBmThreads, NW = NT / 32;
+  constexpr int LD = BmSmem<D>::LD;
+  constexpr int CH = D / 8;                   // 16-byte pieces of a bf16 row
+  extern __shared__ __align__(16) unsigned char bm_raw[];
+  BmSmem<D>& S = *reinterpret_cast<BmSmem<D>*>(bm_raw);
+  float2* sml = reinterpret_cast<float2*>(bm_raw + bm_align16(sizeof(BmSmem<D>)));
+  float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) +
+                                        bm_align16((size_t)p.group * sch * sizeof(float2)));
 
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
   const int G = p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gq = lane >> 2, t4 = lane & 3;
   const PadEventDesc ev = p.events[e];
   const PadVideoDesc vd = p.videos[ev.video];
-
-  for (int i = tid; i < MAXG * D; i += NT) {
-    int g = i / D, d = i - g * D;
-    sq[g][d] = g < G ? __bfloat162float(q[((size_t)e * p.h_q + kvh * G + g) * D + d]) : 0.f;
-    so[g][d] = 0.f;
-  }
-  if (tid < MAXG) {
-    s_m[tid] = kNegInf;
-    s_l[tid] = 0.f;
-  }
-  __syncthreads();
-
-  float acc[MAXG][VPL];
-#pragma unroll
-  for (int g = 0; g < MAXG; ++g)
-#pragma unroll
-    for (int i = 0; i < VPL; ++i) acc[g][i] = 0.f;
-  const int nk = ev.len + 1;
-  const int ps = p.page_size;
-  const size_t head_off = (size_t)kvh * ps * D;
-  const size_t page_stride = (size_t)p.h_kv * ps * D;
-
-  for (int c0 = 0; c0 < nk; c0 += NT) {
-    const int k = c0 + tid;
-    bool valid = k < nk;
-    int page = -1;
-    if (valid) {
-      const int pi = k / ps;
-      page = p.page_table[(size_t)e * p.max_pages + pi];
-      if (page < 0 || page >= p.n_pages) {
-        set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
-        valid = false;
-        page = -1;
-      }
-    }
-    spage[tid] = page;
-    float s[MAXG];
-#pragma unroll
-    for (int g = 0; g < MAXG; ++g) s[g] = 0.f;
-    if (valid) {
-      const uint4* kr = reinterpret_cast<const uint4*>(kpool + (size_t)page * page_stride + head_off +
-                                                       (size_t)(k % ps) * D);
-      uint4 raw[D / 8];
-#pragma unroll
-      for (int d8 = 0; d8 < D / 8; ++d8) raw[d8] = __ldg(kr + d8);
-#pragma unroll
-      for (int d8 = 0; d8 < D / 8; ++d8) {
-        float kf[8];
-        unpack8(raw[d8], kf);
-#pragma unroll
-        for (int g = 0; g < MAXG; ++g) {
-          if (g < G) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j) s[g] = fmaf(sq[g][d8 * 8 + j], kf[j], s[g]);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int g = 0; g < MAXG; ++g) {
-      s[g] = valid ? s[g] * p.scale_log2 : kNegInf;
-      float wm = warp_max(s[g]);
-      if (lane == 0) sred[warp][g] = wm;
-    }
-    __syncthreads();
-    if (tid < G) {
-      float cm = kNegInf;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) cm = fmaxf(cm, sred[w][tid]);
-      const float mo = s_m[tid];
-      float mn = fmaxf(mo, cm);
-      if (mn == kNegInf) mn = 0.f;  // only if every key so far failed its bounds check
-      s_a[tid] = ex2(mo - mn);
-      s_m[tid] = mn;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int g = 0; g < MAXG; ++g) {
-      float pr = 0.f;
-      if (g < G) pr = ex2(s[g] - s_m[g]);
-      sp[g][tid] = pr;
-      float ws = warp_sum(pr);
-      if (lane == 0) sred[warp][g] = ws;
-    }
-    __syncthreads();
-    if (tid < G) {
-      float cs = 0.f;
-#pragma unroll
-      for (int w = 0; w < NW; ++w) cs += sred[w][tid];
-      s_l[tid] = s_l[tid] * s_a[tid] + cs;
-    }
-#pragma unroll
-    for (int g = 0; g < MAXG; ++g) {
-      const float a = s_a[g];
-#pragma unroll
-      for (int i = 0; i < VPL; ++i) acc[g][i] *= a;
-    }
-    const int nv = min(NT, nk - c0);
-#pragma unroll 2
-    for (int j = warp; j < nv; j += NW) {
-      const int pg = spage[j];
-      if (pg < 0) continue;
-      const int kk = c0 + j;
-      const __nv_bfloat16* vr = vpool + (size_t)pg * page_stride + head_off + (size_t)(kk % ps) * D +
-                                lane * VPL;
-      float vf[VPL];
-      if constexpr (VPL == 4) {
-        uint2 raw = __ldg(reinterpret_cast<const uint2*>(vr));
-        vf[0] = bf16_lo(raw.x); vf[1] = bf16_hi(raw.x); vf[2] = bf16_lo(raw.y); vf[3] = bf16_hi(raw.y);
-      } else {
-        uint32_t raw = __ldg(reinterpret_cast<const unsigned int*>(vr));
-        vf[0] = bf16_lo(raw); vf[1] = bf16_hi(raw);
-      }
-#pragma unroll
-      for (int g = 0; g < MAXG; ++g) {
-        if (g < G) {
-          const float pj = sp[g][j];
-#pragma unroll
-          for (int i = 0; i < VPL; ++i) acc[g][i] = fmaf(pj, vf[i], acc[g][i]);
-        }
-      }
-    }
-    __syncthreads();
-  }
-  // deterministic reduction of the warps' p.v partial sums (fixed order: warp 0, 1, ...)
-  for (int w = 0; w < NW; ++w) {
-    if (warp == w) {
-#pragma unroll
-      for (int g = 0; g < MAXG; ++g) {
-        if (g < G) {
-#pragma unroll
-          for (int i = 0; i < VPL; ++i) so[g][lane * VPL + i] += acc[g][i];
-        }
-      }
-    }
-    __syncthreads();
-  }
-
-  // a5 stage 1: row maxima and sums over the branch and every prefix split.
   const int R = vd.n_events * G;
   const int ns = vd.n_splits;
   const int rbase = ev.local * G;
-  {
-    const int g = tid >> 4, part = tid & 15;  // 16 threads per row
-    float mm = kNegInf;
-    if (g < G) {
-      if (part == 0) mm = s_m[g];
-      for (int sidx = part; sidx < ns; sidx += 16)
-        mm = fmaxf(mm, p.part_ml[part_row(vd, kvh, sidx, R, rbase + g)].x);
+  const int nk = ev.len + 1;
+  const int ps = p.page_size;
+
+  // q rows are inputs of the step, not outputs of the kernels before this one: stage them
+  // while those may still run; everything after griddepcontrol.wait may read their results
+  for (int i = tid; i < 16 * CH; i += NT) {
+    const int g = i / CH, c = i - (i / CH) * CH;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (g < G) v = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)e * p.h_q + kvh * G + g) * D) + c);
+    *reinterpret_cast<uint4*>(&S.q[g][c * 8]) = v;
+  }
+  if (tid < 16) {
+    S.m[tid] = kNegInf;
+    S.l[tid] = 0.f;
+  }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  // stage the prefix partials of the first `sch` splits (group 0)
+  auto stage_partials = [&](int s0, int nch) {
+    for (int i = tid; i < G * nch; i += NT) {
+      const int g = i / nch, sl = i - (i / nch) * nch;
+      sml[g * sch + sl] = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
     }
+    constexpr int PC = D / 4;  // 16-byte pieces of one fp32 O row
+    for (int i = tid; i < G * nch * PC; i += NT) {
+      const int c = i % PC, rs = i / PC;
+      const int g = rs / nch, sl = rs - (rs / nch) * nch;
+      cp_async16(spo + ((size_t)g * sch + sl) * D + c * 4,
+                 p.part_o + part_row(vd, kvh, s0 + sl, R, rbase + g) * D + c * 4, true);
+    }
+    cp_async_commit();
+  };
+  if (ns > 0) stage_partials(0, min(sch, ns));
+
+  // O of this warp: rows gq, gq+8 x head-dim columns of d-blocks (2 per warp for D=128)
+  constexpr int DB = D / 8 / NW > 0 ? D / 8 / NW : 1;   // d-blocks per warp (2 or 1)
+  float o[DB][4];
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, o));
-    float ll = 0.f;
-    if (g < G) {
-      if (part == 0) ll = s_l[g] * ex2(s_m[g] - mm);
-      for (int sidx = part; sidx < ns; sidx += 16) {
-        const float2 ml = p.part_ml[part_row(vd, kvh, sidx, R, rbase + g)];
-        ll = fmaf(ml.y, ex2(ml.x - mm), ll);
+  for (int i = 0; i < DB; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  const int db0 = warp * DB;                  // first d-block of this warp (D=64: warps 0-7)
+
+  for (int c0 = 0; c0 < nk; c0 += kBmKeys) {
+    const int nv = min(kBmKeys, nk - c0);
+    const int nv16 = (nv + 15) & ~15;         // keys padded to the MMA K step (zero rows)
+    if (tid < kBmKeys) {
+      int page = -1;
+      if (tid < nv) {
+        const int pi = (c0 + tid) / ps;
+        page = p.page_table[(size_t)e * p.max_pages + pi];
+        if (page < 0 || page >= p.n_pages) {
+          set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
+          page = -1;
+        }
+      }
+      S.page[tid] = page;
+    }
+    __syncthreads();
+    // K and V rows of the chunk (rows past nv or with a bad page: zeros)
+    for (int i = tid; i < nv16 * CH; i += NT) {
+      const int k = i / CH, c = i - (i / CH) * CH;
+      const int pg = k < nv ? S.page[k] : -1;
+      const bool ok = pg >= 0;
+      const size_t off = (((size_t)(ok ? pg : 0) * p.h_kv + kvh) * ps + ((c0 + k) % ps)) * D + c * 8;
+      cp_async16(&S.k[k][c * 8], kpool + off, ok);
+      cp_async16(&S.v[k][c * 8], vpool + off, ok);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+
+    // S = Q K^T: warp w takes 8-key blocks w, w+8, ...
+    for (int nb = warp; nb * 8 < nv16; nb += NW) {
+      float sacc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        uint32_t a[4], b0, b1;
+        ldsm_x4(a[0], a[1], a[2], a[3], &S.q[(lane & 15)][kk * 16 + (lane >> 4) * 8]);
+        uint32_t b2, b3;
+        ldsm_x4(b0, b1, b2, b3, &S.k[nb * 8 + (lane & 7)][kk * 16 + ((lane >> 3) & 1) * 8]);
+        (void)b2;
+        (void)b3;
+        mma_bf16(sacc, a, b0, b1);
+      }
+      const int col = nb * 8 + 2 * t4;
+      S.sc[gq][col] = sacc[0] * p.scale_log2;
+      S.sc[gq][col + 1] = sacc[1] * p.scale_log2;
+      S.sc[gq + 8][col] = sacc[2] * p.scale_log2;
+      S.sc[gq + 8][col + 1] = sacc[3] * p.scale_log2;
+    }
+    __syncthreads();
+    // row softmax of the chunk: warp w takes rows w and w+8
+    for (int g = warp; g < 16; g += NW) {
+      if (g < G) {
+        float mx = kNegInf;
+        for (int k = lane; k < nv; k += 32)
+          if (S.page[k] >= 0) mx = fmaxf(mx, S.sc[g][k]);
+        mx = warp_max(mx);
+        const float mo = S.m[g];
+        float mn = fmaxf(mo, mx);
+        if (mn == kNegInf) mn = 0.f;  // only if every key so far failed its bounds check
+        float sum = 0.f;
+        for (int k = lane; k < nv16; k += 32) {
+          const float pr = (k < nv && S.page[k] >= 0) ? ex2(S.sc[g][k] - mn) : 0.f;
+          sum += pr;
+          S.pb[g][k] = __float2bfloat16_rn(pr);
+        }
+        sum = warp_sum(sum);
+        if (lane == 0) {
+          const float al = ex2(mo - mn);
+          S.a[g] = al;
+          S.l[g] = S.l[g] * al + sum;
+          S.m[g] = mn;
+        }
+      } else {
+        for (int k = lane; k < nv16; k += 32) S.pb[g][k] = __float2bfloat16_rn(0.f);
+        if (lane == 0) S.a[g] = 1.f;
       }
     }
+    __syncthreads();
+    // O = O * alpha + P V: warp w owns d-blocks db0 .. db0+DB-1
+    if (db0 < D / 8) {
+      const float al_lo = S.a[gq], al_hi = S.a[gq + 8];
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) ll += __shfl_xor_sync(0xffffffffu, ll, o);
-    if (g < G && part == 0) {
-      sM[g] = mm;
-      sL[g] = ll;
+      for (int i = 0; i < DB; ++i) {
+        o[i][0] *= al_lo;
+        o[i][1] *= al_lo;
+        o[i][2] *= al_hi;
+        o[i][3] *= al_hi;
+      }
+      for (int ks = 0; ks * 16 < nv16; ++ks) {
+        uint32_t a[4];
+        ldsm_x4(a[0], a[1], a[2], a[3], &S.pb[(lane & 15)][ks * 16 + (lane >> 4) * 8]);
+#pragma unroll
+        for (int i = 0; i < DB; ++i) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(b0, b1, b2, b3, &S.v[ks * 16 + ((lane >> 3) & 1) * 8 + (lane & 7)][(db0 + i) * 8]);
+          (void)b2;
+          (void)b3;
+          mma_bf16(o[i], a, b0, b1);
+        }
+      }
+    }
+    __syncthreads();
+  }
+  // branch O to shared memory (rows < G)
+  if (db0 < D / 8) {
+#pragma unroll
+    for (int i = 0; i < DB; ++i) {
+      const int d = (db0 + i) * 8 + 2 * t4;
+      if (gq < G) {
+        S.ob[gq][d] = o[i][0];
+        S.ob[gq][d + 1] = o[i][1];
+      }
+      if (gq + 8 < G) {
+        S.ob[gq + 8][d] = o[i][2];
+        S.ob[gq + 8][d + 1] = o[i][3];
+      }
     }
   }
+  if (tid < 16) S.M[tid] = S.m[tid];
   __syncthreads();
 
-  // a5 stage 2: O = (w_b O_b + sum_s w_s O_s) / L, splits in chunks of SCH.
-  constexpr int OUT_PER_T = (MAXG * D + NT - 1) / NT;
-  float oacc[OUT_PER_T];
-#pragma unroll
-  for (int u = 0; u < OUT_PER_T; ++u) {
-    const int idx = tid + u * NT;
-    const int g = idx / D, d = idx - (idx / D) * D;
-    oacc[u] = (g < G) ? so[g][d] * ex2(s_m[g] - sM[g]) : 0.f;
-  }
-  for (int s0 = 0; s0 < ns; s0 += SCH) {
-    const int nch = min(SCH, ns - s0);
+  // ---------------- a5: merge with the prefix partials, in chunks of `sch` splits
+  for (int s0 = 0; s0 < ns; s0 += sch) {
+    const int nch = min(sch, ns - s0);
+    if (s0 > 0) stage_partials(s0, nch);
+    cp_async_wait<0>();
     __syncthreads();
-    for (int i = tid; i < MAXG * SCH; i += NT) {
-      const int g = i / SCH, sl = i - g * SCH;
-      float wv = 0.f;
-      if (g < G && sl < nch) wv = ex2(p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)].x - sM[g]);
-      sw[g][sl] = wv;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int u = 0; u < OUT_PER_T; ++u) {
-      const int idx = tid + u * NT;
-      const int g = idx / D, d = idx - (idx / D) * D;
-      if (g < G) {
-        const float* src = p.part_o + part_row(vd, kvh, s0, R, rbase + g) * D + d;
-        const size_t step = (size_t)R * D;
-        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-        int sl = 0;
-        for (; sl + 4 <= nch; sl += 4) {
-          const float v0 = src[(size_t)(sl + 0) * step], v1 = src[(size_t)(sl + 1) * step];
-          const float v2 = src[(size_t)(sl + 2) * step], v3 = src[(size_t)(sl + 3) * step];
-          a0 = fmaf(sw[g][sl + 0], v0, a0);
-          a1 = fmaf(sw[g][sl + 1], v1, a1);
-          a2 = fmaf(sw[g][sl + 2], v2, a2);
-          a3 = fmaf(sw[g][sl + 3], v3, a3);
-        }
-        for (; sl < nch; ++sl) a0 = fmaf(sw[g][sl], src[(size_t)sl * step], a0);
-        oacc[u] += (a0 + a1) + (a2 + a3);
+    if (tid < G) {
+      const float oldM = S.M[tid];
+      float mm = oldM;
+      for (int sl = 0; sl < nch; ++sl) mm = fmaxf(mm, sml[tid * sch + sl].x);
+      float L = (s0 == 0 ? S.l[tid] : S.L[tid]) * ex2(oldM - mm);
+      for (int sl = 0; sl < nch; ++sl) {
+        const float2 ml = sml[tid * sch + sl];
+        L = fmaf(ml.y, ex2(ml.x - mm), L);
       }
+      S.a[tid] = ex2(oldM - mm);
+      S.M[tid] = mm;
+      S.L[tid] = L;
     }
+    __syncthreads();
+    // split weights 2^(m_s - M) of this chunk (sc is free here: nch <= kBmKeys)
+    for (int i = tid; i < G * nch; i += NT) {
+      const int g = i / nch, sl = i - (i / nch) * nch;
+      S.sc[g][sl] = ex2(sml[g * sch + sl].x - S.M[g]);
+    }
+    __syncthreads();
+    for (int i = tid; i < G * D; i += NT) {
+      const int g = i / D, d = i - g * D;
+      const float* src = spo + (size_t)g * sch * D + d;
+      float a0 = S.ob[g][d] * S.a[g], a1 = 0.f, a2 = 0.f, a3 = 0.f;
+      int sl = 0;
+      for (; sl + 4 <= nch; sl += 4) {
+        a0 = fmaf(S.sc[g][sl], src[(size_t)sl * D], a0);
+        a1 = fmaf(S.sc[g][sl + 1], src[(size_t)(sl + 1) * D], a1);
+        a2 = fmaf(S.sc[g][sl + 2], src[(size_t)(sl + 2) * D], a2);
+        a3 = fmaf(S.sc[g][sl + 3], src[(size_t)(sl + 3) * D], a3);
+      }
+      for (; sl < nch; ++sl) a0 = fmaf(S.sc[g][sl], src[(size_t)sl * D], a0);
+      S.ob[g][d] = (a0 + a1) + (a2 + a3);
+    }
+    __syncthreads();
   }
-#pragma unroll
-  for (int u = 0; u < OUT_PER_T; ++u) {
-    const int idx = tid + u * NT;
-    const int g = idx / D, d = idx - (idx / D) * D;
-    if (g < G) {
-      const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
-      const float res = oacc[u] / sL[g];
-      if (p.out_bf16)
-        reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
-      else
-        reinterpret_cast<float*>(out)[oi] = res;
-      if (lse != nullptr && d == 0)
-        lse[(size_t)e * p.h_q + kvh * G + g] = (sM[g] + log2f(sL[g])) * 0.69314718055994531f;
-    }
+  if (ns == 0 && tid < G) S.L[tid] = S.l[tid];
+  __syncthreads();
+
+  for (int i = tid; i < G * D; i += NT) {
+    const int g = i / D, d = i - g * D;
+    const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
+    const float res = S.ob[g][d] / S.L[g];
+    if (p.out_bf16)
+      reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
+    else
+      reinterpret_cast<float*>(out)[oi] = res;
+    if (lse != nullptr && d == 0)
+      lse[(size_t)e * p.h_q + kvh * G + g] = (S.M[g] + log2f(S.L[g])) * 0.69314718055994531f;
   }
 }
 
@@ -785,25 +803,51 @@ cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, con
   return launch_mma_d<64>(p, max_rows, q, kp, vp, s);
 }
 
-cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
-                                const void* v_pool, void* out, float* lse, cudaStream_t s) {
-  if (p.n_events == 0) return cudaSuccess;
-  dim3 grid(p.n_events * p.h_kv);
-  auto Q = static_cast<const __nv_bfloat16*>(q);
-  auto K = static_cast<const __nv_bfloat16*>(k_pool);
-  auto V = static_cast<const __nv_bfloat16*>(v_pool);
-  if (p.head_dim == 128) {
-    if (p.group <= 8)
-      branch_merge_kernel<128, 8><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
-    else
-      branch_merge_kernel<128, 16><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
-  } else {
-    if (p.group <= 8)
-      branch_merge_kernel<64, 8><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
-    else
-      branch_merge_kernel<64, 16><<<grid, 256, 0, s>>>(p, Q, K, V, out, lse);
+template <int D>
+static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
+                             void* out, float* lse, bool pdl, cudaStream_t s) {
+  const int G = p.group;
+  const size_t base = bm_align16(sizeof(BmSmem<D>));
+  // Staged prefix partials: all splits of a video when one wave of CTAs covers the grid
+  // (then latency decides), else a budget that keeps three CTAs per SM resident.
+  const int n_cta = p.n_events * p.h_kv;
+  const size_t per_split = (size_t)G * (D * sizeof(float) + sizeof(float2));
+  const size_t budget = n_cta > p.n_sms ? (72 * 1024 > base ? 72 * 1024 - base : per_split) : 96 * 1024;
+  int sch = (int)(budget / per_split);
+  if (p.max_splits > 0 && sch > p.max_splits) sch = p.max_splits;
+  sch = sch < 1 ? 1 : (sch > kBmKeys ? kBmKeys : sch);
+  const size_t smem = base + bm_align16((size_t)G * sch * sizeof(float2)) + (size_t)G * sch * D * sizeof(float);
+  constexpr int kMaxSmem = 200 * 1024;
+  if (smem > (size_t)kMaxSmem) return cudaErrorInvalidValue;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(branch_merge_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kMaxSmem);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
   }
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_events * p.h_kv);
+  cfg.blockDim = dim3(kBmThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, branch_merge_kernel<D>, p, static_cast<const __nv_bfloat16*>(q),
+                            static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
+                            out, lse, sch);
+}
+
+cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
+                                const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s) {
+  if (p.n_events == 0) return cudaSuccess;
+  if (p.head_dim == 128) return launch_bm<128>(p, q, k_pool, v_pool, out, lse, pdl, s);
+  return launch_bm<64>(p, q, k_pool, v_pool, out, lse, pdl, s);
 }
 
 }  // namespace pad

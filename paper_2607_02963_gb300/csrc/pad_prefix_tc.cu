@@ -12,13 +12,16 @@
 //               swizzle) into a 3-stage ring; a stage is refilled once the S of
 //               the tile it held has completed
 //   warp 1      MMA issuer (one thread): S = Q K^T into one of three TMEM S
-//               buffers, O += P V with P read back from TMEM; it runs up to two
-//               tiles ahead of the softmax
+//               buffers, O += P V with P read back from TMEM; S runs two tiles ahead
+//               of the softmax and is issued before the P.V that waits for it
 //   warp 2      TMEM allocator (512 columns) and deallocator
 //   warp 3      TMA producer of V tiles (refilled once the P.V of the tile completed)
-//   warps 4-7   softmax: one thread per query row (its TMEM lane), online max and
-//               sum in base 2, P written as packed bf16 over its S columns, lazy
-//               rescaling of O (only when a row maximum grows by more than 2^8)
+//   warps 4-11  softmax: two warps per 32-row lane quarter, each taking 64 of the
+//               tile's 128 columns for one query row per thread; they meet once per
+//               tile to combine their partial row maxima (an mbarrier, so the wait is
+//               bounded); online max and sum in base 2, P written as packed bf16 over
+//               the S columns already read, lazy rescaling of O (only when a row
+//               maximum grows by more than 2^8)
 //
 // Every MMA has N = 128 (S: 128 tokens; P.V: 128 head-dim columns), the size at
 // which one tcgen05.mma carries as much tensor work as it costs to issue.
@@ -39,6 +42,8 @@
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cstdint>
+#include <cstring>
+#include <mutex>
 
 #include "pad_internal.h"
 
@@ -50,7 +55,7 @@ constexpr int kD = 128;
 constexpr int kBN = 128;       // prefix tokens per K/V tile
 constexpr int kStages = 3;
 constexpr int kSBuf = 3;       // S buffers in TMEM
-constexpr int kThreads = 256;
+constexpr int kThreads = 384;
 constexpr uint32_t kHalfBytes = kBN * 128;         // 128 tokens x 64 bf16 = 16 KB
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 32 KB
 constexpr uint32_t kQHalfBytes = 128 * 128;        // 128 rows x 64 bf16 = 16 KB
@@ -59,10 +64,19 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kQTileBytes;
 constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
-constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;   // + slack for 1024-byte alignment
+constexpr uint32_t kOffX = kOffBar + 256;               // partial row maxima: [2][2][128] fp32
+constexpr uint32_t kSmemBytes = kOffX + 2 * 2 * 128 * 4;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 384;
 constexpr float kLazyRescale = 8.0f;                  // log2 units
+#ifdef PAD_MUFU_PAIRS
+constexpr int kMufuPairs = PAD_MUFU_PAIRS;
+#else
+// Exponential pairs (of every 16) on the MUFU unit; the rest use exp2_poly2 on the FMA
+// pipe.  Measured on GB300, the softmax here is latency-bound rather than MUFU-bound, so
+// the extra polynomial instructions cost more than they save: all 16 go to MUFU.
+constexpr int kMufuPairs = 16;
+#endif
 constexpr unsigned long long kWaitNs = 1000000000ull; // one second per wait
 static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 
@@ -74,6 +88,8 @@ struct TcBars {
   uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (4 warp arrivals)
   uint64_t pvdone[2];         // P.V of tile j completes pvdone[j & 1]
   uint64_t drain;
+  uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
+  uint64_t xchg[4];           // the two softmax warps of a lane quarter met (64 thread arrivals)
   uint32_t tmem_base;
   int32_t abort;
 };
@@ -117,6 +133,89 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
+
+// ---------------------------------------------------------------- packed fp32 pairs
+// Blackwell executes two fp32 lanes per instruction (.f32x2); a pair lives in a b64.
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+  return ((uint64_t)__float_as_uint(hi) << 32) | __float_as_uint(lo);
+}
+__device__ __forceinline__ float f2lo(uint64_t v) { return __uint_as_float((uint32_t)v); }
+__device__ __forceinline__ float f2hi(uint64_t v) { return __uint_as_float((uint32_t)(v >> 32)); }
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2_rm(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rm.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// 2^x for a pair on the FMA pipe, to take part of the load off the MUFU unit.
+// Cody-Waite split x = n + f with n = floor(x) and f in [0, 1): adding 1.5 * 2^23 with
+// round-toward-minus-infinity leaves n in the low mantissa bits of t (exact for
+// |x| < 2^22), and (bits(t) << 23) is n << 23 because the low nine bits of 1.5 * 2^23
+// are zero.  2^f is a cubic fitted to 2^f on [0, 1) for the least maximum relative error
+// (7.5e-5; 1.5e-4 after fp32 rounding), far below the bf16 rounding P gets next.
+// x is clamped to -125: the cubic lies in [0.99, 2), so the exponent field stays normal.
+constexpr float kExpC0 = 0.99992512554644490f;
+constexpr float kExpC1 = 0.69583399210713630f;
+constexpr float kExpC2 = 0.22606707273041300f;
+constexpr float kExpC3 = 0.07802403102605904f;
+__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x) {
+  const float x0 = fmaxf(f2lo(x), -125.f), x1 = fmaxf(f2hi(x), -125.f);
+  const uint64_t xc = f2pack(x0, x1);
+  const uint64_t magic = f2pack(12582912.f, 12582912.f);
+  const uint64_t t = fadd2_rm(xc, magic);
+  const uint64_t n = fadd2(t, f2pack(-12582912.f, -12582912.f));
+  const uint64_t f = fadd2(xc, n ^ 0x8000000080000000ull);  // x - n
+  uint64_t q = ffma2(f, f2pack(kExpC3, kExpC3), f2pack(kExpC2, kExpC2));
+  q = ffma2(f, q, f2pack(kExpC1, kExpC1));
+  q = ffma2(f, q, f2pack(kExpC0, kExpC0));
+  const uint32_t lo = (uint32_t)q + ((uint32_t)t << 23);
+  const uint32_t hi = (uint32_t)(q >> 32) + ((uint32_t)(t >> 32) << 23);
+  return ((uint64_t)hi << 32) | lo;
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Maximum of the raw scores of one softmax warp's 64 columns (eight chains of three-input
+// max); with MASK, columns at or past `valid` are left out.
+template <bool MASK>
+__device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], int valid) {
+  float mxa[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) mxa[u] = -__builtin_huge_valf();
+#pragma unroll
+  for (int c = 0; c < 2; ++c)
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      float a = __uint_as_float(sr[c][i]), b = __uint_as_float(sr[c][i + 1]);
+      if (MASK) {
+        if (32 * c + i >= valid) a = -__builtin_huge_valf();
+        if (32 * c + i + 1 >= valid) b = -__builtin_huge_valf();
+      }
+      const int u = (16 * c + i / 2) & 7;
+      mxa[u] = max3f(mxa[u], a, b);
+    }
+  return fmaxf(max3f(mxa[0], mxa[1], mxa[2]), max3f(max3f(mxa[3], mxa[4], mxa[5]), mxa[6], mxa[7]));
+}
+
+// P = 2^(s * scale_log2 - m) for one softmax warp's 64 columns, written as packed bf16
+// over the S columns already read; returns the fp32 sum of the P values.
+template <bool MASK>
+__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], int valid, float sl2,
+                                              float m, uint32_t taddr_p);
 
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -250,8 +349,57 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// The registers written by tcgen05.ld are valid only after tcgen05.wait::ld; listing them
+// as operands of the wait makes every later use depend on it in the compiler's view too.
+__device__ __forceinline__ void tmem_wait_ld_dep(uint32_t* r) {
+  asm volatile(
+      "tcgen05.wait::ld.sync.aligned;"
+      : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+        "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+        "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]),
+        "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]),
+        "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+      :
+      : "memory");
+}
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+template <bool MASK>
+__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], int valid, float sl2,
+                                              float m, uint32_t taddr_p) {
+  const uint64_t sc2 = f2pack(sl2, sl2), nm2 = f2pack(-m, -m);
+  uint64_t lacc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int col = 32 * c + 2 * i;
+      const uint64_t x =
+          ffma2(f2pack(__uint_as_float(sr[c][2 * i]), __uint_as_float(sr[c][2 * i + 1])), sc2, nm2);
+      float p0, p1;
+      if (i < kMufuPairs) {
+        p0 = ex2(f2lo(x));
+        p1 = ex2(f2hi(x));
+      } else {
+        const uint64_t e = exp2_poly2(x);
+        p0 = f2lo(e);
+        p1 = f2hi(e);
+      }
+      if (MASK) {
+        if (col >= valid) p0 = 0.f;
+        if (col + 1 >= valid) p1 = 0.f;
+      }
+      lacc[i & 3] = fadd2(lacc[i & 3], f2pack(p0, p1));
+      pk[i] = pack_bf16(p0, p1);
+    }
+    // P of tokens 32c .. 32c+31 of this half, two per column
+    tmem_st16(taddr_p + 16 * c, pk);
+  }
+  const uint64_t ls = fadd2(fadd2(lacc[0], lacc[1]), fadd2(lacc[2], lacc[3]));
+  return f2lo(ls) + f2hi(ls);
 }
 
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
@@ -263,10 +411,12 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
+  if (sbase & 1023u) {  // the 128-byte swizzle atoms need 1024-byte alignment (never expected)
+    if (threadIdx.x == 0) set_error(p.header, PAD_ERR_UNSUPPORTED, (int)blockIdx.x, (int)sbase, 0);
+    return;
+  }
   TcBars* bars = reinterpret_cast<TcBars*>(smem + kOffBar);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -289,11 +439,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < kSBuf; ++b) {
       mbar_init(&bars->sfull[b], 1);
-      mbar_init(&bars->pfull[b], 4);  // one arrival per softmax warp
+      mbar_init(&bars->pfull[b], 8);  // one arrival per softmax warp
     }
     mbar_init(&bars->pvdone[0], 1);
     mbar_init(&bars->pvdone[1], 1);
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->qready, 8);
+    for (int qq = 0; qq < 4; ++qq) mbar_init(&bars->xchg[qq], 64);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -305,27 +457,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
 
-  // Q rows of this group into the 128-byte-swizzled K-major layout the MMA reads:
-  // half h (head-dim 64h..64h+63), row r, 16-byte chunk c at
-  // h*16K + r*128 + ((c ^ (r & 7)) << 4).  Rows past R are zero.
-  for (int idx = threadIdx.x; idx < 128 * 16; idx += kThreads) {
-    const int r = idx >> 4, c = idx & 15;
-    const int h = c >> 3, cc = c & 7;
-    const int grow = row0 + r;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (grow < R) {
-      const int el = grow / p.group;
-      const int gh = grow - el * p.group;
-      const __nv_bfloat16* src =
-          q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * kD + c * 8;
-      v = __ldg(reinterpret_cast<const uint4*>(src));
-    }
-    *reinterpret_cast<uint4*>(smem + kOffQ + h * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = v;
-  }
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   fence_before();
   __syncthreads();
   fence_after();
+  // The grid launched after this one (the branch/merge pass) may start its own
+  // prologue now; it waits for this grid's completion before it reads partials.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const uint32_t tmem = bars->tmem_base;
   const int tok0 = (int)(vd.prefix_off + it.tok_begin);
 
@@ -390,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
                  kk > 0 ? 1u : acc0);
       };
-      bool ok = true;
+      bool ok = mbar_wait(&bars->qready, 0u, bars, p.header, 11);
       for (int t = 0; t < min(2, n_tiles) && ok; ++t) {
         ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
         if (!ok) break;
@@ -399,15 +536,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&bars->sfull[t % kSBuf]);
       }
       for (int j = 0; j < n_tiles && ok; ++j) {
-        const int s = j % kStages;
-        ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
-        if (!ok) break;
-        ok = mbar_wait(&bars->pfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
-        if (!ok) break;
-        fence_after();
-        issue_PV(j);
-        mma_commit(&bars->pvdone[j & 1]);
-        mma_commit(&bars->vempty[s]);
+        // S of tile j+2 first: it needs only its K tile and a free S buffer, so it runs
+        // on the tensor pipe while the softmax still works on tile j
         const int t = j + 2;
         if (t < n_tiles) {
           ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 6);
@@ -420,6 +550,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_S(t);
           mma_commit(&bars->sfull[t % kSBuf]);
         }
+        const int s = j % kStages;
+        ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
+        if (!ok) break;
+        ok = mbar_wait(&bars->pfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
+        if (!ok) break;
+        fence_after();
+        issue_PV(j);
+        mma_commit(&bars->pvdone[j & 1]);
+        mma_commit(&bars->vempty[s]);
       }
       // every MMA issued by this thread has completed once this commit lands
       mma_commit(&bars->drain);
@@ -427,10 +566,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax
-    const int lane_base = 32 * (warp & 3);
-    const int grow = row0 + lane_base + lane;
-    const bool warp_active = (row0 + lane_base) < R;
+    const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31 (query rows)
+    const int half = (warp - 4) >> 2;          // columns 64*half .. +63 of every tile
+    const int lane_base = 32 * quarter;
+    // Q rows of this quarter, head-dim half `half`, into the 128-byte-swizzled K-major
+    // layout the MMA reads (the K/V loads are already in flight): row r, 16-byte chunk
+    // cc of half h at h*16K + r*128 + ((cc ^ (r & 7)) << 4).  Rows past R are zero.
+    for (int idx = lane; idx < 32 * 8; idx += 32) {
+      const int r = lane_base + (idx >> 3), cc = idx & 7;
+      const int qrow = row0 + r;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (qrow < R) {
+        const int el = qrow / p.group;
+        const int gh = qrow - el * p.group;
+        const __nv_bfloat16* src = q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * kD +
+                                   half * 64 + cc * 8;
+        v = __ldg(reinterpret_cast<const uint4*>(src));
+      }
+      *reinterpret_cast<uint4*>(smem + kOffQ + half * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = v;
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bars->qready);
+    const int row = lane_base + lane;
+    const int grow = row0 + row;
+    const bool warp_active = (row0 + lane_base) < R;  // same for both warps of the quarter
     const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
+    const uint32_t col0 = 64u * (uint32_t)half;       // first S column (token) of this warp
+    float* xmax = reinterpret_cast<float*>(smem + kOffX);  // [tile parity][half][row]
+    uint64_t* xbar = &bars->xchg[quarter];
     const float sl2 = p.scale_log2;
     float m_run = -__builtin_huge_valf(), l_run = 0.f;
     bool ok = true;
@@ -442,56 +606,45 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       fence_after();
       if (warp_active) {
-        const int valid = min(kBN, ntok - j * kBN);
-        float mx = -__builtin_huge_valf();
-#pragma unroll
-        for (int c = 0; c < kBN / 32; ++c) {
-          tmem_ld32(tl + cS + 32 * c, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
-        }
-        mx *= sl2;
+        const int valid = min(kBN, ntok - j * kBN) - (int)col0;  // valid columns of this half
+        uint32_t sr[2][32];
+        tmem_ld32(tl + cS + col0, sr[0]);
+        tmem_ld32(tl + cS + col0 + 32, sr[1]);
+        tmem_wait_ld_dep(sr[0]);
+        tmem_wait_ld_dep(sr[1]);
+        const float pmax = valid >= 64 ? half_row_max<false>(sr, valid) : half_row_max<true>(sr, valid);
+        // meet the other half: this also orders both warps' S reads before either
+        // writes P over columns the other one read
+        xmax[(j & 1) * 256 + half * 128 + row] = pmax;
+        mbar_arrive(xbar);
+        ok = mbar_wait(xbar, (uint32_t)(j & 1), bars, p.header, 12);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        const float mx = fmaxf(pmax, xmax[(j & 1) * 256 + (1 - half) * 128 + row]) * sl2;
         const float m_new = fmaxf(m_run, mx);
         const bool need = m_new > m_run + kLazyRescale;
         if (__any_sync(0xffffffffu, need && j > 0)) {
-          // O must hold P.V of tile j-1 before it is rescaled
+          // O must hold P.V of tile j-1 before it is rescaled (each half rescales its
+          // own 64 head-dim columns; both halves take the same decision per row)
           ok = mbar_wait(&bars->pvdone[(j - 1) & 1], (uint32_t)(((j - 1) >> 1) & 1), bars, p.header, 9);
           ok = __all_sync(0xffffffffu, ok);
           if (!ok) break;
           fence_after();
           const float alpha = need ? ex2(m_run - m_new) : 1.f;
 #pragma unroll
-          for (int c = 0; c < kD / 32; ++c) {
-            tmem_ld32(tl + kColO + 32 * c, r);
-            tmem_wait_ld();
+          for (int c = 0; c < 2; ++c) {
+            tmem_ld32(tl + kColO + col0 + 32 * c, r);
+            tmem_wait_ld_dep(r);
 #pragma unroll
             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tmem_st32(tl + kColO + 32 * c, r);
+            tmem_st32(tl + kColO + col0 + 32 * c, r);
           }
           tmem_wait_st();
           if (need) l_run *= alpha;
         }
         if (need) m_run = m_new;
-#pragma unroll
-        for (int c = 0; c < kBN / 32; ++c) {
-          tmem_ld32(tl + cS + 32 * c, r);
-          tmem_wait_ld();
-          uint32_t pk[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int col = 32 * c + 2 * i;
-            const float p0 = col < valid ? ex2(fmaf(__uint_as_float(r[2 * i]), sl2, -m_run)) : 0.f;
-            const float p1 =
-                col + 1 < valid ? ex2(fmaf(__uint_as_float(r[2 * i + 1]), sl2, -m_run)) : 0.f;
-            l_run += p0 + p1;
-            pk[i] = pack_bf16(p0, p1);
-          }
-          // P over the first half of this S buffer; S chunk c sits at columns 32c..32c+31,
-          // so P chunk c (columns 16c..16c+15) only overwrites S values already read.
-          tmem_st16(tl + cS + 16 * c, pk);
-        }
+        l_run += valid >= 64 ? half_row_exp<false>(sr, valid, sl2, m_run, tl + cS + col0 / 2)
+                             : half_row_exp<true>(sr, valid, sl2, m_run, tl + cS + col0 / 2);
         tmem_wait_st();
       }
       fence_before();
@@ -505,23 +658,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_after();
       const int64_t pr = (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + it.split) * R + grow;
 #pragma unroll
-      for (int c = 0; c < kD / 32; ++c) {
-        tmem_ld32(tl + kColO + 32 * c, r);
-        tmem_wait_ld();
+      for (int c = 0; c < 2; ++c) {
+        tmem_ld32(tl + kColO + col0 + 32 * c, r);
+        tmem_wait_ld_dep(r);
         if (grow < R) {
-          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + 32 * c);
+          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + col0 + 32 * c);
 #pragma unroll
           for (int i = 0; i < 8; ++i)
             dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
                                  __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
         }
       }
-      if (grow < R) p.part_ml[pr] = make_float2(m_run, l_run);
+      // row sum = both halves' partial sums (slot n_tiles & 1 was last read two tiles ago)
+      xmax[(n_tiles & 1) * 256 + half * 128 + row] = l_run;
+      mbar_arrive(xbar);
+      ok = mbar_wait(xbar, (uint32_t)(n_tiles & 1), bars, p.header, 13);
+      if (ok && half == 0 && grow < R)
+        p.part_ml[pr] = make_float2(m_run, l_run + xmax[(n_tiles & 1) * 256 + 128 + row]);
     }
   }
 
   __syncwarp();
   fence_before();
+  // This grid may run alongside the append kernel before it (it reads nothing that
+  // kernel writes); waiting for it here makes the completion of this grid imply the
+  // completion of the append, which the branch/merge pass after it relies on.
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
   __syncthreads();
   if (warp == 2) {
     fence_after();
@@ -558,19 +720,59 @@ bool make_map(CUtensorMap* map, const void* base, int h_kv, int64_t tokens) {
   return r == CUDA_SUCCESS;
 }
 
+// The tensor maps of the last few (K, V) prefix buffers, so a step does not re-encode
+// them (an encode costs microseconds of host time; the maps depend only on the base
+// address, the head count and the token extent).
+struct MapCacheEntry {
+  const void* k;
+  const void* v;
+  int h_kv;
+  int64_t tokens;
+  int dev;
+  CUtensorMap mk, mv;
+};
+std::mutex g_map_mu;
+MapCacheEntry g_maps[8];
+int g_maps_n = 0, g_maps_next = 0;
+
+bool get_maps(const void* kp, const void* vp, int h_kv, int64_t tokens, int dev, CUtensorMap* mk,
+              CUtensorMap* mv) {
+  std::lock_guard<std::mutex> lk(g_map_mu);
+  for (int i = 0; i < g_maps_n; ++i) {
+    const MapCacheEntry& e = g_maps[i];
+    if (e.k == kp && e.v == vp && e.h_kv == h_kv && e.tokens == tokens && e.dev == dev) {
+      std::memcpy(mk, &e.mk, sizeof(CUtensorMap));
+      std::memcpy(mv, &e.mv, sizeof(CUtensorMap));
+      return true;
+    }
+  }
+  MapCacheEntry ne;
+  ne.k = kp;
+  ne.v = vp;
+  ne.h_kv = h_kv;
+  ne.tokens = tokens;
+  ne.dev = dev;
+  if (!make_map(&ne.mk, kp, h_kv, tokens) || !make_map(&ne.mv, vp, h_kv, tokens)) return false;
+  g_maps[g_maps_next] = ne;
+  g_maps_next = (g_maps_next + 1) % 8;
+  if (g_maps_n < 8) ++g_maps_n;
+  std::memcpy(mk, &ne.mk, sizeof(CUtensorMap));
+  std::memcpy(mv, &ne.mv, sizeof(CUtensorMap));
+  return true;
+}
+
 }  // namespace
 
 cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
-                             const void* vp, int64_t total_prefix_tokens, cudaStream_t s) {
+                             const void* vp, int64_t total_prefix_tokens, bool pdl, cudaStream_t s) {
   if (p.n_items == 0) return cudaSuccess;
   if (p.head_dim != kD || total_prefix_tokens <= 0 || total_prefix_tokens > (int64_t)INT32_MAX)
     return cudaErrorInvalidValue;
-  CUtensorMap mk, mv;
-  if (!make_map(&mk, kp, p.h_kv, total_prefix_tokens) || !make_map(&mv, vp, p.h_kv, total_prefix_tokens))
-    return cudaErrorInvalidValue;
-  static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
+  CUtensorMap mk, mv;
+  if (!get_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
+  static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
     cudaError_t e = cudaFuncSetAttribute(prefix_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
@@ -578,10 +780,17 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
     configured[dev] = true;
   }
   const int n_groups = (max_rows + 127) / 128;
-  dim3 grid(p.n_items * n_groups);
-  prefix_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, static_cast<const __nv_bfloat16*>(q),
-                                                      n_groups, mk, mv);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_items * n_groups);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, prefix_tc_kernel, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv);
 }
 
 }  // namespace pad

@@ -2,7 +2,7 @@ import pytest
 """Randomised model of the tensor-core prefix kernel's mbarrier protocol.
 
 The kernel (csrc/pad_prefix_tc.cu) runs a K producer, a V producer, one MMA issuer
-and four softmax warps that hand 128-token tiles to each other through mbarriers
+and eight softmax warps that hand 128-token tiles to each other through mbarriers
 waited on by phase parity: 3 K/V stages, 3 S buffers in TMEM (P written over S),
 per-buffer P-ready barriers and P.V completions alternating over two barriers.
 This model mirrors that schedule with asynchronous loads and MMAs that complete
@@ -27,7 +27,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False):
     rnd = random.Random(seed)
     kfull = [Bar(1) for _ in range(ST)]; vfull = [Bar(1) for _ in range(ST)]
     vempty = [Bar(1) for _ in range(ST)]; sfull = [Bar(1) for _ in range(SB)]
-    pfull = [Bar(4) for _ in range(SB)]; pvdone = [Bar(1), Bar(1)]; drain = Bar(1)
+    pfull = [Bar(8) for _ in range(SB)]; pvdone = [Bar(1), Bar(1)]; drain = Bar(1)
     if single_barriers:
         pfull = [pfull[0]] * SB
         pvdone = [pvdone[0]] * 2
@@ -94,10 +94,6 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False):
             yield (kfull[t % ST], (t // ST) & 1)
             issue_S(t); commit(sfull[t % SB])
         for j in range(n):
-            s = j % ST
-            yield (vfull[s], (j // ST) & 1)
-            yield (pfull[j % SB], (j // SB) & 1) if not single_barriers else (pfull[0], j & 1)
-            issue_PV(j); commit(pvdone[j & 1]); commit(vempty[s])
             t = j + 2
             if t < n:
                 yield (kfull[t % ST], (t // ST) & 1)
@@ -105,6 +101,10 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False):
                     yield ((pvdone[(j - 1) & 1], ((j - 1) >> 1) & 1) if not single_barriers
                            else (pvdone[0], (j - 1) & 1))
                 issue_S(t); commit(sfull[t % SB])
+            s = j % ST
+            yield (vfull[s], (j // ST) & 1)
+            yield (pfull[j % SB], (j // SB) & 1) if not single_barriers else (pfull[0], j & 1)
+            issue_PV(j); commit(pvdone[j & 1]); commit(vempty[s])
         commit(drain)
         yield (drain, 0)
     def softmax(w):
@@ -122,7 +122,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False):
             pfull[j % SB].arrive()
         yield (drain, 0)
         assert len(PV_done) == n, "epilogue before all P.V done"
-    actors = [kprod(), vprod(), mma_thread()] + [softmax(w) for w in range(4)]
+    actors = [kprod(), vprod(), mma_thread()] + [softmax(w) for w in range(8)]
     waiting = [None] * len(actors); alive = [True] * len(actors)
     # P_written must be set before any of the 4 arrivals completes the barrier: mark at first
     steps = 0
