@@ -278,16 +278,16 @@ def cpu_baseline(w, budget_s=10.0):
     smp = OracleSample(w)
     t0 = time.perf_counter()
     n = 0
-    while n < w.n_events:
-        smp.run(n)
+    while True:  # whole events, cycling over the workload until the budget is spent
+        smp.run(n % w.n_events)
         n += 1
-        if time.perf_counter() - t0 >= budget_s:
+        if time.perf_counter() - t0 >= budget_s and n >= min(w.n_events, 1):
             break
     dt = time.perf_counter() - t0
     return {"value": n / dt, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
-            "sample": f"{n} of {w.n_events} events of the workload (all {w.h_q} q-heads each; "
-                      f"numpy fp64 with the explicit event mask; inputs widened to fp64 before "
-                      f"timing), {dt:.1f} s"}
+            "sample": f"{n} event decodes ({n / w.n_events:.1f} passes over the {w.n_events} events "
+                      f"of the workload; all {w.h_q} q-heads each; numpy fp64 with the explicit "
+                      f"event mask; inputs widened to fp64 before timing), {dt:.1f} s"}
 
 
 # ---------------------------------------------------------------------------
