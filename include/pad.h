@@ -189,6 +189,27 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
                                  const void* v_prefix, const void* k_pool, const void* v_pool,
                                  void* out, float* lse, pad_stream_t stream);
 
+/* Allocation-free variant of pad_event_decode_attn (the paper has no counterpart; this
+ * is an interface for callers, not part of the method).  Same arguments and result.  It
+ * is meant for callers that cannot give the library device scratch memory, for example a
+ * plugin API that hands out tensors but no allocator, or a serving loop whose device
+ * memory is reserved up front and must not change while it runs.  Instead of the plan's
+ * workspace it uses a 16 MiB device array inside the library (held by every GPU that
+ * loads the library until the process exits) for the plan image and the split-KV partial
+ * states; it calls no cudaMalloc, cudaFree or other allocating routine.
+ *   plan      from pad_plan; its workspace may be NULL (a host-only plan), but it must
+ *             carry the page table.  Plans needing more than 16 MiB of scratch
+ *             (pad_plan_get_info().workspace_bytes) fail with PAD_ERR_WORKSPACE_TOO_SMALL.
+ *   The branch keys are read from the pools, so this step's K/V must already be there.
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ * and caches it, so make that first call before any stream capture.  All calls share the
+ * array: calls that overlap on the GPU (other streams or threads) race on it; calls in
+ * order on one stream are safe (each re-uploads the plan image, clearing the status word).
+ * pad_device_status does not read this array's status word. */
+pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q, const void* k_prefix,
+                                        const void* v_prefix, const void* k_pool, const void* v_pool,
+                                        void* out, float* lse, pad_stream_t stream);
+
 /* Synchronise the stream and read the plan's device status word:
  * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream);

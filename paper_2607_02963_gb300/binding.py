@@ -67,6 +67,8 @@ _SIGNATURES = {
     "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "pad_event_decode_attn": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                         c_void_p, c_void_p, c_void_p, c_void_p]),
+    "pad_event_decode_attn_static": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                               c_void_p, c_void_p, c_void_p, c_void_p]),
     "pad_device_status": (c_int32, [c_void_p, c_void_p]),
     "pad_last_error": (ctypes.c_char_p, []),
     "pad_status_string": (ctypes.c_char_p, [c_int32]),
@@ -248,6 +250,14 @@ def pad_event_decode_attn(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out
     _check(lib().pad_event_decode_attn(plan.handle, _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
                                        _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
                                        _stream(stream)))
+
+
+def pad_event_decode_attn_static(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,
+                                 stream=None):
+    """pad_event_decode_attn with the library's static scratch instead of a workspace."""
+    _check(lib().pad_event_decode_attn_static(plan.handle, _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
+                                              _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
+                                              _stream(stream)))
 
 
 def pad_device_status(plan: Plan, stream=None):

@@ -691,3 +691,109 @@ pad_status pad_timing_read(float* total_ms, int32_t* n_launches) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of pad_event_decode_attn.
+//
+// Some callers have no way to hand this library device memory for scratch: a host
+// application's plugin interface that gives out tensors but no allocator, a serving
+// loop whose memory is reserved up front and must not grow or fragment while it
+// runs, or a process whose device memory is owned by an allocator it cannot call
+// into.  For them the plan image and the split-KV partial states live in the array
+// below instead of a caller workspace; the caller still passes every input and output.
+//
+// The array is a file-scope device variable: every GPU that loads this library keeps
+// kStaticScratchBytes of device memory for it until the process exits.  Its device
+// address is fetched once per device (cudaGetSymbolAddress on the first call made with
+// that device current) and cached.  All calls share the array, so two calls whose work
+// overlaps on the GPU (different streams, or different host threads) race on it; calls
+// ordered on one stream are safe, each one re-uploading the plan image, which also
+// clears the status word.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kStaticScratchBytes = 16u << 20;  // 16 MiB
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_static_mu;
+void* g_static_ptr[64] = {};
+
+}  // namespace
+
+extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q,
+                                                   const void* k_prefix, const void* v_prefix,
+                                                   const void* k_pool, const void* v_pool, void* out,
+                                                   float* lse, pad_stream_t stream) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (plan->n_events == 0) return PAD_OK;
+  if (plan->lay.total_bytes > kStaticScratchBytes)
+    return fail(PAD_ERR_WORKSPACE_TOO_SMALL,
+                "plan needs %zu bytes of scratch; the static scratch array holds %zu bytes",
+                plan->lay.total_bytes, kStaticScratchBytes);
+  if (!plan->page_table) return fail(PAD_ERR_INVALID_ARG, "plan has no page table");
+  if (!q || !k_pool || !v_pool || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (plan->lay.n_items > 0 && (!k_prefix || !v_prefix))
+    return fail(PAD_ERR_INVALID_ARG, "k_prefix / v_prefix is NULL");
+  if (!aligned16(q) || !aligned16(k_prefix) || !aligned16(v_prefix) || !aligned16(k_pool) ||
+      !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(PAD_ERR_UNSUPPORTED, "device index %d", dev);
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_static_mu);
+    if (!g_static_ptr[dev]) {
+      void* ptr = nullptr;
+      e = cudaGetSymbolAddress(&ptr, g_static_scratch);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
+      g_static_ptr[dev] = ptr;
+    }
+    scratch = g_static_ptr[dev];
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // plan image (header with a zero status word, video and event descriptors, work items);
+  // a copy from the plan's own pageable host buffer, staged by the driver
+  e = cudaMemcpyAsync(scratch, plan->host_image.data(), plan->lay.upload_bytes, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e, "static scratch plan upload");
+
+  KParams p;
+  const pad_problem& pr = plan->prob;
+  p.h_q = pr.h_q;
+  p.h_kv = pr.h_kv;
+  p.group = pr.h_q / pr.h_kv;
+  p.head_dim = pr.head_dim;
+  p.page_size = pr.page_size;
+  p.max_pages = plan->max_pages;
+  p.n_pages = plan->n_pages;
+  p.n_videos = plan->n_videos;
+  p.n_events = plan->n_events;
+  p.n_items = (int32_t)plan->lay.n_items;
+  p.out_bf16 = pr.out_dtype == 1;
+  p.n_sms = plan->lay.n_sms;
+  p.max_splits = 0;
+  for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
+  p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
+  auto* ws = static_cast<uint8_t*>(scratch);
+  p.header = reinterpret_cast<PadDevHeader*>(ws);
+  p.videos = reinterpret_cast<const PadVideoDesc*>(ws + plan->lay.off_videos);
+  p.events = reinterpret_cast<const PadEventDesc*>(ws + plan->lay.off_events);
+  p.items = reinterpret_cast<const PadWorkItem*>(ws + plan->lay.off_items);
+  p.part_ml = reinterpret_cast<float2*>(ws + plan->lay.off_ml);
+  p.part_o = reinterpret_cast<float*>(ws + plan->lay.off_o);
+  p.page_table = plan->page_table;
+
+  switch (plan->lay.prefix_kernel) {
+    case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
+    case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
+    case PAD_FLAG_PREFIX_TC:
+      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, false, s);
+      break;
+    default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "prefix launch (static scratch)");
+  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, false, s);
+  if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch (static scratch)");
+  return PAD_OK;
+}
