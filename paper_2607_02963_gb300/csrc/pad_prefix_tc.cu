@@ -11,10 +11,10 @@
 //   warp 0      TMA producer of K tiles (128 tokens: two 64-column halves, 128-byte
 //               swizzle) into a 3-stage ring; a stage is refilled once the S of
 //               the tile it held has completed
-//   warp 1      MMA issuer (one thread): S = Q K^T into one of three TMEM S
-//               buffers, O += P V with P read back from TMEM; S runs two tiles ahead
-//               of the softmax and is issued before the P.V that waits for it
-//   warp 2      TMEM allocator (512 columns) and deallocator
+//   warp 1      S issuer (one thread): S = Q K^T into one of three TMEM S buffers,
+//               up to three tiles ahead of the softmax
+//   warp 2      TMEM allocator (512 columns) and deallocator; its lane 0 issues
+//               O += P V with P read back from TMEM
 //   warp 3      TMA producer of V tiles (refilled once the P.V of the tile completed)
 //   warps 4-11  softmax: two warps per 32-row lane quarter, each taking 64 of the
 //               tile's 128 columns for one query row per thread; they meet once per
@@ -83,11 +83,11 @@ static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 struct TcBars {
   uint64_t kfull[kStages];
   uint64_t vfull[kStages];
-  uint64_t vempty[kStages];   // P.V of the tile in this V stage has completed
+  uint64_t pvfree[kStages];   // P.V of the tile in this stage / S buffer has completed
   uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
   uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (4 warp arrivals)
-  uint64_t pvdone[2];         // P.V of tile j completes pvdone[j & 1]
-  uint64_t drain;
+  uint64_t drain_s;           // every S MMA has completed (S issuer)
+  uint64_t drain_pv;          // every P.V MMA has completed (P.V issuer)
   uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
   uint64_t xchg[4];           // the two softmax warps of a lane quarter met (64 thread arrivals)
   uint32_t tmem_base;
@@ -435,15 +435,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bars->kfull[s], 1);
       mbar_init(&bars->vfull[s], 1);
-      mbar_init(&bars->vempty[s], 1);
+      mbar_init(&bars->pvfree[s], 1);
     }
     for (int b = 0; b < kSBuf; ++b) {
       mbar_init(&bars->sfull[b], 1);
       mbar_init(&bars->pfull[b], 8);  // one arrival per softmax warp
     }
-    mbar_init(&bars->pvdone[0], 1);
-    mbar_init(&bars->pvdone[1], 1);
-    mbar_init(&bars->drain, 1);
+    mbar_init(&bars->drain_s, 1);
+    mbar_init(&bars->drain_pv, 1);
     mbar_init(&bars->qready, 8);
     for (int qq = 0; qq < 4; ++qq) mbar_init(&bars->xchg[qq], 64);
     bars->abort = 0;
@@ -478,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = t % kStages;
         if (t >= kStages) {
           // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
-          uint64_t* freed = isK ? &bars->sfull[s] : &bars->vempty[s];
+          uint64_t* freed = isK ? &bars->sfull[s] : &bars->pvfree[s];
           ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
           if (!ok) break;
         }
@@ -497,8 +496,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == 2) {
+    // ------------------------------------------------------------ MMA issuers
+    // Two threads feed the tensor pipe so that one's waits and commits overlap the
+    // other's MMAs: warp 1 issues S = Q K^T, warp 2 (after allocating TMEM) issues
+    // O += P V.  A commit tracks only its own thread's MMAs, so each has its own
+    // completion barriers (sfull / pvfree) and drain.
     if (lane == 0) {
       // Descriptors are built once; a K-step moves the start address, i.e. adds
       // (byte offset >> 4) to the low field (no carry: addresses stay below 256 KB).
@@ -507,62 +510,50 @@ __global__ void __launch_bounds__(kThreads, 1)
       // V tile, N(=head-dim)-major: 16 tokens per step (2048 bytes), the second
       // 64-column half at +kHalfBytes (leading byte offset), 8-row groups 1024 apart.
       const uint64_t dV = sdesc(sbase + kOffV, kHalfBytes, 1024);
-      auto issue_S = [&](int t) {
-        const uint32_t s = (uint32_t)(t % kStages), b = (uint32_t)(t % kSBuf);
-        const uint32_t d = tmem + 128u * b;
-        const uint64_t kb = dK + (s * kTileBytes >> 4);
-#pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t off = (uint32_t)(kk >> 2) * kQHalfBytes + (uint32_t)(kk & 3) * 32;
-          mma_ss(d, dQ + (off >> 4), kb + (off >> 4), kIdescS, kk > 0 ? 1u : 0u);
-        }
-      };
-      auto issue_PV = [&](int t) {
-        const uint32_t s = (uint32_t)(t % kStages), b = (uint32_t)(t % kSBuf);
-        const uint32_t a = tmem + 128u * b;
-        const uint64_t vb = dV + (s * kTileBytes >> 4);
-        const uint32_t acc0 = t > 0 ? 1u : 0u;
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk)
-          mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
-                 kk > 0 ? 1u : acc0);
-      };
-      bool ok = mbar_wait(&bars->qready, 0u, bars, p.header, 11);
-      for (int t = 0; t < min(2, n_tiles) && ok; ++t) {
-        ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
-        if (!ok) break;
-        fence_after();
-        issue_S(t);
-        mma_commit(&bars->sfull[t % kSBuf]);
-      }
-      for (int j = 0; j < n_tiles && ok; ++j) {
-        // S of tile j+2 first: it needs only its K tile and a free S buffer, so it runs
-        // on the tensor pipe while the softmax still works on tile j
-        const int t = j + 2;
-        if (t < n_tiles) {
-          ok = mbar_wait(&bars->kfull[t % kStages], (uint32_t)((t / kStages) & 1), bars, p.header, 6);
+      bool ok = true;
+      if (warp == 1) {
+        ok = mbar_wait(&bars->qready, 0u, bars, p.header, 11);
+        for (int t = 0; t < n_tiles && ok; ++t) {
+          const uint32_t s = (uint32_t)(t % kStages);
+          ok = mbar_wait(&bars->kfull[s], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
           if (!ok) break;
-          // S buffer t % 3 == (j - 1) % 3 holds P of tile j - 1 until that P.V completes
-          if (j >= 1)
-            ok = mbar_wait(&bars->pvdone[(j - 1) & 1], (uint32_t)(((j - 1) >> 1) & 1), bars, p.header, 7);
+          // S buffer s holds P of tile t-3 until that P.V completes
+          if (t >= kStages)
+            ok = mbar_wait(&bars->pvfree[s], (uint32_t)((t / kStages - 1) & 1), bars, p.header, 6);
           if (!ok) break;
           fence_after();
-          issue_S(t);
-          mma_commit(&bars->sfull[t % kSBuf]);
+          const uint32_t d = tmem + 128u * s;
+          const uint64_t kb = dK + (s * kTileBytes >> 4);
+#pragma unroll
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint32_t off = (uint32_t)(kk >> 2) * kQHalfBytes + (uint32_t)(kk & 3) * 32;
+            mma_ss(d, dQ + (off >> 4), kb + (off >> 4), kIdescS, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&bars->sfull[s]);
         }
-        const int s = j % kStages;
-        ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
-        if (!ok) break;
-        ok = mbar_wait(&bars->pfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
-        if (!ok) break;
-        fence_after();
-        issue_PV(j);
-        mma_commit(&bars->pvdone[j & 1]);
-        mma_commit(&bars->vempty[s]);
+        mma_commit(&bars->drain_s);
+        drain_wait(&bars->drain_s, 0u);
+      } else {
+        for (int j = 0; j < n_tiles && ok; ++j) {
+          const uint32_t s = (uint32_t)(j % kStages);
+          ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
+          if (!ok) break;
+          ok = mbar_wait(&bars->pfull[s], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
+          if (!ok) break;
+          fence_after();
+          const uint32_t a = tmem + 128u * s;
+          const uint64_t vb = dV + (s * kTileBytes >> 4);
+          const uint32_t acc0 = j > 0 ? 1u : 0u;
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
+                   kk > 0 ? 1u : acc0);
+          mma_commit(&bars->pvfree[s]);
+        }
+        // O is final once every P.V has completed
+        mma_commit(&bars->drain_pv);
+        drain_wait(&bars->drain_pv, 0u);
       }
-      // every MMA issued by this thread has completed once this commit lands
-      mma_commit(&bars->drain);
-      drain_wait(&bars->drain, 0u);
     }
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax
@@ -626,7 +617,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (__any_sync(0xffffffffu, need && j > 0)) {
           // O must hold P.V of tile j-1 before it is rescaled (each half rescales its
           // own 64 head-dim columns; both halves take the same decision per row)
-          ok = mbar_wait(&bars->pvdone[(j - 1) & 1], (uint32_t)(((j - 1) >> 1) & 1), bars, p.header, 9);
+          ok = mbar_wait(&bars->pvfree[(j - 1) % kStages], (uint32_t)(((j - 1) / kStages) & 1), bars,
+                         p.header, 9);
           ok = __all_sync(0xffffffffu, ok);
           if (!ok) break;
           fence_after();
@@ -651,8 +643,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->pfull[j % kSBuf]);
     }
-    // the issuer commits `drain` after its last MMA: O is final once it lands
-    if (ok) ok = mbar_wait(&bars->drain, 0u, bars, p.header, 10);
+    // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
+    if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
     ok = __all_sync(0xffffffffu, ok);
     if (ok && warp_active) {
       fence_after();
