@@ -473,11 +473,14 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
     for (int h = 0; h < prob->h_kv; ++h) {
       for (int s = 0; s < L.n_splits[b]; ++s) {
         PadWorkItem it;
-        it.video = b;
-        it.kvh = (int16_t)h;
-        it.split = (int16_t)s;
         it.tok_begin = s * L.split_len;
         it.tok_end = std::min(prefix_len[b], (s + 1) * L.split_len);
+        it.tok0 = vids[b].prefix_off + it.tok_begin;
+        it.first_event = L.ev_first[b];
+        it.n_events = L.ev_count[b];
+        it.part_row0 = L.part_base[b] + (h * L.n_splits[b] + s) * (L.ev_count[b] * L.group);
+        it.kvh = (int16_t)h;
+        it.split = (int16_t)s;
         items.push_back(it);
       }
     }

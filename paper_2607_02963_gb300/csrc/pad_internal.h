@@ -50,14 +50,19 @@ struct PadEventDesc {
 };
 static_assert(sizeof(PadEventDesc) == 16, "event desc is 16 bytes");
 
+// One prefix split of one (video, kv-head).  It carries copies of the owning video's
+// fields so that a CTA can start after a single 32-byte load.
 struct PadWorkItem {
-  int32_t video;
-  int16_t kvh;
-  int16_t split;
+  int64_t tok0;         // first token of the split in k_prefix / v_prefix (prefix_off + tok_begin)
   int32_t tok_begin;    // [tok_begin, tok_end) relative to the video's prefix start
   int32_t tok_end;
+  int32_t first_event;  // the video's first event and event count
+  int32_t n_events;
+  int32_t part_row0;    // partial row of (this split, row 0): part_base + (kvh * n_splits + split) * R
+  int16_t kvh;
+  int16_t split;
 };
-static_assert(sizeof(PadWorkItem) == 16, "work item is 16 bytes");
+static_assert(sizeof(PadWorkItem) == 32, "work item is 32 bytes");
 
 // Everything a kernel needs, passed by value.
 struct KParams {

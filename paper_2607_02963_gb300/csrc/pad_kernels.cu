@@ -94,11 +94,11 @@ __device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a, uint32_t b
 }
 
 // Query row r of (video, kv-head): event e_local = r / G, head kvh*G + r % G.
-__device__ __forceinline__ const __nv_bfloat16* q_row(const KParams& p, const PadVideoDesc& vd,
+__device__ __forceinline__ const __nv_bfloat16* q_row(const KParams& p, int first_event,
                                                       const __nv_bfloat16* q, int kvh, int r) {
   int el = r / p.group;
   int gh = r - el * p.group;
-  return q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * p.head_dim;
+  return q + ((size_t)(first_event + el) * p.h_q + kvh * p.group + gh) * p.head_dim;
 }
 
 __device__ __forceinline__ int64_t part_row(const PadVideoDesc& vd, int kvh, int split, int R, int r) {
@@ -160,15 +160,14 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
   __shared__ float so[MAXR][D];
 
   const PadWorkItem it = p.items[blockIdx.x];
-  const PadVideoDesc vd = p.videos[it.video];
-  const int R = vd.n_events * p.group;
+  const int R = it.n_events * p.group;
   const int kvh = it.kvh;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   for (int i = threadIdx.x; i < MAXR * D; i += blockDim.x) {
     int r = i / D, d = i - r * D;
     float v = 0.f;
-    if (r < R) v = __bfloat162float(q_row(p, vd, q, kvh, r)[d]);
+    if (r < R) v = __bfloat162float(q_row(p, it.first_event, q, kvh, r)[d]);
     sq[r][d] = v;
     so[r][d] = 0.f;
   }
@@ -186,8 +185,8 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
 
   const int ntok = it.tok_end - it.tok_begin;
   const size_t row_stride = (size_t)p.h_kv * D;
-  const __nv_bfloat16* kbase = kp + ((size_t)vd.prefix_off + it.tok_begin) * row_stride + (size_t)kvh * D;
-  const __nv_bfloat16* vbase = vp + ((size_t)vd.prefix_off + it.tok_begin) * row_stride + (size_t)kvh * D;
+  const __nv_bfloat16* kbase = kp + (size_t)it.tok0 * row_stride + (size_t)kvh * D;
+  const __nv_bfloat16* vbase = vp + (size_t)it.tok0 * row_stride + (size_t)kvh * D;
 
   for (int c0 = warp * 32; c0 < ntok; c0 += NW * 32) {
     const int t = c0 + lane;
@@ -278,7 +277,7 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
     float M = kNegInf;
 #pragma unroll
     for (int w = 0; w < NW; ++w) M = fmaxf(M, sm[w][r]);
-    int64_t pr = part_row(vd, kvh, it.split, R, r);
+    int64_t pr = (int64_t)it.part_row0 + r;
     if (d == 0) {
       float L = 0.f;
 #pragma unroll
@@ -309,8 +308,7 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
   __nv_bfloat16* sV = sK + 2 * TN * LDS;
 
   const PadWorkItem it = p.items[blockIdx.x];
-  const PadVideoDesc vd = p.videos[it.video];
-  const int R = vd.n_events * p.group;
+  const int R = it.n_events * p.group;
   const int row0 = blockIdx.y * 64;
   if (row0 >= R) return;
   const int kvh = it.kvh;
@@ -320,8 +318,8 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
   const int rlo = row0 + warp * 16 + g, rhi = rlo + 8;
   uint32_t qa[KSTEPS][4];
   {
-    const __nv_bfloat16* ql = rlo < R ? q_row(p, vd, q, kvh, rlo) : nullptr;
-    const __nv_bfloat16* qh = rhi < R ? q_row(p, vd, q, kvh, rhi) : nullptr;
+    const __nv_bfloat16* ql = rlo < R ? q_row(p, it.first_event, q, kvh, rlo) : nullptr;
+    const __nv_bfloat16* qh = rhi < R ? q_row(p, it.first_event, q, kvh, rhi) : nullptr;
 #pragma unroll
     for (int kk = 0; kk < KSTEPS; ++kk) {
       const int c = kk * 16 + 2 * t4;
@@ -333,8 +331,9 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
   }
 
   const size_t row_stride = (size_t)p.h_kv * D;
-  const __nv_bfloat16* kbase = kp + (size_t)vd.prefix_off * row_stride + (size_t)kvh * D;
-  const __nv_bfloat16* vbase = vp + (size_t)vd.prefix_off * row_stride + (size_t)kvh * D;
+  // token t of the video's prefix (t relative to its start) is row (it.tok0 - it.tok_begin) + t
+  const __nv_bfloat16* kbase = kp + (size_t)(it.tok0 - it.tok_begin) * row_stride + (size_t)kvh * D;
+  const __nv_bfloat16* vbase = vp + (size_t)(it.tok0 - it.tok_begin) * row_stride + (size_t)kvh * D;
   const int ntiles = (it.tok_end - it.tok_begin + TN - 1) / TN;
 
   auto load_tile = [&](int tile, int stage) {
@@ -446,7 +445,7 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
   l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 1);
   l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 2);
   if (rlo < R) {
-    const int64_t pr = part_row(vd, kvh, it.split, R, rlo);
+    const int64_t pr = (int64_t)it.part_row0 + rlo;
     if (t4 == 0) p.part_ml[pr] = make_float2(m_lo, l_lo);
     float* dst = p.part_o + pr * D;
 #pragma unroll
@@ -454,7 +453,7 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
       *reinterpret_cast<float2*>(dst + db * 8 + 2 * t4) = make_float2(o[db][0], o[db][1]);
   }
   if (rhi < R) {
-    const int64_t pr = part_row(vd, kvh, it.split, R, rhi);
+    const int64_t pr = (int64_t)it.part_row0 + rhi;
     if (t4 == 0) p.part_ml[pr] = make_float2(m_hi, l_hi);
     float* dst = p.part_o + pr * D;
 #pragma unroll
@@ -465,18 +464,22 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
 
 // ---------------------------------------------------------------------------
 // a4 + a5: one CTA (256 threads, 8 warps) per (event, kv-head).
-//   At entry the prefix partials (m, l, O of the branch's G rows for up to `sch`
-//   splits) start streaming into shared memory with cp.async, so they land while
-//   the branch is computed.
-//   a4, the own-branch part of the mask of Sec. 3.4: the branch's len+1 keys, in
-//   chunks of 128, are staged (K and V rows through the page table, cp.async) and
-//   processed as a small flash-attention on the warp-level MMA: the G <= 16 query
-//   rows form one m16 tile; S = Q K^T (warps split the keys), a row softmax (one
-//   warp per row), O += P V (warps split the head dimension).
-//   a5: the log-sum-exp merge of the branch state with the staged partials.
+//   a4, the own-branch part of the mask of Sec. 3.4: the branch's len+1 keys.
+//   Keys 0..len-1 were appended by earlier steps and this step's append writes only
+//   key `len` (and, for a new page, the page-table entry of that key), so the pass over
+//   keys 0..len-1 reads nothing the grids launched before this one write: it runs
+//   before griddepcontrol.wait, overlapping the tail of the shared-prefix pass.  Those
+//   keys are staged in blocks of 128 (K and V rows through the page table, cp.async)
+//   and processed as a small flash-attention on the warp-level MMA: the G <= 16 query
+//   rows form one m16 tile; S = Q K^T (warps split the keys), a row softmax (one warp
+//   per row), O += P V (warps split the head dimension).
+//   After the wait, key `len` (written by this step's append) and the prefix partials
+//   (m, l, O of the branch's G rows for up to `sch` splits) arrive in one round trip;
+//   the key is folded into the branch state in fp32 and then
+//   a5: the log-sum-exp merge of the branch state with the partials.
 // ---------------------------------------------------------------------------
 constexpr int kBmThreads = 256;
-constexpr int kBmKeys = 64;                   // branch keys per chunk
+constexpr int kBmKeys = 128;                  // branch keys per staged block
 
 __host__ __device__ constexpr size_t bm_align16(size_t x) { return (x + 15) / 16 * 16; }
 
@@ -484,14 +487,16 @@ template <int D>
 struct BmSmem {
   static constexpr int LD = D + 8;            // padded bf16 row: ldmatrix rows in distinct banks
   __nv_bfloat16 q[16][LD];
-  __nv_bfloat16 k[kBmKeys][LD];
-  __nv_bfloat16 v[kBmKeys][LD];
-  __nv_bfloat16 pb[16][kBmKeys + 8];          // P of the chunk (bf16, A operand of P.V)
-  float sc[16][kBmKeys];                      // scaled scores of the chunk
+  __nv_bfloat16 pb[16][kBmKeys + 8];          // P of the block (bf16, A operand of P.V)
+  float sc[16][kBmKeys];                      // scaled scores of the block; later split weights
   float ob[16][D];                            // branch O, then the merged numerator
+  __nv_bfloat16 knew[D], vnew[D];             // key `len` of the branch
   int page[kBmKeys];
-  float m[16], l[16], a[16];
+  float m[16], l[16], a[16], pn[16];
   float M[16], L[16];
+  // K and V rows of one block; once the branch pass is done the same bytes hold the
+  // staged prefix partials (float2 m,l per row and split, then fp32 O rows)
+  alignas(16) __nv_bfloat16 kv[2][kBmKeys][LD];
 };
 
 template <int D>
@@ -503,17 +508,18 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
                                                                   float* __restrict__ lse,
                                                                   int sch) {
   constexpr int NT = kBmThreads, NW = NT / 32;
-  constexpr int LD = BmSmem<D>::LD;
   constexpr int CH = D / 8;                   // 16-byte pieces of a bf16 row
   extern __shared__ __align__(16) unsigned char bm_raw[];
   BmSmem<D>& S = *reinterpret_cast<BmSmem<D>*>(bm_raw);
-  float2* sml = reinterpret_cast<float2*>(bm_raw + bm_align16(sizeof(BmSmem<D>)));
-  float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) +
-                                        bm_align16((size_t)p.group * sch * sizeof(float2)));
+  auto sK = S.kv[0];
+  auto sV = S.kv[1];
+  float2* sml = reinterpret_cast<float2*>(&S.kv[0][0][0]);
 
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
   const int G = p.group;
+  float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) +
+                                        bm_align16((size_t)G * sch * sizeof(float2)));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, t4 = lane & 3;
   const PadEventDesc ev = p.events[e];
@@ -521,11 +527,9 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
   const int R = vd.n_events * G;
   const int ns = vd.n_splits;
   const int rbase = ev.local * G;
-  const int nk = ev.len + 1;
+  const int len = ev.len;                     // keys before this step; key `len` is this step's
   const int ps = p.page_size;
 
-  // q rows are inputs of the step, not outputs of the kernels before this one: stage them
-  // while those may still run; everything after griddepcontrol.wait may read their results
   for (int i = tid; i < 16 * CH; i += NT) {
     const int g = i / CH, c = i - (i / CH) * CH;
     uint4 v = make_uint4(0u, 0u, 0u, 0u);
@@ -536,24 +540,6 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
     S.m[tid] = kNegInf;
     S.l[tid] = 0.f;
   }
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-
-  // stage the prefix partials of the first `sch` splits (group 0)
-  auto stage_partials = [&](int s0, int nch) {
-    for (int i = tid; i < G * nch; i += NT) {
-      const int g = i / nch, sl = i - (i / nch) * nch;
-      sml[g * sch + sl] = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
-    }
-    constexpr int PC = D / 4;  // 16-byte pieces of one fp32 O row
-    for (int i = tid; i < G * nch * PC; i += NT) {
-      const int c = i % PC, rs = i / PC;
-      const int g = rs / nch, sl = rs - (rs / nch) * nch;
-      cp_async16(spo + ((size_t)g * sch + sl) * D + c * 4,
-                 p.part_o + part_row(vd, kvh, s0 + sl, R, rbase + g) * D + c * 4, true);
-    }
-    cp_async_commit();
-  };
-  if (ns > 0) stage_partials(0, min(sch, ns));
 
   // O of this warp: rows gq, gq+8 x head-dim columns of d-blocks (2 per warp for D=128)
   constexpr int DB = D / 8 / NW > 0 ? D / 8 / NW : 1;   // d-blocks per warp (2 or 1)
@@ -562,8 +548,9 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
   for (int i = 0; i < DB; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   const int db0 = warp * DB;                  // first d-block of this warp (D=64: warps 0-7)
 
-  for (int c0 = 0; c0 < nk; c0 += kBmKeys) {
-    const int nv = min(kBmKeys, nk - c0);
+  // ---------------- a4 over keys 0..len-1 (state of earlier steps only)
+  for (int c0 = 0; c0 < len; c0 += kBmKeys) {
+    const int nv = min(kBmKeys, len - c0);
     const int nv16 = (nv + 15) & ~15;         // keys padded to the MMA K step (zero rows)
     if (tid < kBmKeys) {
       int page = -1;
@@ -578,14 +565,14 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
       S.page[tid] = page;
     }
     __syncthreads();
-    // K and V rows of the chunk (rows past nv or with a bad page: zeros)
+    // K and V rows of the block (rows past nv or with a bad page: zeros)
     for (int i = tid; i < nv16 * CH; i += NT) {
       const int k = i / CH, c = i - (i / CH) * CH;
       const int pg = k < nv ? S.page[k] : -1;
       const bool ok = pg >= 0;
       const size_t off = (((size_t)(ok ? pg : 0) * p.h_kv + kvh) * ps + ((c0 + k) % ps)) * D + c * 8;
-      cp_async16(&S.k[k][c * 8], kpool + off, ok);
-      cp_async16(&S.v[k][c * 8], vpool + off, ok);
+      cp_async16(&sK[k][c * 8], kpool + off, ok);
+      cp_async16(&sV[k][c * 8], vpool + off, ok);
     }
     cp_async_commit();
     cp_async_wait<0>();
@@ -596,10 +583,9 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
       float sacc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
-        uint32_t a[4], b0, b1;
+        uint32_t a[4], b0, b1, b2, b3;
         ldsm_x4(a[0], a[1], a[2], a[3], &S.q[(lane & 15)][kk * 16 + (lane >> 4) * 8]);
-        uint32_t b2, b3;
-        ldsm_x4(b0, b1, b2, b3, &S.k[nb * 8 + (lane & 7)][kk * 16 + ((lane >> 3) & 1) * 8]);
+        ldsm_x4(b0, b1, b2, b3, &sK[nb * 8 + (lane & 7)][kk * 16 + ((lane >> 3) & 1) * 8]);
         (void)b2;
         (void)b3;
         mma_bf16(sacc, a, b0, b1);
@@ -611,7 +597,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
       S.sc[gq + 8][col + 1] = sacc[3] * p.scale_log2;
     }
     __syncthreads();
-    // row softmax of the chunk: warp w takes rows w and w+8
+    // row softmax of the block: warp w takes rows w and w+8
     for (int g = warp; g < 16; g += NW) {
       if (g < G) {
         float mx = kNegInf;
@@ -656,7 +642,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
 #pragma unroll
         for (int i = 0; i < DB; ++i) {
           uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(b0, b1, b2, b3, &S.v[ks * 16 + ((lane >> 3) & 1) * 8 + (lane & 7)][(db0 + i) * 8]);
+          ldsm_x4_t(b0, b1, b2, b3, &sV[ks * 16 + ((lane >> 3) & 1) * 8 + (lane & 7)][(db0 + i) * 8]);
           (void)b2;
           (void)b3;
           mma_bf16(o[i], a, b0, b1);
@@ -665,7 +651,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
     }
     __syncthreads();
   }
-  // branch O to shared memory (rows < G)
+  // branch O so far to shared memory (rows < G)
   if (db0 < D / 8) {
 #pragma unroll
     for (int i = 0; i < DB; ++i) {
@@ -680,15 +666,83 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
       }
     }
   }
+
+  // ---------------- after the shared-prefix pass (and, through it, the append) completed
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  // key `len`: its page is the one this step took, else the table's entry
+  const int pi_new = len / ps;
+  int page_new = ev.new_page >= 0 ? ev.new_page : p.page_table[(size_t)e * p.max_pages + pi_new];
+  const bool new_ok = page_new >= 0 && page_new < p.n_pages;
+  if (!new_ok && tid == 0) set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi_new, page_new);
+  if (tid < 2 * CH) {
+    const int c = tid % CH;
+    const size_t off = (((size_t)(new_ok ? page_new : 0) * p.h_kv + kvh) * ps + (len % ps)) * D + c * 8;
+    if (tid < CH)
+      cp_async16(&S.knew[c * 8], kpool + off, new_ok);
+    else
+      cp_async16(&S.vnew[c * 8], vpool + off, new_ok);
+  }
+  // stage the prefix partials of splits s0 .. s0+nch-1
+  auto stage_partials = [&](int s0, int nch) {
+    for (int i = tid; i < G * nch; i += NT) {
+      const int g = i / nch, sl = i - (i / nch) * nch;
+      sml[g * sch + sl] = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
+    }
+    constexpr int PC = D / 4;  // 16-byte pieces of one fp32 O row
+    for (int i = tid; i < G * nch * PC; i += NT) {
+      const int c = i % PC, rs = i / PC;
+      const int g = rs / nch, sl = rs - (rs / nch) * nch;
+      cp_async16(spo + ((size_t)g * sch + sl) * D + c * 4,
+                 p.part_o + part_row(vd, kvh, s0 + sl, R, rbase + g) * D + c * 4, true);
+    }
+    cp_async_commit();
+  };
+  if (ns > 0)
+    stage_partials(0, min(sch, ns));
+  else
+    cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // fold key `len` into the branch state (fp32): warp w takes rows w and w+8
+  for (int g = warp; g < 16; g += NW) {
+    if (g < G && new_ok) {
+      float dot = 0.f;
+      for (int d = lane; d < D; d += 32)
+        dot = fmaf(__bfloat162float(S.q[g][d]), __bfloat162float(S.knew[d]), dot);
+      const float s = warp_sum(dot) * p.scale_log2;
+      if (lane == 0) {
+        const float mo = S.m[g];
+        const float mn = fmaxf(mo, s);
+        const float al = ex2(mo - mn);
+        const float pnew = ex2(s - mn);
+        S.a[g] = al;
+        S.pn[g] = pnew;
+        S.l[g] = S.l[g] * al + pnew;
+        S.m[g] = mn;
+      }
+    } else if (lane == 0) {
+      S.a[g] = 1.f;
+      S.pn[g] = 0.f;
+    }
+  }
+  __syncthreads();
+  for (int i = tid; i < G * D; i += NT) {
+    const int g = i / D, d = i - g * D;
+    S.ob[g][d] = fmaf(S.pn[g], __bfloat162float(S.vnew[d]), S.ob[g][d] * S.a[g]);
+  }
   if (tid < 16) S.M[tid] = S.m[tid];
   __syncthreads();
 
   // ---------------- a5: merge with the prefix partials, in chunks of `sch` splits
   for (int s0 = 0; s0 < ns; s0 += sch) {
     const int nch = min(sch, ns - s0);
-    if (s0 > 0) stage_partials(s0, nch);
-    cp_async_wait<0>();
-    __syncthreads();
+    if (s0 > 0) {
+      stage_partials(s0, nch);
+      cp_async_wait<0>();
+      __syncthreads();
+    }
     if (tid < G) {
       const float oldM = S.M[tid];
       float mm = oldM;
@@ -807,18 +861,17 @@ template <int D>
 static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
                              void* out, float* lse, bool pdl, cudaStream_t s) {
   const int G = p.group;
-  const size_t base = bm_align16(sizeof(BmSmem<D>));
-  // Staged prefix partials: all splits of a video when one wave of CTAs covers the grid
-  // (then latency decides), else a budget that keeps three CTAs per SM resident.
-  const int n_cta = p.n_events * p.h_kv;
+  // Staged prefix partials share the bytes of the branch K/V block: as many splits of a
+  // chunk as fit there.
+  constexpr size_t region = sizeof(BmSmem<D>::kv);
   const size_t per_split = (size_t)G * (D * sizeof(float) + sizeof(float2));
-  const size_t budget = n_cta > p.n_sms ? (72 * 1024 > base ? 72 * 1024 - base : per_split) : 96 * 1024;
-  int sch = (int)(budget / per_split);
+  int sch = (int)((region - 16) / per_split);
   if (p.max_splits > 0 && sch > p.max_splits) sch = p.max_splits;
   sch = sch < 1 ? 1 : (sch > kBmKeys ? kBmKeys : sch);
-  const size_t smem = base + bm_align16((size_t)G * sch * sizeof(float2)) + (size_t)G * sch * D * sizeof(float);
-  constexpr int kMaxSmem = 200 * 1024;
-  if (smem > (size_t)kMaxSmem) return cudaErrorInvalidValue;
+  if (bm_align16((size_t)G * sch * sizeof(float2)) + (size_t)G * sch * D * sizeof(float) > region)
+    return cudaErrorInvalidValue;
+  const size_t smem = sizeof(BmSmem<D>);
+  constexpr int kMaxSmem = (int)sizeof(BmSmem<D>);
   static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);

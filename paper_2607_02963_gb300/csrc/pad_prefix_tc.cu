@@ -66,6 +66,8 @@ constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
 constexpr uint32_t kOffX = kOffBar + 256;               // partial row maxima: [2][2][128] fp32
 constexpr uint32_t kSmemBytes = kOffX + 2 * 2 * 128 * 4;
+constexpr int kOStage = kD + 4;                       // fp32 row stride of the O staging rows
+static_assert(128 * kOStage * 4 <= kStages * kTileBytes, "O staging fits the K stages");
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 384;
 constexpr float kLazyRescale = 8.0f;                  // log2 units
@@ -85,10 +87,11 @@ struct TcBars {
   uint64_t vfull[kStages];
   uint64_t pvfree[kStages];   // P.V of the tile in this stage / S buffer has completed
   uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
-  uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (4 warp arrivals)
+  uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (8 warp arrivals)
   uint64_t drain_s;           // every S MMA has completed (S issuer)
   uint64_t drain_pv;          // every P.V MMA has completed (P.V issuer)
   uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
+  uint64_t tdone;             // the softmax warps are done with TMEM (8 warp arrivals)
   uint64_t xchg[4];           // the two softmax warps of a lane quarter met (64 thread arrivals)
   uint32_t tmem_base;
   int32_t abort;
@@ -423,13 +426,34 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int item = blockIdx.x / n_groups;
   const int group = blockIdx.x - item * n_groups;
   const PadWorkItem it = p.items[item];
-  const PadVideoDesc vd = p.videos[it.video];
-  const int R = vd.n_events * p.group;
+  const int R = it.n_events * p.group;
   const int row0 = group * 128;
   if (row0 >= R) return;  // uniform over the CTA, before any barrier or allocation
   const int ntok = it.tok_end - it.tok_begin;
   const int n_tiles = (ntok + kBN - 1) / kBN;
   const int kvh = it.kvh;
+  const int tok0 = (int)it.tok0;
+
+  // The softmax warps load their Q rows now, so that the loads overlap barrier set-up
+  // and TMEM allocation; they are stored to shared memory after the block barrier.
+  // Lane `lane` of warp w holds row 32*(w&3) + (lane+32i)/8, 16-byte chunk (lane+32i)%8
+  // of head-dim half (w-4)/4.  Rows past R are zero.
+  uint4 qv[8];
+  if (warp >= 4) {
+    const int lane_base = 32 * (warp & 3), half = (warp - 4) >> 2;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int idx = lane + 32 * i;
+      const int qrow = row0 + lane_base + (idx >> 3);
+      qv[i] = make_uint4(0u, 0u, 0u, 0u);
+      if (qrow < R) {
+        const int el = qrow / p.group;
+        const int gh = qrow - el * p.group;
+        qv[i] = __ldg(reinterpret_cast<const uint4*>(
+            q + ((size_t)(it.first_event + el) * p.h_q + kvh * p.group + gh) * kD + half * 64 + (idx & 7) * 8));
+      }
+    }
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -444,9 +468,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bars->drain_s, 1);
     mbar_init(&bars->drain_pv, 1);
     mbar_init(&bars->qready, 8);
+    mbar_init(&bars->tdone, 8);
     for (int qq = 0; qq < 4; ++qq) mbar_init(&bars->xchg[qq], 64);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // The first kStages K and V tiles go out before TMEM allocation and the block
+    // barrier; the producer warps issue the rest.
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    for (int t = 0; t < kStages && t < n_tiles; ++t) {
+      mbar_expect_tx(&bars->kfull[t], kTileBytes);
+      tma_load_3d(sbase + kOffK + t * kTileBytes, &tmK, 0, kvh, tok0 + t * kBN, &bars->kfull[t]);
+      tma_load_3d(sbase + kOffK + t * kTileBytes + kHalfBytes, &tmK, 64, kvh, tok0 + t * kBN, &bars->kfull[t]);
+      mbar_expect_tx(&bars->vfull[t], kTileBytes);
+      tma_load_3d(sbase + kOffV + t * kTileBytes, &tmV, 0, kvh, tok0 + t * kBN, &bars->vfull[t]);
+      tma_load_3d(sbase + kOffV + t * kTileBytes + kHalfBytes, &tmV, 64, kvh, tok0 + t * kBN, &bars->vfull[t]);
+    }
   }
   if (warp == 2) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -463,19 +501,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   // prologue now; it waits for this grid's completion before it reads partials.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const uint32_t tmem = bars->tmem_base;
-  const int tok0 = (int)(vd.prefix_off + it.tok_begin);
 
   if (warp == 0 || warp == 3) {
     // ------------------------------------------------------------ TMA producers
     if (lane == 0) {
       const bool isK = warp == 0;
       const CUtensorMap* map = isK ? &tmK : &tmV;
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-      int issued = 0;
+      int issued = min(kStages, n_tiles);  // tiles 0..kStages-1 went out in the prologue
       bool ok = true;
-      for (int t = 0; t < n_tiles && ok; ++t) {
+      for (int t = kStages; t < n_tiles && ok; ++t) {
         const int s = t % kStages;
-        if (t >= kStages) {
+        {
           // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
           uint64_t* freed = isK ? &bars->sfull[s] : &bars->pvfree[s];
           ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
@@ -560,21 +596,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31 (query rows)
     const int half = (warp - 4) >> 2;          // columns 64*half .. +63 of every tile
     const int lane_base = 32 * quarter;
-    // Q rows of this quarter, head-dim half `half`, into the 128-byte-swizzled K-major
-    // layout the MMA reads (the K/V loads are already in flight): row r, 16-byte chunk
-    // cc of half h at h*16K + r*128 + ((cc ^ (r & 7)) << 4).  Rows past R are zero.
-    for (int idx = lane; idx < 32 * 8; idx += 32) {
+    // Q rows (loaded in the prologue) into the 128-byte-swizzled K-major layout the
+    // MMA reads: row r, 16-byte chunk cc of half h at h*16K + r*128 + ((cc ^ (r & 7)) << 4).
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int idx = lane + 32 * i;
       const int r = lane_base + (idx >> 3), cc = idx & 7;
-      const int qrow = row0 + r;
-      uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (qrow < R) {
-        const int el = qrow / p.group;
-        const int gh = qrow - el * p.group;
-        const __nv_bfloat16* src = q + ((size_t)(vd.first_event + el) * p.h_q + kvh * p.group + gh) * kD +
-                                   half * 64 + cc * 8;
-        v = __ldg(reinterpret_cast<const uint4*>(src));
-      }
-      *reinterpret_cast<uint4*>(smem + kOffQ + half * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = v;
+      *reinterpret_cast<uint4*>(smem + kOffQ + half * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = qv[i];
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncwarp();
@@ -646,27 +674,41 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
     if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
     ok = __all_sync(0xffffffffu, ok);
+    // O leaves through shared memory: TMEM gives one row per thread, which stored straight
+    // to global memory would touch 32 lines per instruction.  Rows are staged in the K
+    // stages (idle once every MMA has completed) at a padded stride, so that eight
+    // consecutive rows fall in distinct banks, then written one 512-byte row per warp
+    // instruction.
+    float* ostage = reinterpret_cast<float*>(smem + kOffK);
     if (ok && warp_active) {
       fence_after();
-      const int64_t pr = (int64_t)vd.part_base + ((int64_t)kvh * vd.n_splits + it.split) * R + grow;
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         tmem_ld32(tl + kColO + col0 + 32 * c, r);
         tmem_wait_ld_dep(r);
-        if (grow < R) {
-          float4* dst = reinterpret_cast<float4*>(p.part_o + pr * kD + col0 + 32 * c);
+        float4* dst = reinterpret_cast<float4*>(ostage + row * kOStage + col0 + 32 * c);
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
-                                 __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
-        }
+        for (int i = 0; i < 8; ++i)
+          dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                               __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
       }
       // row sum = both halves' partial sums (slot n_tiles & 1 was last read two tiles ago)
       xmax[(n_tiles & 1) * 256 + half * 128 + row] = l_run;
       mbar_arrive(xbar);
       ok = mbar_wait(xbar, (uint32_t)(n_tiles & 1), bars, p.header, 13);
       if (ok && half == 0 && grow < R)
-        p.part_ml[pr] = make_float2(m_run, l_run + xmax[(n_tiles & 1) * 256 + 128 + row]);
+        p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_run, l_run + xmax[(n_tiles & 1) * 256 + 128 + row]);
+    }
+    // TMEM is freed by warp 2 only after every softmax warp has arrived here
+    fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bars->tdone);
+    // every softmax warp reaches this barrier exactly once (the loop above only breaks)
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    const int nrows = min(128, R - row0);
+    for (int rr = warp - 4; rr < nrows; rr += 8) {
+      const float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
+      *reinterpret_cast<float4*>(p.part_o + ((int64_t)it.part_row0 + row0 + rr) * kD + 4 * lane) = v;
     }
   }
 
@@ -678,6 +720,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) asm volatile("griddepcontrol.wait;" ::: "memory");
   __syncthreads();
   if (warp == 2) {
+    // The block barrier above is not relied on to order the softmax warps' last TMEM
+    // reads before the deallocation (it was measured to let the role warps through
+    // before them); their own arrivals are.
+    drain_wait(&bars->tdone, 0u);
     fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
                  : "memory");

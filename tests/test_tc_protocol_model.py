@@ -11,7 +11,8 @@ This model mirrors that schedule with asynchronous loads and MMAs that complete 
 random delays and in any order, and checks under many random interleavings that no stage
 or buffer is reused while something still reads it, that O is rescaled only when no P.V
 is in flight, and that nothing deadlocks.  A schedule that shares one P-ready barrier and
-one P.V barrier across tiles (so that a waiter can miss a phase) fails it.
+one P.V barrier across tiles (so that a waiter can miss a phase) fails it.  TMEM is
+freed only after all eight softmax warps have arrived on their own completion barrier.
 """
 import random
 
@@ -45,6 +46,8 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
     pfull = [Bar(n_softmax) for _ in range(ST)]
     pvfree = [Bar(1) for _ in range(ST)]
     drain_s, drain_pv = Bar(1), Bar(1)
+    tdone = Bar(n_softmax)
+    tmem_users = [True] * n_softmax
     if single_barriers:
         pfull = [pfull[0]] * ST
         pvfree = [pvfree[0]] * ST
@@ -162,8 +165,17 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
             pfull[j % ST].arrive()
         yield (drain_pv, 0)
         assert len(PV_done) == n, "epilogue before every P.V completed"
+        for _ in range(rnd.randint(0, 3)):  # reads O out of TMEM
+            yield None
+        tmem_users[w] = False
+        tdone.arrive()
 
-    actors = [kprod(), vprod(), s_issuer(), pv_issuer()] + [softmax(w) for w in range(n_softmax)]
+    def dealloc():
+        # warp 2 frees TMEM once every softmax warp has arrived on tdone
+        yield (tdone, 0)
+        assert not any(tmem_users), "TMEM freed while a softmax warp still reads it"
+
+    actors = [kprod(), vprod(), s_issuer(), pv_issuer(), dealloc()] + [softmax(w) for w in range(n_softmax)]
     waiting = [None] * len(actors)
     alive = [True] * len(actors)
     steps = 0
