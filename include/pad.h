@@ -10,22 +10,28 @@
  * step), never to another branch's tokens.
  *
  * A step is three calls, all stream-ordered and asynchronous:
- *   pad_plan              host: validate, allocate pages, build the work list,
- *                         upload it into the caller's device workspace;
+ *   pad_plan              host: validate, allocate pages, build the work list in a
+ *                         library-owned page-locked image that the kernels read in
+ *                         place (nothing is put on the stream);
  *   pad_kv_append         device: write each branch's new K/V into its page;
  *   pad_event_decode_attn device: shared-prefix split-KV pass, private-suffix
  *                         pass and log-sum-exp merge; writes O and LSE.
  *
  * Ownership: the caller owns every device buffer (prefix KV, page pools, page
  * table, Q, outputs, workspace); the library never allocates device memory.
- * A pad_plan_t holds host metadata only, plus offsets into the workspace; it
- * stays valid until pad_plan_destroy and is tied to the workspace it was built
- * on (a later pad_plan on the same workspace overwrites it in stream order).
+ * A pad_plan_t holds host metadata and a page-locked, device-mapped image of the
+ * step's descriptors (from a per-device pool of library-owned buffers, kept until
+ * exit); it stays valid until pad_plan_destroy, which may follow its launches at
+ * once: an image is rewritten only after the launches that read it have completed.
+ * A plan is tied to the workspace it was built on, which holds the status word and
+ * the split-KV partial states; steps that share a workspace run in stream order.
  *
  * Errors: every call validates its arguments on the host and returns a
  * pad_status before launching anything; pad_last_error() gives a message
  * (thread-local).  Errors found by a kernel (a page id outside the pool) set a
- * status word in the workspace, which pad_device_status() reads.
+ * status word in the workspace, tagged with the plan's generation (a number drawn
+ * per plan), which pad_device_status() reads; an error recorded by another plan's
+ * kernels does not show up as this plan's.
  *
  * Layouts (row-major, element type bf16 unless stated):
  *   q          [n_events, h_q, head_dim]
@@ -139,13 +145,12 @@ size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32
  *                  new-page entries are written by pad_kv_append
  *   max_pages      columns of page_table; event_len[e] / page_size must be < max_pages
  *   workspace      device, 256-byte aligned, at least pad_workspace_size(...) bytes;
- *                  NULL plans on the host only (no upload; the plan cannot be launched)
- *   stream         stream the plan upload (one cudaMemcpyAsync) is ordered on; the copy is
- *                  made from library-owned page-locked staging memory (eight slots per
- *                  device, allocated on first use and kept until exit), so pad_plan does
- *                  not wait for work already queued on the stream
+ *                  NULL plans on the host only (no image; the plan cannot be launched)
+ *   stream         unused (kept for the interface): pad_plan enqueues nothing; it may
+ *                  wait for the launches of an earlier plan whose image it reuses, once
+ *                  eight or more images of the device have been released
  *   plan_out       receives the new plan (free with pad_plan_destroy)
- * On any error nothing changes: no page is taken and nothing is uploaded. */
+ * On any error nothing changes: no page is taken. */
 pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
                     const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
                     const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
@@ -204,7 +209,7 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
  * and caches it, so make that first call before any stream capture.  All calls share the
  * array: calls that overlap on the GPU (other streams or threads) race on it; calls in
- * order on one stream are safe (each re-uploads the plan image, clearing the status word).
+ * order on one stream are safe (each copies the plan image into it).
  * pad_device_status does not read this array's status word. */
 pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q, const void* k_prefix,
                                         const void* v_prefix, const void* k_pool, const void* v_pool,

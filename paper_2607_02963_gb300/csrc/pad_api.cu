@@ -5,7 +5,11 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
+#include <chrono>
+#include <deque>
 #include <mutex>
+#include <random>
 #include <string>
 #include <vector>
 
@@ -196,59 +200,96 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   return PAD_OK;
 }
 
-// Pinned staging for the plan upload.  A pageable cudaMemcpyAsync may wait for
-// the stream, which would stall the host behind the previous step; copying
-// from page-locked memory keeps pad_plan asynchronous.  Eight slots per device
-// are reused round-robin; a slot is rewritten only after the event recorded
-// behind its last copy has completed.  Slots are allocated on first use (and
-// grown when a larger plan arrives) and kept until the process exits.
-struct StagingSlot {
+// Plan images in pinned, device-mapped host memory.  The kernels read a plan's video and
+// event descriptors and its work items in place, so a step puts no copy on the stream
+// between the previous step's last kernel and its own first one.  An image belongs to
+// its plan until pad_plan_destroy; it then joins its device's FIFO and is rewritten only
+// after the event recorded behind the last launch that read it has completed.  Up to
+// kImagesInFlight images per device are cycled; more are allocated while plans are held.
+struct PlanImage {
   void* host = nullptr;
+  void* dev = nullptr;
   size_t cap = 0;
   cudaEvent_t done = nullptr;
-  bool pending = false;
+  bool recorded = false;
+  int device = 0;
 };
-struct StagingRing {
+constexpr int kImagesInFlight = 8;
+struct ImagePool {
   std::mutex mu;
-  StagingSlot slot[8];
-  int next = 0;
+  std::deque<PlanImage*> fifo;
+  int count = 0;
 };
-StagingRing g_staging[64];
+ImagePool g_images[64];
 
-cudaError_t upload_plan(void* dst, const void* src, size_t n, cudaStream_t s) {
+cudaError_t image_alloc(PlanImage* img, size_t n) {
+  if (img->host) cudaFreeHost(img->host);
+  img->host = img->dev = nullptr;
+  img->cap = 0;
+  const size_t cap = std::max<size_t>(n, 64 * 1024);
+  cudaError_t e = cudaHostAlloc(&img->host, cap, cudaHostAllocMapped | cudaHostAllocPortable);
+  if (e != cudaSuccess) return e;
+  e = cudaHostGetDevicePointer(&img->dev, img->host, 0);
+  if (e != cudaSuccess) return e;
+  img->cap = cap;
+  return cudaSuccess;
+}
+
+cudaError_t image_acquire(size_t n, PlanImage** out) {
+  *out = nullptr;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  StagingRing& ring = g_staging[dev];
-  std::lock_guard<std::mutex> lk(ring.mu);
-  StagingSlot& sl = ring.slot[ring.next];
-  ring.next = (ring.next + 1) % 8;
-  if (sl.pending) {
-    e = cudaEventSynchronize(sl.done);
-    if (e != cudaSuccess) return e;
-    sl.pending = false;
+  ImagePool& pool = g_images[dev];
+  PlanImage* img = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(pool.mu);
+    if (pool.count >= kImagesInFlight && !pool.fifo.empty()) {
+      img = pool.fifo.front();
+      pool.fifo.pop_front();
+    } else {
+      ++pool.count;
+    }
   }
-  if (sl.cap < n) {
-    if (sl.host) cudaFreeHost(sl.host);
-    sl.host = nullptr;
-    sl.cap = 0;
-    const size_t cap = std::max<size_t>(n, 64 * 1024);
-    e = cudaHostAlloc(&sl.host, cap, cudaHostAllocDefault);
-    if (e != cudaSuccess) return e;
-    sl.cap = cap;
+  if (!img) {
+    img = new PlanImage();
+    img->device = dev;
+    e = cudaEventCreateWithFlags(&img->done, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = image_alloc(img, n);
+  } else {
+    if (img->recorded) e = cudaEventSynchronize(img->done);
+    img->recorded = false;
+    if (e == cudaSuccess && img->cap < n) e = image_alloc(img, n);
   }
-  if (!sl.done) {
-    e = cudaEventCreateWithFlags(&sl.done, cudaEventDisableTiming);
-    if (e != cudaSuccess) return e;
+  if (e != cudaSuccess) {
+    std::lock_guard<std::mutex> lk(pool.mu);
+    pool.fifo.push_back(img);
+    return e;
   }
-  std::memcpy(sl.host, src, n);
-  e = cudaMemcpyAsync(dst, sl.host, n, cudaMemcpyHostToDevice, s);
-  if (e != cudaSuccess) return e;
-  e = cudaEventRecord(sl.done, s);
-  if (e != cudaSuccess) return e;
-  sl.pending = true;
+  *out = img;
   return cudaSuccess;
+}
+
+void image_release(PlanImage* img) {
+  if (!img) return;
+  ImagePool& pool = g_images[img->device];
+  std::lock_guard<std::mutex> lk(pool.mu);
+  pool.fifo.push_back(img);
+}
+
+// Generations of plans: 56-bit, nonzero, from a per-process random start.
+uint64_t next_generation() {
+  static std::atomic<uint64_t> ctr{0};
+  static const uint64_t base = [] {
+    std::random_device rd;
+    return ((uint64_t)rd() << 32) ^ (uint64_t)rd() ^
+           (uint64_t)std::chrono::steady_clock::now().time_since_epoch().count();
+  }();
+  for (;;) {
+    const uint64_t g = (base + ctr.fetch_add(1)) & ((1ull << 56) - 1);
+    if (g != 0) return g;
+  }
 }
 
 // Timing of the dominant kernel (process-global measurement aid).
@@ -303,7 +344,13 @@ struct pad_plan_t {
   int64_t total_prefix_tokens = 0;
   int32_t n_new_pages = 0;
   std::vector<int32_t> new_pages;
-  std::vector<uint8_t> host_image;  // header + videos + events + items, as uploaded
+  std::vector<uint8_t> host_image;  // header + videos + events + items
+  PlanImage* image = nullptr;       // the same bytes in pinned memory, read by the kernels
+                                    // when they do not fit the launch parameters
+  std::vector<uint8_t> param_image; // videos | events | items, packed, for KParams::img
+  int32_t img_videos = 0, img_events = 0, img_items = 0;
+  uint64_t gen = 0;                 // generation tagging this plan's device errors
+  ~pad_plan_t() { image_release(image); }
 };
 
 extern "C" {
@@ -516,16 +563,31 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   if (!items.empty())
     std::memcpy(plan->host_image.data() + L.off_items, items.data(), items.size() * sizeof(PadWorkItem));
 
-  if (workspace) {
-    cudaError_t ce = upload_plan(workspace, plan->host_image.data(), L.upload_bytes,
-                                 reinterpret_cast<cudaStream_t>(stream));
+  plan->gen = next_generation();
+  {
+    const size_t nv = vids.size() * sizeof(PadVideoDesc), ne = evs.size() * sizeof(PadEventDesc);
+    const size_t ni = items.size() * sizeof(PadWorkItem);
+    plan->img_videos = 0;
+    plan->img_events = (int32_t)align_up(nv, 16);
+    plan->img_items = (int32_t)(plan->img_events + align_up(ne, 16));
+    const size_t total = plan->img_items + ni;
+    if (n_events > 0 && total <= (size_t)kParamImageBytes) {
+      plan->param_image.assign(total, 0);
+      if (nv) std::memcpy(plan->param_image.data(), vids.data(), nv);
+      if (ne) std::memcpy(plan->param_image.data() + plan->img_events, evs.data(), ne);
+      if (ni) std::memcpy(plan->param_image.data() + plan->img_items, items.data(), ni);
+    }
+  }
+  if (workspace && n_events > 0 && plan->param_image.empty()) {
+    cudaError_t ce = image_acquire(L.upload_bytes, &plan->image);
     if (ce != cudaSuccess) {
       for (int e = 0; e < n_events; ++e)
         if (plan->new_pages[e] >= 0) cache->set(plan->new_pages[e], false);
       cache->free_count += need;
       delete plan;
-      return cuda_fail(ce, "plan upload");
+      return cuda_fail(ce, "plan image");
     }
+    std::memcpy(plan->image->host, plan->host_image.data(), L.upload_bytes);
   }
   plan->prob = *prob;
   plan->n_videos = n_videos;
@@ -564,8 +626,7 @@ pad_status pad_plan_destroy(pad_plan_t* plan) {
   return PAD_OK;
 }
 
-static KParams make_params(const pad_plan_t* plan) {
-  KParams p;
+static void make_params(const pad_plan_t* plan, KParams& p) {
   const pad_problem& pr = plan->prob;
   p.h_q = pr.h_q;
   p.h_kv = pr.h_kv;
@@ -582,15 +643,27 @@ static KParams make_params(const pad_plan_t* plan) {
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
+  p.gen = plan->gen;
   auto* ws = static_cast<uint8_t*>(plan->workspace);
   p.header = reinterpret_cast<PadDevHeader*>(ws);
-  p.videos = reinterpret_cast<const PadVideoDesc*>(ws + plan->lay.off_videos);
-  p.events = reinterpret_cast<const PadEventDesc*>(ws + plan->lay.off_events);
-  p.items = reinterpret_cast<const PadWorkItem*>(ws + plan->lay.off_items);
+  p.img_n = (int32_t)plan->param_image.size();
+  p.img_videos = plan->img_videos;
+  p.img_events = plan->img_events;
+  p.img_items = plan->img_items;
+  if (p.img_n > 0) {
+    std::memcpy(p.img, plan->param_image.data(), plan->param_image.size());
+    p.videos = nullptr;
+    p.events = nullptr;
+    p.items = nullptr;
+  } else {
+    auto* im = static_cast<const uint8_t*>(plan->image->dev);
+    p.videos = reinterpret_cast<const PadVideoDesc*>(im + plan->lay.off_videos);
+    p.events = reinterpret_cast<const PadEventDesc*>(im + plan->lay.off_events);
+    p.items = reinterpret_cast<const PadWorkItem*>(im + plan->lay.off_items);
+  }
   p.part_ml = reinterpret_cast<float2*>(ws + plan->lay.off_ml);
   p.part_o = reinterpret_cast<float*>(ws + plan->lay.off_o);
   p.page_table = plan->page_table;
-  return p;
 }
 
 pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new,
@@ -601,9 +674,16 @@ pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* 
   if (!k_new || !v_new || !k_pool || !v_pool) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_pool) || !aligned16(v_pool))
     return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
-  cudaError_t e = launch_append(make_params(plan), k_new, v_new, k_pool, v_pool,
-                                reinterpret_cast<cudaStream_t>(stream));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  KParams p;
+  make_params(plan, p);
+  cudaError_t e = launch_append(p, k_new, v_new, k_pool, v_pool, s);
   if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  if (plan->image) {
+    e = cudaEventRecord(plan->image->done, s);
+    if (e != cudaSuccess) return cuda_fail(e, "plan image event");
+    plan->image->recorded = true;
+  }
   return PAD_OK;
 }
 
@@ -620,7 +700,8 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
       !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
     return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  const KParams p = make_params(plan);
+  KParams p;
+  make_params(plan, p);
   const bool timed = g_timing.on && g_timing.n < g_timing.max;
   if (timed) cudaEventRecord(g_timing.ev[2 * g_timing.n], s);
   cudaError_t e = cudaSuccess;
@@ -644,6 +725,11 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
   const bool pdl = !timed && plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC;
   e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, pdl, s);
   if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
+  if (plan->image) {
+    e = cudaEventRecord(plan->image->done, s);
+    if (e != cudaSuccess) return cuda_fail(e, "plan image event");
+    plan->image->recorded = true;
+  }
   return PAD_OK;
 }
 
@@ -655,9 +741,10 @@ pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
   cudaError_t e = cudaMemcpyAsync(&h, plan->workspace, sizeof(h), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "reading device status");
-  if (h.status != PAD_OK)
-    return fail((pad_status)h.status, "device reported %s (detail %d %d %d)",
-                pad_status_string((pad_status)h.status), h.info[0], h.info[1], h.info[2]);
+  const int code = (int)(h.word & 0xffull);
+  if ((h.word >> 8) == plan->gen && code != PAD_OK)
+    return fail((pad_status)code, "device reported %s (detail %d %d %d)",
+                pad_status_string((pad_status)code), h.info[0], h.info[1], h.info[2]);
   return PAD_OK;
 }
 
@@ -778,6 +865,8 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
+  p.gen = plan->gen;
+  p.img_n = 0;
   auto* ws = static_cast<uint8_t*>(scratch);
   p.header = reinterpret_cast<PadDevHeader*>(ws);
   p.videos = reinterpret_cast<const PadVideoDesc*>(ws + plan->lay.off_videos);

@@ -1,11 +1,11 @@
 // Internal declarations shared by the host planner (pad_api.cu) and the kernels.
 // The device-side plan is a flat block at the start of the caller's workspace:
 //
-//   [0, 256)            PadDevHeader (status word; reset by every plan upload)
+//   [0, 256)            PadDevHeader (status word, tagged with the plan's generation)
 //   videos              PadVideoDesc[n_videos]
 //   events              PadEventDesc[n_events]
 //   items               PadWorkItem[n_work_items]       (prefix split-KV work list)
-//   -- end of the uploaded part --
+//   -- end of the plan image --
 //   part_ml             float2[partial_rows]            (m in log2 units, l)
 //   part_o              float[partial_rows * head_dim]  (unnormalised O)
 //
@@ -24,12 +24,33 @@ namespace pad {
 constexpr int kSplitGranule = 128;   // prefix splits are multiples of this many tokens
 constexpr int kMaxGroup = 16;        // G = h_q / h_kv supported by the kernels
 
+// Status word of a workspace.  Each plan carries a fresh 56-bit generation; kernels record
+// the first error of their generation as (generation << 8) | pad_status, and a word that
+// carries another generation counts as clear, so nothing resets it between steps.
 struct PadDevHeader {
-  int32_t status;      // pad_status written by kernels (first error wins)
-  int32_t info[3];     // kernel-specific detail of the first error (e.g. event, page)
-  int32_t pad[60];
+  unsigned long long word;
+  int32_t info[3];     // kernel-specific detail of that error (e.g. event, page)
+  int32_t pad[59];
 };
 static_assert(sizeof(PadDevHeader) == 256, "header is 256 bytes");
+
+#ifdef __CUDACC__
+__device__ __forceinline__ void pad_set_error(PadDevHeader* h, uint64_t gen, int code, int a, int b,
+                                              int c) {
+  const unsigned long long want = ((unsigned long long)gen << 8) | (unsigned)code;
+  unsigned long long cur = *reinterpret_cast<volatile unsigned long long*>(&h->word);
+  while ((cur >> 8) != gen || (cur & 0xffull) == 0) {
+    const unsigned long long prev = atomicCAS(&h->word, cur, want);
+    if (prev == cur) {
+      h->info[0] = a;
+      h->info[1] = b;
+      h->info[2] = c;
+      return;
+    }
+    cur = prev;
+  }
+}
+#endif
 
 struct PadVideoDesc {
   int64_t prefix_off;   // first token of the prefix in k_prefix / v_prefix
@@ -64,6 +85,8 @@ struct PadWorkItem {
 };
 static_assert(sizeof(PadWorkItem) == 32, "work item is 32 bytes");
 
+constexpr int kParamImageBytes = 8192 - 256;  // descriptor bytes carried in KParams
+
 // Everything a kernel needs, passed by value.
 struct KParams {
   int32_t h_q, h_kv, group, head_dim, page_size, max_pages, n_pages;
@@ -72,6 +95,7 @@ struct KParams {
   int32_t n_sms;                  // SMs the grid sizes were planned for
   int32_t max_splits;             // largest per-video prefix split count of the batch
   float scale_log2;               // scale * log2(e)
+  uint64_t gen;                   // generation of the plan (tags errors in the status word)
   PadDevHeader* header;
   const PadVideoDesc* videos;
   const PadEventDesc* events;
@@ -79,7 +103,28 @@ struct KParams {
   float2* part_ml;
   float* part_o;
   int32_t* page_table;
+  // The descriptors themselves when they fit (img_n > 0): carried in the launch's
+  // parameter block, so a CTA reads them from the constant bank instead of from the
+  // plan's page-locked host image.  Sections start at the img_* byte offsets.
+  int32_t img_n;                  // bytes used, 0 = read videos / events / items instead
+  int32_t img_videos, img_events, img_items;
+  alignas(16) unsigned char img[kParamImageBytes];
 };
+static_assert(sizeof(KParams) <= 8192, "kernel parameters stay at 8 KB");
+
+#ifdef __CUDACC__
+// Kernels take their KParams as a __grid_constant__ parameter, so these point into the
+// parameter block itself.
+__device__ __forceinline__ const PadVideoDesc* plan_videos(const KParams& p) {
+  return p.img_n > 0 ? reinterpret_cast<const PadVideoDesc*>(p.img + p.img_videos) : p.videos;
+}
+__device__ __forceinline__ const PadEventDesc* plan_events(const KParams& p) {
+  return p.img_n > 0 ? reinterpret_cast<const PadEventDesc*>(p.img + p.img_events) : p.events;
+}
+__device__ __forceinline__ const PadWorkItem* plan_items(const KParams& p) {
+  return p.img_n > 0 ? reinterpret_cast<const PadWorkItem*>(p.img + p.img_items) : p.items;
+}
+#endif
 
 // Launchers (pad_kernels.cu, pad_prefix_tc.cu).  Return the launch error.
 cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,

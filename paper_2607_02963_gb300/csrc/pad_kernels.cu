@@ -18,13 +18,6 @@ namespace {
 
 constexpr float kNegInf = -__builtin_huge_valf();
 
-__device__ __forceinline__ void set_error(PadDevHeader* h, int code, int a, int b, int c) {
-  if (atomicCAS(&h->status, 0, code) == 0) {
-    h->info[0] = a;
-    h->info[1] = b;
-    h->info[2] = c;
-  }
-}
 
 // Hardware base-2 exponential (MUFU.EX2); exp2(-inf) = 0.
 __device__ __forceinline__ float ex2(float x) {
@@ -108,7 +101,7 @@ __device__ __forceinline__ int64_t part_row(const PadVideoDesc& vd, int kvh, int
 // ---------------------------------------------------------------------------
 // a2: fused append.  One thread per 16-byte chunk of one (event, kv-head) row.
 // ---------------------------------------------------------------------------
-__global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
+__global__ void append_kernel(const __grid_constant__ KParams p, const uint4* __restrict__ k_new,
                               const uint4* __restrict__ v_new, uint4* __restrict__ k_pool,
                               uint4* __restrict__ v_pool) {
   // the shared-prefix pass launched after this kernel reads nothing it writes
@@ -121,7 +114,7 @@ __global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
   const int rem = idx - e * per_event;
   const int h = rem / chunks;
   const int c = rem - h * chunks;
-  const PadEventDesc ev = p.events[e];
+  const PadEventDesc ev = plan_events(p)[e];
   const int pidx = ev.len / p.page_size;
   const int slot = ev.len - pidx * p.page_size;
   int page;
@@ -132,7 +125,7 @@ __global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
     page = p.page_table[(size_t)e * p.max_pages + pidx];
   }
   if (page < 0 || page >= p.n_pages) {
-    set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pidx, page);
+    pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pidx, page);
     return;
   }
   const size_t dst = (((size_t)page * p.h_kv + h) * p.page_size + slot) * chunks + c;
@@ -147,7 +140,7 @@ __global__ void append_kernel(KParams p, const uint4* __restrict__ k_new,
 // head_dim slice for p.v; the 8 warps' states are merged through shared memory.
 // ---------------------------------------------------------------------------
 template <int D, int MAXR>
-__global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
+__global__ void __launch_bounds__(256) prefix_simt_kernel(const __grid_constant__ KParams p,
                                                           const __nv_bfloat16* __restrict__ q,
                                                           const __nv_bfloat16* __restrict__ kp,
                                                           const __nv_bfloat16* __restrict__ vp) {
@@ -159,7 +152,7 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
   __shared__ float sl[NW][MAXR];
   __shared__ float so[MAXR][D];
 
-  const PadWorkItem it = p.items[blockIdx.x];
+  const PadWorkItem it = plan_items(p)[blockIdx.x];
   const int R = it.n_events * p.group;
   const int kvh = it.kvh;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -294,7 +287,7 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(KParams p,
 // 4 warps x 16 query rows; 64-token K/V tiles double-buffered with cp.async.
 // ---------------------------------------------------------------------------
 template <int D>
-__global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
+__global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__ KParams p,
                                                          const __nv_bfloat16* __restrict__ q,
                                                          const __nv_bfloat16* __restrict__ kp,
                                                          const __nv_bfloat16* __restrict__ vp) {
@@ -307,7 +300,7 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(KParams p,
   __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw);
   __nv_bfloat16* sV = sK + 2 * TN * LDS;
 
-  const PadWorkItem it = p.items[blockIdx.x];
+  const PadWorkItem it = plan_items(p)[blockIdx.x];
   const int R = it.n_events * p.group;
   const int row0 = blockIdx.y * 64;
   if (row0 >= R) return;
@@ -500,7 +493,7 @@ struct BmSmem {
 };
 
 template <int D>
-__global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
+__global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_constant__ KParams p,
                                                                   const __nv_bfloat16* __restrict__ q,
                                                                   const __nv_bfloat16* __restrict__ kpool,
                                                                   const __nv_bfloat16* __restrict__ vpool,
@@ -522,8 +515,8 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
                                         bm_align16((size_t)G * sch * sizeof(float2)));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, t4 = lane & 3;
-  const PadEventDesc ev = p.events[e];
-  const PadVideoDesc vd = p.videos[ev.video];
+  const PadEventDesc ev = plan_events(p)[e];
+  const PadVideoDesc vd = plan_videos(p)[ev.video];
   const int R = vd.n_events * G;
   const int ns = vd.n_splits;
   const int rbase = ev.local * G;
@@ -558,7 +551,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
         const int pi = (c0 + tid) / ps;
         page = p.page_table[(size_t)e * p.max_pages + pi];
         if (page < 0 || page >= p.n_pages) {
-          set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
+          pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
           page = -1;
         }
       }
@@ -674,7 +667,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(KParams p,
   const int pi_new = len / ps;
   int page_new = ev.new_page >= 0 ? ev.new_page : p.page_table[(size_t)e * p.max_pages + pi_new];
   const bool new_ok = page_new >= 0 && page_new < p.n_pages;
-  if (!new_ok && tid == 0) set_error(p.header, PAD_ERR_DEVICE_BOUNDS, e, pi_new, page_new);
+  if (!new_ok && tid == 0) pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi_new, page_new);
   if (tid < 2 * CH) {
     const int c = tid % CH;
     const size_t off = (((size_t)(new_ok ? page_new : 0) * p.h_kv + kvh) * ps + (len % ps)) * D + c * 8;

@@ -93,6 +93,7 @@ struct TcBars {
   uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
   uint64_t tdone;             // the softmax warps are done with TMEM (8 warp arrivals)
   uint64_t xchg[4];           // the two softmax warps of a lane quarter met (64 thread arrivals)
+  uint64_t gen;               // the plan's generation, for the status word
   uint32_t tmem_base;
   int32_t abort;
 };
@@ -118,13 +119,6 @@ __device__ __forceinline__ unsigned long long globaltimer() {
   return t;
 }
 
-__device__ __forceinline__ void set_error(PadDevHeader* h, int code, int a, int b, int c) {
-  if (atomicCAS(&h->status, 0, code) == 0) {
-    h->info[0] = a;
-    h->info[1] = b;
-    h->info[2] = c;
-  }
-}
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -252,7 +246,7 @@ __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, TcBa
     if ((i & 63u) == 0) {
       if (*reinterpret_cast<volatile int32_t*>(&bars->abort)) return false;
       if (globaltimer() - t0 > kWaitNs) {
-        set_error(hdr, PAD_ERR_DEVICE_TIMEOUT, (int)blockIdx.x, where, (int)threadIdx.x);
+        pad_set_error(hdr, bars->gen, PAD_ERR_DEVICE_TIMEOUT, (int)blockIdx.x, where, (int)threadIdx.x);
         *reinterpret_cast<volatile int32_t*>(&bars->abort) = 1;
         return false;
       }
@@ -412,12 +406,12 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    prefix_tc_kernel(const KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
+    prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
   if (sbase & 1023u) {  // the 128-byte swizzle atoms need 1024-byte alignment (never expected)
-    if (threadIdx.x == 0) set_error(p.header, PAD_ERR_UNSUPPORTED, (int)blockIdx.x, (int)sbase, 0);
+    if (threadIdx.x == 0) pad_set_error(p.header, p.gen, PAD_ERR_UNSUPPORTED, (int)blockIdx.x, (int)sbase, 0);
     return;
   }
   TcBars* bars = reinterpret_cast<TcBars*>(smem + kOffBar);
@@ -425,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int item = blockIdx.x / n_groups;
   const int group = blockIdx.x - item * n_groups;
-  const PadWorkItem it = p.items[item];
+  const PadWorkItem it = plan_items(p)[item];
   const int R = it.n_events * p.group;
   const int row0 = group * 128;
   if (row0 >= R) return;  // uniform over the CTA, before any barrier or allocation
@@ -471,6 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bars->tdone, 8);
     for (int qq = 0; qq < 4; ++qq) mbar_init(&bars->xchg[qq], 64);
     bars->abort = 0;
+    bars->gen = p.gen;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     // The first kStages K and V tiles go out before TMEM allocation and the block
