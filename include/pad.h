@@ -171,6 +171,9 @@ typedef struct {
   int32_t n_new_pages;
   int64_t partial_rows;     /* rows of (m, l, O) partial softmax states in the workspace */
   int64_t workspace_bytes;  /* bytes of workspace this plan uses */
+  int32_t param_descriptor_bytes; /* bytes of descriptors carried in each launch's parameters;
+                                     0 = the kernels read them from the plan's page-locked image */
+  int32_t reserved;
 } pad_plan_info;
 pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info);
 pad_status pad_plan_destroy(pad_plan_t* plan);

@@ -41,7 +41,8 @@ class Problem(ctypes.Structure):
 class PlanInfo(ctypes.Structure):
     _fields_ = [("n_videos", c_int32), ("n_events", c_int32), ("n_work_items", c_int32),
                 ("split_len", c_int32), ("prefix_kernel", c_int32), ("n_new_pages", c_int32),
-                ("partial_rows", c_int64), ("workspace_bytes", c_int64)]
+                ("partial_rows", c_int64), ("workspace_bytes", c_int64),
+                ("param_descriptor_bytes", c_int32), ("reserved", c_int32)]
 
 
 _I32P = POINTER(c_int32)

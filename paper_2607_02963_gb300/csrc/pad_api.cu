@@ -618,6 +618,8 @@ pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
   info->n_new_pages = plan->n_new_pages;
   info->partial_rows = plan->lay.partial_rows;
   info->workspace_bytes = (int64_t)plan->lay.total_bytes;
+  info->param_descriptor_bytes = (int32_t)plan->param_image.size();
+  info->reserved = 0;
   return PAD_OK;
 }
 

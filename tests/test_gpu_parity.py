@@ -261,6 +261,55 @@ def test_repeated_steps_are_deterministic():
     assert torch.equal(o1, db.out)
 
 
+@pytest.mark.parametrize("D,h_q", [(64, 4), (128, 8)])
+def test_large_batch_reads_descriptors_from_host_image(D, h_q):
+    """A batch whose descriptors do not fit the launch parameters (500 events): the
+    kernels read them from the plan's page-locked image instead; results are the same,
+    also after more steps than the library cycles images through."""
+    rng = np.random.default_rng(11)
+    lens = [int(x) for x in rng.integers(0, 40, size=500)]
+    w = _w([96, 40, 0, 130, 64], [100] * 5, lens, seed=11, h_q=h_q, h_kv=2, D=D)
+    ev = [0, 99, 100, 250, 299, 300, 401, 499]
+    db, plan = run_sampled(w, ev)
+    assert plan.info()["param_descriptor_bytes"] == 0
+    o1 = db.out.clone()
+    for _ in range(12):  # more than the images kept in flight per device
+        db.release_new_pages()
+        db.run_step()
+    torch.cuda.synchronize()
+    B.pad_device_status(db.plan)
+    assert torch.equal(o1, db.out)
+
+
+def test_small_batch_carries_descriptors_in_parameters():
+    w = synth.tiny()
+    db = DeviceBatch(w)
+    plan = db.plan_step()
+    n = plan.info()["param_descriptor_bytes"]
+    assert 0 < n <= 8192
+    db.release_new_pages(plan)
+
+
+def test_status_word_reports_only_its_own_plan():
+    """The status word is not reset between steps: each plan's errors are tagged with its
+    generation, so a clean step on the same workspace after a failing one reports OK."""
+    w = _w([200], [2], [5, 3])
+    db = DeviceBatch(w)
+    good = int(db.page_table[1, 0])
+    db.page_table[1, 0] = w.n_pages + 5
+    bad = db.run_step()
+    with pytest.raises(B.PadError) as ei:
+        B.pad_device_status(bad)
+    assert ei.value.status == 7
+    db.release_new_pages(bad)
+    db.page_table[1, 0] = good
+    p2 = db.run_step()
+    B.pad_device_status(p2)
+    torch.cuda.synchronize()
+    ref_o, ref_lse = oracle.decode_step(w)
+    check_outputs(db.out.cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, "after a failed step")
+
+
 def test_device_bounds_check_reports_bad_page():
     """A page id outside the pool in the page table is caught by the kernels' own bounds
     checks (the access is skipped) and reported through the status word."""
