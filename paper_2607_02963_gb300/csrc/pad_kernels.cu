@@ -466,13 +466,16 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
 //   and processed as a small flash-attention on the warp-level MMA: the G <= 16 query
 //   rows form one m16 tile; S = Q K^T (warps split the keys), a row softmax (one warp
 //   per row), O += P V (warps split the head dimension).
-//   After the wait, key `len` (written by this step's append) and the prefix partials
-//   (m, l, O of the branch's G rows for up to `sch` splits) arrive in one round trip;
-//   the key is folded into the branch state in fp32 and then
-//   a5: the log-sum-exp merge of the branch state with the partials.
+//   After the wait, key `len` (written by this step's append) arrives with the prefix
+//   partials: one bulk copy per split brings the G contiguous fp32 O rows of this event
+//   into shared memory while the warps read the (m, l) pairs; the key is folded into the
+//   branch state in fp32 and then
+//   a5: the log-sum-exp merge of the branch state with the partials (Eq. for combining
+//   softmax states: M = max of the maxima, each state weighted by 2^(m_s - M)).
 // ---------------------------------------------------------------------------
 constexpr int kBmThreads = 256;
 constexpr int kBmKeys = 128;                  // branch keys per staged block
+constexpr unsigned long long kBmWaitNs = 1000000000ull;  // one second per bounded wait
 
 __host__ __device__ constexpr size_t bm_align16(size_t x) { return (x + 15) / 16 * 16; }
 
@@ -486,11 +489,35 @@ struct BmSmem {
   __nv_bfloat16 knew[D], vnew[D];             // key `len` of the branch
   int page[kBmKeys];
   float m[16], l[16], a[16], pn[16];
-  float M[16], L[16];
+  unsigned long long bar;                     // completion of a chunk's bulk copies
   // K and V rows of one block; once the branch pass is done the same bytes hold the
-  // staged prefix partials (float2 m,l per row and split, then fp32 O rows)
+  // staged fp32 O rows of the prefix partials, [split][row][d]
   alignas(16) __nv_bfloat16 kv[2][kBmKeys][LD];
 };
+
+__device__ __forceinline__ uint32_t bm_smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ unsigned long long bm_globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait for the phase of the given parity of the chunk barrier; false = gave up.
+__device__ __forceinline__ bool bm_wait(unsigned long long* bar, uint32_t parity) {
+  const unsigned long long t0 = bm_globaltimer();
+  for (;;) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bm_smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if (bm_globaltimer() - t0 > kBmWaitNs) return false;
+  }
+}
 
 template <int D>
 __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_constant__ KParams p,
@@ -506,13 +533,11 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
   BmSmem<D>& S = *reinterpret_cast<BmSmem<D>*>(bm_raw);
   auto sK = S.kv[0];
   auto sV = S.kv[1];
-  float2* sml = reinterpret_cast<float2*>(&S.kv[0][0][0]);
+  float* spo = reinterpret_cast<float*>(&S.kv[0][0][0]);
 
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
   const int G = p.group;
-  float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) +
-                                        bm_align16((size_t)G * sch * sizeof(float2)));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, t4 = lane & 3;
   const PadEventDesc ev = plan_events(p)[e];
@@ -522,7 +547,15 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
   const int rbase = ev.local * G;
   const int len = ev.len;                     // keys before this step; key `len` is this step's
   const int ps = p.page_size;
+  const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
 
+  // the first block's page ids go out together with the Q loads
+  int my_page = -1;
+  if (tid < kBmKeys && tid < len) my_page = ptab[tid / ps];
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bm_smem_u32(&S.bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
   for (int i = tid; i < 16 * CH; i += NT) {
     const int g = i / CH, c = i - (i / CH) * CH;
     uint4 v = make_uint4(0u, 0u, 0u, 0u);
@@ -546,10 +579,10 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
     const int nv = min(kBmKeys, len - c0);
     const int nv16 = (nv + 15) & ~15;         // keys padded to the MMA K step (zero rows)
     if (tid < kBmKeys) {
+      const int pi = (c0 + tid) / ps;
       int page = -1;
       if (tid < nv) {
-        const int pi = (c0 + tid) / ps;
-        page = p.page_table[(size_t)e * p.max_pages + pi];
+        page = c0 == 0 ? my_page : ptab[pi];
         if (page < 0 || page >= p.n_pages) {
           pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
           page = -1;
@@ -659,13 +692,34 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
       }
     }
   }
+  // the K/V block is reused for the partials below
+  __syncthreads();
 
   // ---------------- after the shared-prefix pass (and, through it, the append) completed
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
+  // one bulk copy per split of chunk [s0, s0 + nch): G rows x D fp32, contiguous
+  const uint32_t chunk_bytes_per_split = (uint32_t)(G * D * sizeof(float));
+  auto issue_chunk = [&](int s0, int nch) {
+    // the block's earlier reads of these bytes (generic proxy) before the copies' writes
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bm_smem_u32(&S.bar)),
+                 "r"(chunk_bytes_per_split * (uint32_t)nch)
+                 : "memory");
+    for (int sl = 0; sl < nch; ++sl) {
+      const float* src = p.part_o + part_row(vd, kvh, s0 + sl, R, rbase) * D;
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              bm_smem_u32(spo + (size_t)sl * G * D)),
+          "l"(src), "r"(chunk_bytes_per_split), "r"(bm_smem_u32(&S.bar))
+          : "memory");
+    }
+  };
+  if (tid == 0 && ns > 0) issue_chunk(0, min(sch, ns));
+
   // key `len`: its page is the one this step took, else the table's entry
   const int pi_new = len / ps;
-  int page_new = ev.new_page >= 0 ? ev.new_page : p.page_table[(size_t)e * p.max_pages + pi_new];
+  int page_new = ev.new_page >= 0 ? ev.new_page : ptab[pi_new];
   const bool new_ok = page_new >= 0 && page_new < p.n_pages;
   if (!new_ok && tid == 0) pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi_new, page_new);
   if (tid < 2 * CH) {
@@ -676,25 +730,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
     else
       cp_async16(&S.vnew[c * 8], vpool + off, new_ok);
   }
-  // stage the prefix partials of splits s0 .. s0+nch-1
-  auto stage_partials = [&](int s0, int nch) {
-    for (int i = tid; i < G * nch; i += NT) {
-      const int g = i / nch, sl = i - (i / nch) * nch;
-      sml[g * sch + sl] = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
-    }
-    constexpr int PC = D / 4;  // 16-byte pieces of one fp32 O row
-    for (int i = tid; i < G * nch * PC; i += NT) {
-      const int c = i % PC, rs = i / PC;
-      const int g = rs / nch, sl = rs - (rs / nch) * nch;
-      cp_async16(spo + ((size_t)g * sch + sl) * D + c * 4,
-                 p.part_o + part_row(vd, kvh, s0 + sl, R, rbase + g) * D + c * 4, true);
-    }
-    cp_async_commit();
-  };
-  if (ns > 0)
-    stage_partials(0, min(sch, ns));
-  else
-    cp_async_commit();
+  cp_async_commit();
   cp_async_wait<0>();
   __syncthreads();
 
@@ -725,66 +761,76 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
     const int g = i / D, d = i - g * D;
     S.ob[g][d] = fmaf(S.pn[g], __bfloat162float(S.vnew[d]), S.ob[g][d] * S.a[g]);
   }
-  if (tid < 16) S.M[tid] = S.m[tid];
   __syncthreads();
 
   // ---------------- a5: merge with the prefix partials, in chunks of `sch` splits
-  for (int s0 = 0; s0 < ns; s0 += sch) {
+  bool staged_ok = true;
+  for (int s0 = 0, chunk = 0; s0 < ns; s0 += sch, ++chunk) {
     const int nch = min(sch, ns - s0);
     if (s0 > 0) {
-      stage_partials(s0, nch);
-      cp_async_wait<0>();
-      __syncthreads();
+      if (tid == 0) issue_chunk(s0, nch);
     }
-    if (tid < G) {
-      const float oldM = S.M[tid];
-      float mm = oldM;
-      for (int sl = 0; sl < nch; ++sl) mm = fmaxf(mm, sml[tid * sch + sl].x);
-      float L = (s0 == 0 ? S.l[tid] : S.L[tid]) * ex2(oldM - mm);
-      for (int sl = 0; sl < nch; ++sl) {
-        const float2 ml = sml[tid * sch + sl];
-        L = fmaf(ml.y, ex2(ml.x - mm), L);
+    // row statistics, one warp per row, lanes over splits: M = max(m, m_s), the split
+    // weights 2^(m_s - M) (into sc) and L = l 2^(m - M) + sum_s l_s 2^(m_s - M)
+    for (int g = warp; g < G; g += NW) {
+      float mx = kNegInf;
+      for (int sl = lane; sl < nch; sl += 32) mx = fmaxf(mx, p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)].x);
+      mx = warp_max(mx);
+      const float mo = S.m[g];
+      const float mn = fmaxf(mo, mx);
+      float sum = 0.f;
+      for (int sl = lane; sl < nch; sl += 32) {
+        const float2 ml = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
+        const float wgt = ex2(ml.x - mn);
+        S.sc[g][sl] = wgt;
+        sum = fmaf(ml.y, wgt, sum);
       }
-      S.a[tid] = ex2(oldM - mm);
-      S.M[tid] = mm;
-      S.L[tid] = L;
+      sum = warp_sum(sum);
+      if (lane == 0) {
+        const float al = ex2(mo - mn);
+        S.a[g] = al;
+        S.l[g] = S.l[g] * al + sum;
+        S.m[g] = mn;
+      }
+    }
+    if (!bm_wait(&S.bar, (uint32_t)(chunk & 1))) {
+      staged_ok = false;
+      if (tid == 0) pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_TIMEOUT, e, -1, chunk);
     }
     __syncthreads();
-    // split weights 2^(m_s - M) of this chunk (sc is free here: nch <= kBmKeys)
-    for (int i = tid; i < G * nch; i += NT) {
-      const int g = i / nch, sl = i - (i / nch) * nch;
-      S.sc[g][sl] = ex2(sml[g * sch + sl].x - S.M[g]);
+    if (!__syncthreads_and(staged_ok)) {
+      // the copies must land before this CTA's shared memory is released
+      bm_wait(&S.bar, (uint32_t)(chunk & 1));
+      break;
     }
-    __syncthreads();
     for (int i = tid; i < G * D; i += NT) {
       const int g = i / D, d = i - g * D;
-      const float* src = spo + (size_t)g * sch * D + d;
+      const float* src = spo + (size_t)g * D + d;
+      const size_t step = (size_t)G * D;
       float a0 = S.ob[g][d] * S.a[g], a1 = 0.f, a2 = 0.f, a3 = 0.f;
       int sl = 0;
       for (; sl + 4 <= nch; sl += 4) {
-        a0 = fmaf(S.sc[g][sl], src[(size_t)sl * D], a0);
-        a1 = fmaf(S.sc[g][sl + 1], src[(size_t)(sl + 1) * D], a1);
-        a2 = fmaf(S.sc[g][sl + 2], src[(size_t)(sl + 2) * D], a2);
-        a3 = fmaf(S.sc[g][sl + 3], src[(size_t)(sl + 3) * D], a3);
+        a0 = fmaf(S.sc[g][sl], src[sl * step], a0);
+        a1 = fmaf(S.sc[g][sl + 1], src[(sl + 1) * step], a1);
+        a2 = fmaf(S.sc[g][sl + 2], src[(sl + 2) * step], a2);
+        a3 = fmaf(S.sc[g][sl + 3], src[(sl + 3) * step], a3);
       }
-      for (; sl < nch; ++sl) a0 = fmaf(S.sc[g][sl], src[(size_t)sl * D], a0);
+      for (; sl < nch; ++sl) a0 = fmaf(S.sc[g][sl], src[sl * step], a0);
       S.ob[g][d] = (a0 + a1) + (a2 + a3);
     }
     __syncthreads();
   }
-  if (ns == 0 && tid < G) S.L[tid] = S.l[tid];
-  __syncthreads();
 
   for (int i = tid; i < G * D; i += NT) {
     const int g = i / D, d = i - g * D;
     const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
-    const float res = S.ob[g][d] / S.L[g];
+    const float res = S.ob[g][d] / S.l[g];
     if (p.out_bf16)
       reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
     else
       reinterpret_cast<float*>(out)[oi] = res;
     if (lse != nullptr && d == 0)
-      lse[(size_t)e * p.h_q + kvh * G + g] = (S.M[g] + log2f(S.L[g])) * 0.69314718055994531f;
+      lse[(size_t)e * p.h_q + kvh * G + g] = (S.m[g] + log2f(S.l[g])) * 0.69314718055994531f;
   }
 }
 
@@ -855,14 +901,12 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
                              void* out, float* lse, bool pdl, cudaStream_t s) {
   const int G = p.group;
   // Staged prefix partials share the bytes of the branch K/V block: as many splits of a
-  // chunk as fit there.
+  // chunk as fit there ([split][row][d] fp32).
   constexpr size_t region = sizeof(BmSmem<D>::kv);
-  const size_t per_split = (size_t)G * (D * sizeof(float) + sizeof(float2));
-  int sch = (int)((region - 16) / per_split);
+  const size_t per_split = (size_t)G * D * sizeof(float);
+  int sch = (int)(region / per_split);
   if (p.max_splits > 0 && sch > p.max_splits) sch = p.max_splits;
   sch = sch < 1 ? 1 : (sch > kBmKeys ? kBmKeys : sch);
-  if (bm_align16((size_t)G * sch * sizeof(float2)) + (size_t)G * sch * D * sizeof(float) > region)
-    return cudaErrorInvalidValue;
   const size_t smem = sizeof(BmSmem<D>);
   constexpr int kMaxSmem = (int)sizeof(BmSmem<D>);
   static bool configured[64] = {};
