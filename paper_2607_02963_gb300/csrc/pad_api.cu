@@ -339,6 +339,7 @@ struct pad_plan_t {
   Layout lay;
   int32_t n_videos = 0, n_events = 0;
   int32_t max_pages = 0, n_pages = 0;
+  int32_t max_event_len = 0;        // longest branch (private tokens before this step)
   int32_t* page_table = nullptr;
   void* workspace = nullptr;
   int64_t total_prefix_tokens = 0;
@@ -592,6 +593,8 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   plan->prob = *prob;
   plan->n_videos = n_videos;
   plan->n_events = n_events;
+  plan->max_event_len = 0;
+  for (int e = 0; e < n_events; ++e) plan->max_event_len = std::max(plan->max_event_len, event_len[e]);
   plan->max_pages = max_pages;
   plan->n_pages = cache->n_pages;
   plan->page_table = page_table;
@@ -644,6 +647,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.n_sms = plan->lay.n_sms;
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
+  p.branch_rows = std::min(128, (plan->max_event_len + 1 + 15) / 16 * 16);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   p.gen = plan->gen;
   auto* ws = static_cast<uint8_t*>(plan->workspace);
@@ -866,6 +870,7 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.n_sms = plan->lay.n_sms;
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
+  p.branch_rows = std::min(128, (plan->max_event_len + 1 + 15) / 16 * 16);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   p.gen = plan->gen;
   p.img_n = 0;

@@ -94,6 +94,8 @@ struct KParams {
   int32_t out_bf16;
   int32_t n_sms;                  // SMs the grid sizes were planned for
   int32_t max_splits;             // largest per-video prefix split count of the batch
+  int32_t branch_rows;            // branch keys staged per round: the longest branch's
+                                  // len + 1 rounded up to 16, at most 128
   float scale_log2;               // scale * log2(e)
   uint64_t gen;                   // generation of the plan (tags errors in the status word)
   PadDevHeader* header;

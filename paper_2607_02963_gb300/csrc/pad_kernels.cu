@@ -8,6 +8,7 @@
 // Partial softmax states (m, l, O) keep m in log2 units of the scaled score:
 // m = max_k s_k * scale * log2(e), l = sum_k 2^(s_k*scale*log2(e) - m), O = sum_k 2^(...) v_k.
 #include <cuda_bf16.h>
+#include <cstddef>
 #include <cstdint>
 
 #include "pad_internal.h"
@@ -457,43 +458,54 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
 
 // ---------------------------------------------------------------------------
 // a4 + a5: one CTA (256 threads, 8 warps) per (event, kv-head).
-//   a4, the own-branch part of the mask of Sec. 3.4: the branch's len+1 keys.
-//   Keys 0..len-1 were appended by earlier steps and this step's append writes only
-//   key `len` (and, for a new page, the page-table entry of that key), so the pass over
-//   keys 0..len-1 reads nothing the grids launched before this one write: it runs
-//   before griddepcontrol.wait, overlapping the tail of the shared-prefix pass.  Those
-//   keys are staged in blocks of 128 (K and V rows through the page table, cp.async)
-//   and processed as a small flash-attention on the warp-level MMA: the G <= 16 query
-//   rows form one m16 tile; S = Q K^T (warps split the keys), a row softmax (one warp
-//   per row), O += P V (warps split the head dimension).
-//   After the wait, key `len` (written by this step's append) arrives with the prefix
-//   partials: one bulk copy per split brings the G contiguous fp32 O rows of this event
-//   into shared memory while the warps read the (m, l) pairs; the key is folded into the
-//   branch state in fp32 and then
-//   a5: the log-sum-exp merge of the branch state with the partials (Eq. for combining
-//   softmax states: M = max of the maxima, each state weighted by 2^(m_s - M)).
+//   a4, the own-branch part of the mask of Sec. 3.4: the branch's keys 0..len, its
+//   private tokens and the one appended at this step, staged in rounds of kBmKeys (K and
+//   V rows through the page table, cp.async); each warp takes 16 of a round's keys and
+//   keeps a flash-attention state held in registers in the manner of the warp-level MMA
+//   kernels (the G <= 16 query rows form one m16 tile, S = Q K^T, online softmax on the
+//   accumulators in base 2, O += P V with P re-packed from the S accumulators).
+//   a5: the eight warp states and the prefix splits' partial states are merged by
+//   log-sum-exp: M = max of the maxima, every state weighted by 2^(m - M).
+//   The CTA starts as the shared-prefix pass's CTAs retire.  Before griddepcontrol.wait it
+//   stages what the grids ahead do not write: Q rows, the branch's page ids and the K/V
+//   rows of its earlier keys.  After it, in one round trip: key `len` (written by this
+//   step's append), the splits' (m, l) pairs and (one bulk copy per split, on an
+//   mbarrier) their fp32 O rows.
 // ---------------------------------------------------------------------------
 constexpr int kBmThreads = 256;
-constexpr int kBmKeys = 128;                  // branch keys per staged block
+constexpr int kBmWarps = kBmThreads / 32;
+constexpr int kBmKeys = 16 * kBmWarps;        // branch keys staged per round
+constexpr int kBmMaxChunk = 64;               // prefix splits merged per staged chunk
 constexpr unsigned long long kBmWaitNs = 1000000000ull;  // one second per bounded wait
 
 __host__ __device__ constexpr size_t bm_align16(size_t x) { return (x + 15) / 16 * 16; }
 
+// Shared memory: this head, then three regions sized per launch (16-byte aligned):
+//   kv   K rows [nkr][LD] and V rows [nkr][LD] of a round (nkr = KParams::branch_rows);
+//        after the branch pass the warps' O rows, fp32 [warp][G][D]
+//   ml   the splits' (m, l) pairs of a chunk, [G][sch]
+//   po   the splits' O rows of a chunk, fp32 [sch][G][D]
 template <int D>
-struct BmSmem {
+struct BmHead {
   static constexpr int LD = D + 8;            // padded bf16 row: ldmatrix rows in distinct banks
   __nv_bfloat16 q[16][LD];
-  __nv_bfloat16 pb[16][kBmKeys + 8];          // P of the block (bf16, A operand of P.V)
-  float sc[16][kBmKeys];                      // scaled scores of the block; later split weights
-  float ob[16][D];                            // branch O, then the merged numerator
-  __nv_bfloat16 knew[D], vnew[D];             // key `len` of the branch
   int page[kBmKeys];
-  float m[16], l[16], a[16], pn[16];
+  float wm[kBmWarps][16], wl[kBmWarps][16];   // each warp's branch state per row
+  float sc[16][kBmMaxChunk];                  // state weights 2^(m - M)
+  float ob[16][D];                            // merged numerator
+  float M[16], L[16], a[16];
   unsigned long long bar;                     // completion of a chunk's bulk copies
-  // K and V rows of one block; once the branch pass is done the same bytes hold the
-  // staged fp32 O rows of the prefix partials, [split][row][d]
-  alignas(16) __nv_bfloat16 kv[2][kBmKeys][LD];
 };
+__host__ __device__ constexpr size_t bm_max(size_t a, size_t b) { return a > b ? a : b; }
+template <int D>
+__host__ __device__ constexpr size_t bm_kv_bytes(int nkr, int G) {
+  return bm_align16(bm_max((size_t)2 * nkr * BmHead<D>::LD * 2, (size_t)kBmWarps * G * D * 4));
+}
+template <int D>
+__host__ __device__ constexpr size_t bm_smem_bytes(int nkr, int G, int sch) {
+  return bm_align16(sizeof(BmHead<D>)) + bm_kv_bytes<D>(nkr, G) + bm_align16((size_t)G * sch * 8) +
+         (size_t)sch * G * D * 4;
+}
 
 __device__ __forceinline__ uint32_t bm_smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -518,6 +530,10 @@ __device__ __forceinline__ bool bm_wait(unsigned long long* bar, uint32_t parity
     if (bm_globaltimer() - t0 > kBmWaitNs) return false;
   }
 }
+__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
+  unsigned s = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(s), "l"(gmem));
+}
 
 template <int D>
 __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_constant__ KParams p,
@@ -527,17 +543,24 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
                                                                   void* __restrict__ out,
                                                                   float* __restrict__ lse,
                                                                   int sch) {
-  constexpr int NT = kBmThreads, NW = NT / 32;
+  constexpr int NT = kBmThreads;
   constexpr int CH = D / 8;                   // 16-byte pieces of a bf16 row
+  constexpr int KS = D / 16;                  // k-steps of S = Q K^T
+  constexpr int OT = D / 8;                   // n8 tiles of O
+  constexpr int LD = BmHead<D>::LD;
   extern __shared__ __align__(16) unsigned char bm_raw[];
-  BmSmem<D>& S = *reinterpret_cast<BmSmem<D>*>(bm_raw);
-  auto sK = S.kv[0];
-  auto sV = S.kv[1];
-  float* spo = reinterpret_cast<float*>(&S.kv[0][0][0]);
+  BmHead<D>& S = *reinterpret_cast<BmHead<D>*>(bm_raw);
+  const int G = p.group;
+  const int nkr = p.branch_rows;              // keys per round (multiple of 16, <= kBmKeys)
+  unsigned char* kv_raw = bm_raw + bm_align16(sizeof(BmHead<D>));
+  __nv_bfloat16 (*sK)[LD] = reinterpret_cast<__nv_bfloat16 (*)[LD]>(kv_raw);
+  __nv_bfloat16 (*sV)[LD] = reinterpret_cast<__nv_bfloat16 (*)[LD]>(kv_raw + (size_t)nkr * LD * 2);
+  float* wo = reinterpret_cast<float*>(kv_raw);  // [warp][G][d] after the branch pass
+  float2* sml = reinterpret_cast<float2*>(kv_raw + bm_kv_bytes<D>(nkr, G));
+  float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) + bm_align16((size_t)G * sch * 8));
 
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
-  const int G = p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, t4 = lane & 3;
   const PadEventDesc ev = plan_events(p)[e];
@@ -546,241 +569,244 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
   const int ns = vd.n_splits;
   const int rbase = ev.local * G;
   const int len = ev.len;                     // keys before this step; key `len` is this step's
+  const int nk = len + 1;
   const int ps = p.page_size;
   const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
 
-  // the first block's page ids go out together with the Q loads
-  int my_page = -1;
-  if (tid < kBmKeys && tid < len) my_page = ptab[tid / ps];
+  // page of key c0 + tid: the page this step took for key `len`, else the table's entry
+  // (written by an earlier step)
+  auto page_of = [&](int key) -> int {
+    const int pi = key / ps;
+    int page = (pi == len / ps && ev.new_page >= 0) ? ev.new_page : ptab[pi];
+    if (page < 0 || page >= p.n_pages) {
+      pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
+      page = -1;
+    }
+    return page;
+  };
+  // Before the wait: Q rows, the first round's page ids (key `len`'s page is the one this
+  // step took, else the table's entry of an earlier step) and its K/V rows except key
+  // `len`, which this step's append writes
+  const int nv0 = min(nkr, nk);
+  if (tid < nkr) S.page[tid] = tid < nv0 ? page_of(tid) : -1;
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bm_smem_u32(&S.bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   for (int i = tid; i < 16 * CH; i += NT) {
     const int g = i / CH, c = i - (i / CH) * CH;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (g < G) v = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)e * p.h_q + kvh * G + g) * D) + c);
-    *reinterpret_cast<uint4*>(&S.q[g][c * 8]) = v;
+    const bool in = g < G;
+    cp_async16(&S.q[g][c * 8], q + ((size_t)e * p.h_q + kvh * G + (in ? g : 0)) * D + c * 8, in);
   }
+  for (int i = tid; i < G * D; i += NT) S.ob[i / D][i % D] = 0.f;
   if (tid < 16) {
-    S.m[tid] = kNegInf;
-    S.l[tid] = 0.f;
+    S.M[tid] = kNegInf;
+    S.L[tid] = 0.f;
   }
-
-  // O of this warp: rows gq, gq+8 x head-dim columns of d-blocks (2 per warp for D=128)
-  constexpr int DB = D / 8 / NW > 0 ? D / 8 / NW : 1;   // d-blocks per warp (2 or 1)
-  float o[DB][4];
-#pragma unroll
-  for (int i = 0; i < DB; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  const int db0 = warp * DB;                  // first d-block of this warp (D=64: warps 0-7)
-
-  // ---------------- a4 over keys 0..len-1 (state of earlier steps only)
-  for (int c0 = 0; c0 < len; c0 += kBmKeys) {
-    const int nv = min(kBmKeys, len - c0);
-    const int nv16 = (nv + 15) & ~15;         // keys padded to the MMA K step (zero rows)
-    if (tid < kBmKeys) {
-      const int pi = (c0 + tid) / ps;
-      int page = -1;
-      if (tid < nv) {
-        page = c0 == 0 ? my_page : ptab[pi];
-        if (page < 0 || page >= p.n_pages) {
-          pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
-          page = -1;
-        }
-      }
-      S.page[tid] = page;
-    }
-    __syncthreads();
-    // K and V rows of the block (rows past nv or with a bad page: zeros)
-    for (int i = tid; i < nv16 * CH; i += NT) {
-      const int k = i / CH, c = i - (i / CH) * CH;
+  __syncthreads();
+  auto stage_keys = [&](int r0, int nv, int k_lo, int k_hi) {  // rows k_lo..k_hi-1 of the round
+    for (int i = tid; i < (k_hi - k_lo) * CH; i += NT) {
+      const int k = k_lo + i / CH, c = i - (i / CH) * CH;
       const int pg = k < nv ? S.page[k] : -1;
-      const bool ok = pg >= 0;
-      const size_t off = (((size_t)(ok ? pg : 0) * p.h_kv + kvh) * ps + ((c0 + k) % ps)) * D + c * 8;
-      cp_async16(&sK[k][c * 8], kpool + off, ok);
-      cp_async16(&sV[k][c * 8], vpool + off, ok);
+      const bool in = pg >= 0;
+      const size_t off = (((size_t)(in ? pg : 0) * p.h_kv + kvh) * ps + ((r0 + k) % ps)) * D + c * 8;
+      cp_async16(&sK[k][c * 8], kpool + off, in);
+      cp_async16(&sV[k][c * 8], vpool + off, in);
+    }
+  };
+  const int nv0_16 = (nv0 + 15) & ~15;
+  const bool len_in_first = len < nkr;
+  // rows 0..nv0_16-1 except key `len` (rows past nv0 are zero-filled)
+  if (len_in_first) {
+    stage_keys(0, nv0, 0, len);
+    stage_keys(0, nv0, len + 1, nv0_16);
+  } else {
+    stage_keys(0, nv0, 0, nv0_16);
+  }
+  cp_async_commit();
+
+  // ---------------- after the shared-prefix pass (and, through it, the append) completed
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (len_in_first) stage_keys(0, nv0, len, len + 1);
+
+  const uint32_t bytes_per_split = (uint32_t)(G * D * sizeof(float));
+  // the splits' O rows (bulk copies) and (m, l) pairs of chunk [s0, s0 + nch)
+  auto stage_chunk = [&](int s0, int nch) {
+    if (tid == 0) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bm_smem_u32(&S.bar)),
+                   "r"(bytes_per_split * (uint32_t)nch)
+                   : "memory");
+      for (int sl = 0; sl < nch; ++sl)
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                bm_smem_u32(spo + (size_t)sl * G * D)),
+            "l"(p.part_o + part_row(vd, kvh, s0 + sl, R, rbase) * D), "r"(bytes_per_split),
+            "r"(bm_smem_u32(&S.bar))
+            : "memory");
+    }
+    for (int i = tid; i < G * nch; i += NT) {
+      const int g = i / nch, sl = i - g * nch;
+      cp_async8(&sml[g * sch + sl], &p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)]);
+    }
+  };
+  if (ns > 0) stage_chunk(0, min(sch, ns));
+
+  // ---------------- a4: the branch pass
+  float o[OT][4];
+#pragma unroll
+  for (int i = 0; i < OT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m_lo = kNegInf, m_hi = kNegInf;       // rows gq, gq + 8 (log2 units)
+  float l_lo = 0.f, l_hi = 0.f;               // this lane's share of the row sums
+  uint32_t qa[KS][4];
+  const int kb0 = 16 * warp;                  // this warp's keys within a round
+  for (int r0 = 0; r0 < nk; r0 += nkr) {
+    const int nv = min(nkr, nk - r0);
+    if (r0 > 0) {
+      if (tid < nkr) S.page[tid] = tid < nv ? page_of(r0 + tid) : -1;
+      __syncthreads();
+      stage_keys(r0, nv, 0, (nv + 15) & ~15);
     }
     cp_async_commit();
     cp_async_wait<0>();
     __syncthreads();
-
-    // S = Q K^T: warp w takes 8-key blocks w, w+8, ...
-    for (int nb = warp; nb * 8 < nv16; nb += NW) {
-      float sacc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (r0 == 0) {
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        uint32_t a[4], b0, b1, b2, b3;
-        ldsm_x4(a[0], a[1], a[2], a[3], &S.q[(lane & 15)][kk * 16 + (lane >> 4) * 8]);
-        ldsm_x4(b0, b1, b2, b3, &sK[nb * 8 + (lane & 7)][kk * 16 + ((lane >> 3) & 1) * 8]);
-        (void)b2;
-        (void)b3;
-        mma_bf16(sacc, a, b0, b1);
-      }
-      const int col = nb * 8 + 2 * t4;
-      S.sc[gq][col] = sacc[0] * p.scale_log2;
-      S.sc[gq][col + 1] = sacc[1] * p.scale_log2;
-      S.sc[gq + 8][col] = sacc[2] * p.scale_log2;
-      S.sc[gq + 8][col + 1] = sacc[3] * p.scale_log2;
+      for (int kk = 0; kk < KS; ++kk)
+        ldsm_x4(qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], &S.q[lane & 15][kk * 16 + (lane >> 4) * 8]);
     }
-    __syncthreads();
-    // row softmax of the block: warp w takes rows w and w+8
-    for (int g = warp; g < 16; g += NW) {
-      if (g < G) {
-        float mx = kNegInf;
-        for (int k = lane; k < nv; k += 32)
-          if (S.page[k] >= 0) mx = fmaxf(mx, S.sc[g][k]);
-        mx = warp_max(mx);
-        const float mo = S.m[g];
-        float mn = fmaxf(mo, mx);
-        if (mn == kNegInf) mn = 0.f;  // only if every key so far failed its bounds check
-        float sum = 0.f;
-        for (int k = lane; k < nv16; k += 32) {
-          const float pr = (k < nv && S.page[k] >= 0) ? ex2(S.sc[g][k] - mn) : 0.f;
-          sum += pr;
-          S.pb[g][k] = __float2bfloat16_rn(pr);
-        }
-        sum = warp_sum(sum);
-        if (lane == 0) {
-          const float al = ex2(mo - mn);
-          S.a[g] = al;
-          S.l[g] = S.l[g] * al + sum;
-          S.m[g] = mn;
-        }
-      } else {
-        for (int k = lane; k < nv16; k += 32) S.pb[g][k] = __float2bfloat16_rn(0.f);
-        if (lane == 0) S.a[g] = 1.f;
-      }
-    }
-    __syncthreads();
-    // O = O * alpha + P V: warp w owns d-blocks db0 .. db0+DB-1
-    if (db0 < D / 8) {
-      const float al_lo = S.a[gq], al_hi = S.a[gq + 8];
+    if (kb0 < nv) {
+      float s[2][4];
 #pragma unroll
-      for (int i = 0; i < DB; ++i) {
+      for (int nt = 0; nt < 2; ++nt) {
+        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < KS; kk += 2) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(b0, b1, b2, b3, &sK[kb0 + nt * 8 + (lane & 7)][kk * 16 + (lane >> 3) * 8]);
+          mma_bf16(s[nt], qa[kk], b0, b1);
+          mma_bf16(s[nt], qa[kk + 1], b2, b3);
+        }
+      }
+      float mx_lo = kNegInf, mx_hi = kNegInf;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const int k = kb0 + nt * 8 + 2 * t4 + j;
+          const bool in = k < nv && S.page[k] >= 0;
+          s[nt][j] = in ? s[nt][j] * p.scale_log2 : kNegInf;
+          s[nt][2 + j] = in ? s[nt][2 + j] * p.scale_log2 : kNegInf;
+          mx_lo = fmaxf(mx_lo, s[nt][j]);
+          mx_hi = fmaxf(mx_hi, s[nt][2 + j]);
+        }
+      }
+      mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, 1));
+      mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, 2));
+      mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 1));
+      mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 2));
+      float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);
+      if (mn_lo == kNegInf) mn_lo = 0.f;  // only while every key so far failed its bounds check
+      if (mn_hi == kNegInf) mn_hi = 0.f;
+      const float al_lo = ex2(m_lo - mn_lo), al_hi = ex2(m_hi - mn_hi);
+      m_lo = mn_lo;
+      m_hi = mn_hi;
+      float pr[2][4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) pr[h][j] = ex2(s[h][j] - (j < 2 ? mn_lo : mn_hi));
+      l_lo = l_lo * al_lo + (pr[0][0] + pr[0][1]) + (pr[1][0] + pr[1][1]);
+      l_hi = l_hi * al_hi + (pr[0][2] + pr[0][3]) + (pr[1][2] + pr[1][3]);
+      uint32_t a[4];
+      a[0] = pack_bf16(pr[0][0], pr[0][1]);
+      a[1] = pack_bf16(pr[0][2], pr[0][3]);
+      a[2] = pack_bf16(pr[1][0], pr[1][1]);
+      a[3] = pack_bf16(pr[1][2], pr[1][3]);
+#pragma unroll
+      for (int i = 0; i < OT; i += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(b0, b1, b2, b3, &sV[kb0 + (lane & 15)][(i + (lane >> 4)) * 8]);
         o[i][0] *= al_lo;
         o[i][1] *= al_lo;
         o[i][2] *= al_hi;
         o[i][3] *= al_hi;
-      }
-      for (int ks = 0; ks * 16 < nv16; ++ks) {
-        uint32_t a[4];
-        ldsm_x4(a[0], a[1], a[2], a[3], &S.pb[(lane & 15)][ks * 16 + (lane >> 4) * 8]);
-#pragma unroll
-        for (int i = 0; i < DB; ++i) {
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(b0, b1, b2, b3, &sV[ks * 16 + ((lane >> 3) & 1) * 8 + (lane & 7)][(db0 + i) * 8]);
-          (void)b2;
-          (void)b3;
-          mma_bf16(o[i], a, b0, b1);
-        }
+        o[i + 1][0] *= al_lo;
+        o[i + 1][1] *= al_lo;
+        o[i + 1][2] *= al_hi;
+        o[i + 1][3] *= al_hi;
+        mma_bf16(o[i], a, b0, b1);
+        mma_bf16(o[i + 1], a, b2, b3);
       }
     }
-    __syncthreads();
+    __syncthreads();                          // the next round (or the O rows below) overwrite k / v
   }
-  // branch O so far to shared memory (rows < G)
-  if (db0 < D / 8) {
+  l_lo += __shfl_xor_sync(0xffffffffu, l_lo, 1);
+  l_lo += __shfl_xor_sync(0xffffffffu, l_lo, 2);
+  l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 1);
+  l_hi += __shfl_xor_sync(0xffffffffu, l_hi, 2);
+  // this warp's state: (m, l) per row and its O rows
+  if (t4 == 0) {
+    S.wm[warp][gq] = m_lo;
+    S.wl[warp][gq] = l_lo;
+    S.wm[warp][gq + 8] = m_hi;
+    S.wl[warp][gq + 8] = l_hi;
+  }
+  if (gq < G) {
+    float* dst = wo + ((size_t)warp * G + gq) * D;
 #pragma unroll
-    for (int i = 0; i < DB; ++i) {
-      const int d = (db0 + i) * 8 + 2 * t4;
-      if (gq < G) {
-        S.ob[gq][d] = o[i][0];
-        S.ob[gq][d + 1] = o[i][1];
-      }
-      if (gq + 8 < G) {
-        S.ob[gq + 8][d] = o[i][2];
-        S.ob[gq + 8][d + 1] = o[i][3];
-      }
-    }
+    for (int i = 0; i < OT; ++i) *reinterpret_cast<float2*>(dst + i * 8 + 2 * t4) = make_float2(o[i][0], o[i][1]);
   }
-  // the K/V block is reused for the partials below
+  if (gq + 8 < G) {
+    float* dst = wo + ((size_t)warp * G + gq + 8) * D;
+#pragma unroll
+    for (int i = 0; i < OT; ++i) *reinterpret_cast<float2*>(dst + i * 8 + 2 * t4) = make_float2(o[i][2], o[i][3]);
+  }
   __syncthreads();
 
-  // ---------------- after the shared-prefix pass (and, through it, the append) completed
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-
-  // one bulk copy per split of chunk [s0, s0 + nch): G rows x D fp32, contiguous
-  const uint32_t chunk_bytes_per_split = (uint32_t)(G * D * sizeof(float));
-  auto issue_chunk = [&](int s0, int nch) {
-    // the block's earlier reads of these bytes (generic proxy) before the copies' writes
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bm_smem_u32(&S.bar)),
-                 "r"(chunk_bytes_per_split * (uint32_t)nch)
-                 : "memory");
-    for (int sl = 0; sl < nch; ++sl) {
-      const float* src = p.part_o + part_row(vd, kvh, s0 + sl, R, rbase) * D;
-      asm volatile(
-          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-              bm_smem_u32(spo + (size_t)sl * G * D)),
-          "l"(src), "r"(chunk_bytes_per_split), "r"(bm_smem_u32(&S.bar))
-          : "memory");
-    }
-  };
-  if (tid == 0 && ns > 0) issue_chunk(0, min(sch, ns));
-
-  // key `len`: its page is the one this step took, else the table's entry
-  const int pi_new = len / ps;
-  int page_new = ev.new_page >= 0 ? ev.new_page : ptab[pi_new];
-  const bool new_ok = page_new >= 0 && page_new < p.n_pages;
-  if (!new_ok && tid == 0) pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi_new, page_new);
-  if (tid < 2 * CH) {
-    const int c = tid % CH;
-    const size_t off = (((size_t)(new_ok ? page_new : 0) * p.h_kv + kvh) * ps + (len % ps)) * D + c * 8;
-    if (tid < CH)
-      cp_async16(&S.knew[c * 8], kpool + off, new_ok);
-    else
-      cp_async16(&S.vnew[c * 8], vpool + off, new_ok);
-  }
-  cp_async_commit();
-  cp_async_wait<0>();
-  __syncthreads();
-
-  // fold key `len` into the branch state (fp32): warp w takes rows w and w+8
-  for (int g = warp; g < 16; g += NW) {
-    if (g < G && new_ok) {
-      float dot = 0.f;
-      for (int d = lane; d < D; d += 32)
-        dot = fmaf(__bfloat162float(S.q[g][d]), __bfloat162float(S.knew[d]), dot);
-      const float s = warp_sum(dot) * p.scale_log2;
-      if (lane == 0) {
-        const float mo = S.m[g];
-        const float mn = fmaxf(mo, s);
-        const float al = ex2(mo - mn);
-        const float pnew = ex2(s - mn);
-        S.a[g] = al;
-        S.pn[g] = pnew;
-        S.l[g] = S.l[g] * al + pnew;
-        S.m[g] = mn;
-      }
-    } else if (lane == 0) {
-      S.a[g] = 1.f;
-      S.pn[g] = 0.f;
+  // ---------------- a5: the warp states, then the prefix splits in chunks of `sch`
+  // (M, L, numerator) = log-sum-exp merge of the warps' states: one warp per row
+  for (int g = warp; g < G; g += kBmWarps) {
+    const float mw = lane < kBmWarps ? S.wm[lane][g] : kNegInf;
+    float mx = warp_max(mw);
+    if (mx == kNegInf) mx = 0.f;              // no key of the branch passed its bounds check
+    const float wgt = lane < kBmWarps ? ex2(mw - mx) : 0.f;
+    const float sum = warp_sum(lane < kBmWarps ? S.wl[lane][g] * wgt : 0.f);
+    if (lane < kBmWarps) S.sc[g][lane] = wgt;
+    if (lane == 0) {
+      S.M[g] = mx;
+      S.L[g] = sum;
     }
   }
   __syncthreads();
   for (int i = tid; i < G * D; i += NT) {
     const int g = i / D, d = i - g * D;
-    S.ob[g][d] = fmaf(S.pn[g], __bfloat162float(S.vnew[d]), S.ob[g][d] * S.a[g]);
+    float acc = 0.f;
+#pragma unroll
+    for (int w = 0; w < kBmWarps; ++w) acc = fmaf(S.sc[g][w], wo[((size_t)w * G + g) * D + d], acc);
+    S.ob[g][d] = acc;
   }
-  __syncthreads();
 
-  // ---------------- a5: merge with the prefix partials, in chunks of `sch` splits
   bool staged_ok = true;
   for (int s0 = 0, chunk = 0; s0 < ns; s0 += sch, ++chunk) {
     const int nch = min(sch, ns - s0);
     if (s0 > 0) {
-      if (tid == 0) issue_chunk(s0, nch);
+      __syncthreads();                        // the previous chunk's rows are consumed
+      stage_chunk(s0, nch);
     }
-    // row statistics, one warp per row, lanes over splits: M = max(m, m_s), the split
-    // weights 2^(m_s - M) (into sc) and L = l 2^(m - M) + sum_s l_s 2^(m_s - M)
-    for (int g = warp; g < G; g += NW) {
+    cp_async_commit();
+    cp_async_wait<0>();                       // the (m, l) pairs
+    __syncthreads();
+    // row statistics, one warp per row, lanes over splits
+    for (int g = warp; g < G; g += kBmWarps) {
       float mx = kNegInf;
-      for (int sl = lane; sl < nch; sl += 32) mx = fmaxf(mx, p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)].x);
+      for (int sl = lane; sl < nch; sl += 32) mx = fmaxf(mx, sml[g * sch + sl].x);
       mx = warp_max(mx);
-      const float mo = S.m[g];
+      const float mo = S.M[g];
       const float mn = fmaxf(mo, mx);
       float sum = 0.f;
       for (int sl = lane; sl < nch; sl += 32) {
-        const float2 ml = p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)];
+        const float2 ml = sml[g * sch + sl];
         const float wgt = ex2(ml.x - mn);
         S.sc[g][sl] = wgt;
         sum = fmaf(ml.y, wgt, sum);
@@ -789,15 +815,14 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
       if (lane == 0) {
         const float al = ex2(mo - mn);
         S.a[g] = al;
-        S.l[g] = S.l[g] * al + sum;
-        S.m[g] = mn;
+        S.L[g] = S.L[g] * al + sum;
+        S.M[g] = mn;
       }
     }
     if (!bm_wait(&S.bar, (uint32_t)(chunk & 1))) {
       staged_ok = false;
       if (tid == 0) pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_TIMEOUT, e, -1, chunk);
     }
-    __syncthreads();
     if (!__syncthreads_and(staged_ok)) {
       // the copies must land before this CTA's shared memory is released
       bm_wait(&S.bar, (uint32_t)(chunk & 1));
@@ -818,19 +843,19 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
       for (; sl < nch; ++sl) a0 = fmaf(S.sc[g][sl], src[sl * step], a0);
       S.ob[g][d] = (a0 + a1) + (a2 + a3);
     }
-    __syncthreads();
   }
+  __syncthreads();
 
   for (int i = tid; i < G * D; i += NT) {
     const int g = i / D, d = i - g * D;
     const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
-    const float res = S.ob[g][d] / S.l[g];
+    const float res = S.ob[g][d] / S.L[g];
     if (p.out_bf16)
       reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
     else
       reinterpret_cast<float*>(out)[oi] = res;
     if (lse != nullptr && d == 0)
-      lse[(size_t)e * p.h_q + kvh * G + g] = (S.m[g] + log2f(S.l[g])) * 0.69314718055994531f;
+      lse[(size_t)e * p.h_q + kvh * G + g] = (S.M[g] + log2f(S.L[g])) * 0.69314718055994531f;
   }
 }
 
@@ -900,15 +925,20 @@ template <int D>
 static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
                              void* out, float* lse, bool pdl, cudaStream_t s) {
   const int G = p.group;
-  // Staged prefix partials share the bytes of the branch K/V block: as many splits of a
-  // chunk as fit there ([split][row][d] fp32).
-  constexpr size_t region = sizeof(BmSmem<D>::kv);
-  const size_t per_split = (size_t)G * D * sizeof(float);
-  int sch = (int)(region / per_split);
+  const int nkr = p.branch_rows;
+  if (nkr <= 0 || nkr > kBmKeys || nkr % 16 != 0) return cudaErrorInvalidValue;
+  // Staged prefix partials: as many splits per chunk as a budget allows; a grid larger than
+  // one wave keeps two CTAs per SM.
+  const int n_cta = p.n_events * p.h_kv;
+  const size_t budget = n_cta > p.n_sms ? 110 * 1024 : 200 * 1024;
+  const size_t fixed = bm_align16(sizeof(BmHead<D>)) + bm_kv_bytes<D>(nkr, G) + 16;
+  const size_t per_split = (size_t)G * D * sizeof(float) + sizeof(float2);
+  int sch = fixed + per_split <= budget ? (int)((budget - fixed) / per_split) : 1;
   if (p.max_splits > 0 && sch > p.max_splits) sch = p.max_splits;
-  sch = sch < 1 ? 1 : (sch > kBmKeys ? kBmKeys : sch);
-  const size_t smem = sizeof(BmSmem<D>);
-  constexpr int kMaxSmem = (int)sizeof(BmSmem<D>);
+  sch = sch < 1 ? 1 : (sch > kBmMaxChunk ? kBmMaxChunk : sch);
+  const size_t smem = bm_smem_bytes<D>(nkr, G, sch);
+  constexpr int kMaxSmem = 227 * 1024;
+  if (smem > (size_t)kMaxSmem) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
