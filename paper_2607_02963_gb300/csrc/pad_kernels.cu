@@ -492,7 +492,7 @@ struct BmHead {
   int page[kBmKeys];
   float wm[kBmWarps][16], wl[kBmWarps][16];   // each warp's branch state per row
   float sc[16][kBmMaxChunk];                  // state weights 2^(m - M)
-  float ob[16][D];                            // merged numerator
+  alignas(16) float ob[16][D];                // merged numerator (read as float4)
   float M[16], L[16], a[16];
   unsigned long long bar;                     // completion of a chunk's bulk copies
 };
@@ -628,11 +628,12 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
   // ---------------- after the shared-prefix pass (and, through it, the append) completed
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (len_in_first) stage_keys(0, nv0, len, len + 1);
+  cp_async_commit();                          // this round's keys
 
   const uint32_t bytes_per_split = (uint32_t)(G * D * sizeof(float));
   // the splits' O rows (bulk copies) and (m, l) pairs of chunk [s0, s0 + nch)
   auto stage_chunk = [&](int s0, int nch) {
-    if (tid == 0) {
+    if (tid == NT - 1) {
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bm_smem_u32(&S.bar)),
                    "r"(bytes_per_split * (uint32_t)nch)
@@ -651,6 +652,7 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
     }
   };
   if (ns > 0) stage_chunk(0, min(sch, ns));
+  cp_async_commit();                          // the first chunk's (m, l) pairs, waited for in a5
 
   // ---------------- a4: the branch pass
   float o[OT][4];
@@ -666,9 +668,11 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
       if (tid < nkr) S.page[tid] = tid < nv ? page_of(r0 + tid) : -1;
       __syncthreads();
       stage_keys(r0, nv, 0, (nv + 15) & ~15);
+      cp_async_commit();
+      cp_async_wait<0>();
+    } else {
+      cp_async_wait<1>();                     // all but the (m, l) group
     }
-    cp_async_commit();
-    cp_async_wait<0>();
     __syncthreads();
     if (r0 == 0) {
 #pragma unroll
@@ -779,12 +783,20 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
     }
   }
   __syncthreads();
-  for (int i = tid; i < G * D; i += NT) {
-    const int g = i / D, d = i - g * D;
-    float acc = 0.f;
+  constexpr int D4 = D / 4;
+  for (int i = tid; i < G * D4; i += NT) {
+    const int g = i / D4, d4 = i - g * D4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int w = 0; w < kBmWarps; ++w) acc = fmaf(S.sc[g][w], wo[((size_t)w * G + g) * D + d], acc);
-    S.ob[g][d] = acc;
+    for (int w = 0; w < kBmWarps; ++w) {
+      const float c = S.sc[g][w];
+      const float4 v = reinterpret_cast<const float4*>(wo)[(w * G + g) * D4 + d4];
+      acc.x = fmaf(c, v.x, acc.x);
+      acc.y = fmaf(c, v.y, acc.y);
+      acc.z = fmaf(c, v.z, acc.z);
+      acc.w = fmaf(c, v.w, acc.w);
+    }
+    reinterpret_cast<float4*>(&S.ob[g][0])[d4] = acc;
   }
 
   bool staged_ok = true;
@@ -828,33 +840,45 @@ __global__ void __launch_bounds__(kBmThreads) branch_merge_kernel(const __grid_c
       bm_wait(&S.bar, (uint32_t)(chunk & 1));
       break;
     }
-    for (int i = tid; i < G * D; i += NT) {
-      const int g = i / D, d = i - g * D;
-      const float* src = spo + (size_t)g * D + d;
-      const size_t step = (size_t)G * D;
-      float a0 = S.ob[g][d] * S.a[g], a1 = 0.f, a2 = 0.f, a3 = 0.f;
-      int sl = 0;
-      for (; sl + 4 <= nch; sl += 4) {
-        a0 = fmaf(S.sc[g][sl], src[sl * step], a0);
-        a1 = fmaf(S.sc[g][sl + 1], src[(sl + 1) * step], a1);
-        a2 = fmaf(S.sc[g][sl + 2], src[(sl + 2) * step], a2);
-        a3 = fmaf(S.sc[g][sl + 3], src[(sl + 3) * step], a3);
+    for (int i = tid; i < G * D4; i += NT) {
+      const int g = i / D4, d4 = i - g * D4;
+      const float4* src = reinterpret_cast<const float4*>(spo) + g * D4 + d4;
+      const int step = G * D4;
+      const float al = S.a[g];
+      float4 acc = reinterpret_cast<const float4*>(&S.ob[g][0])[d4];
+      acc.x *= al;
+      acc.y *= al;
+      acc.z *= al;
+      acc.w *= al;
+#pragma unroll 4
+      for (int sl = 0; sl < nch; ++sl) {
+        const float c = S.sc[g][sl];
+        const float4 v = src[sl * step];
+        acc.x = fmaf(c, v.x, acc.x);
+        acc.y = fmaf(c, v.y, acc.y);
+        acc.z = fmaf(c, v.z, acc.z);
+        acc.w = fmaf(c, v.w, acc.w);
       }
-      for (; sl < nch; ++sl) a0 = fmaf(S.sc[g][sl], src[sl * step], a0);
-      S.ob[g][d] = (a0 + a1) + (a2 + a3);
+      reinterpret_cast<float4*>(&S.ob[g][0])[d4] = acc;
     }
   }
   __syncthreads();
 
-  for (int i = tid; i < G * D; i += NT) {
-    const int g = i / D, d = i - g * D;
-    const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + d;
-    const float res = S.ob[g][d] / S.L[g];
+  for (int i = tid; i < G * D4; i += NT) {
+    const int g = i / D4, d4 = i - g * D4;
+    const float inv = 1.0f / S.L[g];
+    float4 v = reinterpret_cast<const float4*>(&S.ob[g][0])[d4];
+    v.x *= inv;
+    v.y *= inv;
+    v.z *= inv;
+    v.w *= inv;
+    const size_t oi = ((size_t)e * p.h_q + kvh * G + g) * D + 4 * d4;
     if (p.out_bf16)
-      reinterpret_cast<__nv_bfloat16*>(out)[oi] = __float2bfloat16_rn(res);
+      *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(out) + oi) =
+          make_uint2(pack_bf16(v.x, v.y), pack_bf16(v.z, v.w));
     else
-      reinterpret_cast<float*>(out)[oi] = res;
-    if (lse != nullptr && d == 0)
+      *reinterpret_cast<float4*>(reinterpret_cast<float*>(out) + oi) = v;
+    if (lse != nullptr && d4 == 0)
       lse[(size_t)e * p.h_q + kvh * G + g] = (S.M[g] + log2f(S.L[g])) * 0.69314718055994531f;
   }
 }
