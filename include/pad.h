@@ -161,6 +161,11 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
  * keeps writing into its current page.  new_page has n_events entries (host). */
 pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page);
 
+/* Give the pages this plan took back to `cache` (host bookkeeping only; the device page
+ * table keeps its entries).  For a step that is re-run with the same lengths, such as a
+ * timing loop, or a step that is abandoned.  PAD_ERR_INVALID_ARG if a page is not in use. */
+pad_status pad_plan_release_new_pages(const pad_plan_t* plan, pad_cache_state* cache);
+
 /* Summary of a plan (host): the split-KV decomposition chosen for the prefix pass. */
 typedef struct {
   int32_t n_videos;

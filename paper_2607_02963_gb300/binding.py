@@ -63,6 +63,7 @@ _SIGNATURES = {
                            _I32P, c_void_p, c_int32, c_void_p, c_size_t, c_void_p,
                            POINTER(c_void_p)]),
     "pad_plan_new_pages": (c_int32, [c_void_p, _I32P]),
+    "pad_plan_release_new_pages": (c_int32, [c_void_p, c_void_p]),
     "pad_plan_get_info": (c_int32, [c_void_p, POINTER(PlanInfo)]),
     "pad_plan_destroy": (c_int32, [c_void_p]),
     "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -197,6 +198,10 @@ class Plan:
         _check(lib().pad_plan_new_pages(self._h, out.ctypes.data_as(_I32P)))
         return out
 
+    def release_new_pages(self, cache: "CacheState"):
+        """Give the pages this plan took back to ``cache`` (pad_plan_release_new_pages)."""
+        _check(lib().pad_plan_release_new_pages(self._h, cache.handle))
+
     def info(self) -> dict:
         i = PlanInfo()
         _check(lib().pad_plan_get_info(self._h, ctypes.byref(i)))
@@ -326,11 +331,6 @@ class StepLauncher:
             _check(L.pad_kv_append(h, *self.args_append))
             _check(L.pad_event_decode_attn(h, *self.args_attn))
             if self.release:
-                L.pad_plan_new_pages(h, self.newpp)
-                sel = self.newp[self.newp >= 0]
-                if sel.size:
-                    _check(L.pad_cache_state_release(self.cache.handle,
-                                                     np.ascontiguousarray(sel).ctypes.data_as(_I32P),
-                                                     int(sel.size)))
+                _check(L.pad_plan_release_new_pages(h, self.cache.handle))
         finally:
             L.pad_plan_destroy(h)

@@ -611,6 +611,14 @@ pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page) {
   return PAD_OK;
 }
 
+pad_status pad_plan_release_new_pages(const pad_plan_t* plan, pad_cache_state* cache) {
+  if (!plan || !cache) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  std::vector<int32_t> pages;
+  for (int32_t pg : plan->new_pages)
+    if (pg >= 0) pages.push_back(pg);
+  return pages.empty() ? PAD_OK : set_pages(cache, pages.data(), (int32_t)pages.size(), false);
+}
+
 pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
   if (!plan || !info) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
   info->n_videos = plan->n_videos;

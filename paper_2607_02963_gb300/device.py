@@ -69,11 +69,7 @@ class DeviceBatch:
 
     def release_new_pages(self, plan=None):
         """Return the pages the last plan took (keeps repeated steps idempotent)."""
-        plan = plan or self.plan
-        np_ = plan.new_pages()
-        np_ = np_[np_ >= 0]
-        if np_.size:
-            self.cache.release(np_)
+        (plan or self.plan).release_new_pages(self.cache)
 
     def gather_branch(self, e: int, n_tokens: int):
         """Read branch e's first n_tokens K/V rows back through the device page table."""

@@ -194,3 +194,22 @@ def test_launch_calls_reject_plans_without_workspace(padlib):
         B.lib().pad_kv_append(plan.handle, None, None, None, None, None) and None
         B._check(B.lib().pad_kv_append(plan.handle, None, None, None, None, None))
     assert ei.value.status == 1
+
+
+def test_release_new_pages_returns_exactly_the_plans_pages(padlib):
+    """pad_plan_release_new_pages frees the pages the plan took and nothing else; releasing
+    twice is an error that changes nothing."""
+    cache = B.CacheState(40, used_pages=[0, 1, 2, 5])
+    prob = B.make_problem(4, 1, 64, page_size=16)
+    lens = np.array([16, 3, 32, 0], dtype=np.int32)  # three page starts
+    plan = B.pad_plan(prob, cache, [100], [0, 0, 0, 0], lens, max_pages=4, workspace=None)
+    new = plan.new_pages()
+    assert sorted(new[new >= 0].tolist()) == [3, 4, 6]
+    free_before = cache.free_count
+    plan.release_new_pages(cache)
+    assert cache.free_count == free_before + 3
+    assert sorted(cache.free_pages().tolist()) == [p for p in range(40) if p not in (0, 1, 2, 5)]
+    with pytest.raises(B.PadError) as ei:
+        plan.release_new_pages(cache)
+    assert ei.value.status == 1
+    assert cache.free_count == free_before + 3
