@@ -1,8 +1,8 @@
 #!/usr/bin/env python3
 """Throughput of one event-factorized parallel decode step (one attention layer) on GB300.
 
-A step is the whole hot path: pad_plan (host work list + page allocation, uploaded
-asynchronously), pad_kv_append (each branch's new K/V into its page) and
+A step is the whole hot path: pad_plan (host work list + page allocation, carried
+in the launch parameters), pad_kv_append (each branch's new K/V into its page) and
 pad_event_decode_attn (shared-prefix split-KV pass, private-suffix pass and
 log-sum-exp merge).  The default workload is the long-video case: batch 1,
 H_q=28, H_kv=4, head_dim 128, shared prefix 32768 tokens, 32 events with private
@@ -26,6 +26,11 @@ the events of all ranks divided by the slowest rank's time.
 
 --impl reference times the fp64 oracle (the only other implementation) on the
 host cores with the same metric; each step is a bounded sample of the workload.
+
+--sweep prints one JSON line per event count E of the sweep workload (prefix 16384,
+L = 48): our step's time and HBM rate, and a naive comparator that re-reads the shared
+prefix once per event (one scaled_dot_product_attention call per event over that event's
+own [prefix ; branch] keys, a library kernel used only as a baseline here).
 """
 from __future__ import annotations
 
@@ -537,6 +542,86 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """Per E: our step (cold replicas, back to back) and the naive per-event comparator."""
+    import torch
+    import torch.nn.functional as F
+    from paper_2607_02963_gb300 import binding as B
+    from paper_2607_02963_gb300 import build as pad_build
+    from paper_2607_02963_gb300.device import DeviceBatch
+
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    pad_build.build()
+    B.lib()
+    stream = torch.cuda.current_stream(device)
+    l2 = int(getattr(torch.cuda.get_device_properties(device), "L2_cache_size", 0) or (126 << 20))
+    flush = torch.empty(3 * l2, dtype=torch.uint8, device=device)
+    for E in (1, 2, 4, 8, 16, 32, 64):
+        w = make_workload(f"sweep_e{E}")
+        byt_all = w.bytes_algorithmic()
+        byt = byt_all["total"]
+        first = DeviceBatch(w, device=device, fill_nan=False)
+        per_rep = first.k_prefix.numel() * 4 + first.k_pool.numel() * 4
+        n_rep = max(2, -(-3 * l2 // per_rep))
+        reps = [first] + [DeviceBatch(w, device=device, fill_nan=False) for _ in range(n_rep - 1)]
+        steps = [B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                                db.page_table, w.max_pages, db.workspace, w.prefix_offset, db.q,
+                                db.k_new, db.v_new, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool,
+                                db.out, db.lse, stream) for db in reps]
+        for i in range(max(3, args.warmup)):
+            steps[i % n_rep]()
+        torch.cuda.synchronize()
+        K = args.steps
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(K):
+            steps[i % n_rep]()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ours_us = e0.elapsed_time(e1) * 1e3 / K
+
+        # naive comparator: per event, its visible keys made contiguous once (outside the
+        # timing), then one attention call per event per step; L2 flushed between steps
+        db = first
+        steps[0]()
+        torch.cuda.synchronize()
+        ks, vs, qs = [], [], []
+        for e in range(w.n_events):
+            b_ = int(w.event_video[e])
+            o, P = int(w.prefix_offset[b_]), int(w.prefix_len[b_])
+            kb, vb = db.gather_branch(e, int(w.event_len[e]) + 1)
+            ks.append(torch.cat([db.k_prefix[o:o + P], kb]).transpose(0, 1).unsqueeze(0).contiguous())
+            vs.append(torch.cat([db.v_prefix[o:o + P], vb]).transpose(0, 1).unsqueeze(0).contiguous())
+            qs.append(db.q[e].view(1, w.h_q, 1, w.head_dim))
+        naive_bytes = sum(k.numel() * 2 * 2 for k in ks)
+        outs = [None] * w.n_events
+        times = []
+        for it in range(3 + args.sweep_naive_steps):
+            flush.zero_()
+            a0 = torch.cuda.Event(enable_timing=True)
+            a1 = torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            for e in range(w.n_events):
+                outs[e] = F.scaled_dot_product_attention(qs[e], ks[e], vs[e], scale=float(w.scale),
+                                                         enable_gqa=True)
+            a1.record(stream)
+            torch.cuda.synchronize()
+            if it >= 3:
+                times.append(a0.elapsed_time(a1) * 1e3)
+        naive_us = statistics.median(times)
+        ref = torch.stack([o.view(w.h_q, w.head_dim).float() for o in outs])
+        diff = float((ref - db.out.float()).abs().max())
+        print(json.dumps({"sweep_E": E, "algorithmic_bytes": byt, "prefix_bytes": byt_all["prefix"],
+                          "branch_bytes": byt_all["branch"], "ours_us_per_step": ours_us,
+                          "ours_gbs": byt / ours_us * 1e-3, "naive_bytes_per_step": naive_bytes,
+                          "naive_us_per_step": naive_us, "naive_gbs": naive_bytes / naive_us * 1e-3,
+                          "max_abs_ours_vs_naive": diff, "replicas": n_rep, "steps": K}), flush=True)
+        del reps, steps, first, db, ks, vs, qs, outs
+        torch.cuda.empty_cache()
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -550,8 +635,13 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="per-E table of the sweep workload with the naive per-event comparator")
+    ap.add_argument("--sweep-naive-steps", type=int, default=20)
     args = ap.parse_args(argv)
-    if args.impl == "reference":
+    if args.sweep:
+        run_sweep(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)
