@@ -38,7 +38,7 @@ def sources():
 
 def _stamp(nvcc: str, extra) -> str:
     h = hashlib.sha256()
-    files = sources() + sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".h"))
+    files = sources() + sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh")))
     files.append(os.path.join(INCLUDE, "pad.h"))
     for f in files:
         h.update(f.encode())
