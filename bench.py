@@ -324,6 +324,8 @@ def run_ours(args):
 
     flags = {"auto": 0, "simt": B.FLAG_PREFIX_SIMT, "mma": B.FLAG_PREFIX_MMA,
              "tc": B.FLAG_PREFIX_TC}[args.prefix]
+    if args.fused_merge:
+        flags |= B.FLAG_FUSED_MERGE
     first = DeviceBatch(w, device=device, fill_nan=False, flags=flags)
     per_rep = sum(t.numel() * t.element_size() for t in
                   (first.k_prefix, first.v_prefix, first.k_pool, first.v_pool, first.q, first.k_new,
@@ -336,10 +338,18 @@ def run_ours(args):
         return B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
                               db.page_table, w.max_pages, db.workspace, w.prefix_offset,
                               kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
-                              db.k_pool, db.v_pool, db.out, db.lse, stream)
+                              db.k_pool, db.v_pool, db.out, db.lse, stream,
+                              one_call=not args.two_call)
 
+    one_call = not args.two_call
+    api_path = ("pad_plan + pad_decode_step" if one_call
+                else "pad_plan + pad_kv_append + pad_event_decode_attn")
     steps = [launcher(db) for db in reps]
     info = reps[0].plan_step(stream).info()
+    # kernels of one step: append (two-call path only), prefix pass, branch/merge (unless
+    # the prefix kernel runs it)
+    launches_per_step = ((0 if one_call else 1) + (info["n_work_items"] > 0)
+                         + (0 if info["fused_tail"] else 1))
     reps[0].release_new_pages()
     torch.cuda.synchronize()
 
@@ -414,8 +424,8 @@ def run_ours(args):
     e_units, e_ms = aggregate(float(w.n_events * Ke), e2e_ms, device)
     e2e = {"value": e_units / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
            "d2h_bytes_per_step": d2h, "steps": Ke,
-           "path": "pinned H2D of q/k_new/v_new, pad_plan + pad_kv_append + pad_event_decode_attn "
-                   "through the C ABI, D2H of O and LSE, stream sync every step"}
+           "path": "pinned H2D of q/k_new/v_new, " + api_path + " through the C ABI, D2H of O and "
+                   "LSE, stream sync every step"}
 
     if rank != 0:
         return
@@ -423,7 +433,16 @@ def run_ours(args):
     kern_name = {1: "prefix_simt_kernel", 2: "prefix_mma_kernel", 4: "prefix_tc_kernel"}[
         info["prefix_kernel"]]
     prefix_ms_per_launch = pre_ms / max(1, pre_n)
-    achieved = byt["prefix"] / (prefix_ms_per_launch * 1e-3) / 1e9
+    # the timed kernel's own algorithmic bytes: the prefix pass alone, or, when it also runs
+    # a4 + a5 (and a2 in the one-call step), every byte of the step that it moves
+    fused = bool(info["fused_tail"])
+    if fused:
+        roof_bytes = byt["total"] - (0 if one_call else byt["append"])
+        roof_what = "prefix + branch KV + Q + out/LSE" + (" + append" if one_call else "")
+    else:
+        roof_bytes = byt["prefix"]
+        roof_what = "prefix KV read once"
+    achieved = roof_bytes / (prefix_ms_per_launch * 1e-3) / 1e9
     step_ms = ms / K
     line = {
         "metric": METRIC,
@@ -447,12 +466,13 @@ def run_ours(args):
             "prefix_tokens": int(w.prefix_len.sum()),
             "private_tokens_after_append": int((w.event_len + 1).sum()),
             "prefix_kernel": kern_name, "splits": info["n_work_items"],
+            "fused_tail": bool(info["fused_tail"]), "api": api_path,
             "l2": f"{n_rep} rotating cold replicas of the whole device state "
                   f"({n_rep * per_rep / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
             "parallelism": "replicas" if world > 1 else "single GPU",
         },
         "clocks": clocks,
-        "gpu_launches": K * (1 + (info["n_work_items"] > 0) + 1),
+        "gpu_launches": K * launches_per_step,
         "roofline": {
             "bound": "hbm",
             "kernel": kern_name,
@@ -462,7 +482,9 @@ def run_ours(args):
             "frac": achieved / peak,
             "peak_kind": peak_kind,
             "traffic": recorded_traffic(args.workload, kern_name),
-            "algorithmic_bytes_per_launch": byt["prefix"],
+            "algorithmic_bytes_per_launch": roof_bytes,
+            "algorithmic_bytes_cover": roof_what,
+            "fused_tail": fused,
             "launch_us": prefix_ms_per_launch * 1e3,
             "launches_timed": pre_n,
             "timing": "CUDA events around each launch of the kernel on its stream, in a loop of "
@@ -635,6 +657,10 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fused-merge", action="store_true",
+                    help="a4 + a5 inside the tensor-core prefix kernel where the plan allows it")
+    ap.add_argument("--two-call", action="store_true",
+                    help="pad_kv_append + pad_event_decode_attn instead of pad_decode_step")
     ap.add_argument("--sweep", action="store_true",
                     help="per-E table of the sweep workload with the naive per-event comparator")
     ap.add_argument("--sweep-naive-steps", type=int, default=20)

@@ -23,8 +23,11 @@
  * step's descriptors (from a per-device pool of library-owned buffers, kept until
  * exit); it stays valid until pad_plan_destroy, which may follow its launches at
  * once: an image is rewritten only after the launches that read it have completed.
- * A plan is tied to the workspace it was built on, which holds the status word and
- * the split-KV partial states; steps that share a workspace run in stream order.
+ * A plan is tied to the workspace it was built on, which holds the status word, the
+ * split-KV partial states and the counters by which prefix CTAs tell the fused merge
+ * that their partials are written; steps that share a workspace run in stream order.
+ * Zero-fill a workspace once when it is allocated; every launch leaves its counters at
+ * zero again, and pad_device_status zeroes them after a device error.
  *
  * Errors: every call validates its arguments on the host and returns a
  * pad_status before launching anything; pad_last_error() gives a message
@@ -93,6 +96,12 @@ typedef struct {
 #define PAD_FLAG_PREFIX_SIMT 0x1   /* CUDA-core path */
 #define PAD_FLAG_PREFIX_MMA 0x2    /* warp-level mma.sync path */
 #define PAD_FLAG_PREFIX_TC 0x4     /* tcgen05 / TMEM / TMA path */
+/* Run a4 + a5 inside the tensor-core prefix kernel, after each CTA's split, where every
+ * (event, kv-head) pair can take a prefix CTA and the prefix grid fits one CTA per SM
+ * (pad_plan_info.fused_tail says whether it was chosen).  Off by default: the separate
+ * branch/merge kernel, which starts its branch pass as prefix CTAs retire, was measured
+ * faster on GB300. */
+#define PAD_FLAG_FUSED_MERGE 0x8
 
 /* ---------------------------------------------------------------------------
  * Page pool bookkeeping (host).  Tracks which pages of the private KV pool are
@@ -142,10 +151,11 @@ size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32
  *   event_len      [n_events] host: private tokens of each branch BEFORE this step's append;
  *                  branch e attends to event_len[e] + 1 private keys after the append
  *   page_table     [n_events * max_pages] device: row e lists branch e's pages; the
- *                  new-page entries are written by pad_kv_append
+ *                  new-page entries are written by pad_kv_append (or pad_decode_step)
  *   max_pages      columns of page_table; event_len[e] / page_size must be < max_pages
- *   workspace      device, 256-byte aligned, at least pad_workspace_size(...) bytes;
- *                  NULL plans on the host only (no image; the plan cannot be launched)
+ *   workspace      device, 256-byte aligned, at least pad_workspace_size(...) bytes,
+ *                  zero-filled when allocated (see above); NULL plans on the host only
+ *                  (no image; the plan cannot be launched)
  *   stream         unused (kept for the interface): pad_plan enqueues nothing; it may
  *                  wait for the launches of an earlier plan whose image it reuses, once
  *                  eight or more images of the device have been released
@@ -178,7 +188,8 @@ typedef struct {
   int64_t workspace_bytes;  /* bytes of workspace this plan uses */
   int32_t param_descriptor_bytes; /* bytes of descriptors carried in each launch's parameters;
                                      0 = the kernels read them from the plan's page-locked image */
-  int32_t reserved;
+  int32_t fused_tail;       /* 1: the branch pass and the merge run inside the prefix kernel */
+  uint64_t generation;      /* the number tagging this plan's device status word and counters */
 } pad_plan_info;
 pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info);
 pad_status pad_plan_destroy(pad_plan_t* plan);
@@ -201,6 +212,15 @@ pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* 
 pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
                                  const void* v_prefix, const void* k_pool, const void* v_pool,
                                  void* out, float* lse, pad_stream_t stream);
+
+/* a2-a5 in one call: the same result as pad_kv_append followed by pad_event_decode_attn
+ * (pools, page table, out and lse all end up identical), with one kernel launch fewer.
+ * The shared-prefix pass starts the step; each (event, kv-head) branch task reads its
+ * newest key from k_new / v_new, writes it into the pools (and the page table) itself,
+ * and attends to it.  Arguments as in those two calls; k_pool and v_pool are written. */
+pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_new, const void* v_new,
+                           const void* k_prefix, const void* v_prefix, void* k_pool, void* v_pool,
+                           void* out, float* lse, pad_stream_t stream);
 
 /* Allocation-free variant of pad_event_decode_attn (the paper has no counterpart; this
  * is an interface for callers, not part of the method).  Same arguments and result.  It

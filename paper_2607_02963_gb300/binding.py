@@ -24,6 +24,7 @@ STATUS_NAMES = {
 FLAG_PREFIX_SIMT = 0x1
 FLAG_PREFIX_MMA = 0x2
 FLAG_PREFIX_TC = 0x4
+FLAG_FUSED_MERGE = 0x8
 
 
 class PadError(RuntimeError):
@@ -42,7 +43,8 @@ class PlanInfo(ctypes.Structure):
     _fields_ = [("n_videos", c_int32), ("n_events", c_int32), ("n_work_items", c_int32),
                 ("split_len", c_int32), ("prefix_kernel", c_int32), ("n_new_pages", c_int32),
                 ("partial_rows", c_int64), ("workspace_bytes", c_int64),
-                ("param_descriptor_bytes", c_int32), ("reserved", c_int32)]
+                ("param_descriptor_bytes", c_int32), ("fused_tail", c_int32),
+                ("generation", ctypes.c_uint64)]
 
 
 _I32P = POINTER(c_int32)
@@ -71,6 +73,7 @@ _SIGNATURES = {
                                         c_void_p, c_void_p, c_void_p, c_void_p]),
     "pad_event_decode_attn_static": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                                c_void_p, c_void_p, c_void_p, c_void_p]),
+    "pad_decode_step": (c_int32, [c_void_p] * 11),
     "pad_device_status": (c_int32, [c_void_p, c_void_p]),
     "pad_last_error": (ctypes.c_char_p, []),
     "pad_status_string": (ctypes.c_char_p, [c_int32]),
@@ -258,6 +261,14 @@ def pad_event_decode_attn(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out
                                        _stream(stream)))
 
 
+def pad_decode_step(plan: Plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,
+                    stream=None):
+    """pad_kv_append + pad_event_decode_attn in one call (one kernel launch fewer)."""
+    _check(lib().pad_decode_step(plan.handle, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix),
+                                 _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
+                                 _stream(stream)))
+
+
 def pad_event_decode_attn_static(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,
                                  stream=None):
     """pad_event_decode_attn with the library's static scratch instead of a workspace."""
@@ -282,15 +293,16 @@ def pad_timing_read():
 
 
 class StepLauncher:
-    """One decode step (pad_plan -> pad_kv_append -> pad_event_decode_attn) with every
-    argument converted to ctypes once, so a repeated step costs only the C calls.
+    """One decode step (pad_plan -> pad_decode_step, or pad_plan -> pad_kv_append ->
+    pad_event_decode_attn with ``one_call=False``) with every argument converted to ctypes
+    once, so a repeated step costs only the C calls.
 
     ``release_pages``: return the pages the step took after launching it (keeps a
     repeated identical step idempotent, as when re-running one step for timing)."""
 
     def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
                  page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
-                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True):
+                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True):
         self.L = lib()
         self.problem = problem
         self.cache = cache
@@ -314,6 +326,9 @@ class StepLauncher:
         self.args_append = [_ptr(k_new), _ptr(v_new), _ptr(k_pool), _ptr(v_pool), self.stream]
         self.args_attn = [_ptr(q), _ptr(k_prefix), _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool),
                           _ptr(out), _ptr(lse), self.stream]
+        self.args_step = [_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix), _ptr(v_prefix),
+                          _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse), self.stream]
+        self.one_call = one_call
         self.newp = np.full(self.ne, -1, dtype=np.int32)
         self.newpp = self.newp.ctypes.data_as(_I32P)
         self.release = release_pages
@@ -328,8 +343,11 @@ class StepLauncher:
                           self.ph))
         h = self.h
         try:
-            _check(L.pad_kv_append(h, *self.args_append))
-            _check(L.pad_event_decode_attn(h, *self.args_attn))
+            if self.one_call:
+                _check(L.pad_decode_step(h, *self.args_step))
+            else:
+                _check(L.pad_kv_append(h, *self.args_append))
+                _check(L.pad_event_decode_attn(h, *self.args_attn))
             if self.release:
                 _check(L.pad_plan_release_new_pages(h, self.cache.handle))
         finally:

@@ -77,9 +77,9 @@ pad_status check_problem(const pad_problem* prob) {
   if (prob->out_dtype != 0 && prob->out_dtype != 1)
     return fail(PAD_ERR_INVALID_ARG, "out_dtype=%d (0 = fp32, 1 = bf16)", prob->out_dtype);
   if (prob->num_sms < 0) return fail(PAD_ERR_INVALID_ARG, "num_sms < 0");
-  const int known = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC;
+  const int known = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC | PAD_FLAG_FUSED_MERGE;
   if (prob->flags & ~known) return fail(PAD_ERR_INVALID_ARG, "unknown flags 0x%x", prob->flags);
-  const int f = prob->flags & known;
+  const int f = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
   if (f && (f & (f - 1))) return fail(PAD_ERR_INVALID_ARG, "at most one PAD_FLAG_PREFIX_* flag");
   return PAD_OK;
 }
@@ -94,8 +94,14 @@ struct Layout {
   std::vector<int32_t> ev_first, ev_count, n_splits, part_base;
   int64_t n_items = 0;
   int64_t partial_rows = 0;
-  size_t off_videos = 0, off_events = 0, off_items = 0, upload_bytes = 0;
-  size_t off_ml = 0, off_o = 0, total_bytes = 0;
+  // fused tail of the tensor-core path: per prefix CTA its (event * h_kv + kv-head) task or
+  // -1, and per (video, kv-head, row group) a split counter
+  bool fused = false;
+  int64_t n_ctas = 0;
+  std::vector<int32_t> cta_task, cnt_base;
+  int64_t n_counters = 0;
+  size_t off_videos = 0, off_events = 0, off_items = 0, off_tasks = 0, upload_bytes = 0;
+  size_t off_ml = 0, off_o = 0, off_cnt = 0, total_bytes = 0;
 };
 
 pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32_t* prefix_len,
@@ -183,6 +189,45 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   L->n_items = items;
   L->partial_rows = rows;
 
+  // Fused tail: when every (event, kv-head) task can go to a prefix CTA of its own, the
+  // tensor-core kernel runs a4 + a5 after its split (tasks go first to the CTAs with the
+  // shortest splits, which finish first) and no separate merge kernel is launched.
+  L->cnt_base.assign(n_videos, 0);
+  L->n_counters = 0;
+  L->fused = false;
+  L->n_ctas = 0;
+  L->cta_task.clear();
+  if (kern == PAD_FLAG_PREFIX_TC && items > 0 && (prob->flags & PAD_FLAG_FUSED_MERGE) &&
+      items * groups <= (int64_t)std::max(1, n_sms)) {
+    // (the tail waits for other CTAs' splits: the whole grid must be resident at once,
+    // which one CTA per SM and a grid of at most one wave guarantee)
+    L->n_ctas = items * groups;
+    std::vector<std::pair<int64_t, int64_t>> valid;  // (split tokens, CTA index)
+    int64_t item = 0;
+    for (int b = 0; b < n_videos; ++b) {
+      if (L->ev_count[b] == 0 || L->n_splits[b] == 0) continue;
+      const int R = L->ev_count[b] * L->group;
+      const int gb = (R + 127) / 128;
+      L->cnt_base[b] = (int32_t)L->n_counters;
+      L->n_counters += (int64_t)prob->h_kv * gb;
+      for (int h = 0; h < prob->h_kv; ++h)
+        for (int s = 0; s < L->n_splits[b]; ++s, ++item) {
+          const int64_t tok = std::min<int64_t>(prefix_len[b], (int64_t)(s + 1) * chunk) - (int64_t)s * chunk;
+          for (int g = 0; g < gb; ++g) valid.push_back({tok, item * groups + g});
+        }
+    }
+    const int64_t tasks_n = (int64_t)n_events * prob->h_kv;
+    if (tasks_n <= (int64_t)valid.size()) {
+      std::stable_sort(valid.begin(), valid.end(),
+                       [](const std::pair<int64_t, int64_t>& x, const std::pair<int64_t, int64_t>& y) {
+                         return x.first < y.first;
+                       });
+      L->cta_task.assign(L->n_ctas, -1);
+      for (int64_t t = 0; t < tasks_n; ++t) L->cta_task[valid[t].second] = (int32_t)t;
+      L->fused = true;
+    }
+  }
+
   size_t off = sizeof(PadDevHeader);
   L->off_videos = off;
   off = align_up(off + (size_t)n_videos * sizeof(PadVideoDesc), 256);
@@ -190,12 +235,16 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   off = align_up(off + (size_t)n_events * sizeof(PadEventDesc), 256);
   L->off_items = off;
   off = off + (size_t)items * sizeof(PadWorkItem);
+  L->off_tasks = off;
+  off = off + (size_t)L->cta_task.size() * sizeof(int32_t);
   L->upload_bytes = off;
   off = align_up(off, 256);
   L->off_ml = off;
   off = align_up(off + (size_t)rows * sizeof(float2), 256);
   L->off_o = off;
   off = align_up(off + (size_t)rows * prob->head_dim * sizeof(float), 256);
+  L->off_cnt = off;
+  off = align_up(off + (size_t)L->n_counters * sizeof(unsigned int), 256);
   L->total_bytes = off;
   return PAD_OK;
 }
@@ -349,7 +398,7 @@ struct pad_plan_t {
   PlanImage* image = nullptr;       // the same bytes in pinned memory, read by the kernels
                                     // when they do not fit the launch parameters
   std::vector<uint8_t> param_image; // videos | events | items, packed, for KParams::img
-  int32_t img_videos = 0, img_events = 0, img_items = 0;
+  int32_t img_videos = 0, img_events = 0, img_items = 0, img_tasks = 0;
   uint64_t gen = 0;                 // generation tagging this plan's device errors
   ~pad_plan_t() { image_release(image); }
 };
@@ -513,7 +562,7 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
     v.n_events = L.ev_count[b];
     v.n_splits = L.n_splits[b];
     v.part_base = L.part_base[b];
-    v.pad = 0;
+    v.cnt_base = L.cnt_base[b];
   }
   std::vector<PadWorkItem> items;
   items.reserve(L.n_items);
@@ -563,20 +612,25 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   if (n_events) std::memcpy(plan->host_image.data() + L.off_events, evs.data(), evs.size() * sizeof(PadEventDesc));
   if (!items.empty())
     std::memcpy(plan->host_image.data() + L.off_items, items.data(), items.size() * sizeof(PadWorkItem));
+  if (!L.cta_task.empty())
+    std::memcpy(plan->host_image.data() + L.off_tasks, L.cta_task.data(), L.cta_task.size() * sizeof(int32_t));
 
   plan->gen = next_generation();
   {
     const size_t nv = vids.size() * sizeof(PadVideoDesc), ne = evs.size() * sizeof(PadEventDesc);
     const size_t ni = items.size() * sizeof(PadWorkItem);
+    const size_t nt = L.cta_task.size() * sizeof(int32_t);
     plan->img_videos = 0;
     plan->img_events = (int32_t)align_up(nv, 16);
     plan->img_items = (int32_t)(plan->img_events + align_up(ne, 16));
-    const size_t total = plan->img_items + ni;
+    plan->img_tasks = (int32_t)(plan->img_items + align_up(ni, 16));
+    const size_t total = plan->img_tasks + nt;
     if (n_events > 0 && total <= (size_t)kParamImageBytes) {
       plan->param_image.assign(total, 0);
       if (nv) std::memcpy(plan->param_image.data(), vids.data(), nv);
       if (ne) std::memcpy(plan->param_image.data() + plan->img_events, evs.data(), ne);
       if (ni) std::memcpy(plan->param_image.data() + plan->img_items, items.data(), ni);
+      if (nt) std::memcpy(plan->param_image.data() + plan->img_tasks, L.cta_task.data(), nt);
     }
   }
   if (workspace && n_events > 0 && plan->param_image.empty()) {
@@ -630,7 +684,8 @@ pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
   info->partial_rows = plan->lay.partial_rows;
   info->workspace_bytes = (int64_t)plan->lay.total_bytes;
   info->param_descriptor_bytes = (int32_t)plan->param_image.size();
-  info->reserved = 0;
+  info->fused_tail = plan->lay.fused ? 1 : 0;
+  info->generation = plan->gen;
   return PAD_OK;
 }
 
@@ -664,16 +719,25 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.img_videos = plan->img_videos;
   p.img_events = plan->img_events;
   p.img_items = plan->img_items;
+  p.img_tasks = plan->img_tasks;
+  p.k_new = nullptr;
+  p.v_new = nullptr;
+  p.fused = plan->lay.fused ? 1 : 0;
+  p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
+  p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
+  p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;
   if (p.img_n > 0) {
     std::memcpy(p.img, plan->param_image.data(), plan->param_image.size());
     p.videos = nullptr;
     p.events = nullptr;
     p.items = nullptr;
+    p.tasks = nullptr;
   } else {
     auto* im = static_cast<const uint8_t*>(plan->image->dev);
     p.videos = reinterpret_cast<const PadVideoDesc*>(im + plan->lay.off_videos);
     p.events = reinterpret_cast<const PadEventDesc*>(im + plan->lay.off_events);
     p.items = reinterpret_cast<const PadWorkItem*>(im + plan->lay.off_items);
+    p.tasks = reinterpret_cast<const int32_t*>(im + plan->lay.off_tasks);
   }
   p.part_ml = reinterpret_cast<float2*>(ws + plan->lay.off_ml);
   p.part_o = reinterpret_cast<float*>(ws + plan->lay.off_o);
@@ -701,9 +765,14 @@ pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* 
   return PAD_OK;
 }
 
-pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
-                                 const void* v_prefix, const void* k_pool, const void* v_pool,
-                                 void* out, float* lse, pad_stream_t stream) {
+// a3 (+ a4, a5 in the same kernel when the plan fuses them, else in the branch/merge
+// kernel after it).  k_new == NULL: the append kernel ran just before (the prefix kernel
+// overlaps it through programmatic dependent launch).  k_new set: no append kernel; each
+// branch task appends its own row, and the prefix kernel is the step's first launch.
+static pad_status launch_attention(const pad_plan_t* plan, const void* q, const void* k_new,
+                                   const void* v_new, const void* k_prefix, const void* v_prefix,
+                                   const void* k_pool, const void* v_pool, void* out, float* lse,
+                                   pad_stream_t stream) {
   if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
   if (plan->n_events == 0) return PAD_OK;
   if (!plan->workspace) return fail(PAD_ERR_INVALID_ARG, "plan was built without a workspace");
@@ -711,11 +780,14 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
   if (plan->lay.n_items > 0 && (!k_prefix || !v_prefix))
     return fail(PAD_ERR_INVALID_ARG, "k_prefix / v_prefix is NULL");
   if (!aligned16(q) || !aligned16(k_prefix) || !aligned16(v_prefix) || !aligned16(k_pool) ||
-      !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+      !aligned16(v_pool) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new) ||
+      (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
     return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   KParams p;
   make_params(plan, p);
+  p.k_new = k_new;
+  p.v_new = v_new;
   const bool timed = g_timing.on && g_timing.n < g_timing.max;
   if (timed) cudaEventRecord(g_timing.ev[2 * g_timing.n], s);
   cudaError_t e = cudaSuccess;
@@ -725,9 +797,11 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
     case PAD_FLAG_PREFIX_TC:
       // programmatic dependent launch: the prefix pass overlaps the append kernel and the
       // branch/merge pass's prologue overlaps the prefix pass (not while timing events
-      // are recorded between the kernels)
-      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens,
-                           !timed, s);
+      // are recorded between the kernels).  As the first kernel of a one-call step it
+      // overlaps only the launch with the grid before it, and waits for that grid before
+      // it reads or writes anything.
+      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
+                           v_pool, out, lse, !timed, s);
       break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }
@@ -736,15 +810,30 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
     cudaEventRecord(g_timing.ev[2 * g_timing.n + 1], s);
     g_timing.n++;
   }
-  const bool pdl = !timed && plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC;
-  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, pdl, s);
-  if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
+  if (!plan->lay.fused) {
+    const bool pdl = !timed && plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC;
+    e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, pdl, s);
+    if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
+  }
   if (plan->image) {
     e = cudaEventRecord(plan->image->done, s);
     if (e != cudaSuccess) return cuda_fail(e, "plan image event");
     plan->image->recorded = true;
   }
   return PAD_OK;
+}
+
+pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
+                                 const void* v_prefix, const void* k_pool, const void* v_pool,
+                                 void* out, float* lse, pad_stream_t stream) {
+  return launch_attention(plan, q, nullptr, nullptr, k_prefix, v_prefix, k_pool, v_pool, out, lse, stream);
+}
+
+pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_new, const void* v_new,
+                           const void* k_prefix, const void* v_prefix, void* k_pool, void* v_pool,
+                           void* out, float* lse, pad_stream_t stream) {
+  if (plan && plan->n_events > 0 && (!k_new || !v_new)) return fail(PAD_ERR_INVALID_ARG, "NULL k_new / v_new");
+  return launch_attention(plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse, stream);
 }
 
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
@@ -756,9 +845,18 @@ pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "reading device status");
   const int code = (int)(h.word & 0xffull);
-  if ((h.word >> 8) == plan->gen && code != PAD_OK)
+  if ((h.word >> 8) == plan->gen && code != PAD_OK) {
+    // a failed launch may have left the fused tail's split counters part-way: zero them,
+    // so that the next plan on this workspace starts clean
+    if (plan->lay.n_counters > 0) {
+      e = cudaMemsetAsync(static_cast<uint8_t*>(plan->workspace) + plan->lay.off_cnt, 0,
+                          (size_t)plan->lay.n_counters * sizeof(unsigned int), s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return cuda_fail(e, "clearing split counters");
+    }
     return fail((pad_status)code, "device reported %s (detail %d %d %d)",
                 pad_status_string((pad_status)code), h.info[0], h.info[1], h.info[2]);
+  }
   return PAD_OK;
 }
 
@@ -882,7 +980,14 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   p.gen = plan->gen;
   p.img_n = 0;
+  p.k_new = nullptr;
+  p.v_new = nullptr;
+  p.fused = plan->lay.fused ? 1 : 0;
+  p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   auto* ws = static_cast<uint8_t*>(scratch);
+  p.tasks = reinterpret_cast<const int32_t*>(ws + plan->lay.off_tasks);
+  p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
+  p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;
   p.header = reinterpret_cast<PadDevHeader*>(ws);
   p.videos = reinterpret_cast<const PadVideoDesc*>(ws + plan->lay.off_videos);
   p.events = reinterpret_cast<const PadEventDesc*>(ws + plan->lay.off_events);
@@ -895,12 +1000,19 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
     case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_TC:
-      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, false, s);
+      if (p.n_counters > 0) {  // (the append of a workspace plan zeroes them; none ran on this array)
+        e = cudaMemsetAsync(ws + plan->lay.off_cnt, 0, (size_t)p.n_counters * sizeof(unsigned int), s);
+        if (e != cudaSuccess) return cuda_fail(e, "static scratch counters");
+      }
+      e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
+                           v_pool, out, lse, false, s);
       break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }
   if (e != cudaSuccess) return cuda_fail(e, "prefix launch (static scratch)");
-  e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, false, s);
-  if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch (static scratch)");
+  if (!plan->lay.fused) {
+    e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, false, s);
+    if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch (static scratch)");
+  }
   return PAD_OK;
 }

@@ -12,12 +12,18 @@
 //   log-sum-exp (Eq. for combining softmax states: M = max of the maxima, every state
 //   weighted by 2^(m - M)), and O and the LSE are written once.
 //
+//   a2, when the step is one call (KParams::k_new set): key `len` is read from k_new /
+//   v_new instead of the pools, and this task writes it into them (its page-table entry
+//   too, by the kv-head-0 task of an event that took a new page).  No other task reads
+//   this (event, kv-head)'s branch, so nothing else waits for that write.
+//
 // Staging before griddepcontrol.wait reads nothing the grids ahead write: Q rows, the
 // branch's page ids (key `len`'s page is the one this step took, else the table's entry
-// of an earlier step) and the K/V rows of keys 0..len-1.  After it: key `len` (written
-// by this step's append), and the splits' (m, l) pairs and O rows once the caller says
-// they are complete (`partials_ready`: at once for the standalone kernel, whose wait
-// covers the prefix grid; after the split counters for the tensor-core kernel).
+// of an earlier step) and the K/V rows of keys 0..len-1, and key `len` itself when it
+// comes from k_new / v_new.  After it: key `len` when the append kernel wrote it, and the
+// splits' (m, l) pairs and O rows once the caller says they are complete
+// (`partials_ready`: at once for the standalone kernel, whose wait covers the prefix
+// grid; after the split counters for the tensor-core kernel).
 #pragma once
 
 #include <cuda_bf16.h>
@@ -203,18 +209,42 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     S.L[tid] = 0.f;
   }
   sy.sync();
+  const __nv_bfloat16* knew = static_cast<const __nv_bfloat16*>(p.k_new);
+  const __nv_bfloat16* vnew = static_cast<const __nv_bfloat16*>(p.v_new);
+  const size_t new_row = ((size_t)e * p.h_kv + kvh) * D;
   auto stage_keys = [&](int r0, int nv, int k_lo, int k_hi) {  // rows k_lo..k_hi-1 of the round
     for (int i = tid; i < (k_hi - k_lo) * CH; i += NT) {
       const int k = k_lo + i / CH, c = i - (i / CH) * CH;
       const int pg = k < nv ? S.page[k] : -1;
       const bool in = pg >= 0;
+      if (knew != nullptr && r0 + k == len) {
+        cp_async16(&sK[k][c * 8], knew + new_row + c * 8, in);
+        cp_async16(&sV[k][c * 8], vnew + new_row + c * 8, in);
+        continue;
+      }
       const size_t off = (((size_t)(in ? pg : 0) * p.h_kv + kvh) * ps + ((r0 + k) % ps)) * D + c * 8;
       cp_async16(&sK[k][c * 8], kpool + off, in);
       cp_async16(&sV[k][c * 8], vpool + off, in);
     }
   };
+  if (knew != nullptr) {
+    // a2: this task's row of the new token into the pools (16-byte pieces of K, then V)
+    if (tid < 2 * CH) {
+      const int pg = page_of(len);
+      if (pg >= 0) {
+        const int c = tid % CH;
+        const bool isv = tid >= CH;
+        const size_t dst = (((size_t)pg * p.h_kv + kvh) * ps + (len % ps)) * D + c * 8;
+        const uint4 v = *reinterpret_cast<const uint4*>((isv ? vnew : knew) + new_row + c * 8);
+        *reinterpret_cast<uint4*>(const_cast<__nv_bfloat16*>(isv ? vpool : kpool) + dst) = v;
+      }
+    }
+    if (kvh == 0 && tid == 0 && ev.new_page >= 0 && ev.new_page < p.n_pages)
+      p.page_table[(size_t)e * p.max_pages + len / ps] = ev.new_page;
+  }
   const int nv0_16 = (nv0 + 15) & ~15;
-  const bool len_in_first = len < nkr;
+  // key `len` waits for the grids ahead only when the append kernel wrote it
+  const bool len_in_first = len < nkr && knew == nullptr;
   // rows 0..nv0_16-1 except key `len` (rows past nv0 are zero-filled)
   if (len_in_first) {
     stage_keys(0, nv0, 0, len);

@@ -59,7 +59,7 @@ struct PadVideoDesc {
   int32_t n_events;
   int32_t n_splits;     // prefix splits per kv-head (0 if prefix_len == 0 or no events)
   int32_t part_base;    // first partial row of this video
-  int32_t pad;
+  int32_t cnt_base;     // first split counter of this video (fused tail; see KParams::counters)
 };
 static_assert(sizeof(PadVideoDesc) == 32, "video desc is 32 bytes");
 
@@ -96,6 +96,9 @@ struct KParams {
   int32_t max_splits;             // largest per-video prefix split count of the batch
   int32_t branch_rows;            // branch keys staged per round: the longest branch's
                                   // len + 1 rounded up to 16, at most 128
+  int32_t fused;                  // the tensor-core prefix kernel runs a4 + a5 itself (one
+                                  // (event, kv-head) task per CTA after its split)
+  int32_t tail_chunk;             // split partials merged per staged chunk in that tail
   float scale_log2;               // scale * log2(e)
   uint64_t gen;                   // generation of the plan (tags errors in the status word)
   PadDevHeader* header;
@@ -105,11 +108,23 @@ struct KParams {
   float2* part_ml;
   float* part_o;
   int32_t* page_table;
+  // Set by the one-call step (pad_decode_step): this step's new K/V rows [n_events, h_kv,
+  // head_dim].  Each (event, kv-head) task of a4 then reads its key `len` from here and
+  // writes it into the pools itself (a2 folded into a4; no append kernel runs).
+  const void* k_new;
+  const void* v_new;
+  const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
+  // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
+  // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by
+  // the append kernel of the step; the last task to take a counter zeroes it again, so a
+  // plan launched twice without an append in between starts from zero too.
+  unsigned int* counters;
+  int32_t n_counters;
   // The descriptors themselves when they fit (img_n > 0): carried in the launch's
   // parameter block, so a CTA reads them from the constant bank instead of from the
   // plan's page-locked host image.  Sections start at the img_* byte offsets.
   int32_t img_n;                  // bytes used, 0 = read videos / events / items instead
-  int32_t img_videos, img_events, img_items;
+  int32_t img_videos, img_events, img_items, img_tasks;
   alignas(16) unsigned char img[kParamImageBytes];
 };
 static_assert(sizeof(KParams) <= 8192, "kernel parameters stay at 8 KB");
@@ -126,6 +141,9 @@ __device__ __forceinline__ const PadEventDesc* plan_events(const KParams& p) {
 __device__ __forceinline__ const PadWorkItem* plan_items(const KParams& p) {
   return p.img_n > 0 ? reinterpret_cast<const PadWorkItem*>(p.img + p.img_items) : p.items;
 }
+__device__ __forceinline__ const int32_t* plan_tasks(const KParams& p) {
+  return p.img_n > 0 ? reinterpret_cast<const int32_t*>(p.img + p.img_tasks) : p.tasks;
+}
 #endif
 
 // Launchers (pad_kernels.cu, pad_prefix_tc.cu).  Return the launch error.
@@ -135,8 +153,12 @@ cudaError_t launch_prefix_simt(const KParams& p, int max_rows, const void* q, co
                                const void* vp, cudaStream_t s);
 cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, const void* kp,
                               const void* vp, cudaStream_t s);
+// With p.fused the same launch also runs a4 + a5 (k_pool, v_pool, out, lse used).
+// Split partials merged per staged chunk by that tail (fits the kernel's shared memory).
+int prefix_tc_tail_chunk(int branch_rows, int group, int max_splits);
 cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
-                             const void* vp, int64_t total_prefix_tokens, bool pdl, cudaStream_t s);
+                             const void* vp, int64_t total_prefix_tokens, const void* k_pool,
+                             const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 // pdl: launch with programmatic stream serialization (the kernel waits for its
 // predecessor with griddepcontrol.wait before it reads anything the predecessor wrote).
 cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,

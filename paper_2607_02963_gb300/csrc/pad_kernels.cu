@@ -106,11 +106,15 @@ __device__ __forceinline__ int64_t part_row(const PadVideoDesc& vd, int kvh, int
 __global__ void append_kernel(const __grid_constant__ KParams p, const uint4* __restrict__ k_new,
                               const uint4* __restrict__ v_new, uint4* __restrict__ k_pool,
                               uint4* __restrict__ v_pool) {
-  // the shared-prefix pass launched after this kernel reads nothing it writes
+  // the shared-prefix pass launched after this kernel reads nothing it writes before its
+  // griddepcontrol.wait
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int chunks = p.head_dim / 8;
   const int per_event = p.h_kv * chunks;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  // the split counters of the fused tail start the step at zero (there are fewer of them
+  // than threads here: at most h_kv per event)
+  if (idx < p.n_counters) p.counters[idx] = 0u;
   if (idx >= p.n_events * per_event) return;
   const int e = idx / per_event;
   const int rem = idx - e * per_event;

@@ -27,7 +27,11 @@
 // which one tcgen05.mma carries as much tensor work as it costs to issue.
 // TMEM columns: S[b] at 128*b (b = 0, 1, 2), O at 384.  Output: the partial
 // softmax state (m, l, O) of every row for this split, merged with the other
-// splits and the branch by the branch/merge kernel.
+// splits and the branch by the branch/merge kernel, or, when the plan fuses them
+// (every (event, kv-head) task has a CTA of its own and the grid is one wave), by
+// the softmax warps of this kernel after their split: they publish the split on a
+// counter, then run one task's branch pass, wait for the counters of the task's rows
+// and merge (a4 + a5 as in the standalone kernel, same code).
 //
 // Barrier phases: a thread waits for completion #c of a barrier by its parity, which is
 // only sound while completion #c+1 cannot yet have happened.  Every barrier here is
@@ -41,10 +45,12 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
+#include <algorithm>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
 
+#include "pad_branch_merge.cuh"
 #include "pad_internal.h"
 
 namespace pad {
@@ -405,9 +411,56 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   }
 }
 
+// Split counters of the fused tail, one per (video, kv-head, 128-row group): bits 15-0
+// count the video's splits that have written their partial rows, bits 31-16 the tasks
+// that have taken them.  The append kernel of the step zeroes them; the last task to
+// take a counter zeroes it again for a launch of the same plan without an append.
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* a) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
+  return v;
+}
+// Thread `leader` waits (bounded) until every split of video `vd` has published the rows
+// [r0, r0 + G) of kv-head `kvh`, then takes them; the result is the same for all 256
+// threads of the softmax group.
+__device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadVideoDesc& vd, int kvh,
+                                                    int r0, bool leader) {
+  bool good = true;
+  if (leader) {
+    const int G = p.group;
+    const int gb = (vd.n_events * G + 127) >> 7;
+    const int g0 = r0 >> 7, g1 = (r0 + G - 1) >> 7;
+    unsigned* base = p.counters + vd.cnt_base + (size_t)kvh * gb;
+    const unsigned long long t0 = globaltimer();
+    for (int g = g0; g <= g1 && good; ++g) {
+      while ((int)(ld_acquire_u32(base + g) & 0xffffu) != vd.n_splits) {
+        // give up at once if this plan's kernels already recorded an error (a split that
+        // failed never publishes), else after the usual bound
+        const unsigned long long hw = *reinterpret_cast<volatile unsigned long long*>(&p.header->word);
+        if (((hw >> 8) == p.gen && (hw & 0xffull) != 0) || globaltimer() - t0 > kWaitNs) {
+          pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_TIMEOUT, (int)blockIdx.x, g, 20);
+          good = false;
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    if (good) {
+      for (int g = g0; g <= g1; ++g) {
+        const int lo = (g << 7) / G, hi = min(vd.n_events - 1, ((g << 7) + 127) / G);
+        const unsigned old = atomicAdd(base + g, 1u << 16);
+        if ((int)(old >> 16) + 1 == hi - lo + 1) atomicExch(base + g, 0u);
+      }
+    }
+  }
+  return bm::SyncNamed{1}.all(good);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
-                     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV) {
+                     const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                     const __nv_bfloat16* __restrict__ kpool, const __nv_bfloat16* __restrict__ vpool,
+                     void* __restrict__ out, float* __restrict__ lse) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const uint32_t sbase = smem_u32(smem);
   if (sbase & 1023u) {  // the 128-byte swizzle atoms need 1024-byte alignment (never expected)
@@ -416,6 +469,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   TcBars* bars = reinterpret_cast<TcBars*>(smem + kOffBar);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // One-call step (k_new set): this is the step's first kernel, launched so that it may
+  // start while the grid before it (the previous step, or the caller's own kernel that
+  // wrote q) finishes.  Nothing is read or written before that grid has completed.
+  const bool one_call = p.k_new != nullptr;
+  if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
 
   const int item = blockIdx.x / n_groups;
   const int group = blockIdx.x - item * n_groups;
@@ -493,8 +551,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   fence_after();
   // The grid launched after this one (the branch/merge pass) may start its own
-  // prologue now; it waits for this grid's completion before it reads partials.
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // prologue now; it waits for this grid's completion before it reads partials.  With
+  // the fused tail of a two-call step the next grid is the next step's append, which
+  // must not overwrite partials that the tail still reads: no early release there.  The
+  // next one-call step waits for this grid before it touches anything, so it may start.
+  if (one_call || !p.fused) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const uint32_t tmem = bars->tmem_base;
 
   if (warp == 0 || warp == 3) {
@@ -705,6 +766,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
       *reinterpret_cast<float4*>(p.part_o + ((int64_t)it.part_row0 + row0 + rr) * kD + 4 * lane) = v;
     }
+    if (p.fused) {
+      // ---------------------------------------------------------- fused a4 + a5
+      // Publish this split's rows (every softmax thread's partial stores are ordered
+      // before the counter by the barrier and the fence), then run this CTA's (event,
+      // kv-head) task with all of shared memory below the barriers (the Q, K and V
+      // stages are idle once the last MMA has completed).
+      const bm::SyncNamed sy{1};
+      if (sy.all(ok)) {
+        if (threadIdx.x == 128) {
+          // the append kernel ahead zeroes the counters: wait for it (long complete by now)
+          asm volatile("griddepcontrol.wait;" ::: "memory");
+          __threadfence();
+          const PadVideoDesc vd = plan_videos(p)[plan_events(p)[it.first_event].video];
+          atomicAdd(p.counters + vd.cnt_base + (size_t)kvh * ((R + 127) >> 7) + group, 1u);
+        }
+        const int task = plan_tasks(p)[blockIdx.x];
+        if (task >= 0) {
+          const int te = task / p.h_kv, th = task - (task / p.h_kv) * p.h_kv;
+          bm::run_task<kD>(p, q, kpool, vpool, out, lse, te, th, (int)threadIdx.x - 128, smem, p.tail_chunk, sy,
+                           false, [&]() {
+                             const PadEventDesc ev = plan_events(p)[te];
+                             const PadVideoDesc vd = plan_videos(p)[ev.video];
+                             return tail_partials_ready(p, vd, th, ev.local * p.group, threadIdx.x == 128);
+                           });
+        }
+      }
+    }
   }
 
   __syncwarp();
@@ -796,8 +884,15 @@ bool get_maps(const void* kp, const void* vp, int h_kv, int64_t tokens, int dev,
 
 }  // namespace
 
+int prefix_tc_tail_chunk(int branch_rows, int group, int max_splits) {
+  int sch = std::min(bm::kMaxChunk, std::max(1, max_splits));
+  while (sch > 1 && bm::smem_bytes<kD>(branch_rows, group, sch) > kOffBar) --sch;
+  return sch;
+}
+
 cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
-                             const void* vp, int64_t total_prefix_tokens, bool pdl, cudaStream_t s) {
+                             const void* vp, int64_t total_prefix_tokens, const void* k_pool,
+                             const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s) {
   if (p.n_items == 0) return cudaSuccess;
   if (p.head_dim != kD || total_prefix_tokens <= 0 || total_prefix_tokens > (int64_t)INT32_MAX)
     return cudaErrorInvalidValue;
@@ -823,7 +918,10 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, prefix_tc_kernel, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv);
+  if (p.fused && bm::smem_bytes<kD>(p.branch_rows, p.group, p.tail_chunk) > kOffBar) return cudaErrorInvalidValue;
+  return cudaLaunchKernelEx(&cfg, prefix_tc_kernel, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
+                            static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
+                            out, lse);
 }
 
 }  // namespace pad

@@ -41,7 +41,7 @@ class DeviceBatch:
         ws = B.pad_workspace_size(self.problem, w.prefix_len, w.event_video)
         if ws == 0:
             raise B.PadError(1, B.lib().pad_last_error().decode())
-        self.workspace = torch.empty(ws, dtype=torch.uint8, device=self.device)
+        self.workspace = torch.zeros(ws, dtype=torch.uint8, device=self.device)
         odt = torch.float32 if out_dtype == 0 else torch.bfloat16
         self.out = torch.empty((w.n_events, w.h_q, w.head_dim), dtype=odt, device=self.device)
         self.lse = torch.empty((w.n_events, w.h_q), dtype=torch.float32, device=self.device)
@@ -57,14 +57,23 @@ class DeviceBatch:
                                stream=stream)
         return self.plan
 
-    def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None):
-        """plan + append + attention; returns the plan (its new pages stay allocated)."""
+    def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None,
+                 one_call=False):
+        """plan + append + attention (two calls, or pad_decode_step with ``one_call``);
+        returns the plan (its new pages stay allocated)."""
         plan = self.plan_step(stream)
-        B.pad_kv_append(plan, self.k_new if k_new is None else k_new,
-                        self.v_new if v_new is None else v_new, self.k_pool, self.v_pool, stream)
-        B.pad_event_decode_attn(plan, self.q if q is None else q, self.k_prefix, self.v_prefix,
-                                self.k_pool, self.v_pool, self.out if out is None else out,
-                                self.lse if lse is None else lse, stream)
+        q = self.q if q is None else q
+        k_new = self.k_new if k_new is None else k_new
+        v_new = self.v_new if v_new is None else v_new
+        out = self.out if out is None else out
+        lse = self.lse if lse is None else lse
+        if one_call:
+            B.pad_decode_step(plan, q, k_new, v_new, self.k_prefix, self.v_prefix, self.k_pool,
+                              self.v_pool, out, lse, stream)
+        else:
+            B.pad_kv_append(plan, k_new, v_new, self.k_pool, self.v_pool, stream)
+            B.pad_event_decode_attn(plan, q, self.k_prefix, self.v_prefix, self.k_pool, self.v_pool,
+                                    out, lse, stream)
         return plan
 
     def release_new_pages(self, plan=None):

@@ -324,3 +324,150 @@ def test_device_bounds_check_reports_bad_page():
     db2 = DeviceBatch(_w([64], [1], [2]))
     p2 = db2.run_step()
     B.pad_device_status(p2)
+
+
+# ---------------------------------------------------------------------------
+# a4 + a5 inside the tensor-core prefix kernel
+# ---------------------------------------------------------------------------
+
+# (prefix lengths, events per video, branch lengths): 80 query rows; 140 rows with
+# G = 7, so that event 18's rows 126..132 straddle two 128-row groups; a single event
+_FUSED_CASES = {
+    "few_events": ([4000], [3], [5, 0, 17]),
+    "straddling_rows": ([3000], [20], [(7 * i) % 41 for i in range(20)]),
+    "one_event_long_branch": ([6000], [1], [300]),
+}
+
+
+@pytest.mark.parametrize("case", sorted(_FUSED_CASES))
+def test_fused_tail_and_separate_merge_both_match_oracle(case):
+    prefix, epv, lens = _FUSED_CASES[case]
+    w = _w(prefix, epv, lens, seed=21)
+    db_f, plan_f = run_full(w, flags=B.FLAG_PREFIX_TC | B.FLAG_FUSED_MERGE, what=f"{case} fused")
+    assert plan_f.info()["fused_tail"] == 1
+    db_s, plan_s = run_full(w, flags=B.FLAG_PREFIX_TC, what=f"{case} separate")
+    assert plan_s.info()["fused_tail"] == 0
+    d = (db_f.out - db_s.out).abs().max().item()
+    assert d <= 2e-3, f"fused and separate paths differ by {d:.3e}"
+
+
+def test_fused_tail_same_plan_relaunched():
+    """The split counters are zeroed again by the last task that reads them, so launching
+    one plan again without an append (as a timing loop or a graph replay of the attention
+    alone does) gives the same result; a second plan on the same workspace does too."""
+    w = _w([5000], [6], [3, 9, 0, 33, 12, 4], seed=5)
+    db, plan = run_full(w, flags=B.FLAG_PREFIX_TC | B.FLAG_FUSED_MERGE)
+    assert plan.info()["fused_tail"] == 1
+    o1 = db.out.clone()
+    for _ in range(3):
+        db.out.fill_(float("nan"))
+        B.pad_event_decode_attn(plan, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool, db.out, db.lse)
+        torch.cuda.synchronize()
+        B.pad_device_status(plan)
+        assert torch.equal(o1, db.out)
+    db.release_new_pages(plan)
+    db.run_step()
+    torch.cuda.synchronize()
+    B.pad_device_status(db.plan)
+    assert torch.equal(o1, db.out)
+
+
+def test_fused_tail_wait_runs_out_and_reports_timeout():
+    """A split counter that can never reach its target (set, after the append zeroed it,
+    to a count no launch reaches): the tail's bounded wait gives up, the status word says
+    PAD_ERR_DEVICE_TIMEOUT, and the context stays usable for the next plan."""
+    w = _w([3000], [4], [5, 0, 9, 2], seed=9)
+    db = DeviceBatch(w, flags=B.FLAG_PREFIX_TC | B.FLAG_FUSED_MERGE)
+    plan = db.plan_step()
+    info = plan.info()
+    assert info["fused_tail"] == 1
+    G = w.h_q // w.h_kv
+    n_cnt = w.h_kv * ((4 * G + 127) // 128)
+    off = info["workspace_bytes"] - (n_cnt * 4 + 255) // 256 * 256
+    B.pad_kv_append(plan, db.k_new, db.v_new, db.k_pool, db.v_pool)
+    db.workspace[off:off + n_cnt * 4].view(torch.int32).fill_(0x7000)
+    B.pad_event_decode_attn(plan, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool, db.out, db.lse)
+    with pytest.raises(B.PadError) as ei:
+        B.pad_device_status(plan)
+    assert ei.value.status == 6
+    db.release_new_pages(plan)
+    p2 = db.run_step()
+    B.pad_device_status(p2)
+    torch.cuda.synchronize()
+    ref_o, ref_lse = oracle.decode_step(w)
+    check_outputs(db.out.cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, "after a timed-out tail")
+
+
+# ---------------------------------------------------------------------------
+# pad_decode_step: a2 folded into the branch tasks
+# ---------------------------------------------------------------------------
+
+_ONE_CALL_CASES = {
+    "fused_tc": (lambda: _w([4000], [3], [5, 0, 17], seed=31), B.FLAG_PREFIX_TC | B.FLAG_FUSED_MERGE),
+    "separate_tc": (lambda: _w([4000], [3], [5, 0, 17], seed=31), B.FLAG_PREFIX_TC),
+    "separate_tc_ragged": (lambda: _w([300, 2000, 0, 900], [5, 2, 1, 7], [16, 0, 31, 47, 2, 15, 64, 3, 9, 33,
+                                                                          48, 0, 1, 16, 17], seed=32),
+                           B.FLAG_PREFIX_TC),
+    "mma": (lambda: synth.random_small(33, h_q=8, h_kv=2, max_events=6), B.FLAG_PREFIX_MMA),
+    "simt_d64": (synth.tiny, B.FLAG_PREFIX_SIMT),
+    "gqa_8k": (synth.gqa_8k, 0),
+    "long_branch": (lambda: _w([700], [2], [200, 129], seed=34), B.FLAG_PREFIX_TC),
+}
+
+
+@pytest.mark.parametrize("case", sorted(_ONE_CALL_CASES))
+def test_one_call_step_matches_two_calls(case):
+    """pad_decode_step against pad_kv_append + pad_event_decode_attn on the same inputs:
+    outputs, LSE, both pools and the page table bit-identical, and the oracle's
+    bookkeeping and outputs met."""
+    make, flags = _ONE_CALL_CASES[case]
+    w = make()
+    a = DeviceBatch(w, flags=flags)
+    pa = a.run_step()
+    b = DeviceBatch(w, flags=flags)
+    pb = b.run_step(one_call=True)
+    torch.cuda.synchronize()
+    B.pad_device_status(pa)
+    B.pad_device_status(pb)
+    assert pa.info()["fused_tail"] == pb.info()["fused_tail"]
+    assert torch.equal(a.out, b.out)
+    assert torch.equal(a.lse, b.lse)
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+    assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
+    assert torch.equal(a.page_table, b.page_table)
+    check_bookkeeping(b, w, pb)
+    ref_o, ref_lse = oracle.decode_step(w)
+    check_outputs(b.out.float().cpu().numpy(), b.lse.cpu().numpy(), ref_o, ref_lse, case)
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_one_call_steps_advance_like_a_generation_loop(fused):
+    """Three consecutive steps through pad_decode_step, each branch one token longer than
+    the last (new pages taken as lengths cross page boundaries): the pools and page table
+    after the loop equal those of the same loop through the two-call path."""
+    w = _w([2500], [4], [14, 15, 31, 0], seed=35)
+    flags = B.FLAG_PREFIX_TC | (B.FLAG_FUSED_MERGE if fused else 0)
+    a = DeviceBatch(w, flags=flags)
+    b = DeviceBatch(w, flags=flags)
+    lens = w.event_len.copy()
+    for step in range(3):
+        for db, one in ((a, False), (b, True)):
+            db.plan = B.pad_plan(db.problem, db.cache, w.prefix_len, w.event_video, lens,
+                                 page_table=db.page_table, max_pages=w.max_pages,
+                                 workspace=db.workspace, prefix_offset=w.prefix_offset)
+            if one:
+                B.pad_decode_step(db.plan, db.q, db.k_new, db.v_new, db.k_prefix, db.v_prefix,
+                                  db.k_pool, db.v_pool, db.out, db.lse)
+            else:
+                B.pad_kv_append(db.plan, db.k_new, db.v_new, db.k_pool, db.v_pool)
+                B.pad_event_decode_attn(db.plan, db.q, db.k_prefix, db.v_prefix, db.k_pool,
+                                        db.v_pool, db.out, db.lse)
+        torch.cuda.synchronize()
+        B.pad_device_status(a.plan)
+        B.pad_device_status(b.plan)
+        assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)
+        lens = lens + 1
+    assert torch.equal(a.page_table, b.page_table)
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+    assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
+    assert np.array_equal(a.cache.free_pages(), b.cache.free_pages())

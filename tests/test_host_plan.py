@@ -213,3 +213,35 @@ def test_release_new_pages_returns_exactly_the_plans_pages(padlib):
         plan.release_new_pages(cache)
     assert ei.value.status == 1
     assert cache.free_count == free_before + 3
+
+
+def test_fused_tail_decision(padlib):
+    """The tensor-core plan runs a4 + a5 inside the prefix kernel exactly when every
+    (event, kv-head) task can have a prefix CTA of its own and the prefix grid fits one
+    CTA per SM (the tail waits on other CTAs' splits, so the grid must be resident at
+    once), and only when PAD_FLAG_FUSED_MERGE asks for it."""
+    rng = np.random.default_rng(17)
+    seen = set()
+    for trial in range(80):
+        B_ = int(rng.integers(1, 6))
+        P = rng.integers(0, 30000, size=B_).astype(np.int32)
+        Ev = rng.integers(1, 24, size=B_)
+        ev_video = np.repeat(np.arange(B_, dtype=np.int32), Ev)
+        L = np.zeros(ev_video.size, dtype=np.int32)
+        sms = int(rng.integers(8, 160))
+        for flags in (0, B.FLAG_FUSED_MERGE, B.FLAG_PREFIX_TC | B.FLAG_FUSED_MERGE):
+            prob = B.make_problem(28, 4, 128, num_sms=sms, flags=flags)
+            info = B.pad_plan(prob, B.CacheState(4096), P, ev_video, L, max_pages=2, workspace=None).info()
+            sl = info["split_len"]
+            groups = max(-(-int(Ev[b]) * 7 // 128) for b in range(B_))
+            valid = sum(4 * (-(-int(P[b]) // sl)) * (-(-int(Ev[b]) * 7 // 128)) for b in range(B_))
+            want = (bool(flags & B.FLAG_FUSED_MERGE) and info["n_work_items"] > 0 and info["n_work_items"] * groups <= sms
+                    and int(Ev.sum()) * 4 <= valid)
+            assert info["fused_tail"] == int(want), (trial, flags)
+            seen.add(want)
+    assert seen == {True, False}
+    # the 64-dim problems never take the tensor-core path, hence never the fused tail
+    prob = B.make_problem(8, 2, 64, num_sms=152, flags=B.FLAG_FUSED_MERGE)
+    info = B.pad_plan(prob, B.CacheState(64), np.array([5000], np.int32), np.zeros(2, np.int32),
+                      np.zeros(2, np.int32), max_pages=2, workspace=None).info()
+    assert info["fused_tail"] == 0
