@@ -476,6 +476,10 @@ __global__ void __launch_bounds__(bm::kThreads) branch_merge_kernel(const __grid
                                                                     float* __restrict__ lse,
                                                                     int sch) {
   extern __shared__ __align__(16) unsigned char bm_raw[];
+  // The grid after this one may be scheduled now: in a one-call loop it is the next step's
+  // prefix kernel, which waits for this grid before it touches anything (an append kernel
+  // after it is launched without programmatic serialisation and waits in any case).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
   bm::run_task<D>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,

@@ -471,9 +471,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // One-call step (k_new set): this is the step's first kernel, launched so that it may
   // start while the grid before it (the previous step, or the caller's own kernel that
-  // wrote q) finishes.  Nothing is read or written before that grid has completed.
+  // wrote q) finishes.  Barrier set-up and TMEM allocation overlap that grid; every thread
+  // that touches global memory waits for it first (the Q loads, the first TMA issue),
+  // and the block barrier after them orders everything else, including the release of
+  // the grid behind this one.
   const bool one_call = p.k_new != nullptr;
-  if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
 
   const int item = blockIdx.x / n_groups;
   const int group = blockIdx.x - item * n_groups;
@@ -492,6 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // of head-dim half (w-4)/4.  Rows past R are zero.
   uint4 qv[8];
   if (warp >= 4) {
+    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
     const int lane_base = 32 * (warp & 3), half = (warp - 4) >> 2;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
@@ -530,6 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // barrier; the producer warps issue the rest.
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int t = 0; t < kStages && t < n_tiles; ++t) {
       mbar_expect_tx(&bars->kfull[t], kTileBytes);
       tma_load_3d(sbase + kOffK + t * kTileBytes, &tmK, 0, kvh, tok0 + t * kBN, &bars->kfull[t]);
