@@ -154,6 +154,67 @@ def event_rows(w, e, heads=None):
 
 
 # ---------------------------------------------------------------------------
+# Rotary position embedding at the shared per-step position (Sec. 3.4)
+# ---------------------------------------------------------------------------
+#
+# Sec. 3.4 gives the tokens generated at the same decoding step of different
+# branches identical position indices.  Positions enter attention through the
+# rotary embedding of q and of the new key (values are not rotated); the prefix
+# and earlier branch keys were rotated when they were written.  Reading (listed in
+# the design notes): the rotate-half form over the whole head dimension, with a
+# per-position table whose first D/2 columns hold cos(theta_i) and last D/2
+# columns sin(theta_i); for the caption tokens of the paper's backbone all
+# multimodal position components coincide, so this is the 1-D form.
+
+
+def bf16_round(x32: np.ndarray) -> np.ndarray:
+    """float32 values -> bf16 bit patterns (uint16), round to nearest, ties to even.
+
+    Finite inputs only (the rotated values of finite bf16 rows and a finite table)."""
+    u = np.ascontiguousarray(x32, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    lsb = (u >> np.uint64(16)) & np.uint64(1)
+    return ((u + np.uint64(0x7FFF) + lsb) >> np.uint64(16)).astype(np.uint16)
+
+
+def rope_rotate(x: np.ndarray, cs_row: np.ndarray) -> np.ndarray:
+    """Rotate the rows x[..., D] by the table row cs_row[D] (cos | sin halves).
+
+    Pairs (i, i + D/2): x'_i = x_i cos_i - x_{i+D/2} sin_i and
+    x'_{i+D/2} = x_{i+D/2} cos_i + x_i sin_i.  Works in the dtype of its inputs:
+    float64 for the exact rotation; float32 for the rounding of an unfused pass
+    (each product and each sum rounded to float32, no fused multiply-add).
+    """
+    D = x.shape[-1]
+    h = D // 2
+    c, s = cs_row[:h], cs_row[h:]
+    lo, hi = x[..., :h], x[..., h:]
+    out = np.empty_like(x)
+    out[..., :h] = lo * c - hi * s
+    out[..., h:] = hi * c + lo * s
+    return out
+
+
+def rope_bits(bits: np.ndarray, cs_row32: np.ndarray) -> np.ndarray:
+    """bf16 rows -> their rotation, as bf16 bits: widened exactly to float32,
+    rotated in float32 (rope_rotate), rounded once to bf16."""
+    x32 = bf16_to_f64(bits).astype(np.float32)
+    return bf16_round(rope_rotate(x32, np.asarray(cs_row32, dtype=np.float32)))
+
+
+def rotated_workload(w, positions, cos_sin32):
+    """The workload with q and k_new rotated at each event's position (what an
+    unfused RoPE pass would hand to attention and to the append)."""
+    import dataclasses
+    q = np.array(w.q, copy=True)
+    kn = np.array(w.k_new, copy=True)
+    for e in range(w.n_events):
+        row = cos_sin32[int(positions[e])]
+        q[e] = rope_bits(w.q[e], row)
+        kn[e] = rope_bits(w.k_new[e], row)
+    return dataclasses.replace(w, q=q, k_new=kn)
+
+
+# ---------------------------------------------------------------------------
 # Log-sum-exp merge of partial softmax states (the split-KV identity)
 # ---------------------------------------------------------------------------
 

@@ -134,6 +134,24 @@ class Workload:
                     total=prefix + branch + q + out + append)
 
 
+def rope_table(max_position: int, head_dim: int, theta: float = 1.0e6) -> np.ndarray:
+    """The rotary-embedding table a model keeps for its positions: fp32 [max_position,
+    head_dim], cos(pos * theta^(-2i/D)) in columns i < D/2 and the matching sin in columns
+    D/2 + i (computed in fp64, rounded once).  theta = 1e6 as in the paper's backbone
+    family; an input of the step, like the weights that produce q and k."""
+    h = head_dim // 2
+    inv = theta ** (-np.arange(h, dtype=np.float64) * 2.0 / head_dim)
+    ang = np.arange(max_position, dtype=np.float64)[:, None] * inv[None, :]
+    return np.concatenate([np.cos(ang), np.sin(ang)], axis=1).astype(np.float32)
+
+
+def step_positions(w) -> np.ndarray:
+    """Per-event position of this step's token: the video's prefix length plus the
+    branch's private length before the step, so branches at the same step share it
+    (Sec. 3.4).  int32 [n_events]."""
+    return (w.prefix_len[w.event_video].astype(np.int64) + w.event_len).astype(np.int32)
+
+
 def _normal(rng, shape):
     return rng.standard_normal(size=shape, dtype=np.float32)
 

@@ -291,3 +291,78 @@ def test_bf16_widening_is_exact():
     tie = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8], dtype=np.float32)
     np.testing.assert_array_equal(oracle.bf16_to_f64(synth.f32_to_bf16_bits(tie)),
                                   [1.0, 1.0 + 2.0 ** -6])
+
+
+# ---------------------------------------------------------------------------
+# Rotary embedding at the shared per-step position (Sec. 3.4)
+# ---------------------------------------------------------------------------
+
+def _exact_row(pos, D, theta=1.0e6):
+    h = D // 2
+    ang = pos * theta ** (-np.arange(h) * 2.0 / D)
+    return np.concatenate([np.cos(ang), np.sin(ang)])
+
+
+def test_bf16_round_matches_torch_and_ties_to_even():
+    rng = np.random.default_rng(3)
+    x = (rng.standard_normal(4096) * np.exp(rng.uniform(-20, 20, 4096))).astype(np.float32)
+    want = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(oracle.bf16_round(x), want)
+    # halfway between 1.0 (0x3F80) and the next bf16 up: ties to the even pattern
+    assert oracle.bf16_round(np.array([1.0 + 2.0 ** -8], np.float32))[0] == 0x3F80
+    assert oracle.bf16_round(np.array([1.0 + 3 * 2.0 ** -8], np.float32))[0] == 0x3F82
+
+
+def test_rope_is_a_rotation_of_each_pair():
+    """D = 2 closed form, and the norm of every (i, i + D/2) pair kept (fp64)."""
+    th = 0.7
+    x = np.array([[3.0, -2.0]])
+    got = oracle.rope_rotate(x, np.array([math.cos(th), math.sin(th)]))
+    want = np.array([[3 * math.cos(th) + 2 * math.sin(th), -2 * math.cos(th) + 3 * math.sin(th)]])
+    assert np.allclose(got, want, rtol=0, atol=1e-15)
+    rng = np.random.default_rng(4)
+    D = 16
+    x = rng.standard_normal((5, D))
+    y = oracle.rope_rotate(x, _exact_row(1234, D))
+    n0 = x[:, :D // 2] ** 2 + x[:, D // 2:] ** 2
+    n1 = y[:, :D // 2] ** 2 + y[:, D // 2:] ** 2
+    assert np.allclose(n0, n1, rtol=1e-13, atol=0)
+
+
+def test_rope_scores_depend_on_relative_position_only():
+    """<R(m) q, R(n) k> = <R(m+t) q, R(n+t) k> (fp64, exact tables), and rotations
+    compose: R(b) R(a) x = R(a+b) x."""
+    rng = np.random.default_rng(5)
+    D = 32
+    q, k = rng.standard_normal(D), rng.standard_normal(D)
+    for m, n, t in [(10, 3, 7), (0, 500, 1234), (40000, 39000, 17)]:
+        a = oracle.rope_rotate(q, _exact_row(m, D)) @ oracle.rope_rotate(k, _exact_row(n, D))
+        b = oracle.rope_rotate(q, _exact_row(m + t, D)) @ oracle.rope_rotate(k, _exact_row(n + t, D))
+        assert abs(a - b) <= 1e-9 * (1 + abs(a))
+    x = rng.standard_normal(D)
+    two = oracle.rope_rotate(oracle.rope_rotate(x, _exact_row(300, D)), _exact_row(77, D))
+    assert np.allclose(two, oracle.rope_rotate(x, _exact_row(377, D)), rtol=0, atol=1e-12)
+
+
+def test_rope_bits_identity_at_position_zero_and_float32_rounding():
+    """Position 0 (cos 1, sin 0) gives back the input bits; elsewhere the float32
+    rotation rounded once to bf16 is within one bf16 step of the exact rotation of the
+    same (widened) inputs and table."""
+    rng = np.random.default_rng(6)
+    D = 128
+    bits = synth.f32_to_bf16_bits(rng.standard_normal((7, D)).astype(np.float32))
+    table = synth.rope_table(50000, D)
+    assert np.array_equal(oracle.rope_bits(bits, table[0]), bits)
+    for pos in (1, 8191, 32801, 49999):
+        got = oracle.bf16_to_f64(oracle.rope_bits(bits, table[pos]))
+        exact = oracle.rope_rotate(oracle.bf16_to_f64(bits), table[pos].astype(np.float64))
+        step = np.maximum(np.abs(exact), 2.0 ** -126) * 2.0 ** -7
+        assert np.all(np.abs(got - exact) <= step)
+
+
+def test_rope_table_closed_form():
+    t = synth.rope_table(40000, 128)
+    for pos, i in [(0, 0), (1, 0), (1, 63), (32768, 5), (39999, 40)]:
+        ang = pos * 1.0e6 ** (-2.0 * i / 128)
+        assert t[pos, i] == np.float32(math.cos(ang))
+        assert t[pos, 64 + i] == np.float32(math.sin(ang))
