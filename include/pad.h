@@ -176,6 +176,25 @@ pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page);
  * timing loop, or a step that is abandoned.  PAD_ERR_INVALID_ARG if a page is not in use. */
 pad_status pad_plan_release_new_pages(const pad_plan_t* plan, pad_cache_state* cache);
 
+/* Rotary embedding fused into the step (host; before the plan's launches).  Sec. 3.4 gives
+ * the tokens that different branches generate at the same decoding step the same position
+ * index; positions[e] is the position of event e's token at this step (the caller passes
+ * that shared value), and the step's kernels rotate q (every head of event e) and k_new[e]
+ * at it where they load them, instead of a separate rotation pass.  V is not rotated; the
+ * prefix and earlier branch keys are expected rotated already (they were, when written).
+ * Rotate-half form over the whole head dimension:
+ *   x'_i = x_i cos_i - x_{i+D/2} sin_i,   x'_{i+D/2} = x_{i+D/2} cos_i + x_i sin_i,
+ * each product and sum rounded to fp32 and the result to bf16 (the rotated key is what the
+ * pool receives), exactly as an unfused pass computing in fp32 would store it.
+ *   positions  [n_events] host, each in [0, max_position)
+ *   cos_sin    [max_position, head_dim] device fp32, 16-byte aligned: cos_i in columns
+ *              i < D/2, sin_i in columns D/2 + i (the model's own table; read, not owned)
+ * PAD_ERR_INVALID_ARG (nothing changes) for a NULL or misaligned table, or a position out
+ * of range.  Applies to pad_decode_step, pad_kv_append + pad_event_decode_attn and the
+ * static variant alike. */
+pad_status pad_plan_set_rope(pad_plan_t* plan, const int32_t* positions, const float* cos_sin,
+                             int32_t max_position);
+
 /* Summary of a plan (host): the split-KV decomposition chosen for the prefix pass. */
 typedef struct {
   int32_t n_videos;

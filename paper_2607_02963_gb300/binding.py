@@ -66,6 +66,7 @@ _SIGNATURES = {
                            POINTER(c_void_p)]),
     "pad_plan_new_pages": (c_int32, [c_void_p, _I32P]),
     "pad_plan_release_new_pages": (c_int32, [c_void_p, c_void_p]),
+    "pad_plan_set_rope": (c_int32, [c_void_p, _I32P, c_void_p, c_int32]),
     "pad_plan_get_info": (c_int32, [c_void_p, POINTER(PlanInfo)]),
     "pad_plan_destroy": (c_int32, [c_void_p]),
     "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -204,6 +205,13 @@ class Plan:
     def release_new_pages(self, cache: "CacheState"):
         """Give the pages this plan took back to ``cache`` (pad_plan_release_new_pages)."""
         _check(lib().pad_plan_release_new_pages(self._h, cache.handle))
+
+    def set_rope(self, positions, cos_sin, max_position: int = None):
+        """Rotate q and k_new at these per-event positions in the step's kernels
+        (pad_plan_set_rope); ``cos_sin`` is the device fp32 table [max_position, D]."""
+        pos = np.ascontiguousarray(positions, dtype=np.int32)
+        n = int(cos_sin.shape[0]) if max_position is None else int(max_position)
+        _check(lib().pad_plan_set_rope(self._h, pos.ctypes.data_as(_I32P), _ptr(cos_sin), n))
 
     def info(self) -> dict:
         i = PlanInfo()

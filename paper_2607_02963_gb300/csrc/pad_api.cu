@@ -110,6 +110,7 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   if (n_videos > 0 && !prefix_len) return fail(PAD_ERR_INVALID_ARG, "prefix_len is NULL");
   if (n_events > 0 && !event_video) return fail(PAD_ERR_INVALID_ARG, "event_video is NULL");
   if (n_events > 0 && n_videos == 0) return fail(PAD_ERR_INVALID_ARG, "events without videos");
+  if (n_videos > 65535) return fail(PAD_ERR_UNSUPPORTED, "at most 65535 videos per step; got %d", n_videos);
   L->group = prob->h_q / prob->h_kv;
   L->n_sms = n_sms;
   L->ev_first.assign(n_videos, 0);
@@ -129,8 +130,11 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
     prev = v;
   }
   int max_rows = 0;
-  for (int b = 0; b < n_videos; ++b)
+  for (int b = 0; b < n_videos; ++b) {
+    if (L->ev_count[b] > 65535)
+      return fail(PAD_ERR_UNSUPPORTED, "at most 65535 events per video; video %d has %d", b, L->ev_count[b]);
     if (L->ev_count[b] > 0) max_rows = std::max(max_rows, L->ev_count[b] * L->group);
+  }
   L->max_rows = max_rows;
 
   // Prefix kernel: forced by a flag, else the tensor-core path for head_dim 128 and the
@@ -399,6 +403,7 @@ struct pad_plan_t {
                                     // when they do not fit the launch parameters
   std::vector<uint8_t> param_image; // videos | events | items, packed, for KParams::img
   int32_t img_videos = 0, img_events = 0, img_items = 0, img_tasks = 0;
+  const float* rope_cs = nullptr;   // rotary table (pad_plan_set_rope), else NULL
   uint64_t gen = 0;                 // generation tagging this plan's device errors
   ~pad_plan_t() { image_release(image); }
 };
@@ -589,10 +594,11 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   int cursor = 0;
   for (int e = 0; e < n_events; ++e) {
     PadEventDesc& d = evs[e];
-    d.video = event_video[e];
+    d.video = (uint16_t)event_video[e];
     d.len = event_len[e];
-    d.local = e - L.ev_first[d.video];
+    d.local = (uint16_t)(e - L.ev_first[event_video[e]]);
     d.new_page = -1;
+    d.pos = 0;
     if (event_len[e] % ps == 0) {
       const int pg = cache->next_free(cursor);
       // need <= free_count guarantees a page exists
@@ -659,6 +665,31 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   return PAD_OK;
 }
 
+pad_status pad_plan_set_rope(pad_plan_t* plan, const int32_t* positions, const float* cos_sin,
+                             int32_t max_position) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (!cos_sin) return fail(PAD_ERR_INVALID_ARG, "cos_sin is NULL");
+  if (!aligned16(cos_sin)) return fail(PAD_ERR_INVALID_ARG, "cos_sin must be 16-byte aligned");
+  if (max_position <= 0) return fail(PAD_ERR_INVALID_ARG, "max_position must be > 0");
+  if (plan->n_events > 0 && !positions) return fail(PAD_ERR_INVALID_ARG, "positions is NULL");
+  for (int e = 0; e < plan->n_events; ++e)
+    if (positions[e] < 0 || positions[e] >= max_position)
+      return fail(PAD_ERR_INVALID_ARG, "positions[%d]=%d outside [0, %d)", e, positions[e], max_position);
+  // every copy of the event descriptors: the host image, the launch-parameter image and
+  // the page-locked image (no launch of this plan has read them yet)
+  auto set = [&](uint8_t* base) {
+    auto* ev = reinterpret_cast<PadEventDesc*>(base);
+    for (int e = 0; e < plan->n_events; ++e) ev[e].pos = positions[e];
+  };
+  if (plan->n_events > 0) {
+    set(plan->host_image.data() + plan->lay.off_events);
+    if (!plan->param_image.empty()) set(plan->param_image.data() + plan->img_events);
+    if (plan->image) set(static_cast<uint8_t*>(plan->image->host) + plan->lay.off_events);
+  }
+  plan->rope_cs = cos_sin;
+  return PAD_OK;
+}
+
 pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page) {
   if (!plan || (!new_page && plan->n_events > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
   std::copy(plan->new_pages.begin(), plan->new_pages.end(), new_page);
@@ -722,6 +753,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.img_tasks = plan->img_tasks;
   p.k_new = nullptr;
   p.v_new = nullptr;
+  p.rope_cs = plan->rope_cs;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
@@ -982,6 +1014,7 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.img_n = 0;
   p.k_new = nullptr;
   p.v_new = nullptr;
+  p.rope_cs = plan->rope_cs;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   auto* ws = static_cast<uint8_t*>(scratch);

@@ -152,7 +152,7 @@ struct SyncNamed {
 // One task.  `tid` in [0, 256); `smem` 16-byte aligned, smem_bytes<D>(branch_rows, G, sch)
 // long.  `partials_ready()` is called by all 256 threads and returns false if the
 // partials cannot be read (then only the status word is written).
-template <int D, class Sync, class Ready>
+template <int D, bool ROPE, class Sync, class Ready>
 __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* __restrict__ q,
                                          const __nv_bfloat16* __restrict__ kpool,
                                          const __nv_bfloat16* __restrict__ vpool, void* __restrict__ out,
@@ -198,10 +198,16 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   };
   const int nv0 = min(nkr, nk);
   if (tid < nkr) S.page[tid] = tid < nv0 ? page_of(tid) : -1;
+  // (ROPE: the plan carries positions; a separate instantiation keeps the plain one lean)
+  const float* cs = ROPE ? p.rope_cs + (size_t)ev.pos * D : nullptr;
   for (int i = tid; i < 16 * CH; i += NT) {
     const int g = i / CH, c = i - (i / CH) * CH;
     const bool in = g < G;
-    cp_async16(&S.q[g][c * 8], q + ((size_t)e * p.h_q + kvh * G + (in ? g : 0)) * D + c * 8, in);
+    const __nv_bfloat16* qr = q + ((size_t)e * p.h_q + kvh * G + (in ? g : 0)) * D;
+    if (ROPE)  // rotated here (rows past G are zero)
+      *reinterpret_cast<uint4*>(&S.q[g][c * 8]) = in ? rope_chunk8(qr, D, c * 8, cs) : make_uint4(0u, 0u, 0u, 0u);
+    else
+      cp_async16(&S.q[g][c * 8], qr + c * 8, in);
   }
   for (int i = tid; i < G * D; i += NT) S.ob[i / D][i % D] = 0.f;
   if (tid < 16) {
@@ -218,7 +224,11 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
       const int pg = k < nv ? S.page[k] : -1;
       const bool in = pg >= 0;
       if (knew != nullptr && r0 + k == len) {
-        cp_async16(&sK[k][c * 8], knew + new_row + c * 8, in);
+        if (ROPE)
+          *reinterpret_cast<uint4*>(&sK[k][c * 8]) = in ? rope_chunk8(knew + new_row, D, c * 8, cs)
+                                                        : make_uint4(0u, 0u, 0u, 0u);
+        else
+          cp_async16(&sK[k][c * 8], knew + new_row + c * 8, in);
         cp_async16(&sV[k][c * 8], vnew + new_row + c * 8, in);
         continue;
       }
@@ -235,7 +245,8 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
         const int c = tid % CH;
         const bool isv = tid >= CH;
         const size_t dst = (((size_t)pg * p.h_kv + kvh) * ps + (len % ps)) * D + c * 8;
-        const uint4 v = *reinterpret_cast<const uint4*>((isv ? vnew : knew) + new_row + c * 8);
+        const uint4 v = (ROPE && !isv) ? rope_chunk8(knew + new_row, D, c * 8, cs)
+                                                : *reinterpret_cast<const uint4*>((isv ? vnew : knew) + new_row + c * 8);
         *reinterpret_cast<uint4*>(const_cast<__nv_bfloat16*>(isv ? vpool : kpool) + dst) = v;
       }
     }

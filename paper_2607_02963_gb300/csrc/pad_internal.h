@@ -15,6 +15,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "../../include/pad.h"
@@ -64,10 +65,11 @@ struct PadVideoDesc {
 static_assert(sizeof(PadVideoDesc) == 32, "video desc is 32 bytes");
 
 struct PadEventDesc {
-  int32_t video;
   int32_t len;          // private length before this step
   int32_t new_page;     // page taken this step, or -1
-  int32_t local;        // index of the event within its video
+  int32_t pos;          // position of this step's token (rotary table row; 0 without RoPE)
+  uint16_t video;
+  uint16_t local;       // index of the event within its video
 };
 static_assert(sizeof(PadEventDesc) == 16, "event desc is 16 bytes");
 
@@ -113,6 +115,9 @@ struct KParams {
   // writes it into the pools itself (a2 folded into a4; no append kernel runs).
   const void* k_new;
   const void* v_new;
+  // Rotary table [max_position, head_dim] fp32 (cos | sin halves) when the plan carries
+  // positions (pad_plan_set_rope): q and the new key are rotated where they are loaded.
+  const float* rope_cs;
   const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
   // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
   // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by
@@ -143,6 +148,59 @@ __device__ __forceinline__ const PadWorkItem* plan_items(const KParams& p) {
 }
 __device__ __forceinline__ const int32_t* plan_tasks(const KParams& p) {
   return p.img_n > 0 ? reinterpret_cast<const int32_t*>(p.img + p.img_tasks) : p.tasks;
+}
+
+// Rotary embedding, rotate-half form (the position rule of Sec. 3.4 decides `cs`, the
+// table row of the token's position: cos in columns i < D/2, sin in D/2 + i).  Element
+// d < D/2 becomes x_d cos_d - x_{d+D/2} sin_d, element D/2 + i becomes
+// x_{D/2+i} cos_i + x_i sin_i; each product and sum is rounded to fp32 (no contraction)
+// and the result once to bf16, as an unfused rotation pass would store it.
+__device__ __forceinline__ float rope_one(float own, float partner, float c, float s, bool low) {
+  return low ? __fsub_rn(__fmul_rn(own, c), __fmul_rn(partner, s))
+             : __fadd_rn(__fmul_rn(own, c), __fmul_rn(partner, s));
+}
+// Elements d0 .. d0+7 (d0 a multiple of 8) of a bf16 row of length D, as packed bf16.
+__device__ __forceinline__ uint4 rope_chunk8(const __nv_bfloat16* row, int D, int d0, const float* cs) {
+  const int h = D >> 1;
+  const bool low = d0 < h;
+  const int i0 = low ? d0 : d0 - h;
+  const uint4 xa = *reinterpret_cast<const uint4*>(row + d0);
+  const uint4 xb = *reinterpret_cast<const uint4*>(row + (low ? d0 + h : i0));
+  const float4 c0 = *reinterpret_cast<const float4*>(cs + i0), c1 = *reinterpret_cast<const float4*>(cs + i0 + 4);
+  const float4 s0 = *reinterpret_cast<const float4*>(cs + h + i0),
+               s1 = *reinterpret_cast<const float4*>(cs + h + i0 + 4);
+  const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+  const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+  const uint32_t a[4] = {xa.x, xa.y, xa.z, xa.w}, b[4] = {xb.x, xb.y, xb.z, xb.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&a[j]));
+    const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&b[j]));
+    const __nv_bfloat162 r = __floats2bfloat162_rn(rope_one(x.x, y.x, c[2 * j], s[2 * j], low),
+                                                   rope_one(x.y, y.y, c[2 * j + 1], s[2 * j + 1], low));
+    o[j] = *reinterpret_cast<const uint32_t*>(&r);
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+// Elements d, d+1 (d even) as packed bf16.
+__device__ __forceinline__ uint32_t rope_pair(const __nv_bfloat16* row, int D, int d, const float* cs) {
+  const int h = D >> 1;
+  const bool low = d < h;
+  const int i0 = low ? d : d - h;
+  const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(row + d));
+  const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(row + (low ? d + h : i0)));
+  const float2 c = *reinterpret_cast<const float2*>(cs + i0), s = *reinterpret_cast<const float2*>(cs + h + i0);
+  const __nv_bfloat162 r = __floats2bfloat162_rn(rope_one(x.x, y.x, c.x, s.x, low), rope_one(x.y, y.y, c.y, s.y, low));
+  return *reinterpret_cast<const uint32_t*>(&r);
+}
+// Element d, widened back to fp32 after the bf16 rounding.
+__device__ __forceinline__ float rope_elem(const __nv_bfloat16* row, int D, int d, const float* cs) {
+  const int h = D >> 1;
+  const bool low = d < h;
+  const int i = low ? d : d - h;
+  const float v = rope_one(__bfloat162float(row[d]), __bfloat162float(row[low ? d + h : i]), cs[i], cs[h + i], low);
+  return __bfloat162float(__float2bfloat16_rn(v));
 }
 #endif
 

@@ -136,7 +136,10 @@ __global__ void append_kernel(const __grid_constant__ KParams p, const uint4* __
   }
   const size_t dst = (((size_t)page * p.h_kv + h) * p.page_size + slot) * chunks + c;
   const size_t src = ((size_t)e * p.h_kv + h) * chunks + c;
-  k_pool[dst] = k_new[src];
+  k_pool[dst] = p.rope_cs != nullptr
+                    ? rope_chunk8(reinterpret_cast<const __nv_bfloat16*>(k_new + (src - c)), p.head_dim, 8 * c,
+                                  p.rope_cs + (size_t)ev.pos * p.head_dim)
+                    : k_new[src];
   v_pool[dst] = v_new[src];
 }
 
@@ -166,7 +169,12 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(const __grid_constant_
   for (int i = threadIdx.x; i < MAXR * D; i += blockDim.x) {
     int r = i / D, d = i - r * D;
     float v = 0.f;
-    if (r < R) v = __bfloat162float(q_row(p, it.first_event, q, kvh, r)[d]);
+    if (r < R) {
+      const __nv_bfloat16* qr = q_row(p, it.first_event, q, kvh, r);
+      v = p.rope_cs != nullptr
+              ? rope_elem(qr, D, d, p.rope_cs + (size_t)plan_events(p)[it.first_event + r / p.group].pos * D)
+              : __bfloat162float(qr[d]);
+    }
     sq[r][d] = v;
     so[r][d] = 0.f;
   }
@@ -319,13 +327,26 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
   {
     const __nv_bfloat16* ql = rlo < R ? q_row(p, it.first_event, q, kvh, rlo) : nullptr;
     const __nv_bfloat16* qh = rhi < R ? q_row(p, it.first_event, q, kvh, rhi) : nullptr;
+    if (p.rope_cs != nullptr) {
+      const float* cl = ql ? p.rope_cs + (size_t)plan_events(p)[it.first_event + rlo / p.group].pos * D : nullptr;
+      const float* ch = qh ? p.rope_cs + (size_t)plan_events(p)[it.first_event + rhi / p.group].pos * D : nullptr;
 #pragma unroll
-    for (int kk = 0; kk < KSTEPS; ++kk) {
-      const int c = kk * 16 + 2 * t4;
-      qa[kk][0] = ql ? *reinterpret_cast<const uint32_t*>(ql + c) : 0u;
-      qa[kk][1] = qh ? *reinterpret_cast<const uint32_t*>(qh + c) : 0u;
-      qa[kk][2] = ql ? *reinterpret_cast<const uint32_t*>(ql + c + 8) : 0u;
-      qa[kk][3] = qh ? *reinterpret_cast<const uint32_t*>(qh + c + 8) : 0u;
+      for (int kk = 0; kk < KSTEPS; ++kk) {
+        const int c = kk * 16 + 2 * t4;
+        qa[kk][0] = ql ? rope_pair(ql, D, c, cl) : 0u;
+        qa[kk][1] = qh ? rope_pair(qh, D, c, ch) : 0u;
+        qa[kk][2] = ql ? rope_pair(ql, D, c + 8, cl) : 0u;
+        qa[kk][3] = qh ? rope_pair(qh, D, c + 8, ch) : 0u;
+      }
+    } else {
+#pragma unroll
+      for (int kk = 0; kk < KSTEPS; ++kk) {
+        const int c = kk * 16 + 2 * t4;
+        qa[kk][0] = ql ? *reinterpret_cast<const uint32_t*>(ql + c) : 0u;
+        qa[kk][1] = qh ? *reinterpret_cast<const uint32_t*>(qh + c) : 0u;
+        qa[kk][2] = ql ? *reinterpret_cast<const uint32_t*>(ql + c + 8) : 0u;
+        qa[kk][3] = qh ? *reinterpret_cast<const uint32_t*>(qh + c + 8) : 0u;
+      }
     }
   }
 
@@ -467,8 +488,8 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
 // programmatic dependent launch: its griddepcontrol.wait covers the prefix grid, so the
 // split partials are complete once it returns.
 // ---------------------------------------------------------------------------
-template <int D>
-__global__ void __launch_bounds__(bm::kThreads) branch_merge_kernel(const __grid_constant__ KParams p,
+template <int D, bool ROPE>
+__global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __grid_constant__ KParams p,
                                                                     const __nv_bfloat16* __restrict__ q,
                                                                     const __nv_bfloat16* __restrict__ kpool,
                                                                     const __nv_bfloat16* __restrict__ vpool,
@@ -482,7 +503,7 @@ __global__ void __launch_bounds__(bm::kThreads) branch_merge_kernel(const __grid
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
-  bm::run_task<D>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,
+  bm::run_task<D, ROPE>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,
                   [] { return true; });
 }
 
@@ -578,9 +599,10 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(branch_merge_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kMaxSmem);
-    if (e != cudaSuccess) return e;
+    for (auto fn : {branch_merge_kernel<D, false>, branch_merge_kernel<D, true>}) {
+      cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+      if (e != cudaSuccess) return e;
+    }
     configured[dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
@@ -593,7 +615,8 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, branch_merge_kernel<D>, p, static_cast<const __nv_bfloat16*>(q),
+  return cudaLaunchKernelEx(&cfg, p.rope_cs != nullptr ? branch_merge_kernel<D, true> : branch_merge_kernel<D, false>,
+                            p, static_cast<const __nv_bfloat16*>(q),
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse, sch);
 }

@@ -456,6 +456,7 @@ __device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadV
   return bm::SyncNamed{1}.all(good);
 }
 
+template <bool ROPE>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -504,8 +505,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (qrow < R) {
         const int el = qrow / p.group;
         const int gh = qrow - el * p.group;
-        qv[i] = __ldg(reinterpret_cast<const uint4*>(
-            q + ((size_t)(it.first_event + el) * p.h_q + kvh * p.group + gh) * kD + half * 64 + (idx & 7) * 8));
+        const __nv_bfloat16* qr = q + ((size_t)(it.first_event + el) * p.h_q + kvh * p.group + gh) * kD;
+        const int d0 = half * 64 + (idx & 7) * 8;
+        if (ROPE)
+          qv[i] = rope_chunk8(qr, kD, d0, p.rope_cs + (size_t)plan_events(p)[it.first_event + el].pos * kD);
+        else
+          qv[i] = __ldg(reinterpret_cast<const uint4*>(qr + d0));
       }
     }
   }
@@ -788,7 +793,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int task = plan_tasks(p)[blockIdx.x];
         if (task >= 0) {
           const int te = task / p.h_kv, th = task - (task / p.h_kv) * p.h_kv;
-          bm::run_task<kD>(p, q, kpool, vpool, out, lse, te, th, (int)threadIdx.x - 128, smem, p.tail_chunk, sy,
+          bm::run_task<kD, ROPE>(p, q, kpool, vpool, out, lse, te, th, (int)threadIdx.x - 128, smem, p.tail_chunk, sy,
                            false, [&]() {
                              const PadEventDesc ev = plan_events(p)[te];
                              const PadVideoDesc vd = plan_videos(p)[ev.video];
@@ -906,9 +911,10 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   if (!get_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(prefix_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e != cudaSuccess) return e;
+    for (auto fn : {prefix_tc_kernel<false>, prefix_tc_kernel<true>}) {
+      cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+      if (e != cudaSuccess) return e;
+    }
     configured[dev] = true;
   }
   const int n_groups = (max_rows + 127) / 128;
@@ -923,7 +929,7 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (p.fused && bm::smem_bytes<kD>(p.branch_rows, p.group, p.tail_chunk) > kOffBar) return cudaErrorInvalidValue;
-  return cudaLaunchKernelEx(&cfg, prefix_tc_kernel, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
+  return cudaLaunchKernelEx(&cfg, p.rope_cs != nullptr ? prefix_tc_kernel<true> : prefix_tc_kernel<false>, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse);
 }

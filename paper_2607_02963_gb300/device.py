@@ -46,6 +46,13 @@ class DeviceBatch:
         self.out = torch.empty((w.n_events, w.h_q, w.head_dim), dtype=odt, device=self.device)
         self.lse = torch.empty((w.n_events, w.h_q), dtype=torch.float32, device=self.device)
         self.plan = None
+        self.rope = None           # (positions [E] host int32, cos_sin device fp32 [P, D])
+
+    def set_rope(self, positions, table):
+        """Rotate q and k_new at ``positions`` with the fp32 table ``table`` (numpy
+        [max_position, D]) in every later step."""
+        self.rope = (np.ascontiguousarray(positions, dtype=np.int32),
+                     torch.from_numpy(np.ascontiguousarray(table, dtype=np.float32)).to(self.device))
 
     def plan_step(self, stream=None):
         w = self.w
@@ -55,6 +62,8 @@ class DeviceBatch:
                                page_table=self.page_table, max_pages=w.max_pages,
                                workspace=self.workspace, prefix_offset=w.prefix_offset,
                                stream=stream)
+        if self.rope is not None:
+            self.plan.set_rope(self.rope[0], self.rope[1])
         return self.plan
 
     def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None,

@@ -471,3 +471,51 @@ def test_one_call_steps_advance_like_a_generation_loop(fused):
     assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
     assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
     assert np.array_equal(a.cache.free_pages(), b.cache.free_pages())
+
+
+# ---------------------------------------------------------------------------
+# Rotary embedding fused into the step (same position for a step's branches, Sec. 3.4)
+# ---------------------------------------------------------------------------
+
+_ROPE_CASES = {
+    "tc_gqa_8k": (synth.gqa_8k, 0),
+    "tc_ragged": (lambda: _w([300, 2000, 0, 900], [5, 2, 1, 7], [16, 0, 31, 47, 2, 15, 64, 3, 9, 33,
+                                                               48, 0, 1, 16, 17], seed=42), B.FLAG_PREFIX_TC),
+    "mma_small": (lambda: synth.random_small(41, h_q=8, h_kv=2, max_events=5), B.FLAG_PREFIX_MMA),
+    "simt_tiny_d64": (synth.tiny, 0),
+}
+
+
+@pytest.mark.parametrize("one_call", [False, True])
+@pytest.mark.parametrize("case", sorted(_ROPE_CASES))
+def test_rope_step_matches_oracle(case, one_call):
+    """q and k_new rotated at each event's step position inside the step's kernels: the
+    pools hold the rotated new keys bit for bit, and the outputs match the oracle run on
+    the rotated inputs."""
+    make, flags = _ROPE_CASES[case]
+    w = make()
+    pos = synth.step_positions(w)
+    table = synth.rope_table(int(pos.max()) + 8, w.head_dim)
+    db = DeviceBatch(w, flags=flags)
+    db.set_rope(pos, table)
+    plan = db.run_step(one_call=one_call)
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    wr = oracle.rotated_workload(w, pos, table)
+    check_bookkeeping(db, wr, plan)
+    ref_o, ref_lse = oracle.decode_step(wr)
+    check_outputs(db.out.float().cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, f"{case} rope")
+
+
+def test_rope_at_position_zero_changes_nothing():
+    """A table row of cos 1, sin 0 leaves q and k_new as they are: bit-identical to the
+    step without a rotation."""
+    w = _w([3000], [3], [5, 0, 17], seed=43)
+    a = DeviceBatch(w)
+    a.run_step(one_call=True)
+    b = DeviceBatch(w)
+    b.set_rope(np.zeros(w.n_events, np.int32), synth.rope_table(4, w.head_dim))
+    b.run_step(one_call=True)
+    torch.cuda.synchronize()
+    assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))

@@ -245,3 +245,20 @@ def test_fused_tail_decision(padlib):
     info = B.pad_plan(prob, B.CacheState(64), np.array([5000], np.int32), np.zeros(2, np.int32),
                       np.zeros(2, np.int32), max_pages=2, workspace=None).info()
     assert info["fused_tail"] == 0
+
+
+def test_set_rope_validates_positions_and_table(padlib):
+    import torch
+    prob = B.make_problem(8, 2, 128, num_sms=152)
+    cache = B.CacheState(64)
+    plan = B.pad_plan(prob, cache, np.array([500], np.int32), np.zeros(3, np.int32),
+                      np.array([0, 3, 16], np.int32), max_pages=4, workspace=None)
+    table = torch.zeros((100, 128), dtype=torch.float32)
+    plan.set_rope(np.array([0, 50, 99], np.int32), table)
+    for bad in ([0, 50, 100], [-1, 0, 0]):
+        with pytest.raises(B.PadError) as ei:
+            plan.set_rope(np.array(bad, np.int32), table)
+        assert ei.value.status == 1
+    with pytest.raises(B.PadError) as ei:
+        B._check(B.lib().pad_plan_set_rope(plan.handle, np.zeros(3, np.int32).ctypes.data_as(B._I32P), None, 100))
+    assert ei.value.status == 1
