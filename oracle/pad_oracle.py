@@ -49,17 +49,28 @@ def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
 # The explicit event-factorized mask (Sec. 3.4, Fig. 3)
 # ---------------------------------------------------------------------------
 
-def event_mask(prefix_len: int, branch_lens) -> np.ndarray:
+def event_mask(prefix_len: int, branch_lens, self_g=None) -> np.ndarray:
     """Mask M[e, k] over the key sequence [prefix ; branch 1 ; ... ; branch E].
 
     M[e, k] is True when key k lies in the shared prefix (P and the planning
     tokens) or inside branch e's own block; keys of every other branch are
     False.  ``branch_lens[e]`` counts branch e's keys at this step (L_e + 1).
+
+    ``self_g = (K, g_index)`` selects the "self G-token only" structure of the
+    attention ablation (Tab. 8): the prefix ends with the planning tokens
+    G^1..G^K and S (Sec. 3.3), and event e sees only G^(g_index[e] + 1) of them,
+    besides P, S and its own branch.
     """
     branch_lens = [int(x) for x in branch_lens]
     n_keys = prefix_len + sum(branch_lens)
     M = np.zeros((len(branch_lens), n_keys), dtype=bool)
     M[:, :prefix_len] = True
+    if self_g is not None:
+        K, g_index = int(self_g[0]), [int(x) for x in self_g[1]]
+        g0 = prefix_len - 1 - K                      # G^1 .. G^K, then S at prefix_len - 1
+        for e in range(len(branch_lens)):
+            M[e, g0:g0 + K] = False
+            M[e, g0 + g_index[e]] = True
     start = prefix_len
     for e, n in enumerate(branch_lens):
         M[e, start:start + n] = True
@@ -72,7 +83,7 @@ def event_mask(prefix_len: int, branch_lens) -> np.ndarray:
 # ---------------------------------------------------------------------------
 
 def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return_p=False,
-                    heads=None):
+                    heads=None, self_g=None):
     """Decode attention of one video's events under the event-factorized mask.
 
     q:          [E_b, H_q, D] float64, one query token per event branch
@@ -89,7 +100,7 @@ def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return
     G = H_q // H_kv
     K_all = np.concatenate([k_prefix] + list(k_branches), axis=0)   # [n_keys, H_kv, D]
     V_all = np.concatenate([v_prefix] + list(v_branches), axis=0)
-    M = event_mask(S, [kb.shape[0] for kb in k_branches])             # [E_b, n_keys]
+    M = event_mask(S, [kb.shape[0] for kb in k_branches], self_g)     # [E_b, n_keys]
     n_keys = K_all.shape[0]
     o = np.zeros((E_b, H_q, D), dtype=np.float64)
     lse = np.zeros((E_b, H_q), dtype=np.float64)
@@ -109,12 +120,13 @@ def video_attention(q, k_prefix, v_prefix, k_branches, v_branches, scale, return
     return o, lse, p_all
 
 
-def decode_step(w, return_p=False):
+def decode_step(w, return_p=False, self_g=None):
     """Oracle for a whole batch described by a workload object (see ``synth.Workload``).
 
     Branch e's keys after this step's append are its L_e stored private tokens
     followed by k_new[e] (and likewise for values).  Returns o [E, H_q, D] and
-    lse [E, H_q] in float64 (and p per video when asked).
+    lse [E, H_q] in float64 (and p per video when asked).  ``self_g`` = (K per
+    video, G index per event) selects the "self G-token only" mask (event_mask).
     """
     E = w.n_events
     o = np.zeros((E, w.h_q, w.head_dim), dtype=np.float64)
@@ -129,7 +141,8 @@ def decode_step(w, return_p=False):
         vp = bf16_to_f64(w.prefix_v(b))
         kbs = [np.concatenate([bf16_to_f64(w.priv_k(e)), bf16_to_f64(w.k_new[e:e + 1])]) for e in ev]
         vbs = [np.concatenate([bf16_to_f64(w.priv_v(e)), bf16_to_f64(w.v_new[e:e + 1])]) for e in ev]
-        ob, lb, pb = video_attention(qb, kp, vp, kbs, vbs, w.scale, return_p=return_p)
+        sg = None if self_g is None else (self_g[0][b], [self_g[1][e] for e in ev])
+        ob, lb, pb = video_attention(qb, kp, vp, kbs, vbs, w.scale, return_p=return_p, self_g=sg)
         o[ev] = ob
         lse[ev] = lb
         ps.append(pb)
@@ -138,7 +151,7 @@ def decode_step(w, return_p=False):
     return o, lse
 
 
-def event_rows(w, e, heads=None):
+def event_rows(w, e, heads=None, self_g=None):
     """Oracle output of event e alone (all or selected q-heads), for sampled checks
     at full size: the mask of Sec. 3.4 restricted to row e is prefix + own branch."""
     b = int(w.event_video[e])
@@ -147,7 +160,8 @@ def event_rows(w, e, heads=None):
     vp = bf16_to_f64(w.prefix_v(b))
     kb = np.concatenate([bf16_to_f64(w.priv_k(e)), bf16_to_f64(w.k_new[e:e + 1])])
     vb = np.concatenate([bf16_to_f64(w.priv_v(e)), bf16_to_f64(w.v_new[e:e + 1])])
-    o, lse, _ = video_attention(qb, kp, vp, [kb], [vb], w.scale, heads=heads)
+    sg = None if self_g is None else (self_g[0][b], [self_g[1][e]])
+    o, lse, _ = video_attention(qb, kp, vp, [kb], [vb], w.scale, heads=heads, self_g=sg)
     if heads is not None:
         return o[0, heads], lse[0, heads]
     return o[0], lse[0]

@@ -366,3 +366,64 @@ def test_rope_table_closed_form():
         ang = pos * 1.0e6 ** (-2.0 * i / 128)
         assert t[pos, i] == np.float32(math.cos(ang))
         assert t[pos, 64 + i] == np.float32(math.sin(ang))
+
+
+# ---------------------------------------------------------------------------
+# "Self G-token only" mask variant (Tab. 8): G^1..G^K and S end the prefix
+# ---------------------------------------------------------------------------
+
+def _self_g_case(seed, E=3, S=20, K=4, D=16):
+    rng = np.random.default_rng(seed)
+    L = [int(x) for x in rng.integers(0, 5, size=E)]
+    q, kp, vp, kbs, vbs = _rand_video(rng, E, S, L, D=D)
+    g_index = [int(x) for x in rng.permutation(K)[:E]]
+    return q, kp, vp, kbs, vbs, (K, g_index)
+
+
+def test_self_g_mask_hides_exactly_the_other_events_g_tokens():
+    E, S, K = 3, 20, 4
+    M_full = oracle.event_mask(S, [2, 1, 3])
+    M = oracle.event_mask(S, [2, 1, 3], (K, [2, 0, 3]))
+    g0 = S - 1 - K
+    for e, own in enumerate([2, 0, 3]):
+        diff = np.nonzero(M_full[e] != M[e])[0]
+        assert set(diff.tolist()) == {g0 + g for g in range(K) if g != own}
+        assert M[e, S - 1] and M[e, :g0].all()        # S and P stay visible
+    assert np.array_equal(oracle.event_mask(S, [2, 1, 3], (0, [0, 0, 0])), M_full)
+
+
+def test_self_g_other_events_g_rows_do_not_matter():
+    """Changing the K/V rows of G tokens an event cannot see leaves its output bit for
+    bit; changing its own G row changes it."""
+    q, kp, vp, kbs, vbs, sg = _self_g_case(8)
+    scale = 1 / math.sqrt(q.shape[-1])
+    K, g_index = sg
+    o0, l0, _ = oracle.video_attention(q, kp, vp, kbs, vbs, scale, self_g=sg)
+    S = kp.shape[0]
+    g0 = S - 1 - K
+    other = [g for g in range(K) if g != g_index[0]]
+    kp2, vp2 = kp.copy(), vp.copy()
+    kp2[g0 + other[0]] += 3.0
+    vp2[g0 + other[1]] -= 2.0
+    o1, l1, _ = oracle.video_attention(q, kp2, vp2, kbs, vbs, scale, self_g=sg)
+    assert np.array_equal(o0[0], o1[0]) and np.array_equal(l0[0], l1[0])
+    kp3 = kp.copy()
+    kp3[g0 + g_index[0]] += 3.0
+    o2, _, _ = oracle.video_attention(q, kp3, vp, kbs, vbs, scale, self_g=sg)
+    assert not np.allclose(o0[0], o2[0])
+
+
+def test_self_g_against_sdpa_on_the_visible_keys():
+    """Event e's output equals plain attention over exactly P, its own G, S and its own
+    branch (library routine on the gathered keys)."""
+    q, kp, vp, kbs, vbs, sg = _self_g_case(9, E=2, S=30, K=5, D=8)
+    scale = 1 / math.sqrt(q.shape[-1])
+    K, g_index = sg
+    o, _, _ = oracle.video_attention(q, kp, vp, kbs, vbs, scale, self_g=sg)
+    S = kp.shape[0]
+    g0 = S - 1 - K
+    for e in range(q.shape[0]):
+        rows = list(range(g0)) + [g0 + g_index[e], S - 1]
+        Kv = np.concatenate([kp[rows], kbs[e]])
+        Vv = np.concatenate([vp[rows], vbs[e]])
+        assert np.allclose(o[e], _sdpa_single(q[e], Kv, Vv, scale), rtol=1e-10, atol=1e-12)
