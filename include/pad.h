@@ -148,7 +148,8 @@ size_t pad_workspace_size(const pad_problem* prob, int32_t n_videos, const int32
  *                  or NULL for packed prefixes (exclusive prefix sum of prefix_len)
  *   n_events       active event branches this step (>= 0); 0 gives a plan that launches nothing
  *   event_video    [n_events] host: video of each event, non-decreasing, in [0, n_videos)
- *   event_len      [n_events] host: private tokens of each branch BEFORE this step's append;
+ *   event_len      [n_events] host: private tokens of each branch BEFORE this step's append
+ *                  (at most 65534);
  *                  branch e attends to event_len[e] + 1 private keys after the append
  *   page_table     [n_events * max_pages] device: row e lists branch e's pages; the
  *                  new-page entries are written by pad_kv_append (or pad_decode_step)
@@ -194,6 +195,21 @@ pad_status pad_plan_release_new_pages(const pad_plan_t* plan, pad_cache_state* c
  * static variant alike. */
 pad_status pad_plan_set_rope(pad_plan_t* plan, const int32_t* positions, const float* cos_sin,
                              int32_t max_position);
+
+/* Which planning tokens a branch sees (host; before the plan's launches).  The prefix of a
+ * video ends with its planning tokens G^1..G^K and the end-of-planning token S (Sec. 3.3).
+ *   PAD_G_ALL  (default) every branch sees all of them: the method's mask (Sec. 3.4).
+ *   PAD_G_SELF the "self G-token only" structure of the paper's attention ablation
+ *              (Tab. 8): event e sees P, S and G^(g_index[e]+1) only, besides its branch.
+ *   n_planning [n_videos] host: K of each video (0 = nothing hidden in that video);
+ *              K + 1 <= prefix_len
+ *   g_index    [n_events] host: each event's own planning token, in [0, K)
+ * Ignored (may be NULL) for PAD_G_ALL.  PAD_ERR_INVALID_ARG (nothing changes) on a bad
+ * mode, count or index. */
+#define PAD_G_ALL 0
+#define PAD_G_SELF 1
+pad_status pad_plan_set_g_visibility(pad_plan_t* plan, int32_t mode, const int32_t* n_planning,
+                                     const int32_t* g_index);
 
 /* Summary of a plan (host): the split-KV decomposition chosen for the prefix pass. */
 typedef struct {

@@ -25,6 +25,8 @@ FLAG_PREFIX_SIMT = 0x1
 FLAG_PREFIX_MMA = 0x2
 FLAG_PREFIX_TC = 0x4
 FLAG_FUSED_MERGE = 0x8
+G_ALL = 0
+G_SELF = 1
 
 
 class PadError(RuntimeError):
@@ -67,6 +69,7 @@ _SIGNATURES = {
     "pad_plan_new_pages": (c_int32, [c_void_p, _I32P]),
     "pad_plan_release_new_pages": (c_int32, [c_void_p, c_void_p]),
     "pad_plan_set_rope": (c_int32, [c_void_p, _I32P, c_void_p, c_int32]),
+    "pad_plan_set_g_visibility": (c_int32, [c_void_p, c_int32, _I32P, _I32P]),
     "pad_plan_get_info": (c_int32, [c_void_p, POINTER(PlanInfo)]),
     "pad_plan_destroy": (c_int32, [c_void_p]),
     "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -212,6 +215,16 @@ class Plan:
         pos = np.ascontiguousarray(positions, dtype=np.int32)
         n = int(cos_sin.shape[0]) if max_position is None else int(max_position)
         _check(lib().pad_plan_set_rope(self._h, pos.ctypes.data_as(_I32P), _ptr(cos_sin), n))
+
+    def set_g_visibility(self, mode: int, n_planning=None, g_index=None):
+        """pad_plan_set_g_visibility: G_SELF hides the other events' planning tokens."""
+        if n_planning is None or g_index is None:
+            _check(lib().pad_plan_set_g_visibility(self._h, int(mode), None, None))
+            return
+        k = np.ascontiguousarray(n_planning, dtype=np.int32)
+        g = np.ascontiguousarray(g_index, dtype=np.int32)
+        _check(lib().pad_plan_set_g_visibility(self._h, mode, k.ctypes.data_as(_I32P),
+                                               g.ctypes.data_as(_I32P)))
 
     def info(self) -> dict:
         i = PlanInfo()

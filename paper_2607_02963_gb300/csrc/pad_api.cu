@@ -404,6 +404,7 @@ struct pad_plan_t {
   std::vector<uint8_t> param_image; // videos | events | items, packed, for KParams::img
   int32_t img_videos = 0, img_events = 0, img_items = 0, img_tasks = 0;
   const float* rope_cs = nullptr;   // rotary table (pad_plan_set_rope), else NULL
+  int32_t g_self = 0;               // self G-token mask (pad_plan_set_g_visibility)
   uint64_t gen = 0;                 // generation tagging this plan's device errors
   ~pad_plan_t() { image_release(image); }
 };
@@ -537,6 +538,10 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
       delete plan;
       return fail(PAD_ERR_INVALID_ARG, "event_len[%d]=%d < 0", e, len);
     }
+    if (len > 65534) {
+      delete plan;
+      return fail(PAD_ERR_UNSUPPORTED, "event_len[%d]=%d: branches hold at most 65535 tokens", e, len);
+    }
     if (len / ps >= max_pages) {
       delete plan;
       return fail(PAD_ERR_INVALID_ARG, "event %d: length %d needs page index %d >= max_pages=%d", e,
@@ -565,7 +570,8 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
     v.prefix_len = prefix_len[b];
     v.first_event = L.ev_first[b];
     v.n_events = L.ev_count[b];
-    v.n_splits = L.n_splits[b];
+    v.n_splits = (int16_t)L.n_splits[b];
+    v.n_planning = 0;
     v.part_base = L.part_base[b];
     v.cnt_base = L.cnt_base[b];
   }
@@ -595,10 +601,11 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
   for (int e = 0; e < n_events; ++e) {
     PadEventDesc& d = evs[e];
     d.video = (uint16_t)event_video[e];
-    d.len = event_len[e];
+    d.len = (uint16_t)event_len[e];
     d.local = (uint16_t)(e - L.ev_first[event_video[e]]);
     d.new_page = -1;
     d.pos = 0;
+    d.gidx = 0;
     if (event_len[e] % ps == 0) {
       const int pg = cache->next_free(cursor);
       // need <= free_count guarantees a page exists
@@ -690,6 +697,48 @@ pad_status pad_plan_set_rope(pad_plan_t* plan, const int32_t* positions, const f
   return PAD_OK;
 }
 
+pad_status pad_plan_set_g_visibility(pad_plan_t* plan, int32_t mode, const int32_t* n_planning,
+                                     const int32_t* g_index) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (mode != PAD_G_ALL && mode != PAD_G_SELF) return fail(PAD_ERR_INVALID_ARG, "mode %d", mode);
+  std::vector<int32_t> K(plan->n_videos, 0), gi(plan->n_events, 0);
+  if (mode == PAD_G_SELF) {
+    if ((plan->n_videos > 0 && !n_planning) || (plan->n_events > 0 && !g_index))
+      return fail(PAD_ERR_INVALID_ARG, "n_planning / g_index is NULL");
+    auto* vids = reinterpret_cast<const PadVideoDesc*>(plan->host_image.data() + plan->lay.off_videos);
+    auto* evs = reinterpret_cast<const PadEventDesc*>(plan->host_image.data() + plan->lay.off_events);
+    for (int b = 0; b < plan->n_videos; ++b) {
+      if (n_planning[b] < 0 || n_planning[b] > 32767 || n_planning[b] + 1 > std::max(1, vids[b].prefix_len))
+        return fail(PAD_ERR_INVALID_ARG, "n_planning[%d]=%d: the prefix (%d tokens) must hold G^1..G^K and S", b,
+                    n_planning[b], vids[b].prefix_len);
+      K[b] = n_planning[b];
+    }
+    for (int e = 0; e < plan->n_events; ++e) {
+      const int v = evs[e].video;
+      if (g_index[e] < 0 || g_index[e] >= std::max(1, K[v]) || (K[v] == 0 && g_index[e] != 0))
+        return fail(PAD_ERR_INVALID_ARG, "g_index[%d]=%d outside [0, %d)", e, g_index[e], K[v]);
+      gi[e] = g_index[e];
+    }
+  }
+  // every copy of the descriptors (no launch of this plan has read them yet)
+  auto set = [&](uint8_t* vbase, uint8_t* ebase) {
+    auto* v = reinterpret_cast<PadVideoDesc*>(vbase);
+    auto* ev = reinterpret_cast<PadEventDesc*>(ebase);
+    for (int b = 0; b < plan->n_videos; ++b) v[b].n_planning = (int16_t)K[b];
+    for (int e = 0; e < plan->n_events; ++e) ev[e].gidx = (uint16_t)gi[e];
+  };
+  if (plan->n_events > 0) {
+    set(plan->host_image.data() + plan->lay.off_videos, plan->host_image.data() + plan->lay.off_events);
+    if (!plan->param_image.empty())
+      set(plan->param_image.data() + plan->img_videos, plan->param_image.data() + plan->img_events);
+    if (plan->image)
+      set(static_cast<uint8_t*>(plan->image->host) + plan->lay.off_videos,
+          static_cast<uint8_t*>(plan->image->host) + plan->lay.off_events);
+  }
+  plan->g_self = mode == PAD_G_SELF ? 1 : 0;
+  return PAD_OK;
+}
+
 pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page) {
   if (!plan || (!new_page && plan->n_events > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
   std::copy(plan->new_pages.begin(), plan->new_pages.end(), new_page);
@@ -754,6 +803,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.k_new = nullptr;
   p.v_new = nullptr;
   p.rope_cs = plan->rope_cs;
+  p.g_self = plan->g_self;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
@@ -1015,6 +1065,7 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.k_new = nullptr;
   p.v_new = nullptr;
   p.rope_cs = plan->rope_cs;
+  p.g_self = plan->g_self;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   auto* ws = static_cast<uint8_t*>(scratch);

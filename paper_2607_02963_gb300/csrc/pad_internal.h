@@ -58,18 +58,21 @@ struct PadVideoDesc {
   int32_t prefix_len;
   int32_t first_event;
   int32_t n_events;
-  int32_t n_splits;     // prefix splits per kv-head (0 if prefix_len == 0 or no events)
+  int16_t n_splits;     // prefix splits per kv-head (0 if prefix_len == 0 or no events)
+  int16_t n_planning;   // K of the "self G-token only" mask (its G^1..G^K, S end the
+                        // prefix), 0 = every event sees every prefix token
   int32_t part_base;    // first partial row of this video
   int32_t cnt_base;     // first split counter of this video (fused tail; see KParams::counters)
 };
 static_assert(sizeof(PadVideoDesc) == 32, "video desc is 32 bytes");
 
 struct PadEventDesc {
-  int32_t len;          // private length before this step
   int32_t new_page;     // page taken this step, or -1
   int32_t pos;          // position of this step's token (rotary table row; 0 without RoPE)
+  uint16_t len;         // private length before this step
   uint16_t video;
   uint16_t local;       // index of the event within its video
+  uint16_t gidx;        // its own planning token G^(gidx+1) (self G-token mask only)
 };
 static_assert(sizeof(PadEventDesc) == 16, "event desc is 16 bytes");
 
@@ -118,6 +121,7 @@ struct KParams {
   // Rotary table [max_position, head_dim] fp32 (cos | sin halves) when the plan carries
   // positions (pad_plan_set_rope): q and the new key are rotated where they are loaded.
   const float* rope_cs;
+  int32_t g_self;                 // "self G-token only" mask: videos with n_planning > 0
   const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
   // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
   // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by
@@ -148,6 +152,30 @@ __device__ __forceinline__ const PadWorkItem* plan_items(const KParams& p) {
 }
 __device__ __forceinline__ const int32_t* plan_tasks(const KParams& p) {
   return p.img_n > 0 ? reinterpret_cast<const int32_t*>(p.img + p.img_tasks) : p.tasks;
+}
+
+// "Self G-token only" mask (attention ablation of the paper, Tab. 8): a row of event e
+// does not see the planning tokens G^1..G^K of its video other than its own; the prefix
+// ends with them and S.  Token indices are relative to the video's prefix.
+struct GMask {
+  int lo, hi, own;  // hidden: lo <= t < hi, t != own (lo == hi: nothing hidden)
+};
+__device__ __forceinline__ GMask g_mask_of(const KParams& p, const PadVideoDesc& vd, const PadEventDesc& ev) {
+  if (!p.g_self || vd.n_planning == 0) return GMask{0, 0, -1};
+  const int lo = vd.prefix_len - 1 - vd.n_planning;
+  return GMask{lo, vd.prefix_len - 1, lo + ev.gidx};
+}
+__device__ __forceinline__ bool g_visible(const GMask& g, int t) { return t < g.lo || t >= g.hi || t == g.own; }
+// Visible-column bits of the 64 tokens t0 .. t0+63, given the first `valid` are in range.
+__device__ __forceinline__ uint64_t keep_bits(int valid, const GMask& g, int t0) {
+  uint64_t keep = valid >= 64 ? ~0ull : (valid <= 0 ? 0ull : ((1ull << valid) - 1ull));
+  const int a = max(g.lo - t0, 0), b = min(g.hi - t0, 64);
+  if (a < b) {
+    const uint64_t range = (b >= 64 ? ~0ull : ((1ull << b) - 1ull)) & ~((1ull << a) - 1ull);
+    const int o = g.own - t0;
+    keep &= ~range | ((o >= 0 && o < 64) ? (1ull << o) : 0ull);
+  }
+  return keep;
 }
 
 // Rotary embedding, rotate-half form (the position rule of Sec. 3.4 decides `cs`, the

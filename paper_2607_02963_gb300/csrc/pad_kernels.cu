@@ -160,11 +160,20 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(const __grid_constant_
   __shared__ float sm[NW][MAXR];
   __shared__ float sl[NW][MAXR];
   __shared__ float so[MAXR][D];
+  __shared__ GMask sg[MAXR];
 
   const PadWorkItem it = plan_items(p)[blockIdx.x];
   const int R = it.n_events * p.group;
   const int kvh = it.kvh;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x < MAXR) {
+    GMask g{0, 0, -1};
+    if (p.g_self && (int)threadIdx.x < R) {
+      const PadEventDesc ev = plan_events(p)[it.first_event + threadIdx.x / p.group];
+      g = g_mask_of(p, plan_videos(p)[ev.video], ev);
+    }
+    sg[threadIdx.x] = g;
+  }
 
   for (int i = threadIdx.x; i < MAXR * D; i += blockDim.x) {
     int r = i / D, d = i - r * D;
@@ -219,10 +228,12 @@ __global__ void __launch_bounds__(256) prefix_simt_kernel(const __grid_constant_
 #pragma unroll
     for (int r = 0; r < MAXR; ++r) {
       if (r < R) {
-        float sv = valid ? s[r] * p.scale_log2 : kNegInf;
-        float mn = fmaxf(m[r], warp_max(sv));       // finite: lane 0's token is valid
-        float alpha = ex2(m[r] - mn);
-        float pr = ex2(sv - mn);
+        float sv = valid && g_visible(sg[r], it.tok_begin + t) ? s[r] * p.scale_log2 : kNegInf;
+        float mn = fmaxf(m[r], warp_max(sv));
+        // -inf only while every token so far was hidden by the self G-token mask
+        const float mb = mn == kNegInf ? 0.f : mn;
+        float alpha = ex2(m[r] - mb);
+        float pr = ex2(sv - mb);
         l[r] = l[r] * alpha + warp_sum(pr);
         m[r] = mn;
 #pragma unroll
@@ -323,6 +334,17 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
   const int g = lane >> 2, t4 = lane & 3;
 
   const int rlo = row0 + warp * 16 + g, rhi = rlo + 8;
+  GMask g_lo{0, 0, -1}, g_hi{0, 0, -1};
+  if (p.g_self) {
+    if (rlo < R) {
+      const PadEventDesc ev = plan_events(p)[it.first_event + rlo / p.group];
+      g_lo = g_mask_of(p, plan_videos(p)[ev.video], ev);
+    }
+    if (rhi < R) {
+      const PadEventDesc ev = plan_events(p)[it.first_event + rhi / p.group];
+      g_hi = g_mask_of(p, plan_videos(p)[ev.video], ev);
+    }
+  }
   uint32_t qa[KSTEPS][4];
   {
     const __nv_bfloat16* ql = rlo < R ? q_row(p, it.first_event, q, kvh, rlo) : nullptr;
@@ -401,15 +423,16 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
       }
     }
 
-    const int valid = it.tok_end - (it.tok_begin + tile * TN);
+    const int tb = it.tok_begin + tile * TN;   // prefix token of column 0
+    const int valid = it.tok_end - tb;
     float mx_lo = kNegInf, mx_hi = kNegInf;
 #pragma unroll
     for (int nb = 0; nb < TN / 8; ++nb) {
       const int c0 = nb * 8 + 2 * t4;
-      s[nb][0] = c0 < valid ? s[nb][0] * p.scale_log2 : kNegInf;
-      s[nb][1] = c0 + 1 < valid ? s[nb][1] * p.scale_log2 : kNegInf;
-      s[nb][2] = c0 < valid ? s[nb][2] * p.scale_log2 : kNegInf;
-      s[nb][3] = c0 + 1 < valid ? s[nb][3] * p.scale_log2 : kNegInf;
+      s[nb][0] = c0 < valid && g_visible(g_lo, tb + c0) ? s[nb][0] * p.scale_log2 : kNegInf;
+      s[nb][1] = c0 + 1 < valid && g_visible(g_lo, tb + c0 + 1) ? s[nb][1] * p.scale_log2 : kNegInf;
+      s[nb][2] = c0 < valid && g_visible(g_hi, tb + c0) ? s[nb][2] * p.scale_log2 : kNegInf;
+      s[nb][3] = c0 + 1 < valid && g_visible(g_hi, tb + c0 + 1) ? s[nb][3] * p.scale_log2 : kNegInf;
       mx_lo = fmaxf(mx_lo, fmaxf(s[nb][0], s[nb][1]));
       mx_hi = fmaxf(mx_hi, fmaxf(s[nb][2], s[nb][3]));
     }
@@ -417,17 +440,19 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
     mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, 2));
     mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 1));
     mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, 2));
-    const float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);  // finite (valid >= 1)
-    const float a_lo = ex2(m_lo - mn_lo), a_hi = ex2(m_hi - mn_hi);
+    const float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);
+    // -inf only while every token so far was hidden by the self G-token mask
+    const float mb_lo = mn_lo == kNegInf ? 0.f : mn_lo, mb_hi = mn_hi == kNegInf ? 0.f : mn_hi;
+    const float a_lo = ex2(m_lo - mb_lo), a_hi = ex2(m_hi - mb_hi);
     m_lo = mn_lo;
     m_hi = mn_hi;
     float rs_lo = 0.f, rs_hi = 0.f;
 #pragma unroll
     for (int nb = 0; nb < TN / 8; ++nb) {
-      s[nb][0] = ex2(s[nb][0] - mn_lo);
-      s[nb][1] = ex2(s[nb][1] - mn_lo);
-      s[nb][2] = ex2(s[nb][2] - mn_hi);
-      s[nb][3] = ex2(s[nb][3] - mn_hi);
+      s[nb][0] = ex2(s[nb][0] - mb_lo);
+      s[nb][1] = ex2(s[nb][1] - mb_lo);
+      s[nb][2] = ex2(s[nb][2] - mb_hi);
+      s[nb][3] = ex2(s[nb][3] - mb_hi);
       rs_lo += s[nb][0] + s[nb][1];
       rs_hi += s[nb][2] + s[nb][3];
     }

@@ -194,8 +194,18 @@ __device__ __forceinline__ float max3f(float a, float b, float c) {
 
 // Maximum of the raw scores of one softmax warp's 64 columns (eight chains of three-input
 // max); with MASK, columns at or past `valid` are left out.
-template <bool MASK>
-__device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], int valid) {
+// Visible columns of a warp's 64 (used on the MASK path only): the first `valid` ones (the
+// split's end), or the set bits of `keep` (also the self G-token mask).
+struct ColsValid {
+  int valid;
+  __device__ bool vis(int c) const { return c < valid; }
+};
+struct ColsBits {
+  uint64_t keep;
+  __device__ bool vis(int c) const { return (keep >> c) & 1ull; }
+};
+template <bool MASK, class Cols>
+__device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], Cols cols) {
   float mxa[8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) mxa[u] = -__builtin_huge_valf();
@@ -205,8 +215,8 @@ __device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], int v
     for (int i = 0; i < 32; i += 2) {
       float a = __uint_as_float(sr[c][i]), b = __uint_as_float(sr[c][i + 1]);
       if (MASK) {
-        if (32 * c + i >= valid) a = -__builtin_huge_valf();
-        if (32 * c + i + 1 >= valid) b = -__builtin_huge_valf();
+        if (!cols.vis(32 * c + i)) a = -__builtin_huge_valf();
+        if (!cols.vis(32 * c + i + 1)) b = -__builtin_huge_valf();
       }
       const int u = (16 * c + i / 2) & 7;
       mxa[u] = max3f(mxa[u], a, b);
@@ -216,8 +226,8 @@ __device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], int v
 
 // P = 2^(s * scale_log2 - m) for one softmax warp's 64 columns, written as packed bf16
 // over the S columns already read; returns the fp32 sum of the P values.
-template <bool MASK>
-__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], int valid, float sl2,
+template <bool MASK, class Cols>
+__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
                                               float m, uint32_t taddr_p);
 
 // ---------------------------------------------------------------- mbarrier
@@ -369,8 +379,8 @@ __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-template <bool MASK>
-__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], int valid, float sl2,
+template <bool MASK, class Cols>
+__device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
                                               float m, uint32_t taddr_p) {
   const uint64_t sc2 = f2pack(sl2, sl2), nm2 = f2pack(-m, -m);
   uint64_t lacc[4] = {0ull, 0ull, 0ull, 0ull};
@@ -392,8 +402,8 @@ __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], int v
         p1 = f2hi(e);
       }
       if (MASK) {
-        if (col >= valid) p0 = 0.f;
-        if (col + 1 >= valid) p1 = 0.f;
+        if (!cols.vis(col)) p0 = 0.f;
+        if (!cols.vis(col + 1)) p1 = 0.f;
       }
       lacc[i & 3] = fadd2(lacc[i & 3], f2pack(p0, p1));
       pk[i] = pack_bf16(p0, p1);
@@ -456,7 +466,7 @@ __device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadV
   return bm::SyncNamed{1}.all(good);
 }
 
-template <bool ROPE>
+template <bool ROPE, bool GSELF>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -683,6 +693,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_run = -__builtin_huge_valf(), l_run = 0.f;
     bool ok = true;
     uint32_t r[32];
+    // self G-token mask: the video's planning tokens G^1..G^K (prefix-relative [g_lo, g_hi))
+    int g_lo = 0, g_hi = 0;
+    if (GSELF) {
+      const PadVideoDesc vdg = plan_videos(p)[plan_events(p)[it.first_event].video];
+      if (vdg.n_planning > 0) {
+        g_lo = vdg.prefix_len - 1 - vdg.n_planning;
+        g_hi = vdg.prefix_len - 1;
+      }
+    }
     for (int j = 0; j < n_tiles; ++j) {
       const uint32_t cS = 128u * (uint32_t)(j % kSBuf);
       ok = mbar_wait(&bars->sfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 8);
@@ -696,7 +715,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32(tl + cS + col0 + 32, sr[1]);
         tmem_wait_ld_dep(sr[0]);
         tmem_wait_ld_dep(sr[1]);
-        const float pmax = valid >= 64 ? half_row_max<false>(sr, valid) : half_row_max<true>(sr, valid);
+        // columns to mask: past the split's end, or (GSELF) hidden planning tokens of this
+        // row's event; the path is chosen per warp (tcgen05.st below is warp-collective)
+        float pmax;
+        bool masked;
+        uint64_t keep = ~0ull;
+        if (GSELF) {
+          const int t0 = it.tok_begin + j * kBN + (int)col0;
+          if (valid < 64 || (t0 < g_hi && t0 + 64 > g_lo)) {
+            GMask gm{0, 0, -1};
+            if (g_lo < g_hi && grow < R)
+              gm = GMask{g_lo, g_hi, g_lo + plan_events(p)[it.first_event + grow / p.group].gidx};
+            keep = keep_bits(valid, gm, t0);
+          }
+          masked = __any_sync(0xffffffffu, keep != ~0ull);
+          pmax = masked ? half_row_max<true>(sr, ColsBits{keep}) : half_row_max<false>(sr, ColsBits{keep});
+        } else {
+          masked = valid < 64;
+          pmax = masked ? half_row_max<true>(sr, ColsValid{valid}) : half_row_max<false>(sr, ColsValid{valid});
+        }
         // meet the other half: this also orders both warps' S reads before either
         // writes P over columns the other one read
         xmax[(j & 1) * 256 + half * 128 + row] = pmax;
@@ -728,8 +765,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (need) l_run *= alpha;
         }
         if (need) m_run = m_new;
-        l_run += valid >= 64 ? half_row_exp<false>(sr, valid, sl2, m_run, tl + cS + col0 / 2)
-                             : half_row_exp<true>(sr, valid, sl2, m_run, tl + cS + col0 / 2);
+        if (GSELF)
+          l_run += masked ? half_row_exp<true>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2)
+                          : half_row_exp<false>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2);
+        else
+          l_run += masked ? half_row_exp<true>(sr, ColsValid{valid}, sl2, m_run, tl + cS + col0 / 2)
+                          : half_row_exp<false>(sr, ColsValid{valid}, sl2, m_run, tl + cS + col0 / 2);
         tmem_wait_st();
       }
       fence_before();
@@ -911,7 +952,8 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   if (!get_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    for (auto fn : {prefix_tc_kernel<false>, prefix_tc_kernel<true>}) {
+    for (auto fn : {prefix_tc_kernel<false, false>, prefix_tc_kernel<true, false>, prefix_tc_kernel<false, true>,
+                    prefix_tc_kernel<true, true>}) {
       cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
       if (e != cudaSuccess) return e;
     }
@@ -929,7 +971,9 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (p.fused && bm::smem_bytes<kD>(p.branch_rows, p.group, p.tail_chunk) > kOffBar) return cudaErrorInvalidValue;
-  return cudaLaunchKernelEx(&cfg, p.rope_cs != nullptr ? prefix_tc_kernel<true> : prefix_tc_kernel<false>, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
+  auto fn = p.rope_cs != nullptr ? (p.g_self ? prefix_tc_kernel<true, true> : prefix_tc_kernel<true, false>)
+                                 : (p.g_self ? prefix_tc_kernel<false, true> : prefix_tc_kernel<false, false>);
+  return cudaLaunchKernelEx(&cfg, fn, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse);
 }

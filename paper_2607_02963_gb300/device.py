@@ -47,6 +47,7 @@ class DeviceBatch:
         self.lse = torch.empty((w.n_events, w.h_q), dtype=torch.float32, device=self.device)
         self.plan = None
         self.rope = None           # (positions [E] host int32, cos_sin device fp32 [P, D])
+        self.self_g = None         # (K per video, G index per event) for the self G-token mask
 
     def set_rope(self, positions, table):
         """Rotate q and k_new at ``positions`` with the fp32 table ``table`` (numpy
@@ -64,6 +65,8 @@ class DeviceBatch:
                                stream=stream)
         if self.rope is not None:
             self.plan.set_rope(self.rope[0], self.rope[1])
+        if self.self_g is not None:
+            self.plan.set_g_visibility(B.G_SELF, self.self_g[0], self.self_g[1])
         return self.plan
 
     def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None,

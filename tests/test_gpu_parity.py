@@ -519,3 +519,69 @@ def test_rope_at_position_zero_changes_nothing():
     torch.cuda.synchronize()
     assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)
     assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+
+
+# ---------------------------------------------------------------------------
+# "Self G-token only" mask variant (attention ablation, Tab. 8)
+# ---------------------------------------------------------------------------
+
+def _self_g_spec(w, K=None, seed=0):
+    """K per video (default: E_b + 2, at most prefix - 1) and a distinct G index per event."""
+    rng = np.random.default_rng(seed)
+    Ks, gi = [], np.zeros(w.n_events, np.int32)
+    for b in range(w.n_videos):
+        ev = w.events_of_video(b)
+        k = int(K[b]) if K is not None else min(int(w.prefix_len[b]) - 1, len(ev) + 2)
+        k = max(0, min(k, int(w.prefix_len[b]) - 1))
+        Ks.append(k)
+        if k > 0:
+            pick = rng.permutation(k)
+            gi[ev] = pick[np.arange(len(ev)) % k]
+    return np.array(Ks, np.int32), gi
+
+
+# "tc": prefix 1000 with K = 300 puts a whole 128-token split inside the planning region,
+# so most rows see none of that split's keys
+_SELF_G_CASES = {
+    "tc_wide_planning": (lambda: _w([1000, 2600], [4, 3], [5, 0, 17, 3, 9, 1, 30], seed=51),
+                         B.FLAG_PREFIX_TC, [300, 5]),
+    "tc_gqa_8k": (synth.gqa_8k, 0, None),
+    "mma_small": (lambda: synth.random_small(52, h_q=8, h_kv=2, max_events=5), B.FLAG_PREFIX_MMA, None),
+    "mma_wide_planning": (lambda: _w([1000], [4], [5, 0, 17, 3], seed=53, h_q=8, h_kv=2),
+                          B.FLAG_PREFIX_MMA, [300]),
+    "simt_tiny_d64": (synth.tiny, 0, None),
+    "simt_wide_planning": (lambda: _w([400], [2], [3, 9], seed=54, h_q=4, h_kv=1, D=64),
+                           B.FLAG_PREFIX_SIMT, [200]),
+}
+
+
+@pytest.mark.parametrize("case", sorted(_SELF_G_CASES))
+def test_self_g_mask_matches_oracle(case):
+    make, flags, K = _SELF_G_CASES[case]
+    w = make()
+    Ks, gi = _self_g_spec(w, K, seed=len(case))
+    db = DeviceBatch(w, flags=flags)
+    db.self_g = (Ks, gi)
+    plan = db.run_step(one_call=True)
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    ref_o, ref_lse = oracle.decode_step(w, self_g=(Ks, gi))
+    check_outputs(db.out.float().cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, f"{case} self-G")
+    # and it is not the default mask
+    full_o, _ = oracle.decode_step(w)
+    if Ks.max() > 1:
+        assert np.abs(full_o - ref_o).max() > 1e-3
+
+
+def test_g_all_after_self_g_is_the_default_mask():
+    w = _w([3000], [3], [5, 0, 17], seed=55)
+    a = DeviceBatch(w)
+    a.run_step(one_call=True)
+    b = DeviceBatch(w)
+    plan = b.plan_step()
+    Ks, gi = _self_g_spec(w)
+    plan.set_g_visibility(B.G_SELF, Ks, gi)
+    plan.set_g_visibility(B.G_ALL)
+    B.pad_decode_step(plan, b.q, b.k_new, b.v_new, b.k_prefix, b.v_prefix, b.k_pool, b.v_pool, b.out, b.lse)
+    torch.cuda.synchronize()
+    assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)

@@ -262,3 +262,20 @@ def test_set_rope_validates_positions_and_table(padlib):
     with pytest.raises(B.PadError) as ei:
         B._check(B.lib().pad_plan_set_rope(plan.handle, np.zeros(3, np.int32).ctypes.data_as(B._I32P), None, 100))
     assert ei.value.status == 1
+
+
+def test_set_g_visibility_validates(padlib):
+    prob = B.make_problem(8, 2, 128, num_sms=152)
+    plan = B.pad_plan(prob, B.CacheState(64), np.array([50, 10], np.int32), np.array([0, 0, 1], np.int32),
+                      np.array([0, 3, 16], np.int32), max_pages=4, workspace=None)
+    plan.set_g_visibility(B.G_SELF, [4, 9], [0, 3, 8])
+    plan.set_g_visibility(B.G_ALL)
+    for K, gi in (([50, 0], [0, 0, 0]),      # K + 1 > prefix
+                  ([4, 2], [0, 4, 1]),       # index >= K
+                  ([4, 0], [0, 1, 1]),       # K = 0 needs index 0
+                  ([-1, 2], [0, 0, 0])):
+        with pytest.raises(B.PadError) as ei:
+            plan.set_g_visibility(B.G_SELF, K, gi)
+        assert ei.value.status == 1
+    with pytest.raises(B.PadError):
+        plan.set_g_visibility(7)
