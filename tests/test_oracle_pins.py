@@ -427,3 +427,49 @@ def test_self_g_against_sdpa_on_the_visible_keys():
         Kv = np.concatenate([kp[rows], kbs[e]])
         Vv = np.concatenate([vp[rows], vbs[e]])
         assert np.allclose(o[e], _sdpa_single(q[e], Kv, Vv, scale), rtol=1e-10, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# "Causal attention" mask variant (Tab. 8): generated tokens of all branches visible
+# ---------------------------------------------------------------------------
+
+def test_causal_mask_shape():
+    M = oracle.event_mask(5, [3, 1, 2], causal=True)
+    want = np.zeros((3, 11), bool)
+    want[:, :5] = True
+    want[:, 5:7] = True      # branch 0's two stored tokens
+    want[0, 7] = True        # its token of this step
+    want[1, 8] = True        # branch 1 has no stored token
+    want[:, 9:10] = True     # branch 2's stored token
+    want[2, 10] = True
+    assert np.array_equal(M, want)
+    assert np.array_equal(oracle.event_mask(5, [4], causal=True), oracle.event_mask(5, [4]))
+
+
+def test_causal_sees_stored_tokens_of_other_branches_but_not_their_new_one():
+    rng = np.random.default_rng(11)
+    q, kp, vp, kbs, vbs = _rand_video(rng, 3, 12, [4, 2, 5])
+    scale = 0.3
+    o0, _, _ = oracle.video_attention(q, kp, vp, kbs, vbs, scale, causal=True)
+    k2 = [x.copy() for x in kbs]
+    k2[1][-1] += 5.0                                # branch 1's token of this step
+    o1, _, _ = oracle.video_attention(q, kp, vp, k2, vbs, scale, causal=True)
+    assert np.array_equal(o0[0], o1[0]) and np.array_equal(o0[2], o1[2])
+    assert not np.allclose(o0[1], o1[1])
+    k3 = [x.copy() for x in kbs]
+    k3[1][0] += 5.0                                 # a stored token of branch 1
+    o2, _, _ = oracle.video_attention(q, kp, vp, k3, vbs, scale, causal=True)
+    assert not np.allclose(o0[0], o2[0]) and not np.allclose(o0[2], o2[2])
+
+
+def test_causal_against_sdpa_on_the_visible_keys():
+    rng = np.random.default_rng(12)
+    q, kp, vp, kbs, vbs = _rand_video(rng, 3, 9, [3, 1, 4], D=8)
+    scale = 1 / math.sqrt(8)
+    o, _, _ = oracle.video_attention(q, kp, vp, kbs, vbs, scale, causal=True)
+    stored_k = np.concatenate([kb[:-1] for kb in kbs])
+    stored_v = np.concatenate([vb[:-1] for vb in vbs])
+    for e in range(3):
+        Kv = np.concatenate([kp, stored_k, kbs[e][-1:]])
+        Vv = np.concatenate([vp, stored_v, vbs[e][-1:]])
+        assert np.allclose(o[e], _sdpa_single(q[e], Kv, Vv, scale), rtol=1e-10, atol=1e-12)
