@@ -310,6 +310,7 @@ def run_ours(args):
 
     from paper_2607_02963_gb300 import binding as B
     from paper_2607_02963_gb300 import build as pad_build
+    from paper_2607_02963_gb300 import synth
     from paper_2607_02963_gb300.device import DeviceBatch, bits_to_bf16
 
     if rank == 0 or world == 1:
@@ -334,12 +335,26 @@ def run_ours(args):
     reps = [first] + [DeviceBatch(w, device=device, fill_nan=False, flags=flags)
                       for _ in range(n_rep - 1)]
 
+    rope = self_g = None
+    if args.rope:
+        pos = synth.step_positions(w)
+        rope = (pos, torch.from_numpy(synth.rope_table(int(pos.max()) + 1, w.head_dim)).to(device))
+    if args.self_g:
+        Kp = np.array([min(int(w.prefix_len[b]) - 1, len(w.events_of_video(b)) + 2)
+                       for b in range(w.n_videos)], np.int32)
+        gi = np.zeros(w.n_events, np.int32)
+        for b in range(w.n_videos):
+            ev = w.events_of_video(b)
+            if Kp[b] > 0:
+                gi[ev] = np.arange(len(ev)) % Kp[b]
+        self_g = (Kp, gi)
+
     def launcher(db, **kw):
         return B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
                               db.page_table, w.max_pages, db.workspace, w.prefix_offset,
                               kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
                               db.k_pool, db.v_pool, db.out, db.lse, stream,
-                              one_call=not args.two_call)
+                              one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal)
 
     one_call = not args.two_call
     api_path = ("pad_plan + pad_decode_step" if one_call
@@ -467,6 +482,8 @@ def run_ours(args):
             "private_tokens_after_append": int((w.event_len + 1).sum()),
             "prefix_kernel": kern_name, "splits": info["n_work_items"],
             "fused_tail": bool(info["fused_tail"]), "api": api_path,
+            "variants": {"rope": bool(args.rope), "self_g_only": bool(args.self_g),
+                         "causal": bool(args.causal)},
             "l2": f"{n_rep} rotating cold replicas of the whole device state "
                   f"({n_rep * per_rep / 2**20:.0f} MiB > 3x L2 {l2 / 2**20:.0f} MiB)",
             "parallelism": "replicas" if world > 1 else "single GPU",
@@ -659,6 +676,11 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused-merge", action="store_true",
                     help="a4 + a5 inside the tensor-core prefix kernel where the plan allows it")
+    ap.add_argument("--rope", action="store_true",
+                    help="rotate q and k_new inside the step at the shared step position")
+    ap.add_argument("--self-g", action="store_true",
+                    help="the self G-token only mask (K = events + 2 planning tokens per video)")
+    ap.add_argument("--causal", action="store_true", help="the causal-attention mask variant")
     ap.add_argument("--two-call", action="store_true",
                     help="pad_kv_append + pad_event_decode_attn instead of pad_decode_step")
     ap.add_argument("--sweep", action="store_true",

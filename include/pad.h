@@ -211,6 +211,19 @@ pad_status pad_plan_set_rope(pad_plan_t* plan, const int32_t* positions, const f
 pad_status pad_plan_set_g_visibility(pad_plan_t* plan, int32_t mode, const int32_t* n_planning,
                                      const int32_t* g_index);
 
+/* Which branch tokens a branch sees (host; before the plan's launches).
+ *   PAD_BRANCH_OWN    (default) only its own: the method's mask (Sec. 3.4).
+ *   PAD_BRANCH_CAUSAL the "causal attention" row of the paper's attention ablation
+ *                     (Tab. 8): the tokens every branch of the video generated at earlier
+ *                     steps are visible to all its branches; the token a branch emits at
+ *                     this step only to itself (the branches emit them simultaneously).
+ * Each branch task then reads every stored branch token of its video (no sharing across
+ * tasks; this variant exists for the ablation, not for speed).  PAD_ERR_INVALID_ARG on a
+ * bad mode. */
+#define PAD_BRANCH_OWN 0
+#define PAD_BRANCH_CAUSAL 1
+pad_status pad_plan_set_branch_visibility(pad_plan_t* plan, int32_t mode);
+
 /* Summary of a plan (host): the split-KV decomposition chosen for the prefix pass. */
 typedef struct {
   int32_t n_videos;

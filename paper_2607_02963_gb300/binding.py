@@ -27,6 +27,8 @@ FLAG_PREFIX_TC = 0x4
 FLAG_FUSED_MERGE = 0x8
 G_ALL = 0
 G_SELF = 1
+BRANCH_OWN = 0
+BRANCH_CAUSAL = 1
 
 
 class PadError(RuntimeError):
@@ -70,6 +72,7 @@ _SIGNATURES = {
     "pad_plan_release_new_pages": (c_int32, [c_void_p, c_void_p]),
     "pad_plan_set_rope": (c_int32, [c_void_p, _I32P, c_void_p, c_int32]),
     "pad_plan_set_g_visibility": (c_int32, [c_void_p, c_int32, _I32P, _I32P]),
+    "pad_plan_set_branch_visibility": (c_int32, [c_void_p, c_int32]),
     "pad_plan_get_info": (c_int32, [c_void_p, POINTER(PlanInfo)]),
     "pad_plan_destroy": (c_int32, [c_void_p]),
     "pad_kv_append": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -226,6 +229,10 @@ class Plan:
         _check(lib().pad_plan_set_g_visibility(self._h, mode, k.ctypes.data_as(_I32P),
                                                g.ctypes.data_as(_I32P)))
 
+    def set_branch_visibility(self, mode: int):
+        """pad_plan_set_branch_visibility: BRANCH_CAUSAL shows every branch's stored tokens."""
+        _check(lib().pad_plan_set_branch_visibility(self._h, int(mode)))
+
     def info(self) -> dict:
         i = PlanInfo()
         _check(lib().pad_plan_get_info(self._h, ctypes.byref(i)))
@@ -323,7 +330,10 @@ class StepLauncher:
 
     def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
                  page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
-                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True):
+                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True,
+                 rope=None, self_g=None, causal=False):
+        """``rope`` = (positions [E], device fp32 table [P, D]); ``self_g`` = (K per video, G
+        index per event); ``causal``: the mask variants of the ablation (set per plan)."""
         self.L = lib()
         self.problem = problem
         self.cache = cache
@@ -350,6 +360,18 @@ class StepLauncher:
         self.args_step = [_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix), _ptr(v_prefix),
                           _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse), self.stream]
         self.one_call = one_call
+        self.rope = None
+        if rope is not None:
+            pos = np.ascontiguousarray(rope[0], dtype=np.int32)
+            self._keep.append(pos)
+            self.rope = (pos.ctypes.data_as(_I32P), _ptr(rope[1]), int(rope[1].shape[0]))
+        self.self_g = None
+        if self_g is not None:
+            kk = np.ascontiguousarray(self_g[0], dtype=np.int32)
+            gg = np.ascontiguousarray(self_g[1], dtype=np.int32)
+            self._keep += [kk, gg]
+            self.self_g = (kk.ctypes.data_as(_I32P), gg.ctypes.data_as(_I32P))
+        self.causal = bool(causal)
         self.newp = np.full(self.ne, -1, dtype=np.int32)
         self.newpp = self.newp.ctypes.data_as(_I32P)
         self.release = release_pages
@@ -364,6 +386,12 @@ class StepLauncher:
                           self.ph))
         h = self.h
         try:
+            if self.rope is not None:
+                _check(L.pad_plan_set_rope(h, *self.rope))
+            if self.self_g is not None:
+                _check(L.pad_plan_set_g_visibility(h, G_SELF, *self.self_g))
+            if self.causal:
+                _check(L.pad_plan_set_branch_visibility(h, BRANCH_CAUSAL))
             if self.one_call:
                 _check(L.pad_decode_step(h, *self.args_step))
             else:

@@ -405,6 +405,8 @@ struct pad_plan_t {
   int32_t img_videos = 0, img_events = 0, img_items = 0, img_tasks = 0;
   const float* rope_cs = nullptr;   // rotary table (pad_plan_set_rope), else NULL
   int32_t g_self = 0;               // self G-token mask (pad_plan_set_g_visibility)
+  int32_t causal = 0;               // causal mask (pad_plan_set_branch_visibility)
+  int32_t task_keys = 0;            // most keys one branch task reads (set with causal)
   uint64_t gen = 0;                 // generation tagging this plan's device errors
   ~pad_plan_t() { image_release(image); }
 };
@@ -739,6 +741,25 @@ pad_status pad_plan_set_g_visibility(pad_plan_t* plan, int32_t mode, const int32
   return PAD_OK;
 }
 
+pad_status pad_plan_set_branch_visibility(pad_plan_t* plan, int32_t mode) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (mode != PAD_BRANCH_OWN && mode != PAD_BRANCH_CAUSAL) return fail(PAD_ERR_INVALID_ARG, "mode %d", mode);
+  int64_t most = 0;
+  if (plan->n_events > 0) {
+    auto* vids = reinterpret_cast<const PadVideoDesc*>(plan->host_image.data() + plan->lay.off_videos);
+    auto* evs = reinterpret_cast<const PadEventDesc*>(plan->host_image.data() + plan->lay.off_events);
+    for (int b = 0; b < plan->n_videos; ++b) {
+      int64_t sum = 1;
+      for (int f = 0; f < vids[b].n_events; ++f) sum += evs[vids[b].first_event + f].len;
+      most = std::max(most, sum);
+    }
+  }
+  if (most > INT32_MAX) return fail(PAD_ERR_UNSUPPORTED, "too many branch tokens in one video");
+  plan->causal = mode == PAD_BRANCH_CAUSAL ? 1 : 0;
+  plan->task_keys = (int32_t)most;
+  return PAD_OK;
+}
+
 pad_status pad_plan_new_pages(const pad_plan_t* plan, int32_t* new_page) {
   if (!plan || (!new_page && plan->n_events > 0)) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
   std::copy(plan->new_pages.begin(), plan->new_pages.end(), new_page);
@@ -790,7 +811,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.n_sms = plan->lay.n_sms;
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
-  p.branch_rows = std::min(128, (plan->max_event_len + 1 + 15) / 16 * 16);
+  p.branch_rows = std::min(128, ((plan->causal ? plan->task_keys : plan->max_event_len + 1) + 15) / 16 * 16);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   p.gen = plan->gen;
   auto* ws = static_cast<uint8_t*>(plan->workspace);
@@ -804,6 +825,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.v_new = nullptr;
   p.rope_cs = plan->rope_cs;
   p.g_self = plan->g_self;
+  p.causal = plan->causal;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
@@ -1058,7 +1080,7 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.n_sms = plan->lay.n_sms;
   p.max_splits = 0;
   for (int32_t ns : plan->lay.n_splits) p.max_splits = std::max(p.max_splits, ns);
-  p.branch_rows = std::min(128, (plan->max_event_len + 1 + 15) / 16 * 16);
+  p.branch_rows = std::min(128, ((plan->causal ? plan->task_keys : plan->max_event_len + 1) + 15) / 16 * 16);
   p.scale_log2 = (float)((double)pr.scale * 1.4426950408889634);
   p.gen = plan->gen;
   p.img_n = 0;
@@ -1066,6 +1088,7 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.v_new = nullptr;
   p.rope_cs = plan->rope_cs;
   p.g_self = plan->g_self;
+  p.causal = plan->causal;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   auto* ws = static_cast<uint8_t*>(scratch);

@@ -3,8 +3,10 @@
 // softmax warps take one task each after their prefix split.
 //
 //   a4, the own-branch part of the mask of Sec. 3.4: the branch's keys 0..len, its
-//   private tokens and the one appended at this step, staged in rounds of kKeys (K and V
-//   rows through the page table, cp.async); each warp takes 16 of a round's keys and
+//   private tokens and the one appended at this step (under the "causal attention" mask
+//   of the ablation: the stored tokens of every branch of the video, then its own new
+//   one), staged in rounds of kKeys (K and V rows through the page table, cp.async);
+//   each warp takes 16 of a round's keys and
 //   keeps a flash-attention state in registers in the manner of the warp-level MMA
 //   kernels (the G <= 16 query rows form one m16 tile, S = Q K^T, online softmax on the
 //   accumulators in base 2, O += P V with P re-packed from the S accumulators).
@@ -54,6 +56,7 @@ struct Head {
   static constexpr int LD = D + 8;            // padded bf16 row: ldmatrix rows in distinct banks
   __nv_bfloat16 q[16][LD];
   int page[kKeys];
+  int slot[kKeys];                            // offset of the key within its page
   float wm[kWarps][16], wl[kWarps][16];       // each warp's branch state per row
   float sc[16][kMaxChunk];                    // state weights 2^(m - M)
   alignas(16) float ob[16][D];                // merged numerator (read as float4)
@@ -152,7 +155,9 @@ struct SyncNamed {
 // One task.  `tid` in [0, 256); `smem` 16-byte aligned, smem_bytes<D>(branch_rows, G, sch)
 // long.  `partials_ready()` is called by all 256 threads and returns false if the
 // partials cannot be read (then only the status word is written).
-template <int D, bool ROPE, class Sync, class Ready>
+// CAUSAL: 0 = the method's own-branch keys, 1 = the causal-attention key list, 2 = read
+// KParams::causal at run time (separate instantiations keep the common one lean).
+template <int D, bool ROPE, int CAUSAL, class Sync, class Ready>
 __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* __restrict__ q,
                                          const __nv_bfloat16* __restrict__ kpool,
                                          const __nv_bfloat16* __restrict__ vpool, void* __restrict__ out,
@@ -183,21 +188,51 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   const int ns = vd.n_splits;
   const int rbase = ev.local * G;
   const int len = ev.len;                     // keys before this step; key `len` is this step's
-  const int nk = len + 1;
   const int ps = p.page_size;
-  const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
+  // The task's keys: its own branch's len + 1, or (causal mask) the stored tokens of every
+  // branch of the video, branch by branch, then its own token of this step.  `own` is the
+  // index of that token among them.
+  const bool causal = CAUSAL == 2 ? p.causal != 0 : CAUSAL == 1;
+  int own = len;
+  if (causal) {
+    own = 0;
+    for (int f = 0; f < vd.n_events; ++f) own += plan_events(p)[vd.first_event + f].len;
+  }
+  const int nk = own + 1;
 
-  auto page_of = [&](int key) -> int {
-    const int pi = key / ps;
-    int page = (pi == len / ps && ev.new_page >= 0) ? ev.new_page : ptab[pi];
+  // page of task key `key` (-1 if out of the pool) and, in `slot`, its offset in the page
+  auto page_of = [&](int key, int& slot) -> int {
+    int row = e, t = key;
+    if (causal) {
+      if (key == own) {
+        t = len;
+      } else {
+        row = vd.first_event;
+        for (int lf = plan_events(p)[row].len; t >= lf; lf = plan_events(p)[row].len) {
+          t -= lf;
+          ++row;
+        }
+      }
+    }
+    slot = t % ps;
+    const int pi = t / ps;
+    int page = (row == e && pi == len / ps && ev.new_page >= 0) ? ev.new_page
+                                                              : p.page_table[(size_t)row * p.max_pages + pi];
     if (page < 0 || page >= p.n_pages) {
-      pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, e, pi, page);
+      pad_set_error(p.header, p.gen, PAD_ERR_DEVICE_BOUNDS, row, pi, page);
       page = -1;
     }
     return page;
   };
+  auto locate = [&](int r0, int nv) {         // page ids and offsets of a round's keys
+    if (tid < nkr) {
+      int sl = 0;
+      S.page[tid] = tid < nv ? page_of(r0 + tid, sl) : -1;
+      S.slot[tid] = sl;
+    }
+  };
   const int nv0 = min(nkr, nk);
-  if (tid < nkr) S.page[tid] = tid < nv0 ? page_of(tid) : -1;
+  locate(0, nv0);
   // (ROPE: the plan carries positions; a separate instantiation keeps the plain one lean)
   const float* cs = ROPE ? p.rope_cs + (size_t)ev.pos * D : nullptr;
   for (int i = tid; i < 16 * CH; i += NT) {
@@ -223,7 +258,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
       const int k = k_lo + i / CH, c = i - (i / CH) * CH;
       const int pg = k < nv ? S.page[k] : -1;
       const bool in = pg >= 0;
-      if (knew != nullptr && r0 + k == len) {
+      if (knew != nullptr && r0 + k == own) {
         if (ROPE)
           *reinterpret_cast<uint4*>(&sK[k][c * 8]) = in ? rope_chunk8(knew + new_row, D, c * 8, cs)
                                                         : make_uint4(0u, 0u, 0u, 0u);
@@ -232,7 +267,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
         cp_async16(&sV[k][c * 8], vnew + new_row + c * 8, in);
         continue;
       }
-      const size_t off = (((size_t)(in ? pg : 0) * p.h_kv + kvh) * ps + ((r0 + k) % ps)) * D + c * 8;
+      const size_t off = (((size_t)(in ? pg : 0) * p.h_kv + kvh) * ps + (in ? S.slot[k] : 0)) * D + c * 8;
       cp_async16(&sK[k][c * 8], kpool + off, in);
       cp_async16(&sV[k][c * 8], vpool + off, in);
     }
@@ -240,7 +275,8 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   if (knew != nullptr) {
     // a2: this task's row of the new token into the pools (16-byte pieces of K, then V)
     if (tid < 2 * CH) {
-      const int pg = page_of(len);
+      int sl;
+      const int pg = page_of(own, sl);
       if (pg >= 0) {
         const int c = tid % CH;
         const bool isv = tid >= CH;
@@ -254,12 +290,12 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
       p.page_table[(size_t)e * p.max_pages + len / ps] = ev.new_page;
   }
   const int nv0_16 = (nv0 + 15) & ~15;
-  // key `len` waits for the grids ahead only when the append kernel wrote it
-  const bool len_in_first = len < nkr && knew == nullptr;
-  // rows 0..nv0_16-1 except key `len` (rows past nv0 are zero-filled)
+  // this step's key waits for the grids ahead only when the append kernel wrote it
+  const bool len_in_first = own < nkr && knew == nullptr;
+  // rows 0..nv0_16-1 except that key (rows past nv0 are zero-filled)
   if (len_in_first) {
-    stage_keys(0, nv0, 0, len);
-    stage_keys(0, nv0, len + 1, nv0_16);
+    stage_keys(0, nv0, 0, own);
+    stage_keys(0, nv0, own + 1, nv0_16);
   } else {
     stage_keys(0, nv0, 0, nv0_16);
   }
@@ -267,7 +303,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
 
   // ---------------- after the grids ahead (at least the append) completed
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (len_in_first) stage_keys(0, nv0, len, len + 1);
+  if (len_in_first) stage_keys(0, nv0, own, own + 1);
   cp_async_commit();                          // this round's keys
 
   // the splits' O rows and (m, l) pairs of chunk [s0, s0 + nch)
@@ -299,7 +335,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   for (int r0 = 0; r0 < nk; r0 += nkr) {
     const int nv = min(nkr, nk - r0);
     if (r0 > 0) {
-      if (tid < nkr) S.page[tid] = tid < nv ? page_of(r0 + tid) : -1;
+      locate(r0, nv);
       sy.sync();
       stage_keys(r0, nv, 0, (nv + 15) & ~15);
       cp_async_commit();

@@ -122,6 +122,8 @@ struct KParams {
   // positions (pad_plan_set_rope): q and the new key are rotated where they are loaded.
   const float* rope_cs;
   int32_t g_self;                 // "self G-token only" mask: videos with n_planning > 0
+  int32_t causal;                 // "causal attention" mask: every branch's stored tokens
+                                  // are visible to every branch of the video
   const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
   // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
   // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by

@@ -513,7 +513,7 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
 // programmatic dependent launch: its griddepcontrol.wait covers the prefix grid, so the
 // split partials are complete once it returns.
 // ---------------------------------------------------------------------------
-template <int D, bool ROPE>
+template <int D, bool ROPE, int CAUSAL>
 __global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __grid_constant__ KParams p,
                                                                     const __nv_bfloat16* __restrict__ q,
                                                                     const __nv_bfloat16* __restrict__ kpool,
@@ -528,7 +528,7 @@ __global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __g
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
-  bm::run_task<D, ROPE>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,
+  bm::run_task<D, ROPE, CAUSAL>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,
                   [] { return true; });
 }
 
@@ -624,7 +624,8 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    for (auto fn : {branch_merge_kernel<D, false>, branch_merge_kernel<D, true>}) {
+    for (auto fn : {branch_merge_kernel<D, false, 0>, branch_merge_kernel<D, true, 0>, branch_merge_kernel<D, false, 1>,
+                    branch_merge_kernel<D, true, 1>}) {
       cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
       if (e != cudaSuccess) return e;
     }
@@ -640,8 +641,9 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, p.rope_cs != nullptr ? branch_merge_kernel<D, true> : branch_merge_kernel<D, false>,
-                            p, static_cast<const __nv_bfloat16*>(q),
+  auto fn = p.causal ? (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 1> : branch_merge_kernel<D, false, 1>)
+                     : (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 0> : branch_merge_kernel<D, false, 0>);
+  return cudaLaunchKernelEx(&cfg, fn, p, static_cast<const __nv_bfloat16*>(q),
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse, sch);
 }

@@ -517,10 +517,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int gh = qrow - el * p.group;
         const __nv_bfloat16* qr = q + ((size_t)(it.first_event + el) * p.h_q + kvh * p.group + gh) * kD;
         const int d0 = half * 64 + (idx & 7) * 8;
-        if (ROPE)
-          qv[i] = rope_chunk8(qr, kD, d0, p.rope_cs + (size_t)plan_events(p)[it.first_event + el].pos * kD);
-        else
-          qv[i] = __ldg(reinterpret_cast<const uint4*>(qr + d0));
+        qv[i] = __ldg(reinterpret_cast<const uint4*>(qr + d0));
       }
     }
   }
@@ -679,6 +676,52 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int r = lane_base + (idx >> 3), cc = idx & 7;
       *reinterpret_cast<uint4*>(smem + kOffQ + half * kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4)) = qv[i];
     }
+    if (ROPE) {
+      // Rotation in place: element d < 64 pairs with d + 64, i.e. chunk cc of half 0 with
+      // chunk cc of half 1 of the same row, which the other warp of this lane quarter
+      // stored.  The two warps meet (named barrier 2 + quarter) and split the quarter's
+      // 32 rows x 8 chunk pairs; every table row is fetched once all four are addressed.
+      asm volatile("bar.sync %0, 64;" ::"r"(2 + quarter) : "memory");
+      const int t = half * 32 + lane;
+      const float* cs[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int r = lane_base + ((t + 64 * i) >> 3);
+        cs[i] = row0 + r < R
+                    ? p.rope_cs + (size_t)plan_events(p)[it.first_event + (row0 + r) / p.group].pos * kD
+                    : nullptr;
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (cs[i] == nullptr) continue;
+        const int k = t + 64 * i;
+        const int r = lane_base + (k >> 3), cc = k & 7;
+        uint4* lo = reinterpret_cast<uint4*>(smem + kOffQ + r * 128 + ((cc ^ (r & 7)) << 4));
+        uint4* hi = reinterpret_cast<uint4*>(smem + kOffQ + kQHalfBytes + r * 128 + ((cc ^ (r & 7)) << 4));
+        const uint4 a = *lo, b = *hi;
+        const float4 c0 = *reinterpret_cast<const float4*>(cs[i] + 8 * cc);
+        const float4 c1 = *reinterpret_cast<const float4*>(cs[i] + 8 * cc + 4);
+        const float4 s0 = *reinterpret_cast<const float4*>(cs[i] + 64 + 8 * cc);
+        const float4 s1 = *reinterpret_cast<const float4*>(cs[i] + 64 + 8 * cc + 4);
+        const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+        const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        const uint32_t av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+        uint32_t ol[4], oh[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&av[j]));
+          const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&bv[j]));
+          const __nv_bfloat162 l2 = __floats2bfloat162_rn(rope_one(x.x, y.x, c[2 * j], s[2 * j], true),
+                                                          rope_one(x.y, y.y, c[2 * j + 1], s[2 * j + 1], true));
+          const __nv_bfloat162 h2 = __floats2bfloat162_rn(rope_one(y.x, x.x, c[2 * j], s[2 * j], false),
+                                                          rope_one(y.y, x.y, c[2 * j + 1], s[2 * j + 1], false));
+          ol[j] = *reinterpret_cast<const uint32_t*>(&l2);
+          oh[j] = *reinterpret_cast<const uint32_t*>(&h2);
+        }
+        *lo = make_uint4(ol[0], ol[1], ol[2], ol[3]);
+        *hi = make_uint4(oh[0], oh[1], oh[2], oh[3]);
+      }
+    }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncwarp();
     if (lane == 0) mbar_arrive(&bars->qready);
@@ -834,7 +877,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int task = plan_tasks(p)[blockIdx.x];
         if (task >= 0) {
           const int te = task / p.h_kv, th = task - (task / p.h_kv) * p.h_kv;
-          bm::run_task<kD, ROPE>(p, q, kpool, vpool, out, lse, te, th, (int)threadIdx.x - 128, smem, p.tail_chunk, sy,
+          bm::run_task<kD, ROPE, 2>(p, q, kpool, vpool, out, lse, te, th, (int)threadIdx.x - 128, smem, p.tail_chunk, sy,
                            false, [&]() {
                              const PadEventDesc ev = plan_events(p)[te];
                              const PadVideoDesc vd = plan_videos(p)[ev.video];

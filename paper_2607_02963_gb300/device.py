@@ -48,6 +48,7 @@ class DeviceBatch:
         self.plan = None
         self.rope = None           # (positions [E] host int32, cos_sin device fp32 [P, D])
         self.self_g = None         # (K per video, G index per event) for the self G-token mask
+        self.causal = False        # the causal-attention mask variant
 
     def set_rope(self, positions, table):
         """Rotate q and k_new at ``positions`` with the fp32 table ``table`` (numpy
@@ -67,6 +68,8 @@ class DeviceBatch:
             self.plan.set_rope(self.rope[0], self.rope[1])
         if self.self_g is not None:
             self.plan.set_g_visibility(B.G_SELF, self.self_g[0], self.self_g[1])
+        if self.causal:
+            self.plan.set_branch_visibility(B.BRANCH_CAUSAL)
         return self.plan
 
     def run_step(self, stream=None, q=None, k_new=None, v_new=None, out=None, lse=None,

@@ -585,3 +585,51 @@ def test_g_all_after_self_g_is_the_default_mask():
     B.pad_decode_step(plan, b.q, b.k_new, b.v_new, b.k_prefix, b.v_prefix, b.k_pool, b.v_pool, b.out, b.lse)
     torch.cuda.synchronize()
     assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)
+
+
+# ---------------------------------------------------------------------------
+# "Causal attention" mask variant (attention ablation, Tab. 8)
+# ---------------------------------------------------------------------------
+
+_CAUSAL_CASES = {
+    "tc_ragged": (lambda: _w([300, 2000, 0, 900], [5, 2, 1, 7], [16, 0, 31, 47, 2, 15, 64, 3, 9, 33,
+                                                               48, 0, 1, 16, 17], seed=61), B.FLAG_PREFIX_TC),
+    "tc_many_rounds": (lambda: _w([1500], [6], [90, 70, 0, 33, 128, 1], seed=62), B.FLAG_PREFIX_TC),
+    "mma_small": (lambda: synth.random_small(63, h_q=8, h_kv=2, max_events=5), B.FLAG_PREFIX_MMA),
+    "simt_tiny_d64": (synth.tiny, 0),
+}
+
+
+@pytest.mark.parametrize("one_call", [False, True])
+@pytest.mark.parametrize("case", sorted(_CAUSAL_CASES))
+def test_causal_mask_matches_oracle(case, one_call):
+    make, flags = _CAUSAL_CASES[case]
+    w = make()
+    db = DeviceBatch(w, flags=flags)
+    db.causal = True
+    plan = db.run_step(one_call=one_call)
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    check_bookkeeping(db, w, plan)
+    ref_o, ref_lse = oracle.decode_step(w, causal=True)
+    check_outputs(db.out.float().cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, f"{case} causal")
+
+
+def test_mask_variants_and_rope_compose():
+    """Causal branch visibility, the self G-token mask and the fused rotation together:
+    the oracle with all three (rotated inputs, both mask changes)."""
+    w = _w([1000, 2600], [4, 3], [5, 0, 17, 3, 9, 1, 30], seed=64)
+    Ks, gi = _self_g_spec(w, [300, 5], seed=3)
+    pos = synth.step_positions(w)
+    table = synth.rope_table(int(pos.max()) + 1, w.head_dim)
+    db = DeviceBatch(w, flags=B.FLAG_PREFIX_TC)
+    db.causal = True
+    db.self_g = (Ks, gi)
+    db.set_rope(pos, table)
+    plan = db.run_step(one_call=True)
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    wr = oracle.rotated_workload(w, pos, table)
+    check_bookkeeping(db, wr, plan)
+    ref_o, ref_lse = oracle.decode_step(wr, causal=True, self_g=(Ks, gi))
+    check_outputs(db.out.float().cpu().numpy(), db.lse.cpu().numpy(), ref_o, ref_lse, "all variants")

@@ -279,3 +279,14 @@ def test_set_g_visibility_validates(padlib):
         assert ei.value.status == 1
     with pytest.raises(B.PadError):
         plan.set_g_visibility(7)
+
+
+def test_set_branch_visibility_validates(padlib):
+    prob = B.make_problem(8, 2, 128, num_sms=152)
+    plan = B.pad_plan(prob, B.CacheState(64), np.array([50], np.int32), np.zeros(2, np.int32),
+                      np.array([3, 16], np.int32), max_pages=4, workspace=None)
+    plan.set_branch_visibility(B.BRANCH_CAUSAL)
+    plan.set_branch_visibility(B.BRANCH_OWN)
+    with pytest.raises(B.PadError) as ei:
+        plan.set_branch_visibility(2)
+    assert ei.value.status == 1
