@@ -1,8 +1,10 @@
 """fp64 CPU oracle (test infrastructure only; see pad_oracle.py)."""
 from .pad_oracle import (bf16_to_f64, event_mask, video_attention, decode_step, event_rows,
                          lse_merge, simulate_append, bf16_round, rope_rotate, rope_bits,
-                         rotated_workload, OK, OUT_OF_PAGES, INVALID)
+                         rotated_workload, ground_segment_scores, ground_salient,
+                         attention_aggregate, OK, OUT_OF_PAGES, INVALID)
 
 __all__ = ["bf16_to_f64", "event_mask", "video_attention", "decode_step", "event_rows",
            "lse_merge", "simulate_append", "bf16_round", "rope_rotate", "rope_bits",
-           "rotated_workload", "OK", "OUT_OF_PAGES", "INVALID"]
+           "rotated_workload", "ground_segment_scores", "ground_salient", "attention_aggregate",
+           "OK", "OUT_OF_PAGES", "INVALID"]

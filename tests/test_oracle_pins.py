@@ -473,3 +473,70 @@ def test_causal_against_sdpa_on_the_visible_keys():
         Kv = np.concatenate([kp, stored_k, kbs[e][-1:]])
         Vv = np.concatenate([vp, stored_v, vbs[e][-1:]])
         assert np.allclose(o[e], _sdpa_single(q[e], Kv, Vv, scale), rtol=1e-10, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Grounding readout (Sec. 3.3; inference by similarity matching)
+# ---------------------------------------------------------------------------
+
+def test_grounding_hand_worked_example():
+    with open(os.path.join(os.path.dirname(__file__), "golden", "grounding_example.json")) as f:
+        ex = json.load(f)
+    sc = oracle.ground_segment_scores(ex["g_proj"], ex["f_proj"], ex["offsets"])
+    assert np.allclose(sc, ex["scores"], rtol=0, atol=1e-15)
+    for th in ("0.5", "0.7"):
+        sal, iv = oracle.ground_salient(sc, float(th))
+        assert np.array_equal(sal.astype(int), ex["threshold_" + th]["salient"])
+        assert np.array_equal(iv, ex["threshold_" + th]["interval"])
+    _, iv = oracle.ground_salient(sc, 0.5)
+    out = oracle.attention_aggregate(ex["g_emb"], ex["f_proj"], ex["attn"], iv, ex["offsets"])
+    assert np.allclose(out, ex["aggregate_at_0.5"], rtol=0, atol=1e-12)
+
+
+def test_grounding_scores_brute_force():
+    rng = np.random.default_rng(21)
+    K, T, d = 3, 17, 5
+    g, f = rng.standard_normal((K, d)), rng.standard_normal((T, d))
+    offsets = [0, 4, 5, 11, 17]
+    got = oracle.ground_segment_scores(g, f, offsets)
+    for i in range(K):
+        for s in range(4):
+            tot = 0.0
+            for t in range(offsets[s], offsets[s + 1]):
+                for c in range(d):
+                    tot += g[i, c] * f[t, c]
+            assert abs(got[i, s] - tot) <= 1e-12
+
+
+def test_grounding_threshold_rules():
+    sc = np.array([[4.0, 2.0, 1.9, 4.0], [-3.0, -1.0, -2.0, -1.5]])
+    sal, iv = oracle.ground_salient(sc, 0.5)
+    assert sal[0].tolist() == [True, True, False, True] and iv[0].tolist() == [0, 3]
+    assert sal[1].tolist() == [False, True, False, False] and iv[1].tolist() == [1, 1]  # no positive score
+    rng = np.random.default_rng(22)
+    sc = rng.standard_normal((6, 40)) + 1.0
+    prev = None
+    for th in (0.0, 0.3, 0.5, 0.7, 1.0):
+        sal, _ = oracle.ground_salient(sc, th)
+        assert sal[np.arange(6), sc.argmax(axis=1)].all()
+        if prev is not None:
+            assert not (sal & ~prev).any()                 # a higher fraction keeps a subset
+        prev = sal
+
+
+def test_attention_aggregate_special_cases():
+    rng = np.random.default_rng(23)
+    T, d, K = 12, 4, 2
+    x, g = rng.standard_normal((T, d)), rng.standard_normal((K, d))
+    offsets = [0, 3, 7, 12]
+    iv = np.array([[0, 1], [2, 2]])
+    uni = oracle.attention_aggregate(g, x, np.ones(T), iv, offsets)       # uniform: mean pooling
+    assert np.allclose(uni[0], g[0] + x[0:7].mean(axis=0)) and np.allclose(uni[1], g[1] + x[7:12].mean(axis=0))
+    hot = np.zeros(T)
+    hot[5] = 0.7
+    hot[9] = 0.2
+    out = oracle.attention_aggregate(g, x, hot, iv, offsets)              # one weight in each range
+    assert np.allclose(out[0], g[0] + x[5]) and np.allclose(out[1], g[1] + x[9])
+    a = rng.uniform(0, 1, T)
+    assert np.allclose(oracle.attention_aggregate(g, x, a, iv, offsets),
+                       oracle.attention_aggregate(g, x, 3.5 * a, iv, offsets))  # weights normalised
