@@ -291,6 +291,52 @@ pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q, c
                                         const void* v_prefix, const void* k_pool, const void* v_pool,
                                         void* out, float* lse, pad_stream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * Grounding readout of the planning tokens (Sec. 3.3 and the paper's note on grounding at
+ * inference by similarity matching).  Each generated event token G^i and every
+ * audio-visual prefix token are first mapped by the model's projection (its two-layer
+ * MLP, applied by the caller like any other layer); the dot products of G^i with the
+ * tokens of one time segment are summed into a segment score, and the segments whose
+ * score reaches `fraction` (0.5 or 0.7 in the paper) of the event's best score are its
+ * grounded segments.  Segments are contiguous token ranges [offsets[s], offsets[s+1]).
+ * Since the segment score is linear in the token features, the prefix is pooled once per
+ * segment (pad_ground_pool) and every event is scored against the pooled rows
+ * (pad_ground_score).  All calls are asynchronous on `stream`; argument errors return
+ * before any launch.  pad_ground_pool and pad_attn_aggregate add partial sums of row slices
+ * with atomics: their fp32 results do not depend on the order beyond rounding, but are not
+ * bit-reproducible from run to run.
+ * --------------------------------------------------------------------------- */
+
+/* seg_sum[s, :] = sum of f_proj[t, :] over the tokens t of segment s (fp32).
+ *   f_proj   [n_tokens, d_proj] bf16 device, 16-byte aligned; d_proj a multiple of 8, <= 2048
+ *   offsets  [n_segments + 1] HOST, non-decreasing within [0, n_tokens]; 1 <= n_segments <= 1024
+ *   seg_sum  [n_segments, d_proj] fp32 device, 16-byte aligned (written) */
+pad_status pad_ground_pool(const void* f_proj, int64_t n_tokens, int32_t d_proj, const int32_t* offsets,
+                           int32_t n_segments, float* seg_sum, pad_stream_t stream);
+
+/* scores[i, s] = <g_proj[i], seg_sum[s]>; salient[i, s] = 1 when scores[i, s] >= fraction *
+ * best_i (best_i > 0), else only the first best segment; interval[i] = (first, last)
+ * salient segment.
+ *   g_proj   [n_events, d_proj] bf16 device, 16-byte aligned
+ *   scores   [n_events, n_segments] fp32, salient [n_events, n_segments] uint8,
+ *   interval [n_events, 2] int32, all device (written); fraction in [0, 1] */
+pad_status pad_ground_score(const void* g_proj, int32_t n_events, const float* seg_sum, int32_t n_segments,
+                            int32_t d_proj, float fraction, float* scores, uint8_t* salient, int32_t* interval,
+                            pad_stream_t stream);
+
+/* Attention-guided aggregation (Sec. 3.3, strategy (3)): for event i, the prefix tokens of
+ * its grounded segments interval[i] = (lo, hi), i.e. tokens [offsets[lo], offsets[hi + 1]),
+ * are pooled with weights attn[t] (the attention of the last text-query token on them) and
+ * out[i] = g_emb[i] + sum_t attn[t] x[t] / sum_t attn[t] (g_emb[i] alone when that weight is 0).
+ *   x        [n_tokens, d_model] bf16 device (prefix hidden states), 16-byte aligned;
+ *            d_model a multiple of 64
+ *   attn     [n_tokens] fp32 device; interval [n_events, 2] int32 device (as written by
+ *            pad_ground_score; clamped to the segments); offsets as above (host)
+ *   g_emb    [n_events, d_model] bf16 device; out [n_events, d_model] fp32 device (written) */
+pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, const float* attn,
+                              const int32_t* offsets, int32_t n_segments, const int32_t* interval, int32_t n_events,
+                              const void* g_emb, float* out, pad_stream_t stream);
+
 /* Synchronise the stream and read the plan's device status word:
  * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream);

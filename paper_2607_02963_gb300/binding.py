@@ -81,6 +81,11 @@ _SIGNATURES = {
     "pad_event_decode_attn_static": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                                c_void_p, c_void_p, c_void_p, c_void_p]),
     "pad_decode_step": (c_int32, [c_void_p] * 11),
+    "pad_ground_pool": (c_int32, [c_void_p, c_int64, c_int32, _I32P, c_int32, c_void_p, c_void_p]),
+    "pad_ground_score": (c_int32, [c_void_p, c_int32, c_void_p, c_int32, c_int32, c_float, c_void_p, c_void_p,
+                                   c_void_p, c_void_p]),
+    "pad_attn_aggregate": (c_int32, [c_void_p, c_int64, c_int32, c_void_p, _I32P, c_int32, c_void_p, c_int32,
+                                     c_void_p, c_void_p, c_void_p]),
     "pad_device_status": (c_int32, [c_void_p, c_void_p]),
     "pad_last_error": (ctypes.c_char_p, []),
     "pad_status_string": (ctypes.c_char_p, [c_int32]),
@@ -295,6 +300,28 @@ def pad_decode_step(plan: Plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_p
     _check(lib().pad_decode_step(plan.handle, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix),
                                  _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
                                  _stream(stream)))
+
+
+def pad_ground_pool(f_proj, offsets, seg_sum, stream=None):
+    """Per-segment sums of the projected prefix features (Sec. 3.3 grounding readout)."""
+    off = np.ascontiguousarray(offsets, dtype=np.int32)
+    _check(lib().pad_ground_pool(_ptr(f_proj), int(f_proj.shape[0]), int(f_proj.shape[1]),
+                                 off.ctypes.data_as(_I32P), int(off.size - 1), _ptr(seg_sum), _stream(stream)))
+
+
+def pad_ground_score(g_proj, seg_sum, fraction, scores, salient, interval, stream=None):
+    """Segment scores, salient segments and grounded interval of every event token."""
+    _check(lib().pad_ground_score(_ptr(g_proj), int(g_proj.shape[0]), _ptr(seg_sum), int(seg_sum.shape[0]),
+                                  int(seg_sum.shape[1]), float(fraction), _ptr(scores), _ptr(salient),
+                                  _ptr(interval), _stream(stream)))
+
+
+def pad_attn_aggregate(x, attn, offsets, interval, g_emb, out, stream=None):
+    """Attention-guided pooling of each event's grounded tokens, added to its embedding."""
+    off = np.ascontiguousarray(offsets, dtype=np.int32)
+    _check(lib().pad_attn_aggregate(_ptr(x), int(x.shape[0]), int(x.shape[1]), _ptr(attn),
+                                    off.ctypes.data_as(_I32P), int(off.size - 1), _ptr(interval),
+                                    int(g_emb.shape[0]), _ptr(g_emb), _ptr(out), _stream(stream)))
 
 
 def pad_event_decode_attn_static(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,

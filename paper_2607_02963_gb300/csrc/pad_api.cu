@@ -1123,3 +1123,59 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   }
   return PAD_OK;
 }
+
+// ---------------------------------------------------------------------------
+// Grounding readout (Sec. 3.3)
+// ---------------------------------------------------------------------------
+
+static pad_status check_offsets(const int32_t* offsets, int32_t n_segments, int64_t n_tokens) {
+  if (n_segments < 1 || n_segments > 1024) return fail(PAD_ERR_UNSUPPORTED, "n_segments=%d outside [1, 1024]", n_segments);
+  if (!offsets) return fail(PAD_ERR_INVALID_ARG, "offsets is NULL");
+  for (int s = 0; s <= n_segments; ++s)
+    if (offsets[s] < 0 || offsets[s] > n_tokens || (s > 0 && offsets[s] < offsets[s - 1]))
+      return fail(PAD_ERR_INVALID_ARG, "offsets[%d]=%d: must be non-decreasing within [0, %lld]", s, offsets[s],
+                  (long long)n_tokens);
+  return PAD_OK;
+}
+
+pad_status pad_ground_pool(const void* f_proj, int64_t n_tokens, int32_t d_proj, const int32_t* offsets,
+                           int32_t n_segments, float* seg_sum, pad_stream_t stream) {
+  if (d_proj < 8 || d_proj > 2048 || d_proj % 8) return fail(PAD_ERR_UNSUPPORTED, "d_proj=%d: a multiple of 8 up to 2048", d_proj);
+  if (n_tokens < 0 || n_tokens > INT32_MAX) return fail(PAD_ERR_INVALID_ARG, "n_tokens=%lld", (long long)n_tokens);
+  pad_status st = check_offsets(offsets, n_segments, n_tokens);
+  if (st != PAD_OK) return st;
+  if (!f_proj || !seg_sum) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(f_proj) || !aligned16(seg_sum)) return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaError_t e = launch_ground_pool(f_proj, n_tokens, d_proj, offsets, n_segments, seg_sum,
+                                     reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "ground pool launch");
+}
+
+pad_status pad_ground_score(const void* g_proj, int32_t n_events, const float* seg_sum, int32_t n_segments,
+                            int32_t d_proj, float fraction, float* scores, uint8_t* salient, int32_t* interval,
+                            pad_stream_t stream) {
+  if (d_proj < 8 || d_proj > 2048 || d_proj % 8) return fail(PAD_ERR_UNSUPPORTED, "d_proj=%d: a multiple of 8 up to 2048", d_proj);
+  if (n_segments < 1 || n_segments > 1024) return fail(PAD_ERR_UNSUPPORTED, "n_segments=%d outside [1, 1024]", n_segments);
+  if (n_events < 0) return fail(PAD_ERR_INVALID_ARG, "n_events < 0");
+  if (!(fraction >= 0.f && fraction <= 1.f)) return fail(PAD_ERR_INVALID_ARG, "fraction must be in [0, 1]");
+  if (n_events > 0 && (!g_proj || !seg_sum || !scores || !salient || !interval)) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(g_proj) || !aligned16(seg_sum)) return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaError_t e = launch_ground_score(g_proj, n_events, seg_sum, n_segments, d_proj, fraction, scores, salient,
+                                      interval, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "ground score launch");
+}
+
+pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, const float* attn,
+                              const int32_t* offsets, int32_t n_segments, const int32_t* interval, int32_t n_events,
+                              const void* g_emb, float* out, pad_stream_t stream) {
+  if (d_model < 64 || d_model % 64 || d_model > 65535 * 64) return fail(PAD_ERR_UNSUPPORTED, "d_model=%d: a multiple of 64", d_model);
+  if (n_tokens < 0 || n_tokens > INT32_MAX) return fail(PAD_ERR_INVALID_ARG, "n_tokens=%lld", (long long)n_tokens);
+  pad_status st = check_offsets(offsets, n_segments, n_tokens);
+  if (st != PAD_OK) return st;
+  if (n_events < 0 || n_events > 65535) return fail(PAD_ERR_INVALID_ARG, "n_events=%d", n_events);
+  if (n_events > 0 && (!x || !attn || !interval || !g_emb || !out)) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(x) || !aligned16(g_emb)) return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  cudaError_t e = launch_attn_aggregate(x, n_tokens, d_model, attn, offsets, n_segments, interval, n_events, g_emb,
+                                        out, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "attention aggregate launch");
+}

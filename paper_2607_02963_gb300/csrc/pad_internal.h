@@ -249,6 +249,15 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
                              const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 // pdl: launch with programmatic stream serialization (the kernel waits for its
 // predecessor with griddepcontrol.wait before it reads anything the predecessor wrote).
+// Grounding readout (pad_ground.cu).  cudaErrorInvalidValue for bad segment offsets.
+cudaError_t launch_ground_pool(const void* f_proj, int64_t n_tokens, int32_t d, const int32_t* offsets,
+                               int32_t n_segments, float* seg_sum, cudaStream_t s);
+cudaError_t launch_ground_score(const void* g_proj, int32_t n_events, const float* seg_sum, int32_t n_segments,
+                                int32_t d, float frac, float* scores, uint8_t* salient, int32_t* interval,
+                                cudaStream_t s);
+cudaError_t launch_attn_aggregate(const void* x, int64_t n_tokens, int32_t d, const float* attn,
+                                  const int32_t* offsets, int32_t n_segments, const int32_t* interval,
+                                  int32_t n_events, const void* g_emb, float* out, cudaStream_t s);
 cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
                                 const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 

@@ -280,3 +280,44 @@ def random_small(seed: int, h_q: int = 8, h_kv: int = 2, head_dim: int = 128,
     L = rng.integers(0, max_len + 1, size=int(Ev.sum()))
     return make_workload(f"small_s{seed}", seed, h_q, h_kv, head_dim, P, Ev, L, rng=rng,
                          k_scale_sigma=k_scale_sigma)
+
+
+@dataclasses.dataclass
+class GroundingInputs:
+    """Seeded stand-ins for the grounding readout of one video (Sec. 3.3): projected
+    audio-visual prefix tokens and event tokens, the segment ranges, the prefix hidden
+    states, the last query token's attention on the prefix, and the event embeddings."""
+    offsets: np.ndarray    # [S + 1] int32, token ranges of the time segments
+    f_proj: np.ndarray     # [T, d_proj] bf16 bits
+    g_proj: np.ndarray     # [K, d_proj] bf16 bits
+    x: np.ndarray          # [T, d_model] bf16 bits
+    attn: np.ndarray       # [T] fp32, non-negative, sums to 1 over the prefix
+    g_emb: np.ndarray      # [K, d_model] bf16 bits
+    true_seg: np.ndarray   # [K, 2] the segment range each event token was drawn near
+
+
+def grounding_inputs(seed: int, n_tokens: int, n_segments: int, n_events: int, d_proj: int,
+                     d_model: int, text_tokens: int = 0) -> GroundingInputs:
+    """Segments of near-equal length after `text_tokens` leading text tokens; each event
+    token is the mean projected feature of a random run of 1-4 segments plus noise, so it
+    has a real best interval; attention weights are a softmax of N(0, 1) logits."""
+    rng = np.random.default_rng(seed)
+    av = n_tokens - text_tokens
+    cuts = np.sort(rng.choice(np.arange(1, av), size=n_segments - 1, replace=False)) if n_segments > 1 else []
+    offsets = (text_tokens + np.concatenate([[0], cuts, [av]])).astype(np.int32)
+    f = _normal(rng, (n_tokens, d_proj))
+    seg_mean = np.stack([f[offsets[s]:offsets[s + 1]].mean(axis=0) for s in range(n_segments)])
+    true = np.zeros((n_events, 2), dtype=np.int32)
+    g = np.zeros((n_events, d_proj), dtype=np.float32)
+    for i in range(n_events):
+        w = int(rng.integers(1, 5))
+        s0 = int(rng.integers(0, max(1, n_segments - w + 1)))
+        true[i] = (s0, min(n_segments, s0 + w) - 1)
+        g[i] = 8.0 * seg_mean[s0:s0 + w].mean(axis=0) + 0.1 * _normal(rng, (d_proj,))
+    x = _normal(rng, (n_tokens, d_model))
+    logits = _normal(rng, (n_tokens,)).astype(np.float64)
+    a = np.exp(logits - logits.max())
+    a = (a / a.sum()).astype(np.float32)
+    emb = _normal(rng, (n_events, d_model))
+    return GroundingInputs(offsets=offsets, f_proj=f32_to_bf16_bits(f), g_proj=f32_to_bf16_bits(g),
+                           x=f32_to_bf16_bits(x), attn=a, g_emb=f32_to_bf16_bits(emb), true_seg=true)
