@@ -540,3 +540,60 @@ def test_attention_aggregate_special_cases():
     a = rng.uniform(0, 1, T)
     assert np.allclose(oracle.attention_aggregate(g, x, a, iv, offsets),
                        oracle.attention_aggregate(g, x, 3.5 * a, iv, offsets))  # weights normalised
+
+
+# ---------------------------------------------------------------------------
+# Full-sequence mask for training / prefill (Sec. 3.4, Fig. 3)
+# ---------------------------------------------------------------------------
+
+def test_prefill_mask_hand_worked():
+    M = oracle.prefill_mask(3, [2, 1])
+    want = np.array([[1, 0, 0, 0, 0, 0],
+                     [1, 1, 0, 0, 0, 0],
+                     [1, 1, 1, 0, 0, 0],
+                     [1, 1, 1, 1, 0, 0],
+                     [1, 1, 1, 1, 1, 0],
+                     [1, 1, 1, 0, 0, 1]], dtype=bool)
+    assert np.array_equal(M, want)
+
+
+def test_prefill_without_branches_is_causal_attention():
+    rng = np.random.default_rng(31)
+    N, Hq, Hkv, D = 40, 4, 2, 16
+    q, k, v = rng.standard_normal((N, Hq, D)), rng.standard_normal((N, Hkv, D)), rng.standard_normal((N, Hkv, D))
+    o, _ = oracle.prefill_attention(q, k, v, N, [], 0.25)
+    qt = torch.from_numpy(q).permute(1, 0, 2)
+    kt = torch.from_numpy(k).permute(1, 0, 2).repeat_interleave(2, dim=0)
+    vt = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(2, dim=0)
+    ref = F.scaled_dot_product_attention(qt, kt, vt, is_causal=True, scale=0.25).permute(1, 0, 2).numpy()
+    assert np.allclose(o, ref, rtol=1e-10, atol=1e-12)
+
+
+def test_prefill_last_branch_token_is_the_decode_step():
+    """The last token of each branch in the full-sequence mask is exactly that branch's
+    decode step (the decode oracle over the prefix and the branch's tokens)."""
+    rng = np.random.default_rng(32)
+    S, lens, Hq, Hkv, D = 10, [3, 1, 4], 4, 2, 8
+    N = S + sum(lens)
+    q, k, v = rng.standard_normal((N, Hq, D)), rng.standard_normal((N, Hkv, D)), rng.standard_normal((N, Hkv, D))
+    o, lse = oracle.prefill_attention(q, k, v, S, lens, 0.3)
+    starts = np.cumsum([S] + lens[:-1])
+    last = [int(st + n - 1) for st, n in zip(starts, lens)]
+    kb = [k[st:st + n] for st, n in zip(starts, lens)]
+    vb = [v[st:st + n] for st, n in zip(starts, lens)]
+    od, ld, _ = oracle.video_attention(q[last], k[:S], v[:S], kb, vb, 0.3)
+    assert np.allclose(o[last], od, rtol=1e-12, atol=1e-12) and np.allclose(lse[last], ld, rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_other_branches_do_not_matter():
+    rng = np.random.default_rng(33)
+    S, lens, Hq, Hkv, D = 6, [2, 3], 2, 1, 4
+    N = S + sum(lens)
+    q, k, v = rng.standard_normal((N, Hq, D)), rng.standard_normal((N, Hkv, D)), rng.standard_normal((N, Hkv, D))
+    o0, _ = oracle.prefill_attention(q, k, v, S, lens, 0.5)
+    k2, v2 = k.copy(), v.copy()
+    k2[S + 2:] += 4.0                      # branch 2's tokens
+    v2[S + 2:] -= 1.0
+    o1, _ = oracle.prefill_attention(q, k2, v2, S, lens, 0.5)
+    assert np.array_equal(o0[:S + 2], o1[:S + 2])   # prefix and branch 1 unchanged
+    assert not np.allclose(o0[S + 2:], o1[S + 2:])
