@@ -581,6 +581,100 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_prefill(args):
+    """Whole-sequence forward attention under the event-factorized mask (training /
+    prefill), on the long_32k video: prefix 32768 tokens, then its 32 branches (each the
+    branch's tokens after this step, 2080 in all).  Timed with CUDA events over repeated
+    calls (compute-bound; inputs stay resident).  Comparators on the same tensors: torch's
+    scaled_dot_product_attention with the explicit boolean mask (the generic masked path the
+    paper used), and with is_causal=True (the plain causal kernel, which computes a
+    different mask: a speed reference only)."""
+    import math
+    import numpy as np
+    import torch
+    import torch.nn.functional as F
+    from paper_2607_02963_gb300 import binding as B
+    from paper_2607_02963_gb300 import build as pad_build
+    from paper_2607_02963_gb300 import synth
+
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    pad_build.build()
+    B.lib()
+    w = synth.long_32k()
+    S = int(w.prefix_len[0])
+    lens = (w.event_len + 1).astype(np.int32)
+    H, Hkv, D = w.h_q, w.h_kv, w.head_dim
+    qb, kb, vb = synth.prefill_inputs(11, S, lens, H, Hkv, D, k_scale_sigma=0.5)
+    N = qb.shape[0]
+
+    def dev(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(device)
+
+    q, k, v = dev(qb), dev(kb), dev(vb)
+    out = torch.empty((N, H, D), dtype=torch.float32, device=device)
+    lse = torch.empty((N, H), dtype=torch.float32, device=device)
+    prob = B.make_problem(H, Hkv, D, 16, 1.0 / math.sqrt(D))
+    stream = torch.cuda.current_stream(device)
+
+    def timed(fn, n):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    K = max(3, min(args.steps, 20))
+    ms = timed(lambda: B.pad_prefill_attn(prob, S, lens, q, k, v, out, lse, stream), K)
+    # visible (query, key) pairs: the prefix's causal triangle, plus every branch token's
+    # prefix and its own earlier branch tokens
+    pairs = S * (S + 1) // 2 + sum(int(n) * S + int(n) * (int(n) + 1) // 2 for n in lens)
+    flops = 4.0 * pairs * D * H
+    peak = 1862.7
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            peak = float(json.load(fh)["bf16_tflops"])
+        peak_kind = "measured"
+    except Exception:
+        peak_kind = "fallback"
+    qt = q.permute(1, 0, 2).unsqueeze(0)
+    kt = k.permute(1, 0, 2).repeat_interleave(H // Hkv, dim=0).unsqueeze(0)
+    vt = v.permute(1, 0, 2).repeat_interleave(H // Hkv, dim=0).unsqueeze(0)
+    causal_ms = timed(lambda: F.scaled_dot_product_attention(qt, kt, vt, is_causal=True), K)
+    masked_ms = None
+    try:
+        starts = np.concatenate([[S], S + np.cumsum(lens)[:-1]])
+        pos = torch.arange(N, device=device)
+        br = torch.full((N,), -1, dtype=torch.long, device=device)
+        for b, (st, n) in enumerate(zip(starts, lens)):
+            br[int(st):int(st) + int(n)] = b
+        mask = (pos[None, :] <= pos[:, None]) & ((pos[None, :] < S) | (br[None, :] == br[:, None]))
+        masked_ms = timed(lambda: F.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask), max(2, K // 4))
+        del mask
+    except Exception as ex:  # noqa: BLE001 - the comparator is optional
+        masked_ms = f"unavailable: {type(ex).__name__}"
+    line = {
+        "metric": "prefill_tokens_per_s", "value": N / (ms * 1e-3), "unit": "tokens/s",
+        "higher_is_better": True, "n_gpus": 1, "steps": K, "warmup": 2, "dtype": "bf16 in, fp32 accumulate",
+        "data": "synthetic: seeded N(0,1) bf16 q/k/v of the long_32k video's whole sequence",
+        "config": {"workload": "prefill_long_32k", "prefix_tokens": S, "branches": int(lens.size),
+                   "branch_tokens": int(lens.sum()), "tokens": N, "h_q": H, "h_kv": Hkv, "head_dim": D,
+                   "kernel": "prefill_mma_kernel (mma.sync m16n8k16)"},
+        "ms": ms,
+        "roofline": {"bound": "tensor", "achieved": flops / (ms * 1e-3) / 1e12, "peak": peak, "unit": "TFLOP/s",
+                     "frac": flops / (ms * 1e-3) / 1e12 / peak, "peak_kind": peak_kind,
+                     "flops": flops, "visible_pairs_per_head": pairs},
+        "comparators_ms": {"torch_sdpa_explicit_mask": masked_ms, "torch_sdpa_is_causal": causal_ms},
+        "gpu_launches": K,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_grounding(args):
     """Grounding readout of the long_32k video (Sec. 3.3): segment pooling of the projected
     prefix, scoring of the 32 event tokens, attention-guided aggregation; each kernel timed
@@ -772,6 +866,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused-merge", action="store_true",
                     help="a4 + a5 inside the tensor-core prefix kernel where the plan allows it")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time the whole-sequence masked attention (training / prefill) of the long_32k video")
     ap.add_argument("--grounding", action="store_true",
                     help="time the grounding readout (pool, score, aggregate) of the long_32k video")
     ap.add_argument("--rope", action="store_true",
@@ -785,7 +881,9 @@ def main(argv=None):
                     help="per-E table of the sweep workload with the naive per-event comparator")
     ap.add_argument("--sweep-naive-steps", type=int, default=20)
     args = ap.parse_args(argv)
-    if args.grounding:
+    if args.prefill:
+        run_prefill(args)
+    elif args.grounding:
         run_grounding(args)
     elif args.sweep:
         run_sweep(args)

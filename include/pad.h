@@ -337,6 +337,24 @@ pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, 
                               const int32_t* offsets, int32_t n_segments, const int32_t* interval, int32_t n_events,
                               const void* g_emb, float* out, pad_stream_t stream);
 
+/* Forward attention of a whole sequence under the event-factorized mask (Sec. 3.4, Fig. 3),
+ * as training with teacher forcing (and a prefill of the branches) needs it: the sequence of
+ * one video is [prefix of prefix_len tokens (P, G^1..G^K, S) ; branch 0 ; ... ; branch E-1],
+ * branch b holding branch_len[b] tokens (its anchor and local tokens).  A prefix token
+ * attends causally within the prefix; a branch token attends to the whole prefix and
+ * causally to its own branch; never to another branch.  Block-sparse: each query tile reads
+ * only the key ranges its rows can see.
+ *   prob        h_q, h_kv, head_dim (64 or 128), scale, out_dtype (num_sms, flags, page_size
+ *               unused)
+ *   branch_len  [n_branches] HOST, each >= 0; n_branches <= 1024
+ *   q           [N, h_q, head_dim] bf16, k / v [N, h_kv, head_dim] bf16, N = prefix_len +
+ *               sum(branch_len), token-major; out [N, h_q, head_dim] fp32 or bf16; lse [N, h_q]
+ *               fp32 (natural log) or NULL; all device, 16-byte aligned (lse 4-byte)
+ * One video per call; the work is asynchronous on `stream`. */
+pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t n_branches,
+                            const int32_t* branch_len, const void* q, const void* k, const void* v, void* out,
+                            float* lse, pad_stream_t stream);
+
 /* Synchronise the stream and read the plan's device status word:
  * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream);

@@ -81,6 +81,8 @@ _SIGNATURES = {
     "pad_event_decode_attn_static": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                                c_void_p, c_void_p, c_void_p, c_void_p]),
     "pad_decode_step": (c_int32, [c_void_p] * 11),
+    "pad_prefill_attn": (c_int32, [POINTER(Problem), c_int32, c_int32, _I32P, c_void_p, c_void_p, c_void_p,
+                                   c_void_p, c_void_p, c_void_p]),
     "pad_ground_pool": (c_int32, [c_void_p, c_int64, c_int32, _I32P, c_int32, c_void_p, c_void_p]),
     "pad_ground_score": (c_int32, [c_void_p, c_int32, c_void_p, c_int32, c_int32, c_float, c_void_p, c_void_p,
                                    c_void_p, c_void_p]),
@@ -300,6 +302,13 @@ def pad_decode_step(plan: Plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_p
     _check(lib().pad_decode_step(plan.handle, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix),
                                  _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse),
                                  _stream(stream)))
+
+
+def pad_prefill_attn(problem, prefix_len: int, branch_len, q, k, v, out, lse=None, stream=None):
+    """Whole-sequence forward attention under the event-factorized mask (training / prefill)."""
+    bl = np.ascontiguousarray(branch_len, dtype=np.int32)
+    _check(lib().pad_prefill_attn(ctypes.byref(problem), int(prefix_len), int(bl.size), bl.ctypes.data_as(_I32P),
+                                  _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse), _stream(stream)))
 
 
 def pad_ground_pool(f_proj, offsets, seg_sum, stream=None):

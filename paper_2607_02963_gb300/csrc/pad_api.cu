@@ -1179,3 +1179,31 @@ pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, 
                                         out, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "attention aggregate launch");
 }
+
+// ---------------------------------------------------------------------------
+// Full-sequence prefill / training forward (Sec. 3.4, Fig. 3)
+// ---------------------------------------------------------------------------
+
+pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t n_branches,
+                            const int32_t* branch_len, const void* q, const void* k, const void* v, void* out,
+                            float* lse, pad_stream_t stream) {
+  pad_status st = check_problem(prob);
+  if (st != PAD_OK) return st;
+  if (prefix_len < 0) return fail(PAD_ERR_INVALID_ARG, "prefix_len < 0");
+  if (n_branches < 0 || n_branches > 1024) return fail(PAD_ERR_UNSUPPORTED, "n_branches=%d outside [0, 1024]", n_branches);
+  if (n_branches > 0 && !branch_len) return fail(PAD_ERR_INVALID_ARG, "branch_len is NULL");
+  int64_t n = prefix_len;
+  for (int b = 0; b < n_branches; ++b) {
+    if (branch_len[b] < 0) return fail(PAD_ERR_INVALID_ARG, "branch_len[%d]=%d < 0", b, branch_len[b]);
+    n += branch_len[b];
+  }
+  if (n > INT32_MAX / 2) return fail(PAD_ERR_UNSUPPORTED, "sequence too long");
+  if (n == 0) return PAD_OK;
+  if (!q || !k || !v || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
+  cudaError_t e = launch_prefill((int32_t)n, prefix_len, n_branches, branch_len, prob->h_q, prob->h_kv, prob->head_dim,
+                                 prob->scale, prob->out_dtype == 1, q, k, v, out, lse,
+                                 reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "prefill launch");
+}

@@ -249,6 +249,10 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
                              const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 // pdl: launch with programmatic stream serialization (the kernel waits for its
 // predecessor with griddepcontrol.wait before it reads anything the predecessor wrote).
+// Full-sequence prefill / training forward (pad_prefill.cu).
+cudaError_t launch_prefill(int32_t n_tokens, int32_t prefix_len, int32_t n_branches, const int32_t* branch_len,
+                           int32_t h_q, int32_t h_kv, int32_t head_dim, float scale, int32_t out_bf16, const void* q,
+                           const void* k, const void* v, void* out, float* lse, cudaStream_t s);
 // Grounding readout (pad_ground.cu).  cudaErrorInvalidValue for bad segment offsets.
 cudaError_t launch_ground_pool(const void* f_proj, int64_t n_tokens, int32_t d, const int32_t* offsets,
                                int32_t n_segments, float* seg_sum, cudaStream_t s);

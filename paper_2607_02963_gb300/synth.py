@@ -321,3 +321,17 @@ def grounding_inputs(seed: int, n_tokens: int, n_segments: int, n_events: int, d
     emb = _normal(rng, (n_events, d_model))
     return GroundingInputs(offsets=offsets, f_proj=f32_to_bf16_bits(f), g_proj=f32_to_bf16_bits(g),
                            x=f32_to_bf16_bits(x), attn=a, g_emb=f32_to_bf16_bits(emb), true_seg=true)
+
+
+def prefill_inputs(seed: int, prefix_len: int, branch_lens, h_q: int, h_kv: int, head_dim: int,
+                   k_scale_sigma: Optional[float] = None):
+    """q [N, h_q, D], k / v [N, h_kv, D] bf16 bits for a whole sequence [prefix ; branches]
+    (N = prefix_len + sum(branch_lens)), seeded N(0, 1) like the decode workloads."""
+    rng = np.random.default_rng(seed)
+    N = int(prefix_len) + int(np.sum(branch_lens))
+    q = _normal(rng, (N, h_q, head_dim))
+    k = _normal(rng, (N, h_kv, head_dim))
+    v = _normal(rng, (N, h_kv, head_dim))
+    if k_scale_sigma is not None:
+        k = k * rng.lognormal(0.0, k_scale_sigma, size=(1, h_kv, head_dim)).astype(np.float32)
+    return f32_to_bf16_bits(q), f32_to_bf16_bits(k), f32_to_bf16_bits(v)
