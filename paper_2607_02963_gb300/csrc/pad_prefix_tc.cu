@@ -466,6 +466,40 @@ __device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadV
   return bm::SyncNamed{1}.all(good);
 }
 
+// Once its last K tile is issued (about three tiles before the CTA ends), the K producer
+// warp asks L2 for what the branch/merge kernel after this grid will read first: for the
+// CTA's share of the (event, kv-head) tasks, the branch's stored K/V rows (through the page
+// table, whose entries for those keys no kernel of this step writes), its Q rows and, in the
+// one-call step, its new K/V row.  Those tasks then start on warm lines instead of waiting
+// on HBM behind their page-table reads.  Page ids outside the pool are skipped.
+__device__ __forceinline__ void prefetch_l2(const void* a) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
+}
+__device__ __noinline__ void prefetch_branch_tasks(const KParams& p, const __nv_bfloat16* q,
+                                                   const __nv_bfloat16* kpool, const __nv_bfloat16* vpool,
+                                                   int lane) {
+  const int n_tasks = p.n_events * p.h_kv, G = p.group, ps = p.page_size;
+  for (int t = blockIdx.x; t < n_tasks; t += gridDim.x) {
+    const int e = t / p.h_kv, h = t - (t / p.h_kv) * p.h_kv;
+    const int len = plan_events(p)[e].len;
+    const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
+    for (int k = lane; k < len; k += 32) {
+      const int pg = ptab[k / ps];
+      if (pg < 0 || pg >= p.n_pages) continue;
+      const size_t off = (((size_t)pg * p.h_kv + h) * ps + (k % ps)) * kD;
+      prefetch_l2(kpool + off);
+      prefetch_l2(kpool + off + 64);
+      prefetch_l2(vpool + off);
+      prefetch_l2(vpool + off + 64);
+    }
+    if (lane < 2 * G) prefetch_l2(q + ((size_t)e * p.h_q + h * G + (lane >> 1)) * kD + 64 * (lane & 1));
+    if (p.k_new != nullptr && lane < 4) {
+      const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(lane < 2 ? p.k_new : p.v_new);
+      prefetch_l2(src + ((size_t)e * p.h_kv + h) * kD + 64 * (lane & 1));
+    }
+  }
+}
+
 template <bool ROPE, bool GSELF>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
@@ -604,6 +638,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+    __syncwarp();
+    if (warp == 0 && !p.fused && !p.causal) prefetch_branch_tasks(p, q, kpool, vpool, lane);
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issuers
     // Two threads feed the tensor pipe so that one's waits and commits overlap the
