@@ -468,7 +468,7 @@ __device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadV
 
 // Once its last K tile is issued (about three tiles before the CTA ends), the K producer
 // warp asks L2 for what the branch/merge kernel after this grid will read first: for the
-// CTA's share of the (event, kv-head) tasks, the branch's stored K/V rows (through the page
+// (event, kv-head) task with the CTA's index, if there is one, the branch's stored K/V rows (through the page
 // table, whose entries for those keys no kernel of this step writes), its Q rows and, in the
 // one-call step, its new K/V row.  Those tasks then start on warm lines instead of waiting
 // on HBM behind their page-table reads.  Page ids outside the pool are skipped.
@@ -479,7 +479,9 @@ __device__ __noinline__ void prefetch_branch_tasks(const KParams& p, const __nv_
                                                    const __nv_bfloat16* kpool, const __nv_bfloat16* vpool,
                                                    int lane) {
   const int n_tasks = p.n_events * p.h_kv, G = p.group, ps = p.page_size;
-  for (int t = blockIdx.x; t < n_tasks; t += gridDim.x) {
+  // one task per CTA at most: a warp that walked many tasks here would hold the CTA (and
+  // the grid the branch/merge kernel waits for) open longer than the prefetch saves
+  for (int t = blockIdx.x; t < n_tasks && t < (int)gridDim.x; t += gridDim.x) {
     const int e = t / p.h_kv, h = t - (t / p.h_kv) * p.h_kv;
     const int len = plan_events(p)[e].len;
     const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
