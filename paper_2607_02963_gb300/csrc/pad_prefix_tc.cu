@@ -480,8 +480,10 @@ __device__ __noinline__ void prefetch_branch_tasks(const KParams& p, const __nv_
                                                    int lane) {
   const int n_tasks = p.n_events * p.h_kv, G = p.group, ps = p.page_size;
   // one task per CTA at most: a warp that walked many tasks here would hold the CTA (and
-  // the grid the branch/merge kernel waits for) open longer than the prefetch saves
-  for (int t = blockIdx.x; t < n_tasks && t < (int)gridDim.x; t += gridDim.x) {
+  // the grid the branch/merge kernel waits for) open longer than the prefetch saves.  With
+  // the fused tail, the task this CTA will run itself.
+  const int t0 = p.fused ? plan_tasks(p)[blockIdx.x] : (int)blockIdx.x;
+  for (int t = t0; t >= 0 && t < n_tasks && t < (int)gridDim.x; t += gridDim.x) {
     const int e = t / p.h_kv, h = t - (t / p.h_kv) * p.h_kv;
     const int len = plan_events(p)[e].len;
     const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
@@ -641,7 +643,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-    if (warp == 0 && !p.fused && !p.causal) prefetch_branch_tasks(p, q, kpool, vpool, lane);
+    if (warp == 0 && !p.causal) prefetch_branch_tasks(p, q, kpool, vpool, lane);
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issuers
     // Two threads feed the tensor pipe so that one's waits and commits overlap the
