@@ -631,6 +631,9 @@ def run_prefill(args):
 
     K = max(3, min(args.steps, 20))
     ms = timed(lambda: B.pad_prefill_attn(prob, S, lens, q, k, v, out, lse, stream), K)
+    B.pad_prefill_status(stream)
+    prob_mma = B.make_problem(H, Hkv, D, 16, 1.0 / math.sqrt(D), flags=B.FLAG_PREFIX_MMA)
+    mma_ms = timed(lambda: B.pad_prefill_attn(prob_mma, S, lens, q, k, v, out, lse, stream), max(2, K // 4))
     # visible (query, key) pairs: the prefix's causal triangle, plus every branch token's
     # prefix and its own earlier branch tokens
     pairs = S * (S + 1) // 2 + sum(int(n) * S + int(n) * (int(n) + 1) // 2 for n in lens)
@@ -664,12 +667,13 @@ def run_prefill(args):
         "data": "synthetic: seeded N(0,1) bf16 q/k/v of the long_32k video's whole sequence",
         "config": {"workload": "prefill_long_32k", "prefix_tokens": S, "branches": int(lens.size),
                    "branch_tokens": int(lens.sum()), "tokens": N, "h_q": H, "h_kv": Hkv, "head_dim": D,
-                   "kernel": "prefill_mma_kernel (mma.sync m16n8k16)"},
+                   "kernel": "prefix_tc_kernel (tcgen05, prefill mode)"},
         "ms": ms,
         "roofline": {"bound": "tensor", "achieved": flops / (ms * 1e-3) / 1e12, "peak": peak, "unit": "TFLOP/s",
                      "frac": flops / (ms * 1e-3) / 1e12 / peak, "peak_kind": peak_kind,
                      "flops": flops, "visible_pairs_per_head": pairs},
-        "comparators_ms": {"torch_sdpa_explicit_mask": masked_ms, "torch_sdpa_is_causal": causal_ms},
+        "comparators_ms": {"torch_sdpa_explicit_mask": masked_ms, "torch_sdpa_is_causal": causal_ms,
+                           "ours_mma_sync_kernel": mma_ms},
         "gpu_launches": K,
     }
     print(json.dumps(line), flush=True)

@@ -350,10 +350,17 @@ pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, 
  *   q           [N, h_q, head_dim] bf16, k / v [N, h_kv, head_dim] bf16, N = prefix_len +
  *               sum(branch_len), token-major; out [N, h_q, head_dim] fp32 or bf16; lse [N, h_q]
  *               fp32 (natural log) or NULL; all device, 16-byte aligned (lse 4-byte)
- * One video per call; the work is asynchronous on `stream`. */
+ * One video per call; the work is asynchronous on `stream`.  head_dim 128 runs on the
+ * tensor-core kernel (a CTA: 128 / G tokens x the G heads of one kv-head against its visible
+ * key ranges, output normalised in place); head_dim 64, or flags PAD_FLAG_PREFIX_MMA, on the
+ * warp-level kernel (64 tokens x one head). */
 pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t n_branches,
                             const int32_t* branch_len, const void* q, const void* k, const void* v, void* out,
                             float* lse, pad_stream_t stream);
+
+/* Synchronise the stream and read the status word of the last tensor-core prefill launch
+ * (a bounded wait that gave up: PAD_ERR_DEVICE_TIMEOUT); PAD_OK otherwise. */
+pad_status pad_prefill_status(pad_stream_t stream);
 
 /* Synchronise the stream and read the plan's device status word:
  * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */

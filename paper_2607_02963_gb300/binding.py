@@ -83,6 +83,7 @@ _SIGNATURES = {
     "pad_decode_step": (c_int32, [c_void_p] * 11),
     "pad_prefill_attn": (c_int32, [POINTER(Problem), c_int32, c_int32, _I32P, c_void_p, c_void_p, c_void_p,
                                    c_void_p, c_void_p, c_void_p]),
+    "pad_prefill_status": (c_int32, [c_void_p]),
     "pad_ground_pool": (c_int32, [c_void_p, c_int64, c_int32, _I32P, c_int32, c_void_p, c_void_p]),
     "pad_ground_score": (c_int32, [c_void_p, c_int32, c_void_p, c_int32, c_int32, c_float, c_void_p, c_void_p,
                                    c_void_p, c_void_p]),
@@ -309,6 +310,11 @@ def pad_prefill_attn(problem, prefix_len: int, branch_len, q, k, v, out, lse=Non
     bl = np.ascontiguousarray(branch_len, dtype=np.int32)
     _check(lib().pad_prefill_attn(ctypes.byref(problem), int(prefix_len), int(bl.size), bl.ctypes.data_as(_I32P),
                                   _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse), _stream(stream)))
+
+
+def pad_prefill_status(stream=None):
+    """Status word of the last tensor-core prefill launch (synchronises the stream)."""
+    _check(lib().pad_prefill_status(_stream(stream)))
 
 
 def pad_ground_pool(f_proj, offsets, seg_sum, stream=None):

@@ -1184,6 +1184,8 @@ pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, 
 // Full-sequence prefill / training forward (Sec. 3.4, Fig. 3)
 // ---------------------------------------------------------------------------
 
+static std::atomic<uint64_t> g_prefill_gen{0};  // generation of the last tensor-core prefill launch
+
 pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t n_branches,
                             const int32_t* branch_len, const void* q, const void* k, const void* v, void* out,
                             float* lse, pad_stream_t stream) {
@@ -1202,8 +1204,31 @@ pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t
   if (!q || !k || !v || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
     return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
-  cudaError_t e = launch_prefill((int32_t)n, prefix_len, n_branches, branch_len, prob->h_q, prob->h_kv, prob->head_dim,
-                                 prob->scale, prob->out_dtype == 1, q, k, v, out, lse,
-                                 reinterpret_cast<cudaStream_t>(stream));
+  cudaError_t e;
+  if (prob->head_dim == 128 && !(prob->flags & (PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_SIMT))) {
+    const uint64_t gen = next_generation();
+    g_prefill_gen.store(gen);
+    e = launch_prefill_tc((int32_t)n, prefix_len, n_branches, branch_len, prob->h_q, prob->h_kv, prob->scale,
+                          prob->out_dtype == 1, gen, q, k, v, out, lse, reinterpret_cast<cudaStream_t>(stream));
+  } else {
+    e = launch_prefill((int32_t)n, prefix_len, n_branches, branch_len, prob->h_q, prob->h_kv, prob->head_dim,
+                       prob->scale, prob->out_dtype == 1, q, k, v, out, lse, reinterpret_cast<cudaStream_t>(stream));
+  }
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "prefill launch");
+}
+
+pad_status pad_prefill_status(pad_stream_t stream) {
+  PadDevHeader* hdr = nullptr;
+  cudaError_t e = prefill_header(&hdr);
+  if (e != cudaSuccess) return cuda_fail(e, "prefill status word");
+  PadDevHeader h;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  e = cudaMemcpyAsync(&h, hdr, sizeof(h), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "reading prefill status");
+  const int code = (int)(h.word & 0xffull);
+  if ((h.word >> 8) == g_prefill_gen.load() && code != PAD_OK)
+    return fail((pad_status)code, "prefill kernel reported %s (detail %d %d %d)", pad_status_string((pad_status)code),
+                h.info[0], h.info[1], h.info[2]);
+  return PAD_OK;
 }

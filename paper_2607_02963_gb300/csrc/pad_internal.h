@@ -124,6 +124,13 @@ struct KParams {
   int32_t g_self;                 // "self G-token only" mask: videos with n_planning > 0
   int32_t causal;                 // "causal attention" mask: every branch's stored tokens
                                   // are visible to every branch of the video
+  // Whole-sequence prefill on the tensor-core kernel (pad_prefill_attn): a CTA takes
+  // pf_tpc query tokens x G heads of one kv-head against its visible key ranges and writes
+  // the normalised output; branch b of the sequence starts at token ((int32_t*)img)[b]
+  // (b <= pf_nb, entry 0 = pf_S).
+  int32_t pf_N, pf_S, pf_nb, pf_tpc;
+  void* pf_out;
+  float* pf_lse;
   const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
   // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
   // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by
@@ -253,6 +260,12 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
 cudaError_t launch_prefill(int32_t n_tokens, int32_t prefix_len, int32_t n_branches, const int32_t* branch_len,
                            int32_t h_q, int32_t h_kv, int32_t head_dim, float scale, int32_t out_bf16, const void* q,
                            const void* k, const void* v, void* out, float* lse, cudaStream_t s);
+// The same on the tensor-core kernel (pad_prefix_tc.cu), head_dim 128; device errors go to
+// the library's prefill status word (prefill_header), tagged with `gen`.
+cudaError_t launch_prefill_tc(int32_t n_tokens, int32_t prefix_len, int32_t n_branches, const int32_t* branch_len,
+                              int32_t h_q, int32_t h_kv, float scale, int32_t out_bf16, uint64_t gen, const void* q,
+                              const void* k, const void* v, void* out, float* lse, cudaStream_t s);
+cudaError_t prefill_header(PadDevHeader** out);
 // Grounding readout (pad_ground.cu).  cudaErrorInvalidValue for bad segment offsets.
 cudaError_t launch_ground_pool(const void* f_proj, int64_t n_tokens, int32_t d, const int32_t* offsets,
                                int32_t n_segments, float* seg_sum, cudaStream_t s);

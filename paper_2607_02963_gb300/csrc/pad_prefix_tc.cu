@@ -46,6 +46,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <algorithm>
+#include <cstddef>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -504,7 +505,27 @@ __device__ __noinline__ void prefetch_branch_tasks(const KParams& p, const __nv_
   }
 }
 
-template <bool ROPE, bool GSELF>
+// Whole-sequence prefill (PREFILL): branch start of token p >= pf_S, from the branch
+// offsets carried in the parameters.
+__device__ __forceinline__ int pf_branch_start(const KParams& p, int t) {
+  const int32_t* bs = reinterpret_cast<const int32_t*>(p.img);
+  int lo = 0, hi = p.pf_nb - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (bs[mid] <= t) lo = mid; else hi = mid - 1;
+  }
+  return bs[lo];
+}
+// Bits c of [0, 64) with lo <= c < hi (clamped).
+__device__ __forceinline__ uint64_t range_bits(int lo, int hi) {
+  lo = max(lo, 0);
+  hi = min(hi, 64);
+  if (lo >= hi) return 0ull;
+  const uint64_t up = hi >= 64 ? ~0ull : ((1ull << hi) - 1ull);
+  return up & ~((1ull << lo) - 1ull);
+}
+
+template <bool ROPE, bool GSELF, bool PREFILL>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ KParams p, const __nv_bfloat16* __restrict__ q, const int n_groups,
                      const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -528,7 +549,35 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int item = blockIdx.x / n_groups;
   const int group = blockIdx.x - item * n_groups;
-  const PadWorkItem it = plan_items(p)[item];
+  PadWorkItem it;
+  // PREFILL: the CTA's query tokens [it.first_event, +n_events) of kv-head it.kvh (query
+  // tiles in descending order, so that the longest key ranges start first) see the keys
+  // [0, pf_a_end) of the prefix and [pf_b_lo, pf_b_end) of the branches
+  int pf_a_tiles = 0, pf_b_lo = 0, pf_a_end = 0, pf_last = 0;
+  if (PREFILL) {
+    const int n_qt = (p.pf_N + p.pf_tpc - 1) / p.pf_tpc;
+    const int qt = n_qt - 1 - (int)blockIdx.x / p.h_kv;
+    it.first_event = qt * p.pf_tpc;
+    it.n_events = min(p.pf_tpc, p.pf_N - it.first_event);
+    it.kvh = (int16_t)(blockIdx.x % p.h_kv);
+    it.split = 0;
+    it.tok0 = 0;
+    it.tok_begin = 0;
+    it.part_row0 = 0;
+    const int last = it.first_event + it.n_events - 1;
+    const int a_end = min(p.pf_S, last + 1);
+    pf_a_end = a_end;
+    pf_last = last;
+    pf_a_tiles = (a_end + kBN - 1) / kBN;
+    int b_tiles = 0;
+    if (last >= p.pf_S) {
+      pf_b_lo = pf_branch_start(p, max(it.first_event, p.pf_S));
+      b_tiles = (last + 1 - pf_b_lo + kBN - 1) / kBN;
+    }
+    it.tok_end = (pf_a_tiles + b_tiles) * kBN;  // tile count; columns are masked per tile
+  } else {
+    it = plan_items(p)[item];
+  }
   const int R = it.n_events * p.group;
   const int row0 = group * 128;
   if (row0 >= R) return;  // uniform over the CTA, before any barrier or allocation
@@ -536,6 +585,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_tiles = (ntok + kBN - 1) / kBN;
   const int kvh = it.kvh;
   const int tok0 = (int)it.tok0;
+  // first token of K/V tile t
+  auto tile_tok = [&](int t) -> int {
+    if (PREFILL) return t < pf_a_tiles ? t * kBN : pf_b_lo + (t - pf_a_tiles) * kBN;
+    return tok0 + t * kBN;
+  };
 
   // The softmax warps load their Q rows now, so that the loads overlap barrier set-up
   // and TMEM allocation; they are stored to shared memory after the block barrier.
@@ -586,11 +640,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int t = 0; t < kStages && t < n_tiles; ++t) {
       mbar_expect_tx(&bars->kfull[t], kTileBytes);
-      tma_load_3d(sbase + kOffK + t * kTileBytes, &tmK, 0, kvh, tok0 + t * kBN, &bars->kfull[t]);
-      tma_load_3d(sbase + kOffK + t * kTileBytes + kHalfBytes, &tmK, 64, kvh, tok0 + t * kBN, &bars->kfull[t]);
+      tma_load_3d(sbase + kOffK + t * kTileBytes, &tmK, 0, kvh, tile_tok(t), &bars->kfull[t]);
+      tma_load_3d(sbase + kOffK + t * kTileBytes + kHalfBytes, &tmK, 64, kvh, tile_tok(t), &bars->kfull[t]);
       mbar_expect_tx(&bars->vfull[t], kTileBytes);
-      tma_load_3d(sbase + kOffV + t * kTileBytes, &tmV, 0, kvh, tok0 + t * kBN, &bars->vfull[t]);
-      tma_load_3d(sbase + kOffV + t * kTileBytes + kHalfBytes, &tmV, 64, kvh, tok0 + t * kBN, &bars->vfull[t]);
+      tma_load_3d(sbase + kOffV + t * kTileBytes, &tmV, 0, kvh, tile_tok(t), &bars->vfull[t]);
+      tma_load_3d(sbase + kOffV + t * kTileBytes + kHalfBytes, &tmV, 64, kvh, tile_tok(t), &bars->vfull[t]);
     }
   }
   if (warp == 2) {
@@ -630,8 +684,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint64_t* full = isK ? &bars->kfull[s] : &bars->vfull[s];
         mbar_expect_tx(full, kTileBytes);
         const uint32_t dst = sbase + (isK ? kOffK : kOffV) + s * kTileBytes;
-        tma_load_3d(dst, map, 0, kvh, tok0 + t * kBN, full);
-        tma_load_3d(dst + kHalfBytes, map, 64, kvh, tok0 + t * kBN, full);
+        tma_load_3d(dst, map, 0, kvh, tile_tok(t), full);
+        tma_load_3d(dst + kHalfBytes, map, 64, kvh, tile_tok(t), full);
         issued = t + 1;
       }
       if (!ok) {
@@ -643,7 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
-    if (warp == 0 && !p.causal) prefetch_branch_tasks(p, q, kpool, vpool, lane);
+    if (!PREFILL && warp == 0 && !p.causal) prefetch_branch_tasks(p, q, kpool, vpool, lane);
   } else if (warp == 1 || warp == 2) {
     // ------------------------------------------------------------ MMA issuers
     // Two threads feed the tensor pipe so that one's waits and commits overlap the
@@ -777,6 +831,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     uint32_t r[32];
     // self G-token mask: the video's planning tokens G^1..G^K (prefix-relative [g_lo, g_hi))
+    // PREFILL: this row's token and the first token of its branch (-1 in the prefix)
+    int pf_p = 0, pf_bs = -1;
+    if (PREFILL && grow < R) {
+      pf_p = it.first_event + grow / p.group;
+      pf_bs = pf_p >= p.pf_S ? pf_branch_start(p, pf_p) : -1;
+    }
     int g_lo = 0, g_hi = 0;
     if (GSELF) {
       const PadVideoDesc vdg = plan_videos(p)[plan_events(p)[it.first_event].video];
@@ -803,7 +863,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         float pmax;
         bool masked;
         uint64_t keep = ~0ull;
-        if (GSELF) {
+        if (PREFILL) {
+          // the tile's range end, then this row's rule: a prefix token sees keys up to
+          // itself, a branch token the prefix and its own branch up to itself
+          const int tb = tile_tok(j);
+          const int t0 = tb + (int)col0;
+          keep = range_bits(0, min(kBN, (j < pf_a_tiles ? pf_a_end : pf_last + 1) - tb) - (int)col0);
+          if (grow < R)
+            keep &= pf_bs < 0 ? range_bits(0, pf_p - t0 + 1)
+                              : (range_bits(0, p.pf_S - t0) | range_bits(pf_bs - t0, pf_p - t0 + 1));
+          masked = __any_sync(0xffffffffu, keep != ~0ull);
+          pmax = masked ? half_row_max<true>(sr, ColsBits{keep}) : half_row_max<false>(sr, ColsBits{keep});
+        } else if (GSELF) {
           const int t0 = it.tok_begin + j * kBN + (int)col0;
           if (valid < 64 || (t0 < g_hi && t0 + 64 > g_lo)) {
             GMask gm{0, 0, -1};
@@ -848,7 +919,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (need) l_run *= alpha;
         }
         if (need) m_run = m_new;
-        if (GSELF)
+        if (GSELF || PREFILL)
           l_run += masked ? half_row_exp<true>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2)
                           : half_row_exp<false>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2);
         else
@@ -885,8 +956,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       xmax[(n_tiles & 1) * 256 + half * 128 + row] = l_run;
       mbar_arrive(xbar);
       ok = mbar_wait(xbar, (uint32_t)(n_tiles & 1), bars, p.header, 13);
-      if (ok && half == 0 && grow < R)
-        p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_run, l_run + xmax[(n_tiles & 1) * 256 + 128 + row]);
+      if (ok && half == 0 && grow < R) {
+        const float l_tot = l_run + xmax[(n_tiles & 1) * 256 + 128 + row];
+        if (PREFILL) {
+          // normalised output: 1 / l for the write-out below (the other slot is free once
+          // both halves met here), the LSE now
+          xmax[((n_tiles + 1) & 1) * 256 + row] = 1.0f / l_tot;
+          const int64_t orow = (int64_t)pf_p * p.h_q + kvh * p.group + grow % p.group;
+          if (p.pf_lse != nullptr) p.pf_lse[orow] = (m_run + log2f(l_tot)) * 0.69314718055994531f;
+        } else {
+          p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_run, l_tot);
+        }
+      }
     }
     // TMEM is freed by warp 2 only after every softmax warp has arrived here
     fence_before();
@@ -896,10 +977,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("bar.sync 1, 256;" ::: "memory");
     const int nrows = min(128, R - row0);
     for (int rr = warp - 4; rr < nrows; rr += 8) {
-      const float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
-      *reinterpret_cast<float4*>(p.part_o + ((int64_t)it.part_row0 + row0 + rr) * kD + 4 * lane) = v;
+      float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
+      if (PREFILL) {
+        const float inv = xmax[((n_tiles + 1) & 1) * 256 + rr];
+        v.x *= inv;
+        v.y *= inv;
+        v.z *= inv;
+        v.w *= inv;
+        const int gr = row0 + rr;
+        const size_t oi = ((size_t)(it.first_event + gr / p.group) * p.h_q + kvh * p.group + gr % p.group) * kD + 4 * lane;
+        if (p.out_bf16)
+          *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.pf_out) + oi) =
+              make_uint2(bm::pack_bf16(v.x, v.y), bm::pack_bf16(v.z, v.w));
+        else
+          *reinterpret_cast<float4*>(static_cast<float*>(p.pf_out) + oi) = v;
+      } else {
+        *reinterpret_cast<float4*>(p.part_o + ((int64_t)it.part_row0 + row0 + rr) * kD + 4 * lane) = v;
+      }
     }
-    if (p.fused) {
+    if (!PREFILL && p.fused) {
       // ---------------------------------------------------------- fused a4 + a5
       // Publish this split's rows (every softmax thread's partial stores are ordered
       // before the counter by the barrier and the fence), then run this CTA's (event,
@@ -1035,8 +1131,8 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   if (!get_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    for (auto fn : {prefix_tc_kernel<false, false>, prefix_tc_kernel<true, false>, prefix_tc_kernel<false, true>,
-                    prefix_tc_kernel<true, true>}) {
+    for (auto fn : {prefix_tc_kernel<false, false, false>, prefix_tc_kernel<true, false, false>,
+                    prefix_tc_kernel<false, true, false>, prefix_tc_kernel<true, true, false>}) {
       cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
       if (e != cudaSuccess) return e;
     }
@@ -1054,11 +1150,81 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (p.fused && bm::smem_bytes<kD>(p.branch_rows, p.group, p.tail_chunk) > kOffBar) return cudaErrorInvalidValue;
-  auto fn = p.rope_cs != nullptr ? (p.g_self ? prefix_tc_kernel<true, true> : prefix_tc_kernel<true, false>)
-                                 : (p.g_self ? prefix_tc_kernel<false, true> : prefix_tc_kernel<false, false>);
+  auto fn = p.rope_cs != nullptr
+                ? (p.g_self ? prefix_tc_kernel<true, true, false> : prefix_tc_kernel<true, false, false>)
+                : (p.g_self ? prefix_tc_kernel<false, true, false> : prefix_tc_kernel<false, false, false>);
   return cudaLaunchKernelEx(&cfg, fn, p, static_cast<const __nv_bfloat16*>(q), n_groups, mk, mv,
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse);
+}
+
+// Device status word of the whole-sequence prefill (no plan or workspace is involved).
+__device__ PadDevHeader g_prefill_header;
+
+cudaError_t prefill_header(PadDevHeader** out) {
+  static PadDevHeader* ptr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!ptr[dev]) {
+    void* a = nullptr;
+    e = cudaGetSymbolAddress(&a, g_prefill_header);
+    if (e != cudaSuccess) return e;
+    ptr[dev] = static_cast<PadDevHeader*>(a);
+  }
+  *out = ptr[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_prefill_tc(int32_t n_tokens, int32_t prefix_len, int32_t n_branches, const int32_t* branch_len,
+                              int32_t h_q, int32_t h_kv, float scale, int32_t out_bf16, uint64_t gen, const void* q,
+                              const void* k, const void* v, void* out, float* lse, cudaStream_t s) {
+  const int G = h_q / h_kv;
+  if (G < 1 || G > 128 || n_tokens <= 0) return cudaErrorInvalidValue;
+  if ((size_t)(n_branches + 1) * sizeof(int32_t) > sizeof(KParams::img)) return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  CUtensorMap mk, mv;
+  if (!get_maps(k, v, h_kv, n_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
+  static bool configured[64] = {};
+  if (dev >= 0 && dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(prefix_tc_kernel<false, false, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  KParams p;
+  std::memset(&p, 0, offsetof(KParams, img));
+  p.h_q = h_q;
+  p.h_kv = h_kv;
+  p.group = G;
+  p.head_dim = kD;
+  p.out_bf16 = out_bf16;
+  p.scale_log2 = (float)((double)scale * 1.4426950408889634);
+  p.gen = gen;
+  cudaError_t e = prefill_header(&p.header);
+  if (e != cudaSuccess) return e;
+  p.pf_N = n_tokens;
+  p.pf_S = prefix_len;
+  p.pf_nb = n_branches;
+  p.pf_tpc = 128 / G;
+  p.pf_out = out;
+  p.pf_lse = lse;
+  int32_t* bs = reinterpret_cast<int32_t*>(p.img);
+  bs[0] = prefix_len;
+  for (int b = 0; b < n_branches; ++b) bs[b + 1] = bs[b] + branch_len[b];
+  const int n_qt = (n_tokens + p.pf_tpc - 1) / p.pf_tpc;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_qt * h_kv);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cfg.numAttrs = 0;
+  return cudaLaunchKernelEx(&cfg, prefix_tc_kernel<false, false, true>, p, static_cast<const __nv_bfloat16*>(q), 1,
+                            mk, mv, static_cast<const __nv_bfloat16*>(nullptr),
+                            static_cast<const __nv_bfloat16*>(nullptr), static_cast<void*>(nullptr),
+                            static_cast<float*>(nullptr));
 }
 
 }  // namespace pad

@@ -27,14 +27,15 @@ def _dev(bits):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
 
 
-def _run(prefix, lens, h_q, h_kv, D, seed, out_dtype=0, heads=None, sigma=None):
+def _run(prefix, lens, h_q, h_kv, D, seed, out_dtype=0, heads=None, sigma=None, flags=0):
     qb, kb, vb = synth.prefill_inputs(seed, prefix, lens, h_q, h_kv, D, k_scale_sigma=sigma)
     N = qb.shape[0]
-    prob = B.make_problem(h_q, h_kv, D, 16, 1.0 / math.sqrt(D), out_dtype=out_dtype)
+    prob = B.make_problem(h_q, h_kv, D, 16, 1.0 / math.sqrt(D), out_dtype=out_dtype, flags=flags)
     out = torch.empty((N, h_q, D), dtype=torch.float32 if out_dtype == 0 else torch.bfloat16, device="cuda")
     lse = torch.empty((N, h_q), dtype=torch.float32, device="cuda")
     B.pad_prefill_attn(prob, prefix, lens, _dev(qb), _dev(kb), _dev(vb), out, lse)
     torch.cuda.synchronize()
+    B.pad_prefill_status()
     ro, rl = oracle.prefill_attention(oracle.bf16_to_f64(qb), oracle.bf16_to_f64(kb), oracle.bf16_to_f64(vb),
                                       prefix, lens, 1.0 / math.sqrt(D), heads=heads)
     go, gl = out.float().cpu().numpy(), lse.cpu().numpy()
@@ -54,8 +55,10 @@ def _run(prefix, lens, h_q, h_kv, D, seed, out_dtype=0, heads=None, sigma=None):
     (64, [64, 64]),                 # every boundary on a tile edge
     (1000, [42] * 13),              # the paper's average: 13 events of ~42 caption tokens
 ])
-def test_prefill_matches_oracle_d128(prefix, lens):
-    _run(prefix, lens, 28, 4, 128, seed=prefix + len(lens))
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_MMA])
+def test_prefill_matches_oracle_d128(prefix, lens, flags):
+    """head_dim 128 on the tensor-core kernel (default) and on the warp-level kernel."""
+    _run(prefix, lens, 28, 4, 128, seed=prefix + len(lens), flags=flags)
 
 
 def test_prefill_d64_and_bf16_output():
@@ -66,3 +69,10 @@ def test_prefill_d64_and_bf16_output():
 def test_prefill_long_prefix_sampled_heads():
     """An 8k-token prefix with 13 branches (outlier K channels); two heads checked."""
     _run(8192, [42] * 13, 28, 4, 128, seed=7, heads=[0, 27], sigma=0.5)
+
+
+def test_prefill_tc_group_sizes_and_bf16():
+    """Other GQA groups on the tensor-core kernel (128 / G tokens per CTA), bf16 output."""
+    _run(500, [30, 2, 77], 8, 2, 128, seed=8)            # G = 4: 32 tokens per CTA
+    _run(500, [30, 2, 77], 16, 1, 128, seed=9)           # G = 16: 8 tokens per CTA
+    _run(500, [30, 2, 77], 28, 4, 128, seed=10, out_dtype=1)
