@@ -712,6 +712,7 @@ def run_grounding(args):
     sal = torch.empty((K, S), dtype=torch.uint8, device=device)
     iv = torch.empty((K, 2), dtype=torch.int32, device=device)
     out = torch.empty((K, dm), dtype=torch.float32, device=device)
+    ws = B.aggregate_workspace(T, S, dm, device)
     stream = torch.cuda.current_stream(device)
     W, N = max(3, args.warmup), max(10, min(args.steps, 500))
 
@@ -742,25 +743,31 @@ def run_grounding(args):
 
     pool_us = timed(lambda i, s: B.pad_ground_pool(fs[i % nf], gi.offsets, seg, s))
     score_us = timed(lambda i, s: B.pad_ground_score(g, seg, 0.5, sc, sal, iv, s))
-    agg_us = timed(lambda i, s: B.pad_attn_aggregate(xs[i % nx], attn, gi.offsets, iv, emb, out, s))
+    agg_us = timed(lambda i, s: B.pad_attn_aggregate(xs[i % nx], attn, gi.offsets, iv, emb, out, ws, s))
 
     def whole(i, s):
         B.pad_ground_pool(fs[i % nf], gi.offsets, seg, s)
         B.pad_ground_score(g, seg, 0.5, sc, sal, iv, s)
-        B.pad_attn_aggregate(xs[i % nx], attn, gi.offsets, iv, emb, out, s)
+        B.pad_attn_aggregate(xs[i % nx], attn, gi.offsets, iv, emb, out, ws, s)
 
     all_us = timed(whole)
     ivh = iv.cpu().numpy()
     tok = sum(int(gi.offsets[ivh[i, 1] + 1] - gi.offsets[ivh[i, 0]]) for i in range(K))
+    # the events' intervals overlap: a hidden-state row that several events aggregate needs
+    # to come from HBM once, so the algorithmic bytes count the distinct rows
+    covered = np.zeros(T, dtype=bool)
+    for i in range(K):
+        covered[int(gi.offsets[ivh[i, 0]]):int(gi.offsets[ivh[i, 1] + 1])] = True
+    distinct = int(covered.sum())
     peak, peak_kind = hbm_peak()
     pool_bytes = T * dp * 2 + S * dp * 4
-    agg_bytes = tok * (dm * 2 + 4) + K * dm * (2 + 4)
+    agg_bytes = distinct * dm * 2 + tok * 4 + K * dm * (2 + 4)
     line = {
         "metric": "grounding_readouts_per_s", "value": 1e6 / all_us, "unit": "video readouts/s",
         "higher_is_better": True, "n_gpus": 1, "steps": N, "warmup": W, "dtype": "bf16 in, fp32 accumulate",
         "data": "synthetic: seeded projected features and hidden states shaped like the long_32k video",
         "config": {"workload": "grounding_long_32k", "prefix_tokens": T, "segments": S, "events": K,
-                   "d_proj": dp, "d_model": dm, "fraction": 0.5, "grounded_tokens": tok,
+                   "d_proj": dp, "d_model": dm, "fraction": 0.5, "grounded_tokens": tok, "distinct_grounded_tokens": distinct,
                    "l2": f"{nf} / {nx} rotating replicas of the projected features / hidden states (> 3x L2)"},
         "us": {"pool": pool_us, "score": score_us, "aggregate": agg_us, "readout": all_us},
         "roofline": {

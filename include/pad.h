@@ -302,9 +302,9 @@ pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q, c
  * Since the segment score is linear in the token features, the prefix is pooled once per
  * segment (pad_ground_pool) and every event is scored against the pooled rows
  * (pad_ground_score).  All calls are asynchronous on `stream`; argument errors return
- * before any launch.  pad_ground_pool and pad_attn_aggregate add partial sums of row slices
- * with atomics: their fp32 results do not depend on the order beyond rounding, but are not
- * bit-reproducible from run to run.
+ * before any launch.  pad_ground_pool adds partial sums of row slices with atomics: its fp32
+ * results do not depend on the order beyond rounding, but are not bit-reproducible from run
+ * to run.  pad_attn_aggregate sums in a fixed order: its results are the same on every run.
  * --------------------------------------------------------------------------- */
 
 /* seg_sum[s, :] = sum of f_proj[t, :] over the tokens t of segment s (fp32).
@@ -328,14 +328,25 @@ pad_status pad_ground_score(const void* g_proj, int32_t n_events, const float* s
  * its grounded segments interval[i] = (lo, hi), i.e. tokens [offsets[lo], offsets[hi + 1]),
  * are pooled with weights attn[t] (the attention of the last text-query token on them) and
  * out[i] = g_emb[i] + sum_t attn[t] x[t] / sum_t attn[t] (g_emb[i] alone when that weight is 0).
+ * The weights belong to the tokens, so the hidden states are pooled once, per piece of at
+ * most 256 tokens of a segment, into seg_ws (weighted row sums, then the pieces' weight
+ * sums), and each event adds up the pieces of its segments; overlapping intervals read x
+ * once.
  *   x        [n_tokens, d_model] bf16 device (prefix hidden states), 16-byte aligned;
- *            d_model a multiple of 64
+ *            d_model a multiple of 8
  *   attn     [n_tokens] fp32 device; interval [n_events, 2] int32 device (as written by
  *            pad_ground_score; clamped to the segments); offsets as above (host)
- *   g_emb    [n_events, d_model] bf16 device; out [n_events, d_model] fp32 device (written) */
+ *   g_emb    [n_events, d_model] bf16 device, 16-byte aligned
+ *   seg_ws   device scratch of seg_ws_bytes >= pad_attn_aggregate_workspace_size(n_tokens,
+ *            n_segments, d_model) = (n_segments + ceil(n_tokens / 256)) * (d_model + 1) * 4
+ *            bytes, 16-byte aligned (overwritten; owned by the caller, free for reuse once
+ *            the call's work on `stream` is done); too small: PAD_ERR_WORKSPACE_TOO_SMALL
+ *   out      [n_events, d_model] fp32 device (written) */
+size_t pad_attn_aggregate_workspace_size(int64_t n_tokens, int32_t n_segments, int32_t d_model);
 pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, const float* attn,
                               const int32_t* offsets, int32_t n_segments, const int32_t* interval, int32_t n_events,
-                              const void* g_emb, float* out, pad_stream_t stream);
+                              const void* g_emb, float* seg_ws, size_t seg_ws_bytes, float* out,
+                              pad_stream_t stream);
 
 /* Forward attention of a whole sequence under the event-factorized mask (Sec. 3.4, Fig. 3),
  * as training with teacher forcing (and a prefill of the branches) needs it: the sequence of

@@ -88,7 +88,8 @@ _SIGNATURES = {
     "pad_ground_score": (c_int32, [c_void_p, c_int32, c_void_p, c_int32, c_int32, c_float, c_void_p, c_void_p,
                                    c_void_p, c_void_p]),
     "pad_attn_aggregate": (c_int32, [c_void_p, c_int64, c_int32, c_void_p, _I32P, c_int32, c_void_p, c_int32,
-                                     c_void_p, c_void_p, c_void_p]),
+                                     c_void_p, c_void_p, ctypes.c_size_t, c_void_p, c_void_p]),
+    "pad_attn_aggregate_workspace_size": (ctypes.c_size_t, [c_int64, c_int32, c_int32]),
     "pad_device_status": (c_int32, [c_void_p, c_void_p]),
     "pad_last_error": (ctypes.c_char_p, []),
     "pad_status_string": (ctypes.c_char_p, [c_int32]),
@@ -331,12 +332,21 @@ def pad_ground_score(g_proj, seg_sum, fraction, scores, salient, interval, strea
                                   _ptr(interval), _stream(stream)))
 
 
-def pad_attn_aggregate(x, attn, offsets, interval, g_emb, out, stream=None):
-    """Attention-guided pooling of each event's grounded tokens, added to its embedding."""
+def aggregate_workspace(n_tokens, n_segments, d_model, device="cuda"):
+    """Scratch for pad_attn_aggregate (pad_attn_aggregate_workspace_size bytes of fp32)."""
+    import torch
+    n = int(lib().pad_attn_aggregate_workspace_size(int(n_tokens), int(n_segments), int(d_model)))
+    return torch.empty(max(1, n // 4), dtype=torch.float32, device=device)
+
+
+def pad_attn_aggregate(x, attn, offsets, interval, g_emb, out, seg_ws, stream=None):
+    """Attention-guided pooling of each event's grounded tokens, added to its embedding
+    (seg_ws: aggregate_workspace(n_tokens, n_segments, d_model))."""
     off = np.ascontiguousarray(offsets, dtype=np.int32)
     _check(lib().pad_attn_aggregate(_ptr(x), int(x.shape[0]), int(x.shape[1]), _ptr(attn),
                                     off.ctypes.data_as(_I32P), int(off.size - 1), _ptr(interval),
-                                    int(g_emb.shape[0]), _ptr(g_emb), _ptr(out), _stream(stream)))
+                                    int(g_emb.shape[0]), _ptr(g_emb), _ptr(seg_ws),
+                                    int(seg_ws.numel() * seg_ws.element_size()), _ptr(out), _stream(stream)))
 
 
 def pad_event_decode_attn_static(plan: Plan, q, k_prefix, v_prefix, k_pool, v_pool, out, lse=None,

@@ -1165,18 +1165,28 @@ pad_status pad_ground_score(const void* g_proj, int32_t n_events, const float* s
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "ground score launch");
 }
 
+size_t pad_attn_aggregate_workspace_size(int64_t n_tokens, int32_t n_segments, int32_t d_model) {
+  if (n_tokens < 0 || n_segments < 1 || d_model < 1) return 0;
+  return attn_aggregate_ws_floats(n_tokens, n_segments, d_model) * sizeof(float);
+}
+
 pad_status pad_attn_aggregate(const void* x, int64_t n_tokens, int32_t d_model, const float* attn,
                               const int32_t* offsets, int32_t n_segments, const int32_t* interval, int32_t n_events,
-                              const void* g_emb, float* out, pad_stream_t stream) {
-  if (d_model < 64 || d_model % 64 || d_model > 65535 * 64) return fail(PAD_ERR_UNSUPPORTED, "d_model=%d: a multiple of 64", d_model);
+                              const void* g_emb, float* seg_ws, size_t seg_ws_bytes, float* out,
+                              pad_stream_t stream) {
+  if (d_model < 8 || d_model % 8 || d_model > (1 << 24)) return fail(PAD_ERR_UNSUPPORTED, "d_model=%d: a multiple of 8", d_model);
   if (n_tokens < 0 || n_tokens > INT32_MAX) return fail(PAD_ERR_INVALID_ARG, "n_tokens=%lld", (long long)n_tokens);
   pad_status st = check_offsets(offsets, n_segments, n_tokens);
   if (st != PAD_OK) return st;
   if (n_events < 0 || n_events > 65535) return fail(PAD_ERR_INVALID_ARG, "n_events=%d", n_events);
-  if (n_events > 0 && (!x || !attn || !interval || !g_emb || !out)) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
-  if (!aligned16(x) || !aligned16(g_emb)) return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  if (n_events > 0 && (!x || !attn || !interval || !g_emb || !seg_ws || !out))
+    return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (!aligned16(x) || !aligned16(g_emb) || !aligned16(seg_ws)) return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  const size_t need = attn_aggregate_ws_floats(n_tokens, n_segments, d_model) * sizeof(float);
+  if (n_events > 0 && seg_ws_bytes < need)
+    return fail(PAD_ERR_WORKSPACE_TOO_SMALL, "seg_ws has %zu bytes, the call needs %zu", seg_ws_bytes, need);
   cudaError_t e = launch_attn_aggregate(x, n_tokens, d_model, attn, offsets, n_segments, interval, n_events, g_emb,
-                                        out, reinterpret_cast<cudaStream_t>(stream));
+                                        seg_ws, out, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "attention aggregate launch");
 }
 

@@ -10,8 +10,9 @@
 // the prefix is read once, pooling each segment's projected features (ground_pool_kernel,
 // HBM-bound; loads are issued four at a time per thread, since a latency-bound stream of
 // single loads ran at a twentieth of the bandwidth), and scoring every event against the pooled rows is a small contraction over
-// L2-resident data (ground_score_kernel).  The aggregation reads each event's grounded
-// token range once, in whole rows (attn_aggregate_kernel), weights and sums in fp32.
+// L2-resident data (ground_score_kernel).  The aggregation reads the hidden states once,
+// pooling them per segment with the attention weights, and sums each event's segments
+// (attn_seg_pool_kernel, attn_event_kernel).
 #include <cuda_bf16.h>
 #include <algorithm>
 #include <cstdint>
@@ -213,81 +214,144 @@ __global__ void __launch_bounds__(kThreads) ground_score_kernel(const __nv_bfloa
   }
 }
 
-// Grid (event, slice of kAggSlice rows of its grounded range): each thread owns 16-byte
-// chunks of the row (full rows per CTA, so every row is read as whole contiguous lines),
-// loads four rows together and accumulates attn-weighted sums in fp32; the slice's sums are
-// added into out (zeroed by the launcher) with atomics.  attn_finalize_kernel then divides
-// by the range's total weight and adds the event embedding.  The grounded tokens of event
-// i are [off[lo], off[hi + 1]) for its interval (lo, hi), clamped to the segments.
-constexpr int kAggSlice = 256;
-__device__ __forceinline__ void agg_range(const Offsets& so, const int32_t* interval, int i, int& lo, int& hi) {
-  const int S = so.n;
-  const int s_lo = min(max(interval[2 * i], 0), S - 1), s_hi = min(max(interval[2 * i + 1], s_lo), S - 1);
-  lo = so.off[s_lo];
-  hi = so.off[s_hi + 1];
-}
-__global__ void __launch_bounds__(kThreads) attn_aggregate_kernel(
-    const __grid_constant__ Offsets so, const __nv_bfloat16* __restrict__ x, int d, const float* __restrict__ attn,
-    const int32_t* __restrict__ interval, float* __restrict__ out) {
-  const int i = blockIdx.x;
-  int lo, hi;
-  agg_range(so, interval, i, lo, hi);
-  const int r0 = lo + blockIdx.y * kAggSlice, r1 = min(hi, r0 + kAggSlice);
-  if (r0 >= r1) return;
-  for (int c = threadIdx.x; c < d / 8; c += kThreads) {
-    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    int t = r0;
-    for (; t + 3 < r1; t += 4) {
-      uint4 v[4];
-      ld_stream4(v, reinterpret_cast<const uint4*>(x + (size_t)t * d) + c,
-                 reinterpret_cast<const uint4*>(x + (size_t)(t + 1) * d) + c,
-                 reinterpret_cast<const uint4*>(x + (size_t)(t + 2) * d) + c,
-                 reinterpret_cast<const uint4*>(x + (size_t)(t + 3) * d) + c);
-      const float4 w = make_float4(__ldg(attn + t), __ldg(attn + t + 1), __ldg(attn + t + 2), __ldg(attn + t + 3));
-      const float wv[4] = {w.x, w.y, w.z, w.w};
+// Attention-guided aggregation.  The weights attn[t] belong to the tokens, not to the
+// events, so an event's weighted sum over its grounded segments lo..hi is the sum of the
+// segments' own weighted sums: the hidden states are read once (attn_seg_pool_kernel,
+// HBM-bound), and every event then adds up its segments' rows, which stay in L2
+// (attn_event_kernel).  For balance the token axis is cut into pieces of at most
+// kAggPiece tokens, each inside one segment (segment s owns pieces pbeg[s] .. pbeg[s+1]-1),
+// and the pooled rows are per piece: W[p] = sum_{t in p} attn[t] x[t], A[p] = sum_{t in p}
+// attn[t].  Every element is written once and summed in a fixed order, so the results are
+// the same from run to run.
+constexpr int kAggCols = 256;
+constexpr int kAggPiece = 256;
+constexpr int kAggGroups = kThreads / 32;
+
+struct Pieces {
+  int32_t n;                          // segments
+  int32_t off[kMaxSegments + 1];      // token ranges of the segments
+  int32_t pbeg[kMaxSegments + 1];     // first piece of each segment; pbeg[n] = pieces
+};
+
+// attn_seg_pool_kernel: grid (piece, slice of kAggCols columns).  Eight row groups of 32
+// threads; a thread owns one 16-byte piece (8 columns) of every eighth row and keeps eight
+// rows' loads in flight; the row groups' sums are added in shared memory, in order.
+__global__ void __launch_bounds__(kThreads) attn_seg_pool_kernel(const __grid_constant__ Pieces pm,
+                                                                 const __nv_bfloat16* __restrict__ x, int d,
+                                                                 const float* __restrict__ attn,
+                                                                 float* __restrict__ wsum, float* __restrict__ asum) {
+  __shared__ float red[kAggGroups][kAggCols];
+  __shared__ float ared[kAggGroups];
+  const int pc = blockIdx.x;
+  int sl = 0, sh = pm.n - 1;  // the segment owning piece pc: the last s with pbeg[s] <= pc
+  while (sl < sh) {
+    const int mid = (sl + sh + 1) >> 1;
+    if (pm.pbeg[mid] <= pc)
+      sl = mid;
+    else
+      sh = mid - 1;
+  }
+  const int lo = pm.off[sl] + (pc - pm.pbeg[sl]) * kAggPiece, hi = min(pm.off[sl + 1], lo + kAggPiece);
+  const int lane = threadIdx.x & 31, rg = threadIdx.x >> 5;
+  const int c = blockIdx.y * (kAggCols / 8) + lane;  // 16-byte piece of the row
+  const bool cin = c < d / 8;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  float wacc = 0.f;
+  const uint4* xc = reinterpret_cast<const uint4*>(x) + (cin ? c : 0);
+  const size_t rs = (size_t)d / 8;  // row stride in pieces
+  int t = lo + rg;
+  for (; t + 7 * kAggGroups < hi; t += 8 * kAggGroups) {
+    uint4 v[2][4];
+    ld_stream4(v[0], xc + (size_t)t * rs, xc + (size_t)(t + kAggGroups) * rs, xc + (size_t)(t + 2 * kAggGroups) * rs,
+               xc + (size_t)(t + 3 * kAggGroups) * rs);
+    ld_stream4(v[1], xc + (size_t)(t + 4 * kAggGroups) * rs, xc + (size_t)(t + 5 * kAggGroups) * rs,
+               xc + (size_t)(t + 6 * kAggGroups) * rs, xc + (size_t)(t + 7 * kAggGroups) * rs);
+    float w[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        float f0[8];
-        unpack8(v[u], f0);
+    for (int u = 0; u < 8; ++u) w[u] = __ldg(attn + t + u * kAggGroups);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[j] = fmaf(wv[u], f0[j], acc[j]);
-      }
+    for (int u = 0; u < 8; ++u) {
+      float f[8];
+      unpack8(v[u >> 2][u & 3], f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] = fmaf(w[u], f[j], acc[j]);
+      wacc += w[u];
     }
-    for (; t < r1; ++t) {
-      const float w0 = __ldg(attn + t);
-      float f0[8];
-      unpack8(__ldg(reinterpret_cast<const uint4*>(x + (size_t)t * d) + c), f0);
+  }
+  for (; t < hi; t += kAggGroups) {
+    const float w0 = __ldg(attn + t);
+    float f[8];
+    unpack8(__ldg(xc + (size_t)t * rs), f);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] = fmaf(w0, f0[j], acc[j]);
-    }
+    for (int j = 0; j < 8; ++j) acc[j] = fmaf(w0, f[j], acc[j]);
+    wacc += w0;
+  }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) atomicAdd(out + (size_t)i * d + 8 * c + j, acc[j]);
+  for (int j = 0; j < 8; ++j) red[rg][lane * 8 + j] = acc[j];
+  if (lane == 0) ared[rg] = wacc;  // (every lane of the group summed the same weights)
+  __syncthreads();
+  const int col = blockIdx.y * kAggCols + threadIdx.x;
+  if (col < d) {
+    float tot = 0.f;
+#pragma unroll
+    for (int r = 0; r < kAggGroups; ++r) tot += red[r][threadIdx.x];
+    wsum[(size_t)pc * d + col] = tot;
+  }
+  if (blockIdx.y == 0 && threadIdx.x == 0) {
+    float a = 0.f;
+    for (int r = 0; r < kAggGroups; ++r) a += ared[r];
+    asum[pc] = a;
   }
 }
 
-// One CTA per event: out = g_emb + out / (sum of the range's weights), or g_emb alone when
-// the range is empty or carries no weight.
-__global__ void __launch_bounds__(kThreads) attn_finalize_kernel(const __grid_constant__ Offsets so, int d,
-                                                                 const float* __restrict__ attn,
-                                                                 const int32_t* __restrict__ interval,
-                                                                 const __nv_bfloat16* __restrict__ g_emb,
-                                                                 float* __restrict__ out) {
-  __shared__ float wsum[kThreads / 32];
-  const int i = blockIdx.x;
-  int lo, hi;
-  agg_range(so, interval, i, lo, hi);
-  float w = 0.f;
-  for (int t = lo + threadIdx.x; t < hi; t += kThreads) w += __ldg(attn + t);
+// attn_event_kernel: grid (event, slice of kAggCols columns).  The pieces of the event's
+// interval (lo, hi), clamped to the segments, are spread over the eight warps (warp w takes
+// every eighth piece from the first); a lane adds 8 columns; the warps' sums are added in
+// shared memory, in order, and out = g_emb + sum W / sum A (g_emb alone when sum A is 0).
+__global__ void __launch_bounds__(kThreads) attn_event_kernel(const __grid_constant__ Pieces pm, int d,
+                                                              const int32_t* __restrict__ interval,
+                                                              const float* __restrict__ wsum,
+                                                              const float* __restrict__ asum,
+                                                              const __nv_bfloat16* __restrict__ g_emb,
+                                                              float* __restrict__ out) {
+  __shared__ float red[kAggGroups][kAggCols];
+  __shared__ float ared[kAggGroups];
+  const int i = blockIdx.x, S = pm.n;
+  const int s_lo = min(max(interval[2 * i], 0), S - 1), s_hi = min(max(interval[2 * i + 1], s_lo), S - 1);
+  const int p0 = pm.pbeg[s_lo], p1 = pm.pbeg[s_hi + 1];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int c8 = blockIdx.y * kAggCols + lane * 8;  // first of this lane's 8 columns
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  float a = 0.f;
+  if (c8 < d) {
+    for (int pc = p0 + w; pc < p1; pc += kAggGroups) {
+      const float4* src = reinterpret_cast<const float4*>(wsum + (size_t)pc * d + c8);
+      const float4 u0 = __ldg(src), u1 = __ldg(src + 1);
+      acc[0] += u0.x;
+      acc[1] += u0.y;
+      acc[2] += u0.z;
+      acc[3] += u0.w;
+      acc[4] += u1.x;
+      acc[5] += u1.y;
+      acc[6] += u1.z;
+      acc[7] += u1.w;
+      a += __ldg(asum + pc);
+    }
+  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = w;
+  for (int j = 0; j < 8; ++j) red[w][lane * 8 + j] = acc[j];
+  if (lane == 0) ared[w] = a;
   __syncthreads();
-  float den = 0.f;
-  for (int k = 0; k < kThreads / 32; ++k) den += wsum[k];
-  for (int c = threadIdx.x; c < d; c += kThreads) {
-    const float base = __bfloat162float(g_emb[(size_t)i * d + c]);
-    const size_t o = (size_t)i * d + c;
-    out[o] = den > 0.f ? base + out[o] / den : base;
+  const int col = blockIdx.y * kAggCols + threadIdx.x;
+  if (col < d) {
+    float num = 0.f, den = 0.f;
+#pragma unroll
+    for (int r = 0; r < kAggGroups; ++r) {
+      num += red[r][threadIdx.x];
+      den += ared[r];
+    }
+    const float base = __bfloat162float(g_emb[(size_t)i * d + col]);
+    out[(size_t)i * d + col] = den > 0.f ? base + num / den : base;
   }
 }
 
@@ -329,23 +393,38 @@ cudaError_t launch_ground_score(const void* g_proj, int32_t n_events, const floa
   return cudaGetLastError();
 }
 
+size_t attn_aggregate_ws_floats(int64_t n_tokens, int32_t n_segments, int32_t d) {
+  return ((size_t)n_segments + (size_t)(n_tokens + kAggPiece - 1) / kAggPiece) * ((size_t)d + 1);
+}
+
 cudaError_t launch_attn_aggregate(const void* x, int64_t n_tokens, int32_t d, const float* attn,
                                   const int32_t* offsets, int32_t n_segments, const int32_t* interval,
-                                  int32_t n_events, const void* g_emb, float* out, cudaStream_t s) {
+                                  int32_t n_events, const void* g_emb, float* seg_ws, float* out, cudaStream_t s) {
   Offsets so;
   if (!fill_offsets(so, offsets, n_segments, n_tokens)) return cudaErrorInvalidValue;
   if (n_events == 0) return cudaSuccess;
-  // the longest range any interval can select: all segments
-  const int slices = std::max(1, (so.off[n_segments] - so.off[0] + kAggSlice - 1) / kAggSlice);
+  Pieces pm;
+  pm.n = n_segments;
+  pm.pbeg[0] = 0;
+  for (int i = 0; i < n_segments; ++i) {
+    pm.off[i] = so.off[i];
+    pm.pbeg[i + 1] = pm.pbeg[i] + (so.off[i + 1] - so.off[i] + kAggPiece - 1) / kAggPiece;
+  }
+  pm.off[n_segments] = so.off[n_segments];
+  const int pieces = pm.pbeg[n_segments];
+  const int slices = (d + kAggCols - 1) / kAggCols;
   if (slices > 65535) return cudaErrorInvalidValue;
-  cudaError_t e = cudaMemsetAsync(out, 0, (size_t)n_events * d * sizeof(float), s);
-  if (e != cudaSuccess) return e;
-  attn_aggregate_kernel<<<dim3(n_events, slices), kThreads, 0, s>>>(so, static_cast<const __nv_bfloat16*>(x), d,
-                                                                     attn, interval, out);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  attn_finalize_kernel<<<n_events, kThreads, 0, s>>>(so, d, attn, interval, static_cast<const __nv_bfloat16*>(g_emb),
-                                                      out);
+  // (pieces <= n_segments + n_tokens / kAggPiece: within attn_aggregate_ws_floats)
+  float* wsum = seg_ws;
+  float* asum = seg_ws + (size_t)std::max(pieces, 1) * d;
+  if (pieces > 0) {
+    attn_seg_pool_kernel<<<dim3(pieces, slices), kThreads, 0, s>>>(pm, static_cast<const __nv_bfloat16*>(x), d, attn,
+                                                                   wsum, asum);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  attn_event_kernel<<<dim3(n_events, slices), kThreads, 0, s>>>(pm, d, interval, wsum, asum,
+                                                                 static_cast<const __nv_bfloat16*>(g_emb), out);
   return cudaGetLastError();
 }
 

@@ -274,7 +274,8 @@ cudaError_t launch_ground_score(const void* g_proj, int32_t n_events, const floa
                                 cudaStream_t s);
 cudaError_t launch_attn_aggregate(const void* x, int64_t n_tokens, int32_t d, const float* attn,
                                   const int32_t* offsets, int32_t n_segments, const int32_t* interval,
-                                  int32_t n_events, const void* g_emb, float* out, cudaStream_t s);
+                                  int32_t n_events, const void* g_emb, float* seg_ws, float* out, cudaStream_t s);
+size_t attn_aggregate_ws_floats(int64_t n_tokens, int32_t n_segments, int32_t d);
 cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
                                 const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
 

@@ -41,10 +41,17 @@ def _run(gi, frac):
     sal = torch.empty((K, S), dtype=torch.uint8, device="cuda")
     iv = torch.empty((K, 2), dtype=torch.int32, device="cuda")
     out = torch.empty((K, gi.x.shape[1]), dtype=torch.float32, device="cuda")
+    ws = B.aggregate_workspace(T, S, gi.x.shape[1])
     B.pad_ground_pool(f, gi.offsets, seg)
     B.pad_ground_score(g, seg, frac, scores, sal, iv)
-    B.pad_attn_aggregate(x, attn, gi.offsets, iv, emb, out)
+    B.pad_attn_aggregate(x, attn, gi.offsets, iv, emb, out, ws)
     torch.cuda.synchronize()
+    # every pooled element is written once and summed in a fixed order: a second call
+    # reproduces the output bit for bit
+    out2 = torch.empty_like(out)
+    B.pad_attn_aggregate(x, attn, gi.offsets, iv, emb, out2, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2)
     return seg.cpu().numpy(), scores.cpu().numpy(), sal.cpu().numpy().astype(bool), iv.cpu().numpy(), out.cpu().numpy()
 
 
@@ -108,3 +115,19 @@ def test_grounding_edge_cases():
     with pytest.raises(B.PadError):
         B.pad_ground_pool(_dev_bf16(gi.f_proj), np.array([0, 700], np.int32),
                           torch.empty((1, 16), dtype=torch.float32, device="cuda"))
+
+
+def test_aggregate_long_segment_is_split():
+    """A segment of 3000 tokens is pooled in 12 pieces of at most 256 tokens, and a hidden
+    size that is not a multiple of 256 leaves a partial column slice; a scratch one float
+    short of the documented size is refused."""
+    gi = synth.grounding_inputs(9, 3400, 3, 4, 32, 520, text_tokens=0)
+    gi.offsets[:] = np.array([0, 200, 3200, 3400], np.int32)
+    _check(gi, 0.5)
+    ws = B.aggregate_workspace(3400, 3, 520)
+    assert ws.numel() == (3 + 14) * 521
+    with pytest.raises(B.PadError) as ei:
+        B.pad_attn_aggregate(_dev_bf16(gi.x), torch.from_numpy(gi.attn).cuda(), gi.offsets,
+                             torch.zeros((4, 2), dtype=torch.int32, device="cuda"), _dev_bf16(gi.g_emb),
+                             torch.empty((4, 520), dtype=torch.float32, device="cuda"), ws[:-1])
+    assert ei.value.status == 4

@@ -177,10 +177,19 @@ def test_large_group_and_outlier_channels(flags):
 # Edge cases
 # ---------------------------------------------------------------------------
 
-def _w(prefix, epv, lens, seed=7, h_q=28, h_kv=4, D=128, sigma=None):
+def _w(prefix, epv, lens, seed=7, h_q=28, h_kv=4, D=128, sigma=None, page_size=16):
     rng = np.random.default_rng(seed)
     return synth.make_workload("edge", seed, h_q, h_kv, D, prefix, epv, lens, rng=rng,
-                               k_scale_sigma=sigma)
+                               k_scale_sigma=sigma, page_size=page_size)
+
+
+@pytest.mark.parametrize("ps", [4, 8, 32, 64])
+def test_page_sizes_many_events(ps):
+    """40 events of 7 rows (280 rows: three 128-row groups, two events straddling group
+    boundaries) with branch lengths on and around page boundaries, for page sizes other
+    than 16, over pools whose unwritten slots hold NaN."""
+    lens = [(37 * i) % 131 for i in range(36)] + [ps, ps - 1, 2 * ps + 1, 0]
+    run_full(_w([3000], [40], lens, seed=41 + ps, page_size=ps), flags=B.FLAG_PREFIX_TC, what=f"ps {ps}")
 
 
 @pytest.mark.parametrize("flags", [B.FLAG_PREFIX_SIMT, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
