@@ -584,7 +584,7 @@ def run_reference(args):
 def run_prefill(args):
     """Whole-sequence forward attention under the event-factorized mask (training /
     prefill), on the long_32k video: prefix 32768 tokens, then its 32 branches (each the
-    branch's tokens after this step, 2080 in all).  Timed with CUDA events over repeated
+    branch's tokens after this step, 1917 in all).  Timed with CUDA events over repeated
     calls (compute-bound; inputs stay resident).  Comparators on the same tensors: torch's
     scaled_dot_product_attention with the explicit boolean mask (the generic masked path the
     paper used), and with is_causal=True (the plain causal kernel, which computes a
