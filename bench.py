@@ -211,13 +211,17 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+# The sources that define the dominant kernel of the decode step (the tensor-core prefix
+# kernel, the branch/merge task it can run, and the descriptors both read).
+TRAFFIC_SOURCES = ("pad_internal.h", "pad_branch_merge.cuh", "pad_prefix_tc.cu")
+
+
 def kernel_source_hash():
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_02963_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".h", ".cuh")):
-            with open(os.path.join(csrc, f), "rb") as fh:
-                h.update(fh.read())
+    for f in TRAFFIC_SOURCES:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()[:16]
 
 

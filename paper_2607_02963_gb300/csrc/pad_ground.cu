@@ -136,23 +136,23 @@ __global__ void __launch_bounds__(kThreads) ground_score_kernel(const __nv_bfloa
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int c = threadIdx.x; c < d; c += kThreads) gs[c] = __bfloat162float(g[(size_t)i * d + c]);
   __syncthreads();
-  // a warp per segment row (lanes over its float4 columns), four rows in flight per warp
+  // a warp per segment row (lanes over its float4 columns), eight rows in flight per warp
   float best = -__builtin_huge_valf();
   const int d4 = d / 4;
-  for (int s0 = warp * 4; s0 < S; s0 += 4 * (kThreads / 32)) {
-    float part[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int s0 = warp * 8; s0 < S; s0 += 8 * (kThreads / 32)) {
+    float part[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     for (int c = lane; c < d4; c += 32) {
-      float4 v[4];
+      float4 v[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
-        v[u] = s0 + u < S ? reinterpret_cast<const float4*>(seg_sum + (size_t)(s0 + u) * d)[c]
+      for (int u = 0; u < 8; ++u)
+        v[u] = s0 + u < S ? __ldg(reinterpret_cast<const float4*>(seg_sum + (size_t)(s0 + u) * d) + c)
                           : make_float4(0.f, 0.f, 0.f, 0.f);
       const float g0 = gs[4 * c], g1 = gs[4 * c + 1], g2 = gs[4 * c + 2], g3 = gs[4 * c + 3];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) part[u] += (g0 * v[u].x + g1 * v[u].y) + (g2 * v[u].z + g3 * v[u].w);
+      for (int u = 0; u < 8; ++u) part[u] += (g0 * v[u].x + g1 * v[u].y) + (g2 * v[u].z + g3 * v[u].w);
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       float v = part[u];
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
