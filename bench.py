@@ -353,16 +353,18 @@ def run_ours(args):
                 gi[ev] = np.arange(len(ev)) % Kp[b]
         self_g = (Kp, gi)
 
+    # the library's step executor: one C call per step (pad_step_run), or with the host
+    # copies and the wait included (pad_step_run_host)
     def launcher(db, **kw):
-        return B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
-                              db.page_table, w.max_pages, db.workspace, w.prefix_offset,
-                              kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
-                              db.k_pool, db.v_pool, db.out, db.lse, stream,
-                              one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal)
+        return B.NativeStep(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                            db.page_table, w.max_pages, db.workspace, w.prefix_offset,
+                            kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
+                            db.k_pool, db.v_pool, db.out, db.lse, stream,
+                            one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal)
 
     one_call = not args.two_call
-    api_path = ("pad_plan + pad_decode_step" if one_call
-                else "pad_plan + pad_kv_append + pad_event_decode_attn")
+    api_path = ("pad_step_run (pad_plan + pad_decode_step)" if one_call
+                else "pad_step_run (pad_plan + pad_kv_append + pad_event_decode_attn)")
     steps = [launcher(db) for db in reps]
     info = reps[0].plan_step(stream).info()
     # kernels of one step: append (two-call path only), prefix pass, branch/merge (unless
@@ -424,14 +426,9 @@ def run_ours(args):
     d2h = sum(t.numel() * t.element_size() for t in (hout, hlse))
 
     def e2e_step(i):
-        db = reps[i % n_rep]
-        db.q.copy_(hq, non_blocking=True)
-        db.k_new.copy_(hkn, non_blocking=True)
-        db.v_new.copy_(hvn, non_blocking=True)
-        steps[i % n_rep]()
-        hout.copy_(db.out, non_blocking=True)
-        hlse.copy_(db.lse, non_blocking=True)
-        stream.synchronize()
+        # pad_step_run_host: H2D of q / k_new / v_new, the step, D2H of out and lse, and the
+        # wait for the stream, in one call
+        steps[i % n_rep].run_host(hq, hkn, hvn, hout, hlse)
 
     for i in range(3):
         e2e_step(i)
@@ -443,8 +440,9 @@ def run_ours(args):
     e_units, e_ms = aggregate(float(w.n_events * Ke), e2e_ms, device)
     e2e = {"value": e_units / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
            "d2h_bytes_per_step": d2h, "steps": Ke,
-           "path": "pinned H2D of q/k_new/v_new, " + api_path + " through the C ABI, D2H of O and "
-                   "LSE, stream sync every step"}
+           "path": "pad_step_run_host through the C ABI: pinned H2D of q/k_new/v_new, pad_plan + "
+                   + ("pad_decode_step" if one_call else "pad_kv_append + pad_event_decode_attn")
+                   + ", D2H of O and LSE, stream sync, every step"}
 
     if rank != 0:
         return
@@ -809,7 +807,7 @@ def run_sweep(args):
         per_rep = first.k_prefix.numel() * 4 + first.k_pool.numel() * 4
         n_rep = max(2, -(-3 * l2 // per_rep))
         reps = [first] + [DeviceBatch(w, device=device, fill_nan=False) for _ in range(n_rep - 1)]
-        steps = [B.StepLauncher(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+        steps = [B.NativeStep(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
                                 db.page_table, w.max_pages, db.workspace, w.prefix_offset, db.q,
                                 db.k_new, db.v_new, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool,
                                 db.out, db.lse, stream) for db in reps]

@@ -270,6 +270,45 @@ pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_
                            const void* k_prefix, const void* v_prefix, void* k_pool, void* v_pool,
                            void* out, float* lse, pad_stream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * Step executor (host runtime of a serving loop; the paper has no counterpart).  It holds
+ * every argument of a decode step, so that a step costs one call: pad_step_run plans the
+ * step from the caller's host arrays as they are at that moment and launches it;
+ * pad_step_run_host also copies this step's q, k_new and v_new in from host memory and out
+ * and lse back, then waits for the stream.
+ *   arguments  as pad_plan and pad_decode_step; the host arrays prefix_len, prefix_offset,
+ *              event_video and event_len are borrowed (the caller keeps them alive and may
+ *              change them between runs: a generation loop advances event_len in place);
+ *              workspace and page_table are required
+ *   options    PAD_STEP_TWO_CALL: pad_kv_append + pad_event_decode_attn instead of
+ *              pad_decode_step; PAD_STEP_RELEASE_PAGES: hand the pages a run took back to
+ *              the cache after launching it (to repeat one identical step, e.g. for timing)
+ *   new_page   [n_events] host, may be NULL: the pages the run took (pad_plan_new_pages)
+ * A run that fails before launching hands its pages back and returns the plan's status.
+ * The mask variants and RoPE are set once (pad_step_set_*: the same arguments as the
+ * pad_plan_set_* calls, borrowed the same way) and apply to every later run. */
+typedef struct pad_step_t pad_step_t;
+#define PAD_STEP_TWO_CALL 0x1
+#define PAD_STEP_RELEASE_PAGES 0x2
+pad_status pad_step_create(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
+                           const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
+                           const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
+                           int32_t max_pages, void* workspace, size_t workspace_bytes, const void* q,
+                           const void* k_new, const void* v_new, const void* k_prefix, const void* v_prefix,
+                           void* k_pool, void* v_pool, void* out, float* lse, pad_stream_t stream,
+                           int32_t options, pad_step_t** step_out);
+pad_status pad_step_set_rope(pad_step_t* step, const int32_t* positions, const float* cos_sin, int32_t max_position);
+pad_status pad_step_set_g_visibility(pad_step_t* step, int32_t mode, const int32_t* n_planning,
+                                     const int32_t* g_index);
+pad_status pad_step_set_branch_visibility(pad_step_t* step, int32_t mode);
+pad_status pad_step_run(pad_step_t* step, int32_t* new_page);
+/*   h_q [n_events, h_q, head_dim] bf16, h_k_new / h_v_new [n_events, h_kv, head_dim] bf16,
+ *   h_out [n_events, h_q, head_dim] (the problem's out_dtype), h_lse [n_events, h_q] fp32
+ *   or NULL; host memory (page-locked for asynchronous copies). */
+pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
+                             void* h_out, float* h_lse, int32_t* new_page);
+void pad_step_destroy(pad_step_t* step);
+
 /* Allocation-free variant of pad_event_decode_attn (the paper has no counterpart; this
  * is an interface for callers, not part of the method).  Same arguments and result.  It
  * is meant for callers that cannot give the library device scratch memory, for example a

@@ -70,6 +70,15 @@ _SIGNATURES = {
                            POINTER(c_void_p)]),
     "pad_plan_new_pages": (c_int32, [c_void_p, _I32P]),
     "pad_plan_release_new_pages": (c_int32, [c_void_p, c_void_p]),
+    "pad_step_create": (c_int32, [POINTER(Problem), c_void_p, c_int32, _I32P, _I64P, c_int32, _I32P, _I32P,
+                                  c_void_p, c_int32, c_void_p, c_size_t] + [c_void_p] * 10
+                        + [c_int32, POINTER(c_void_p)]),
+    "pad_step_set_rope": (c_int32, [c_void_p, _I32P, c_void_p, c_int32]),
+    "pad_step_set_g_visibility": (c_int32, [c_void_p, c_int32, _I32P, _I32P]),
+    "pad_step_set_branch_visibility": (c_int32, [c_void_p, c_int32]),
+    "pad_step_run": (c_int32, [c_void_p, _I32P]),
+    "pad_step_run_host": (c_int32, [c_void_p] * 6 + [_I32P]),
+    "pad_step_destroy": (None, [c_void_p]),
     "pad_plan_set_rope": (c_int32, [c_void_p, _I32P, c_void_p, c_int32]),
     "pad_plan_set_g_visibility": (c_int32, [c_void_p, c_int32, _I32P, _I32P]),
     "pad_plan_set_branch_visibility": (c_int32, [c_void_p, c_int32]),
@@ -370,6 +379,73 @@ def pad_timing_read():
     n = c_int32()
     _check(lib().pad_timing_read(ctypes.byref(ms), ctypes.byref(n)))
     return float(ms.value), int(n.value)
+
+
+STEP_TWO_CALL = 0x1
+STEP_RELEASE_PAGES = 0x2
+
+
+class NativeStep:
+    """The library's step executor (pad_step_*): every argument marshalled once in C, so a
+    step is one call (``run``), or one call with the host copies and the wait included
+    (``run_host``).  ``event_len`` is borrowed: update it in place between runs (a
+    generation loop), the next run plans from its current values."""
+
+    def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
+                 page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
+                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True,
+                 rope=None, self_g=None, causal=False):
+        self.L = lib()
+        self.problem = problem
+        self.cache = cache
+        self.prefix_len = np.ascontiguousarray(prefix_len, dtype=np.int32)
+        self.event_video = np.ascontiguousarray(event_video, dtype=np.int32)
+        # the executor reads this array at every run
+        self.event_len = np.array(event_len, dtype=np.int32, copy=True)
+        self.prefix_offset = (None if prefix_offset is None
+                              else np.ascontiguousarray(prefix_offset, dtype=np.int64))
+        self._keep = [q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse, workspace, page_table]
+        self.ne = int(self.event_video.size)
+        opts = (0 if one_call else STEP_TWO_CALL) | (STEP_RELEASE_PAGES if release_pages else 0)
+        h = c_void_p()
+        _check(self.L.pad_step_create(
+            ctypes.byref(problem), cache.handle, int(self.prefix_len.size), self.prefix_len.ctypes.data_as(_I32P),
+            None if self.prefix_offset is None else self.prefix_offset.ctypes.data_as(_I64P), self.ne,
+            self.event_video.ctypes.data_as(_I32P), self.event_len.ctypes.data_as(_I32P), _ptr(page_table),
+            int(max_pages), _ptr(workspace), int(workspace.numel() * workspace.element_size()), _ptr(q),
+            _ptr(k_new), _ptr(v_new), _ptr(k_prefix), _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool), _ptr(out),
+            _ptr(lse), _stream(stream), opts, ctypes.byref(h)))
+        self.handle = h
+        if rope is not None:
+            self.rope_pos = np.ascontiguousarray(rope[0], dtype=np.int32)
+            self._keep.append(rope[1])
+            _check(self.L.pad_step_set_rope(h, self.rope_pos.ctypes.data_as(_I32P), _ptr(rope[1]),
+                                            int(rope[1].shape[0])))
+        if self_g is not None:
+            self.g_k = np.ascontiguousarray(self_g[0], dtype=np.int32)
+            self.g_i = np.ascontiguousarray(self_g[1], dtype=np.int32)
+            _check(self.L.pad_step_set_g_visibility(h, G_SELF, self.g_k.ctypes.data_as(_I32P),
+                                                    self.g_i.ctypes.data_as(_I32P)))
+        if causal:
+            _check(self.L.pad_step_set_branch_visibility(h, BRANCH_CAUSAL))
+        self.new_page = np.full(self.ne, -1, dtype=np.int32)
+        self._np = self.new_page.ctypes.data_as(_I32P)
+        self._run = self.L.pad_step_run
+        self._run_host = self.L.pad_step_run_host
+
+    def __call__(self):
+        _check(self._run(self.handle, self._np))
+
+    def run_host(self, h_q, h_k_new, h_v_new, h_out, h_lse=None):
+        """Host tensors (page-locked): copies in, the step, copies out, stream wait."""
+        _check(self._run_host(self.handle, h_q.data_ptr(), h_k_new.data_ptr(), h_v_new.data_ptr(), h_out.data_ptr(),
+                              None if h_lse is None else h_lse.data_ptr(), self._np))
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h is not None and h.value:
+            self.L.pad_step_destroy(h)
+            self.handle = None
 
 
 class StepLauncher:

@@ -940,6 +940,172 @@ pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_
   return launch_attention(plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse, stream);
 }
 
+// ---------------------------------------------------------------------------
+// Step executor: a serving loop's host side in one call per step.
+// ---------------------------------------------------------------------------
+struct pad_step_t {
+  pad_problem prob{};
+  pad_cache_state* cache = nullptr;
+  int32_t n_videos = 0, n_events = 0, max_pages = 0, options = 0;
+  const int32_t* prefix_len = nullptr;
+  const int64_t* prefix_offset = nullptr;
+  const int32_t* event_video = nullptr;
+  const int32_t* event_len = nullptr;
+  int32_t* page_table = nullptr;
+  void* workspace = nullptr;
+  size_t workspace_bytes = 0;
+  const void *q = nullptr, *k_new = nullptr, *v_new = nullptr, *k_prefix = nullptr, *v_prefix = nullptr;
+  void *k_pool = nullptr, *v_pool = nullptr, *out = nullptr;
+  float* lse = nullptr;
+  pad_stream_t stream = nullptr;
+  const int32_t* rope_pos = nullptr;
+  const float* rope_cs = nullptr;
+  int32_t rope_max = 0;
+  int32_t g_mode = PAD_G_ALL;
+  const int32_t* g_planning = nullptr;
+  const int32_t* g_index = nullptr;
+  int32_t branch_mode = PAD_BRANCH_OWN;
+};
+
+pad_status pad_step_create(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
+                           const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
+                           const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
+                           int32_t max_pages, void* workspace, size_t workspace_bytes, const void* q,
+                           const void* k_new, const void* v_new, const void* k_prefix, const void* v_prefix,
+                           void* k_pool, void* v_pool, void* out, float* lse, pad_stream_t stream,
+                           int32_t options, pad_step_t** step_out) {
+  if (!step_out) return fail(PAD_ERR_INVALID_ARG, "step_out is NULL");
+  *step_out = nullptr;
+  pad_status st = check_problem(prob);
+  if (st != PAD_OK) return st;
+  if (!cache) return fail(PAD_ERR_INVALID_ARG, "cache is NULL");
+  if (options & ~(PAD_STEP_TWO_CALL | PAD_STEP_RELEASE_PAGES)) return fail(PAD_ERR_INVALID_ARG, "unknown options 0x%x", options);
+  if (n_videos < 0 || n_events < 0) return fail(PAD_ERR_INVALID_ARG, "negative batch size");
+  if (n_events > 0 && (!event_video || !event_len || !prefix_len)) return fail(PAD_ERR_INVALID_ARG, "NULL host array");
+  if (!workspace || !page_table) return fail(PAD_ERR_INVALID_ARG, "workspace / page_table is NULL");
+  if (n_events > 0 && (!q || !k_pool || !v_pool || !out || !k_new || !v_new))
+    return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  auto* x = new pad_step_t();
+  x->prob = *prob;
+  x->cache = cache;
+  x->n_videos = n_videos;
+  x->n_events = n_events;
+  x->max_pages = max_pages;
+  x->options = options;
+  x->prefix_len = prefix_len;
+  x->prefix_offset = prefix_offset;
+  x->event_video = event_video;
+  x->event_len = event_len;
+  x->page_table = page_table;
+  x->workspace = workspace;
+  x->workspace_bytes = workspace_bytes;
+  x->q = q;
+  x->k_new = k_new;
+  x->v_new = v_new;
+  x->k_prefix = k_prefix;
+  x->v_prefix = v_prefix;
+  x->k_pool = k_pool;
+  x->v_pool = v_pool;
+  x->out = out;
+  x->lse = lse;
+  x->stream = stream;
+  *step_out = x;
+  return PAD_OK;
+}
+
+pad_status pad_step_set_rope(pad_step_t* step, const int32_t* positions, const float* cos_sin, int32_t max_position) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  if (cos_sin && (max_position <= 0 || !aligned16(cos_sin) || (step->n_events > 0 && !positions)))
+    return fail(PAD_ERR_INVALID_ARG, "positions / cos_sin / max_position");
+  step->rope_pos = cos_sin ? positions : nullptr;
+  step->rope_cs = cos_sin;
+  step->rope_max = cos_sin ? max_position : 0;
+  return PAD_OK;
+}
+
+pad_status pad_step_set_g_visibility(pad_step_t* step, int32_t mode, const int32_t* n_planning,
+                                     const int32_t* g_index) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  if (mode != PAD_G_ALL && mode != PAD_G_SELF) return fail(PAD_ERR_INVALID_ARG, "mode %d", mode);
+  if (mode == PAD_G_SELF && ((step->n_videos > 0 && !n_planning) || (step->n_events > 0 && !g_index)))
+    return fail(PAD_ERR_INVALID_ARG, "n_planning / g_index is NULL");
+  step->g_mode = mode;
+  step->g_planning = n_planning;
+  step->g_index = g_index;
+  return PAD_OK;
+}
+
+pad_status pad_step_set_branch_visibility(pad_step_t* step, int32_t mode) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  if (mode != PAD_BRANCH_OWN && mode != PAD_BRANCH_CAUSAL) return fail(PAD_ERR_INVALID_ARG, "mode %d", mode);
+  step->branch_mode = mode;
+  return PAD_OK;
+}
+
+pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  pad_plan_t* plan = nullptr;
+  pad_status st = pad_plan(&step->prob, step->cache, step->n_videos, step->prefix_len, step->prefix_offset,
+                           step->n_events, step->event_video, step->event_len, step->page_table, step->max_pages,
+                           step->workspace, step->workspace_bytes, step->stream, &plan);
+  if (st != PAD_OK) return st;
+  if (step->rope_cs) st = pad_plan_set_rope(plan, step->rope_pos, step->rope_cs, step->rope_max);
+  if (st == PAD_OK && step->g_mode == PAD_G_SELF)
+    st = pad_plan_set_g_visibility(plan, PAD_G_SELF, step->g_planning, step->g_index);
+  if (st == PAD_OK && step->branch_mode == PAD_BRANCH_CAUSAL) st = pad_plan_set_branch_visibility(plan, PAD_BRANCH_CAUSAL);
+  if (st == PAD_OK) {
+    if (step->options & PAD_STEP_TWO_CALL) {
+      st = pad_kv_append(plan, step->k_new, step->v_new, step->k_pool, step->v_pool, step->stream);
+      if (st == PAD_OK)
+        st = pad_event_decode_attn(plan, step->q, step->k_prefix, step->v_prefix, step->k_pool, step->v_pool,
+                                   step->out, step->lse, step->stream);
+    } else {
+      st = pad_decode_step(plan, step->q, step->k_new, step->v_new, step->k_prefix, step->v_prefix, step->k_pool,
+                           step->v_pool, step->out, step->lse, step->stream);
+    }
+  }
+  if (st == PAD_OK && new_page) st = pad_plan_new_pages(plan, new_page);
+  if (st != PAD_OK || (step->options & PAD_STEP_RELEASE_PAGES)) {
+    // a step that failed before launching hands its pages back; so does a timing loop
+    const pad_status keep = st;
+    pad_plan_release_new_pages(plan, step->cache);
+    st = keep;
+  }
+  pad_plan_destroy(plan);
+  return st;
+}
+
+pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
+                             void* h_out, float* h_lse, int32_t* new_page) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  if (step->n_events > 0 && (!h_q || !h_k_new || !h_v_new || !h_out))
+    return fail(PAD_ERR_INVALID_ARG, "NULL host buffer");
+  if (step->n_events > 0 && h_lse && !step->lse) return fail(PAD_ERR_INVALID_ARG, "h_lse given but the step has no lse");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(step->stream);
+  const pad_problem& pr = step->prob;
+  const size_t E = (size_t)step->n_events, D = (size_t)pr.head_dim;
+  const size_t q_bytes = E * pr.h_q * D * 2, kv_bytes = E * pr.h_kv * D * 2;
+  const size_t o_bytes = E * pr.h_q * D * (pr.out_dtype == 1 ? 2 : 4), l_bytes = E * pr.h_q * sizeof(float);
+  cudaError_t e = cudaSuccess;
+  if (E > 0) {
+    e = cudaMemcpyAsync(const_cast<void*>(step->q), h_q, q_bytes, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->k_new), h_k_new, kv_bytes, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->v_new), h_v_new, kv_bytes, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "step inputs H2D");
+  }
+  pad_status st = pad_step_run(step, new_page);
+  if (st != PAD_OK) return st;
+  if (E > 0) {
+    e = cudaMemcpyAsync(h_out, step->out, o_bytes, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && h_lse) e = cudaMemcpyAsync(h_lse, step->lse, l_bytes, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_fail(e, "step outputs D2H");
+  }
+  e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "step synchronize");
+}
+
+void pad_step_destroy(pad_step_t* step) { delete step; }
+
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
   if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
   if (!plan->workspace) return PAD_OK;

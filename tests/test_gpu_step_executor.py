@@ -1,0 +1,98 @@
+"""The step executor (pad_step_*), the host runtime of a serving loop: one call per step.
+
+Its runs must be the library's own step calls, bit for bit: outputs, LSE, both pools and the
+page table against pad_plan + pad_decode_step (and + pad_kv_append + pad_event_decode_attn
+for the two-call option), the host-buffer run against the device-buffer run, and a
+generation loop that advances event_len in place against the same loop through pad_plan.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_02963_gb300 import binding as B
+from paper_2607_02963_gb300 import synth
+from paper_2607_02963_gb300.device import DeviceBatch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda(padlib):
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.init()
+
+
+def _native(db, w, **kw):
+    return B.NativeStep(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len, db.page_table,
+                        w.max_pages, db.workspace, w.prefix_offset, db.q, db.k_new, db.v_new, db.k_prefix,
+                        db.v_prefix, db.k_pool, db.v_pool, db.out, db.lse, torch.cuda.current_stream(), **kw)
+
+
+def _same_state(a, b):
+    assert torch.equal(a.out, b.out) and torch.equal(a.lse, b.lse)
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+    assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
+    assert torch.equal(a.page_table, b.page_table)
+
+
+@pytest.mark.parametrize("one_call", [True, False])
+@pytest.mark.parametrize("make", [synth.gqa_8k, lambda: synth.random_small(5), synth.tiny])
+def test_run_matches_the_step_calls(make, one_call):
+    w = make()
+    a = DeviceBatch(w)
+    pa = a.run_step(one_call=one_call)
+    b = DeviceBatch(w)
+    st = _native(b, w, release_pages=False, one_call=one_call)
+    st()
+    torch.cuda.synchronize()
+    B.pad_device_status(pa)
+    _same_state(a, b)
+    assert np.array_equal(st.new_page, pa.new_pages())
+    ref_o, ref_lse = oracle.decode_step(w)
+    got = b.out.float().cpu().numpy()
+    assert np.abs(got - ref_o).max() <= 1e-2
+
+
+def test_run_host_copies_in_and_out():
+    w = synth.gqa_8k()
+    a = DeviceBatch(w)
+    a.run_step(one_call=True)
+    torch.cuda.synchronize()
+    b = DeviceBatch(w)
+    hq = b.q.cpu().pin_memory()
+    hk = b.k_new.cpu().pin_memory()
+    hv = b.v_new.cpu().pin_memory()
+    b.q.zero_()
+    b.k_new.zero_()
+    b.v_new.zero_()
+    ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
+    hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
+    st = _native(b, w, release_pages=False)
+    st.run_host(hq, hk, hv, ho, hl)
+    assert torch.equal(ho, a.out.cpu()) and torch.equal(hl, a.lse.cpu())
+    _same_state(a, b)
+
+
+@pytest.mark.parametrize("one_call", [True, False])
+def test_generation_loop_advances_event_len_in_place(one_call):
+    """Three steps; each run plans from the executor's event_len as the loop left it."""
+    w = synth.make_workload("loop", 61, 28, 4, 128, [2500], [4], [14, 15, 31, 0],
+                            rng=np.random.default_rng(61))
+    a = DeviceBatch(w)
+    b = DeviceBatch(w)
+    st = _native(b, w, release_pages=False, one_call=one_call)
+    lens = w.event_len.copy()
+    for step in range(3):
+        a.plan = B.pad_plan(a.problem, a.cache, w.prefix_len, w.event_video, lens, page_table=a.page_table,
+                            max_pages=w.max_pages, workspace=a.workspace, prefix_offset=w.prefix_offset)
+        B.pad_decode_step(a.plan, a.q, a.k_new, a.v_new, a.k_prefix, a.v_prefix, a.k_pool, a.v_pool, a.out, a.lse)
+        st.event_len[:] = lens
+        st()
+        torch.cuda.synchronize()
+        B.pad_device_status(a.plan)
+        assert np.array_equal(st.new_page, a.plan.new_pages())
+        _same_state(a, b)
+        lens = lens + 1
+    assert np.array_equal(a.cache.free_pages(), b.cache.free_pages())

@@ -290,3 +290,40 @@ def test_set_branch_visibility_validates(padlib):
     with pytest.raises(B.PadError) as ei:
         plan.set_branch_visibility(2)
     assert ei.value.status == 1
+
+
+def test_step_executor_validates_and_returns_pages_of_a_failed_run(padlib):
+    """pad_step_create checks its arguments; a run whose launch fails (no device here, or a
+    refused launch) hands the pages its plan took back to the cache."""
+    import ctypes
+    prob = B.make_problem(8, 2, 128, num_sms=152)
+    cache = B.CacheState(64)
+    pl = np.array([500], np.int32)
+    ev = np.zeros(3, np.int32)
+    el = np.array([0, 16, 5], np.int32)  # two events start pages
+    h = ctypes.c_void_p()
+    fake = 1 << 20  # 16-byte aligned addresses, never dereferenced by the host
+    args = [ctypes.byref(prob), cache.handle, 1, pl.ctypes.data_as(B._I32P), None, 3, ev.ctypes.data_as(B._I32P),
+            el.ctypes.data_as(B._I32P), fake, 4, fake, 1 << 24] + [fake] * 9 + [None]
+    for bad_opts in (0x4, -1):
+        with pytest.raises(B.PadError) as ei:
+            B._check(B.lib().pad_step_create(*args, bad_opts, ctypes.byref(h)))
+        assert ei.value.status == 1
+    no_ws = list(args)
+    no_ws[10] = None
+    with pytest.raises(B.PadError) as ei:
+        B._check(B.lib().pad_step_create(*no_ws, 0, ctypes.byref(h)))
+    assert ei.value.status == 1
+    B._check(B.lib().pad_step_create(*args, 0, ctypes.byref(h)))
+    try:
+        import torch
+        if not torch.cuda.is_available():
+            # without a device the launch is refused before any kernel runs (with one, the
+            # fake addresses above must never reach a kernel: this part is skipped)
+            free0 = cache.free_count
+            new = np.full(3, -7, np.int32)
+            st = B.lib().pad_step_run(h, new.ctypes.data_as(B._I32P))
+            assert st != 0
+            assert cache.free_count == free0
+    finally:
+        B.lib().pad_step_destroy(h)
