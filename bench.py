@@ -414,14 +414,19 @@ def run_ours(args):
 
     # e2e through the C ABI with host buffers: H2D inputs, step, D2H outputs, sync.
     Ke = max(3, min(K, args.e2e_steps))
-    hq = torch.empty(reps[0].q.shape, dtype=torch.bfloat16, pin_memory=True)
-    hkn = torch.empty(reps[0].k_new.shape, dtype=torch.bfloat16, pin_memory=True)
-    hvn = torch.empty(reps[0].v_new.shape, dtype=torch.bfloat16, pin_memory=True)
+    # page-locked host buffers laid out like the device ones (q | k_new | v_new, out | lse)
+    h_in = torch.empty(reps[0].io_in.shape, dtype=torch.bfloat16, pin_memory=True)
+    h_out = torch.empty(reps[0].io_out.shape, dtype=torch.uint8, pin_memory=True)
+    qn, kn = w.q.size, w.k_new.size
+    hq = h_in[:qn].view(reps[0].q.shape)
+    hkn = h_in[qn:qn + kn].view(reps[0].k_new.shape)
+    hvn = h_in[qn + kn:].view(reps[0].v_new.shape)
     hq.copy_(bits_to_bf16(w.q, "cpu"))
     hkn.copy_(bits_to_bf16(w.k_new, "cpu"))
     hvn.copy_(bits_to_bf16(w.v_new, "cpu"))
-    hout = torch.empty(reps[0].out.shape, dtype=reps[0].out.dtype, pin_memory=True)
-    hlse = torch.empty(reps[0].lse.shape, dtype=torch.float32, pin_memory=True)
+    ob = reps[0].out.numel() * reps[0].out.element_size()
+    hout = h_out[:ob].view(reps[0].out.dtype).view(reps[0].out.shape)
+    hlse = h_out[ob:].view(torch.float32).view(reps[0].lse.shape)
     h2d = sum(t.numel() * t.element_size() for t in (hq, hkn, hvn))
     d2h = sum(t.numel() * t.element_size() for t in (hout, hlse))
 

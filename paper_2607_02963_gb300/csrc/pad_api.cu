@@ -1086,18 +1086,34 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
   const size_t E = (size_t)step->n_events, D = (size_t)pr.head_dim;
   const size_t q_bytes = E * pr.h_q * D * 2, kv_bytes = E * pr.h_kv * D * 2;
   const size_t o_bytes = E * pr.h_q * D * (pr.out_dtype == 1 ? 2 : 4), l_bytes = E * pr.h_q * sizeof(float);
+  // buffers that follow one another in device memory and in host memory alike go in one copy
+  auto adjacent = [](const void* a, size_t n, const void* b) {
+    return static_cast<const char*>(a) + n == static_cast<const char*>(b);
+  };
   cudaError_t e = cudaSuccess;
   if (E > 0) {
-    e = cudaMemcpyAsync(const_cast<void*>(step->q), h_q, q_bytes, cudaMemcpyHostToDevice, s);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->k_new), h_k_new, kv_bytes, cudaMemcpyHostToDevice, s);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->v_new), h_v_new, kv_bytes, cudaMemcpyHostToDevice, s);
+    char* dq = static_cast<char*>(const_cast<void*>(step->q));
+    const char* hq = static_cast<const char*>(h_q);
+    const bool kq = adjacent(step->q, q_bytes, step->k_new) && adjacent(h_q, q_bytes, h_k_new);
+    const bool vk = adjacent(step->k_new, kv_bytes, step->v_new) && adjacent(h_k_new, kv_bytes, h_v_new);
+    if (kq && vk) {
+      e = cudaMemcpyAsync(dq, hq, q_bytes + 2 * kv_bytes, cudaMemcpyHostToDevice, s);
+    } else {
+      e = cudaMemcpyAsync(dq, hq, q_bytes, cudaMemcpyHostToDevice, s);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->k_new), h_k_new, kv_bytes, cudaMemcpyHostToDevice, s);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->v_new), h_v_new, kv_bytes, cudaMemcpyHostToDevice, s);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "step inputs H2D");
   }
   pad_status st = pad_step_run(step, new_page);
   if (st != PAD_OK) return st;
   if (E > 0) {
-    e = cudaMemcpyAsync(h_out, step->out, o_bytes, cudaMemcpyDeviceToHost, s);
-    if (e == cudaSuccess && h_lse) e = cudaMemcpyAsync(h_lse, step->lse, l_bytes, cudaMemcpyDeviceToHost, s);
+    if (h_lse && adjacent(step->out, o_bytes, step->lse) && adjacent(h_out, o_bytes, h_lse)) {
+      e = cudaMemcpyAsync(h_out, step->out, o_bytes + l_bytes, cudaMemcpyDeviceToHost, s);
+    } else {
+      e = cudaMemcpyAsync(h_out, step->out, o_bytes, cudaMemcpyDeviceToHost, s);
+      if (e == cudaSuccess && h_lse) e = cudaMemcpyAsync(h_lse, step->lse, l_bytes, cudaMemcpyDeviceToHost, s);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "step outputs D2H");
   }
   e = cudaStreamSynchronize(s);

@@ -32,9 +32,17 @@ class DeviceBatch:
         self.v_pool = bits_to_bf16(vp, self.device)
         self.k_prefix = bits_to_bf16(w.k_prefix, self.device)
         self.v_prefix = bits_to_bf16(w.v_prefix, self.device)
-        self.q = bits_to_bf16(w.q, self.device)
-        self.k_new = bits_to_bf16(w.k_new, self.device)
-        self.v_new = bits_to_bf16(w.v_new, self.device)
+        # this step's inputs in one allocation (q | k_new | v_new) and its outputs in another
+        # (out | lse), as a serving loop keeps them: the step executor then moves each group
+        # with one copy
+        qn, kn = w.q.size, w.k_new.size
+        self.io_in = torch.empty(qn + 2 * kn, dtype=torch.bfloat16, device=self.device)
+        self.q = self.io_in[:qn].view(w.q.shape)
+        self.k_new = self.io_in[qn:qn + kn].view(w.k_new.shape)
+        self.v_new = self.io_in[qn + kn:].view(w.v_new.shape)
+        self.q.copy_(bits_to_bf16(w.q, self.device))
+        self.k_new.copy_(bits_to_bf16(w.k_new, self.device))
+        self.v_new.copy_(bits_to_bf16(w.v_new, self.device))
         self.page_table = torch.from_numpy(w.page_table.copy()).to(self.device)
         used = w.page_table[w.page_table >= 0]
         self.cache = B.CacheState(w.n_pages, used_pages=used)
@@ -43,8 +51,11 @@ class DeviceBatch:
             raise B.PadError(1, B.lib().pad_last_error().decode())
         self.workspace = torch.zeros(ws, dtype=torch.uint8, device=self.device)
         odt = torch.float32 if out_dtype == 0 else torch.bfloat16
-        self.out = torch.empty((w.n_events, w.h_q, w.head_dim), dtype=odt, device=self.device)
-        self.lse = torch.empty((w.n_events, w.h_q), dtype=torch.float32, device=self.device)
+        ob = w.n_events * w.h_q * w.head_dim * (4 if out_dtype == 0 else 2)
+        lb = w.n_events * w.h_q * 4
+        self.io_out = torch.empty(ob + lb, dtype=torch.uint8, device=self.device)
+        self.out = self.io_out[:ob].view(odt).view(w.n_events, w.h_q, w.head_dim)
+        self.lse = self.io_out[ob:].view(torch.float32).view(w.n_events, w.h_q)
         self.plan = None
         self.rope = None           # (positions [E] host int32, cos_sin device fp32 [P, D])
         self.self_g = None         # (K per video, G index per event) for the self G-token mask

@@ -55,20 +55,31 @@ def test_run_matches_the_step_calls(make, one_call):
     assert np.abs(got - ref_o).max() <= 1e-2
 
 
-def test_run_host_copies_in_and_out():
+@pytest.mark.parametrize("adjacent", [True, False])
+def test_run_host_copies_in_and_out(adjacent):
+    """Host buffers laid out like the device ones (one copy each way) or apart (five)."""
     w = synth.gqa_8k()
     a = DeviceBatch(w)
     a.run_step(one_call=True)
     torch.cuda.synchronize()
     b = DeviceBatch(w)
-    hq = b.q.cpu().pin_memory()
-    hk = b.k_new.cpu().pin_memory()
-    hv = b.v_new.cpu().pin_memory()
+    if adjacent:
+        h_in = b.io_in.cpu().pin_memory()
+        h_out = torch.empty(b.io_out.shape, dtype=torch.uint8).pin_memory()
+        qn, kn = b.q.numel(), b.k_new.numel()
+        hq, hk, hv = h_in[:qn].view(b.q.shape), h_in[qn:qn + kn].view(b.k_new.shape), h_in[qn + kn:].view(b.v_new.shape)
+        ob = b.out.numel() * b.out.element_size()
+        ho = h_out[:ob].view(b.out.dtype).view(b.out.shape)
+        hl = h_out[ob:].view(torch.float32).view(b.lse.shape)
+    else:
+        hq = b.q.cpu().pin_memory()
+        hk = b.k_new.cpu().pin_memory()
+        hv = b.v_new.cpu().pin_memory()
+        ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
+        hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
     b.q.zero_()
     b.k_new.zero_()
     b.v_new.zero_()
-    ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
-    hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
     st = _native(b, w, release_pages=False)
     st.run_host(hq, hk, hv, ho, hl)
     assert torch.equal(ho, a.out.cpu()) and torch.equal(hl, a.lse.cpu())
