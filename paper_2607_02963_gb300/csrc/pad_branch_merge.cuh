@@ -273,10 +273,11 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     }
   };
   if (knew != nullptr) {
-    // a2: this task's row of the new token into the pools (16-byte pieces of K, then V)
+    // a2: this task's row of the new token into the pools (16-byte pieces of K, then V);
+    // its page was located with the first round's keys when it is among them
     if (tid < 2 * CH) {
-      int sl;
-      const int pg = page_of(own, sl);
+      int sl = 0;
+      const int pg = own < nkr ? S.page[own] : page_of(own, sl);
       if (pg >= 0) {
         const int c = tid % CH;
         const bool isv = tid >= CH;
