@@ -327,3 +327,29 @@ def test_step_executor_validates_and_returns_pages_of_a_failed_run(padlib):
             assert cache.free_count == free0
     finally:
         B.lib().pad_step_destroy(h)
+
+
+def test_attn_aggregate_workspace_and_argument_checks(padlib):
+    """The aggregation's scratch is (n_segments + ceil(n_tokens / 256)) x (d_model + 1) fp32;
+    a smaller one, a hidden size that is not a multiple of 8, a NULL tensor or a misaligned
+    one are refused before anything is launched (no device is touched here)."""
+    import ctypes
+    L = B.lib()
+    for T, S, d in ((32768, 128, 2048), (3400, 3, 520), (1, 1, 8), (256, 1, 64), (257, 1, 64)):
+        assert L.pad_attn_aggregate_workspace_size(T, S, d) == (S + -(-T // 256)) * (d + 1) * 4
+    assert L.pad_attn_aggregate_workspace_size(-1, 1, 8) == 0
+    assert L.pad_attn_aggregate_workspace_size(10, 0, 8) == 0
+    off = np.array([0, 100, 300], np.int32)
+    a = 1 << 20  # 16-byte aligned addresses, never dereferenced: every call below fails its checks
+    need = L.pad_attn_aggregate_workspace_size(300, 2, 64)
+
+    def call(d=64, ws_bytes=need, x=a, ws=a, n_events=3):
+        return L.pad_attn_aggregate(x, 300, d, a, off.ctypes.data_as(B._I32P), 2, a, n_events, a, ws, ws_bytes, a,
+                                    None)
+    assert call(ws_bytes=need - 4) == 4                      # PAD_ERR_WORKSPACE_TOO_SMALL
+    assert call(d=60) == 2                                   # d_model not a multiple of 8
+    assert call(ws=None) == 1                                # NULL scratch
+    assert call(ws=a + 4) == 1                               # misaligned scratch
+    assert call(x=a + 8) == 1                                # misaligned hidden states
+    bad = np.array([0, 301, 300], np.int32)                  # offsets past n_tokens
+    assert L.pad_attn_aggregate(a, 300, 64, a, bad.ctypes.data_as(B._I32P), 2, a, 3, a, a, need, a, None) == 1
