@@ -446,86 +446,3 @@ class NativeStep:
         if h is not None and h.value:
             self.L.pad_step_destroy(h)
             self.handle = None
-
-
-class StepLauncher:
-    """One decode step (pad_plan -> pad_decode_step, or pad_plan -> pad_kv_append ->
-    pad_event_decode_attn with ``one_call=False``) with every argument converted to ctypes
-    once, so a repeated step costs only the C calls.
-
-    ``release_pages``: return the pages the step took after launching it (keeps a
-    repeated identical step idempotent, as when re-running one step for timing)."""
-
-    def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
-                 page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
-                 v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True,
-                 rope=None, self_g=None, causal=False):
-        """``rope`` = (positions [E], device fp32 table [P, D]); ``self_g`` = (K per video, G
-        index per event); ``causal``: the mask variants of the ablation (set per plan)."""
-        self.L = lib()
-        self.problem = problem
-        self.cache = cache
-        self._keep = []
-        pl, self.plp = _i32(prefix_len)
-        ev, self.evp = _i32(event_video)
-        el, self.elp = _i32(event_len)
-        self._keep += [pl, ev, el]
-        self.nv, self.ne = int(pl.size), int(ev.size)
-        if prefix_offset is not None:
-            po = np.ascontiguousarray(prefix_offset, dtype=np.int64)
-            self._keep.append(po)
-            self.pop = po.ctypes.data_as(_I64P)
-        else:
-            self.pop = None
-        self.pt = _ptr(page_table)
-        self.maxp = int(max_pages)
-        self.ws = _ptr(workspace)
-        self.wsb = int(workspace.numel())
-        self.stream = _stream(stream)
-        self.args_append = [_ptr(k_new), _ptr(v_new), _ptr(k_pool), _ptr(v_pool), self.stream]
-        self.args_attn = [_ptr(q), _ptr(k_prefix), _ptr(v_prefix), _ptr(k_pool), _ptr(v_pool),
-                          _ptr(out), _ptr(lse), self.stream]
-        self.args_step = [_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_prefix), _ptr(v_prefix),
-                          _ptr(k_pool), _ptr(v_pool), _ptr(out), _ptr(lse), self.stream]
-        self.one_call = one_call
-        self.rope = None
-        if rope is not None:
-            pos = np.ascontiguousarray(rope[0], dtype=np.int32)
-            self._keep.append(pos)
-            self.rope = (pos.ctypes.data_as(_I32P), _ptr(rope[1]), int(rope[1].shape[0]))
-        self.self_g = None
-        if self_g is not None:
-            kk = np.ascontiguousarray(self_g[0], dtype=np.int32)
-            gg = np.ascontiguousarray(self_g[1], dtype=np.int32)
-            self._keep += [kk, gg]
-            self.self_g = (kk.ctypes.data_as(_I32P), gg.ctypes.data_as(_I32P))
-        self.causal = bool(causal)
-        self.newp = np.full(self.ne, -1, dtype=np.int32)
-        self.newpp = self.newp.ctypes.data_as(_I32P)
-        self.release = release_pages
-        self.h = c_void_p()
-        self.ph = ctypes.byref(self.h)
-        self.pprob = ctypes.byref(problem)
-
-    def __call__(self):
-        L = self.L
-        _check(L.pad_plan(self.pprob, self.cache.handle, self.nv, self.plp, self.pop, self.ne,
-                          self.evp, self.elp, self.pt, self.maxp, self.ws, self.wsb, self.stream,
-                          self.ph))
-        h = self.h
-        try:
-            if self.rope is not None:
-                _check(L.pad_plan_set_rope(h, *self.rope))
-            if self.self_g is not None:
-                _check(L.pad_plan_set_g_visibility(h, G_SELF, *self.self_g))
-            if self.causal:
-                _check(L.pad_plan_set_branch_visibility(h, BRANCH_CAUSAL))
-            if self.one_call:
-                _check(L.pad_decode_step(h, *self.args_step))
-            else:
-                _check(L.pad_kv_append(h, *self.args_append))
-                _check(L.pad_event_decode_attn(h, *self.args_attn))
-            if self.release:
-                _check(L.pad_plan_release_new_pages(h, self.cache.handle))
-        finally:
-            L.pad_plan_destroy(h)
