@@ -304,7 +304,8 @@ pad_status pad_step_set_branch_visibility(pad_step_t* step, int32_t mode);
 pad_status pad_step_run(pad_step_t* step, int32_t* new_page);
 /*   h_q [n_events, h_q, head_dim] bf16, h_k_new / h_v_new [n_events, h_kv, head_dim] bf16,
  *   h_out [n_events, h_q, head_dim] (the problem's out_dtype), h_lse [n_events, h_q] fp32
- *   or NULL; host memory (page-locked for asynchronous copies).  Where q, k_new and v_new
+ *   or NULL; host memory (page-locked for asynchronous copies).  The call returns after the
+ *   stream has finished with them, also when it fails.  Where q, k_new and v_new
  *   follow one another in device memory and their host buffers do too, they go in one copy;
  *   so do out and lse. */
 pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,

@@ -1103,10 +1103,18 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
       if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->k_new), h_k_new, kv_bytes, cudaMemcpyHostToDevice, s);
       if (e == cudaSuccess) e = cudaMemcpyAsync(const_cast<void*>(step->v_new), h_v_new, kv_bytes, cudaMemcpyHostToDevice, s);
     }
-    if (e != cudaSuccess) return cuda_fail(e, "step inputs H2D");
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(s);  // the host buffers are the caller's again when this returns
+      return cuda_fail(e, "step inputs H2D");
+    }
   }
   pad_status st = pad_step_run(step, new_page);
-  if (st != PAD_OK) return st;
+  if (st != PAD_OK) {
+    const std::string msg = g_last_error;
+    cudaStreamSynchronize(s);
+    g_last_error = msg;
+    return st;
+  }
   if (E > 0) {
     if (h_lse && adjacent(step->out, o_bytes, step->lse) && adjacent(h_out, o_bytes, h_lse)) {
       e = cudaMemcpyAsync(h_out, step->out, o_bytes + l_bytes, cudaMemcpyDeviceToHost, s);
@@ -1114,7 +1122,10 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
       e = cudaMemcpyAsync(h_out, step->out, o_bytes, cudaMemcpyDeviceToHost, s);
       if (e == cudaSuccess && h_lse) e = cudaMemcpyAsync(h_lse, step->lse, l_bytes, cudaMemcpyDeviceToHost, s);
     }
-    if (e != cudaSuccess) return cuda_fail(e, "step outputs D2H");
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(s);
+      return cuda_fail(e, "step outputs D2H");
+    }
   }
   e = cudaStreamSynchronize(s);
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "step synchronize");
