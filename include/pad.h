@@ -284,7 +284,8 @@ pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_
  *              pad_decode_step; PAD_STEP_RELEASE_PAGES: hand the pages a run took back to
  *              the cache after launching it (to repeat one identical step, e.g. for timing)
  *   new_page   [n_events] host, may be NULL: the pages the run took (pad_plan_new_pages)
- * A run that fails before launching hands its pages back and returns the plan's status.
+ * A run that fails before a kernel wrote its new pages into the page table hands them back
+ * to the cache and returns the failing call's status.
  * The mask variants and RoPE are set once (pad_step_set_*: the same arguments as the
  * pad_plan_set_* calls, borrowed the same way) and apply to every later run. */
 typedef struct pad_step_t pad_step_t;

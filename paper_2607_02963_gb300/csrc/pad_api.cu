@@ -1053,9 +1053,11 @@ pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
   if (st == PAD_OK && step->g_mode == PAD_G_SELF)
     st = pad_plan_set_g_visibility(plan, PAD_G_SELF, step->g_planning, step->g_index);
   if (st == PAD_OK && step->branch_mode == PAD_BRANCH_CAUSAL) st = pad_plan_set_branch_visibility(plan, PAD_BRANCH_CAUSAL);
+  bool wrote_pages = false;  // the append kernel has been launched: the pages are in the table
   if (st == PAD_OK) {
     if (step->options & PAD_STEP_TWO_CALL) {
       st = pad_kv_append(plan, step->k_new, step->v_new, step->k_pool, step->v_pool, step->stream);
+      wrote_pages = st == PAD_OK;
       if (st == PAD_OK)
         st = pad_event_decode_attn(plan, step->q, step->k_prefix, step->v_prefix, step->k_pool, step->v_pool,
                                    step->out, step->lse, step->stream);
@@ -1065,8 +1067,10 @@ pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
     }
   }
   if (st == PAD_OK && new_page) st = pad_plan_new_pages(plan, new_page);
-  if (st != PAD_OK || (step->options & PAD_STEP_RELEASE_PAGES)) {
-    // a step that failed before launching hands its pages back; so does a timing loop
+  if ((st != PAD_OK && !wrote_pages) || (step->options & PAD_STEP_RELEASE_PAGES)) {
+    // a step that failed before any kernel wrote its pages into the table hands them back
+    // (in the one-call step the branch/merge kernel writes them, and it is launched last);
+    // so does a timing loop
     const pad_status keep = st;
     pad_plan_release_new_pages(plan, step->cache);
     st = keep;
