@@ -353,3 +353,36 @@ def test_attn_aggregate_workspace_and_argument_checks(padlib):
     assert call(x=a + 8) == 1                                # misaligned hidden states
     bad = np.array([0, 301, 300], np.int32)                  # offsets past n_tokens
     assert L.pad_attn_aggregate(a, 300, 64, a, bad.ctypes.data_as(B._I32P), 2, a, 3, a, a, need, a, None) == 1
+
+
+def test_step_executor_setters_validate(padlib):
+    """pad_step_set_*: a NULL executor, an unknown mode, and the arrays a mode needs."""
+    import ctypes
+    L = B.lib()
+    assert L.pad_step_run(None, None) == 1
+    assert L.pad_step_set_branch_visibility(None, B.BRANCH_CAUSAL) == 1
+    prob = B.make_problem(8, 2, 128, num_sms=152)
+    cache = B.CacheState(64)
+    pl = np.array([500], np.int32)
+    ev = np.zeros(2, np.int32)
+    el = np.array([3, 7], np.int32)
+    fake = 1 << 20  # never dereferenced: nothing below launches
+    h = ctypes.c_void_p()
+    B._check(L.pad_step_create(ctypes.byref(prob), cache.handle, 1, pl.ctypes.data_as(B._I32P), None, 2,
+                               ev.ctypes.data_as(B._I32P), el.ctypes.data_as(B._I32P), fake, 4, fake, 1 << 24,
+                               *([fake] * 9), None, 0, ctypes.byref(h)))
+    try:
+        assert L.pad_step_set_branch_visibility(h, 2) == 1
+        assert L.pad_step_set_branch_visibility(h, B.BRANCH_CAUSAL) == 0
+        assert L.pad_step_set_branch_visibility(h, B.BRANCH_OWN) == 0
+        assert L.pad_step_set_g_visibility(h, 5, None, None) == 1
+        assert L.pad_step_set_g_visibility(h, B.G_SELF, None, None) == 1   # K / G indices needed
+        assert L.pad_step_set_g_visibility(h, B.G_ALL, None, None) == 0
+        assert L.pad_step_set_rope(h, None, fake, 100) == 1                # positions needed
+        assert L.pad_step_set_rope(h, None, fake + 4, 100) == 1            # misaligned table
+        pos = np.zeros(2, np.int32)
+        assert L.pad_step_set_rope(h, pos.ctypes.data_as(B._I32P), fake, 0) == 1
+        assert L.pad_step_set_rope(h, pos.ctypes.data_as(B._I32P), fake, 100) == 0
+        assert L.pad_step_set_rope(h, None, None, 0) == 0                  # off again
+    finally:
+        L.pad_step_destroy(h)
