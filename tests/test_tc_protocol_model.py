@@ -38,7 +38,10 @@ class Bar:
 ST = 3  # K/V stages = S buffers
 
 
-def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
+def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=False):
+    """prefetch: the softmax warps load tile j + 1's S during tile j (after the two halves
+    meet, before P(j) is released), as a softmax that hides the load behind the
+    exponentials would."""
     rnd = random.Random(seed)
     kfull = [Bar(1) for _ in range(ST)]
     vfull = [Bar(1) for _ in range(ST)]
@@ -59,6 +62,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
     kst = [None] * ST
     vst = [None] * ST
     S_done, PV_done, P_written, PV_issued = set(), set(), set(), set()
+    holding = [set() for _ in range(n_softmax)]  # tiles whose S a softmax warp has loaded, unconsumed
     inflight = []
     commits = []
     issued = {"S": [], "PV": []}  # per-issuer MMA ops (a commit tracks only its own)
@@ -92,6 +96,8 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
                     raise AssertionError(f"S({t}) overwrites P({j}) still read by its P.V")
             if t >= ST:
                 assert (t - ST) in PV_done, f"S({t}) before P.V({t - ST}) done"
+            for h in holding:
+                assert (t - ST) not in h, f"S({t}) overwrites S({t - ST}) that a softmax warp still holds"
         mma("S", chk, lambda: S_done.add(t))
 
     def issue_PV(j):
@@ -149,9 +155,23 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
         yield (drain_pv, 0)
 
     def softmax(w):
+        if prefetch and n > 0:
+            yield (sfull[0], 0)
+            assert 0 in S_done, "softmax loads S(0) before it is done"
+            holding[w].add(0)
         for j in range(n):
-            yield (sfull[j % ST], (j // ST) & 1)
-            assert j in S_done, f"softmax reads S({j}) before it is done"
+            if prefetch:
+                assert j in holding[w], f"softmax uses S({j}) it has not loaded"
+            else:
+                yield (sfull[j % ST], (j // ST) & 1)
+                assert j in S_done, f"softmax reads S({j}) before it is done"
+                holding[w].add(j)
+            for _ in range(rnd.randint(0, 2)):  # the row maximum, the halves meeting
+                yield None
+            if prefetch and j + 1 < n:
+                yield (sfull[(j + 1) % ST], ((j + 1) // ST) & 1)
+                assert (j + 1) in S_done, f"softmax loads S({j + 1}) before it is done"
+                holding[w].add(j + 1)
             if j > 0 and rnd.random() < lazy_prob:
                 yield ((pvfree[(j - 1) % ST], ((j - 1) // ST) & 1) if not single_barriers
                        else (pvfree[0], (j - 1) & 1))
@@ -162,6 +182,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
                 yield None
             if w == 0:
                 P_written.add(j)
+            holding[w].discard(j)
             pfull[j % ST].arrive()
         yield (drain_pv, 0)
         assert len(PV_done) == n, "epilogue before every P.V completed"
@@ -224,6 +245,14 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8):
 def test_tc_kernel_barrier_protocol(n):
     for seed in range(120):
         assert run(n, seed * 131 + n)
+
+
+@pytest.mark.parametrize("n", range(1, 13))
+def test_prefetching_softmax_keeps_the_protocol(n):
+    """Loading tile j + 1's S during tile j (waiting for its S-done barrier before releasing
+    P(j)) neither deadlocks nor lets an S MMA overwrite a buffer a softmax warp still holds."""
+    for seed in range(120):
+        assert run(n, seed * 173 + n, prefetch=True)
 
 
 def test_model_detects_phase_aliasing():
