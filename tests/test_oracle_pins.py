@@ -597,3 +597,155 @@ def test_prefill_other_branches_do_not_matter():
     o1, _ = oracle.prefill_attention(q, k2, v2, S, lens, 0.5)
     assert np.array_equal(o0[:S + 2], o1[:S + 2])   # prefix and branch 1 unchanged
     assert not np.allclose(o0[S + 2:], o1[S + 2:])
+
+
+# ---------------------------------------------------------------------------
+# event_rows, rotated_workload and decode_step on several videos
+# ---------------------------------------------------------------------------
+# The full-size GPU checks call event_rows (one event at a time) and the RoPE checks
+# call rotated_workload, so both are pinned here against things fixed outside the
+# oracle: keys gathered by hand from the raw workload arrays, the library's SDPA, and
+# a hand-worked rotation table.
+
+def _widen(bits):
+    """bf16 bits -> float64 through torch's own bf16 type (independent of the oracle)."""
+    t = torch.from_numpy(np.ascontiguousarray(bits, dtype=np.uint16).view(np.int16))
+    return t.view(torch.bfloat16).double().numpy()
+
+
+def _hand_keys(w, e, causal=False, self_g=None):
+    """Event e's visible keys and values in decode order, gathered from the raw arrays.
+
+    Plain mask: its video's prefix rows, its stored branch rows, its new row.  With
+    ``causal``: the prefix, the stored rows of every branch of its video, its new row.
+    With ``self_g = (K per video, G index per event)``: prefix rows outside the video's
+    planning tokens, plus its own G token."""
+    b = int(w.event_video[e])
+    off, n = int(w.prefix_offset[b]), int(w.prefix_len[b])
+    rows = list(range(off, off + n))
+    if self_g is not None and int(self_g[0][b]) > 0:
+        K = int(self_g[0][b])
+        g0 = off + n - 1 - K
+        rows = [r for r in rows if not (g0 <= r < g0 + K) or r == g0 + int(self_g[1][e])]
+    ks, vs = [w.k_prefix[rows]], [w.v_prefix[rows]]
+    owners = [f for f in range(w.n_events) if int(w.event_video[f]) == b] if causal else [e]
+    for f in owners:
+        ks.append(w.k_priv[int(w.priv_off[f]):int(w.priv_off[f + 1])])
+        vs.append(w.v_priv[int(w.priv_off[f]):int(w.priv_off[f + 1])])
+    ks.append(w.k_new[e:e + 1])
+    vs.append(w.v_new[e:e + 1])
+    return _widen(np.concatenate(ks)), _widen(np.concatenate(vs))
+
+
+def _multi_video(seed):
+    """A small ragged batch of at least two videos whose prefixes differ."""
+    for s in range(seed, seed + 200):
+        w = synth.random_small(s, h_q=6, h_kv=2, head_dim=16, max_videos=3, max_prefix=40,
+                               max_events=4, max_len=9)
+        if w.n_videos >= 2 and len(set(w.event_video.tolist())) >= 2:
+            return w
+    raise AssertionError("no multi-video workload drawn")
+
+
+@pytest.mark.parametrize("seed", [31, 57])
+def test_event_rows_match_the_step_and_sdpa_on_several_videos(seed):
+    w = _multi_video(seed)
+    o, lse = oracle.decode_step(w)
+    for e in range(w.n_events):
+        oe, le = oracle.event_rows(w, e)
+        np.testing.assert_allclose(oe, o[e], rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(le, lse[e], rtol=1e-13, atol=1e-13)
+        oh, lh = oracle.event_rows(w, e, heads=[1, 4])
+        np.testing.assert_allclose(oh, o[e, [1, 4]], rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(lh, lse[e, [1, 4]], rtol=1e-13, atol=1e-13)
+        K, V = _hand_keys(w, e)
+        ref = _sdpa_single(_widen(w.q[e]), K, V, w.scale)
+        np.testing.assert_allclose(oe, ref, rtol=1e-11, atol=1e-12)
+
+
+def _rope_case():
+    """D = 4, one kv-head, four events: q and k_new rows [1, 2, 3, 4] (and 5..8 for
+    event 1), v_new rows distinct.  Table rows: 0 = identity; 1 = pair 0 turned by
+    90 degrees, pair 1 by 180; 2 = pair 0 by 180, pair 1 by 90 (all exact in fp32)."""
+    w = synth.make_workload("rope_d4", 5, 2, 1, 4, [6], [4], [0, 1, 2, 3])
+    base = np.array([1.0, 2.0, 3.0, 4.0], np.float32)
+    q = np.tile(base, (4, 2, 1))
+    q[1] = np.array([5.0, 6.0, 7.0, 8.0], np.float32)
+    kn = np.tile(base, (4, 1, 1))
+    kn[1] = np.array([5.0, 6.0, 7.0, 8.0], np.float32)
+    w.q = synth.f32_to_bf16_bits(q)
+    w.k_new = synth.f32_to_bf16_bits(kn)
+    table = np.array([[1, 1, 0, 0], [0, -1, 1, 0], [-1, 0, 0, 1]], np.float32)
+    return w, table
+
+
+def test_rotated_workload_hand_worked_d4():
+    w, table = _rope_case()
+    pos = np.array([1, 2, 0, 1], np.int32)
+    r = oracle.rotated_workload(w, pos, table)
+    # x' = (x0 c0 - x2 s0, x1 c1 - x3 s1, x2 c0 + x0 s0, x3 c1 + x1 s1), worked by hand:
+    want_q = {0: [-3.0, -2.0, 1.0, -4.0],     # [1,2,3,4] at row 1
+              1: [-5.0, -8.0, -7.0, 6.0],     # [5,6,7,8] at row 2
+              2: [1.0, 2.0, 3.0, 4.0],        # row 0: unchanged
+              3: [-3.0, -2.0, 1.0, -4.0]}     # same input, same position as event 0
+    for e, row in want_q.items():
+        assert np.array_equal(_widen(r.q[e]), np.array([row, row])), e
+        assert np.array_equal(_widen(r.k_new[e]), np.array([row])), e
+    # values, the prefix and the stored branch keys are never rotated
+    for name in ("v_new", "k_prefix", "v_prefix", "k_priv", "v_priv", "page_table"):
+        assert np.array_equal(getattr(r, name), getattr(w, name)), name
+    # the caller's workload is left as it was
+    assert np.array_equal(_widen(w.q[0, 0]), [1.0, 2.0, 3.0, 4.0])
+
+
+def test_rotated_workload_uses_each_events_own_position():
+    """Only the events whose position is not 0 change; two events with equal rows at
+    the same position get the same rotation (Sec. 3.4: one position per step)."""
+    rng = np.random.default_rng(8)
+    w = synth.make_workload("rope_pos", 8, 4, 2, 16, [30], [5], [1, 0, 2, 3, 1], rng=rng)
+    w.q[3] = w.q[1]
+    w.k_new[3] = w.k_new[1]
+    table = synth.rope_table(64, 16)
+    for moved in range(w.n_events):
+        pos = np.zeros(w.n_events, np.int32)
+        pos[moved] = 37
+        r = oracle.rotated_workload(w, pos, table)
+        for e in range(w.n_events):
+            same_q = np.array_equal(r.q[e], w.q[e])
+            same_k = np.array_equal(r.k_new[e], w.k_new[e])
+            assert same_q == same_k == (e != moved), (moved, e)
+        assert np.array_equal(r.v_new, w.v_new)
+    pos = np.array([5, 37, 9, 37, 2], np.int32)
+    r = oracle.rotated_workload(w, pos, table)
+    assert np.array_equal(r.q[1], r.q[3]) and np.array_equal(r.k_new[1], r.k_new[3])
+    pos[3] = 38
+    r2 = oracle.rotated_workload(w, pos, table)
+    assert not np.array_equal(r2.q[1], r2.q[3])
+    # each rotated row is within one bf16 step of the exact rotation of its own row
+    for e in range(w.n_events):
+        c, s = table[pos[e], :8].astype(np.float64), table[pos[e], 8:].astype(np.float64)
+        x = _widen(w.k_new[e])
+        exact = np.concatenate([x[..., :8] * c - x[..., 8:] * s, x[..., 8:] * c + x[..., :8] * s], -1)
+        got = _widen(r2.k_new[e])
+        assert np.all(np.abs(got - exact) <= np.maximum(np.abs(exact), 2.0 ** -126) * 2.0 ** -7)
+
+
+@pytest.mark.parametrize("variant", ["self_g", "causal"])
+def test_decode_step_variants_on_several_videos_against_sdpa(variant):
+    """decode_step with the mask variants over a batch of videos: each event against the
+    library's SDPA over the keys its video and the variant make visible, gathered by hand."""
+    w = _multi_video(77)
+    sg = None
+    if variant == "self_g":
+        Kp = np.array([min(int(w.prefix_len[b]) - 1, 3 + b) for b in range(w.n_videos)], np.int32)
+        gi = np.zeros(w.n_events, np.int32)
+        for b in range(w.n_videos):
+            ev = w.events_of_video(b)
+            if Kp[b] > 0:
+                gi[ev] = (np.arange(len(ev)) * 2 + b) % Kp[b]
+        sg = (Kp, gi)
+    o, lse = oracle.decode_step(w, self_g=sg, causal=(variant == "causal"))
+    for e in range(w.n_events):
+        K, V = _hand_keys(w, e, causal=(variant == "causal"), self_g=sg)
+        ref = _sdpa_single(_widen(w.q[e]), K, V, w.scale)
+        np.testing.assert_allclose(o[e], ref, rtol=1e-11, atol=1e-12)
