@@ -328,7 +328,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream(device)
 
     flags = {"auto": 0, "simt": B.FLAG_PREFIX_SIMT, "mma": B.FLAG_PREFIX_MMA,
-             "tc": B.FLAG_PREFIX_TC}[args.prefix]
+             "tc": B.FLAG_PREFIX_TC, "dual": B.FLAG_PREFIX_DUAL}[args.prefix]
     if args.fused_merge:
         flags |= B.FLAG_FUSED_MERGE
     first = DeviceBatch(w, device=device, fill_nan=False, flags=flags)
@@ -452,7 +452,8 @@ def run_ours(args):
     if rank != 0:
         return
     peak, peak_kind = hbm_peak()
-    kern_name = {1: "prefix_simt_kernel", 2: "prefix_mma_kernel", 4: "prefix_tc_kernel"}[
+    kern_name = {1: "prefix_simt_kernel", 2: "prefix_mma_kernel", 4: "prefix_tc_kernel",
+                 16: "prefix_dual_kernel"}[
         info["prefix_kernel"]]
     prefix_ms_per_launch = pre_ms / max(1, pre_n)
     # the timed kernel's own algorithmic bytes: the prefix pass alone, or, when it also runs
@@ -877,7 +878,7 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="long_32k")
     ap.add_argument("--replicas", type=int, default=0, help="cold replicas (0 = enough for 3x L2)")
-    ap.add_argument("--prefix", choices=["auto", "simt", "mma", "tc"], default="auto",
+    ap.add_argument("--prefix", choices=["auto", "simt", "mma", "tc", "dual"], default="auto",
                     help="shared-prefix kernel (auto = the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")

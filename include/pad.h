@@ -95,7 +95,12 @@ typedef struct {
 /* Force one implementation of the shared-prefix pass (tests and benchmarks). */
 #define PAD_FLAG_PREFIX_SIMT 0x1   /* CUDA-core path */
 #define PAD_FLAG_PREFIX_MMA 0x2    /* warp-level mma.sync path */
-#define PAD_FLAG_PREFIX_TC 0x4     /* tcgen05 / TMEM / TMA path */
+#define PAD_FLAG_PREFIX_TC 0x4     /* tcgen05 / TMEM / TMA path, one 128-row group per CTA */
+/* tcgen05 / TMEM / TMA path with two softmax groups per CTA that take turns with the tensor
+ * pipe: up to 256 query rows share each K/V tile (rows > 128), or two tile parities of the
+ * same <= 128 rows alternate.  Forced only: it halves the traffic per row but doubles the
+ * split partials the merge reads, and was measured no faster than PAD_FLAG_PREFIX_TC. */
+#define PAD_FLAG_PREFIX_DUAL 0x10
 /* Run a4 + a5 inside the tensor-core prefix kernel, after each CTA's split, where every
  * (event, kv-head) pair can take a prefix CTA and the prefix grid fits one CTA per SM
  * (pad_plan_info.fused_tail says whether it was chosen).  Off by default: the separate
@@ -249,7 +254,10 @@ pad_status pad_plan_destroy(pad_plan_t* plan);
 /* a2: write k_new[e] / v_new[e] (bf16 [n_events, h_kv, head_dim], 16-byte aligned) into
  * slot event_len[e] of branch e (page page_table[e][event_len[e] / page_size], offset
  * event_len[e] % page_size) of k_pool / v_pool, and write the new page-table entries.
- * One new token per branch per step (Eq. 3). */
+ * One new token per branch per step (Eq. 3).  A plan built without a workspace (host-only)
+ * is accepted too: its descriptors and status word then live in the library's static scratch
+ * array (see pad_event_decode_attn_static, whose rules apply), so a caller with no device
+ * scratch can run a whole step as pad_kv_append + pad_event_decode_attn_static. */
 pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new,
                          void* k_pool, void* v_pool, pad_stream_t stream);
 
@@ -324,12 +332,17 @@ void pad_step_destroy(pad_step_t* step);
  *   plan      from pad_plan; its workspace may be NULL (a host-only plan), but it must
  *             carry the page table.  Plans needing more than 16 MiB of scratch
  *             (pad_plan_get_info().workspace_bytes) fail with PAD_ERR_WORKSPACE_TOO_SMALL.
- *   The branch keys are read from the pools, so this step's K/V must already be there.
+ *   The branch keys are read from the pools, so this step's K/V must already be there:
+ *   call pad_kv_append with the same plan first (it also takes host-only plans).
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress)
  * and caches it, so make that first call before any stream capture.  All calls share the
  * array: calls that overlap on the GPU (other streams or threads) race on it; calls in
- * order on one stream are safe (each copies the plan image into it).
- * pad_device_status does not read this array's status word. */
+ * order on one stream are safe (each copies the plan image into it).  That copy comes
+ * from the plan's pageable host memory, so the call blocks until the driver has staged
+ * it, and a graph captured around the call keeps the plan's host address: the plan must
+ * outlive such a graph.  Device errors (an out-of-pool page id, a bounded wait that gave
+ * up) go to the array's status word, tagged with the plan; pad_device_status(plan) reads
+ * it for a plan without a workspace. */
 pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q, const void* k_prefix,
                                         const void* v_prefix, const void* k_pool, const void* v_pool,
                                         void* out, float* lse, pad_stream_t stream);
@@ -417,7 +430,9 @@ pad_status pad_prefill_attn(const pad_problem* prob, int32_t prefix_len, int32_t
 pad_status pad_prefill_status(pad_stream_t stream);
 
 /* Synchronise the stream and read the plan's device status word:
- * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT. */
+ * PAD_OK, PAD_ERR_DEVICE_BOUNDS or PAD_ERR_DEVICE_TIMEOUT.  For a plan without a workspace
+ * the word is the static scratch array's (pad_event_decode_attn_static); PAD_OK if no call
+ * has used that array on the current device. */
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream);
 
 /* Message for the last error on this thread ("" if none). */

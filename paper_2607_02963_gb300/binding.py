@@ -25,6 +25,7 @@ FLAG_PREFIX_SIMT = 0x1
 FLAG_PREFIX_MMA = 0x2
 FLAG_PREFIX_TC = 0x4
 FLAG_FUSED_MERGE = 0x8
+FLAG_PREFIX_DUAL = 0x10
 G_ALL = 0
 G_SELF = 1
 BRANCH_OWN = 0

@@ -51,8 +51,12 @@ def _stamp(nvcc: str, extra) -> str:
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile every CUDA source for sm_103a and link libpad.so.  Returns its path."""
+    """Compile every CUDA source for sm_103a and link libpad.so.  Returns its path.
+
+    PAD_NVCC_FLAGS (environment, whitespace-separated) adds compiler flags, e.g. a kernel
+    tuning macro (-DPAD_DUAL_POLY_EVERY=4); they are part of the rebuild stamp."""
     nvcc = _nvcc()
+    extra_flags = tuple(extra_flags) + tuple(os.environ.get("PAD_NVCC_FLAGS", "").split())
     os.makedirs(BUILD, exist_ok=True)
     stamp_file = os.path.join(BUILD, "libpad.stamp")
     stamp = _stamp(nvcc, extra_flags)

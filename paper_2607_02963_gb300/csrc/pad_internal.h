@@ -254,6 +254,11 @@ int prefix_tc_tail_chunk(int branch_rows, int group, int max_splits);
 cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, const void* kp,
                              const void* vp, int64_t total_prefix_tokens, const void* k_pool,
                              const void* v_pool, void* out, float* lse, bool pdl, cudaStream_t s);
+// The prefix pass with two softmax groups per CTA (pad_prefix_dual.cu), head_dim 128, not
+// fused: up to 256 rows per CTA.
+cudaError_t launch_prefix_dual(const KParams& p, int max_rows, const void* q, const void* kp, const void* vp,
+                               int64_t total_prefix_tokens, const void* k_pool, const void* v_pool, bool pdl,
+                               cudaStream_t s);
 // pdl: launch with programmatic stream serialization (the kernel waits for its
 // predecessor with griddepcontrol.wait before it reads anything the predecessor wrote).
 // Full-sequence prefill / training forward (pad_prefill.cu).

@@ -53,10 +53,13 @@
 
 #include "pad_branch_merge.cuh"
 #include "pad_internal.h"
+#include "pad_tc_common.cuh"
 
 namespace pad {
 
 namespace {
+
+using namespace tc;
 
 constexpr int kD = 128;
 constexpr int kBN = 128;       // prefix tokens per K/V tile
@@ -86,7 +89,6 @@ constexpr int kMufuPairs = PAD_MUFU_PAIRS;
 // the extra polynomial instructions cost more than they save: all 16 go to MUFU.
 constexpr int kMufuPairs = 16;
 #endif
-constexpr unsigned long long kWaitNs = 1000000000ull; // one second per wait
 static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 
 struct TcBars {
@@ -106,92 +108,8 @@ struct TcBars {
 };
 static_assert(sizeof(TcBars) <= 256, "barrier block fits its slot");
 
-// Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1), A and B
-// bf16 (bits 7-9, 10-12 = 1), K-major A (bit 15 = 0), B major-ness in bit 16,
-// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-constexpr uint32_t make_idesc(int M, int N, bool b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
-         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
-}
 constexpr uint32_t kIdescS = make_idesc(128, kBN, false);   // S = Q K^T: B = K tile, K-major
 constexpr uint32_t kIdescPV = make_idesc(128, kD, true);    // O += P V: B = V tile, N(=d)-major
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ unsigned long long globaltimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// ---------------------------------------------------------------- packed fp32 pairs
-// Blackwell executes two fp32 lanes per instruction (.f32x2); a pair lives in a b64.
-__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
-  return ((uint64_t)__float_as_uint(hi) << 32) | __float_as_uint(lo);
-}
-__device__ __forceinline__ float f2lo(uint64_t v) { return __uint_as_float((uint32_t)v); }
-__device__ __forceinline__ float f2hi(uint64_t v) { return __uint_as_float((uint32_t)(v >> 32)); }
-__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t fadd2_rm(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rm.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-
-// 2^x for a pair on the FMA pipe, to take part of the load off the MUFU unit.
-// Cody-Waite split x = n + f with n = floor(x) and f in [0, 1): adding 1.5 * 2^23 with
-// round-toward-minus-infinity leaves n in the low mantissa bits of t (exact for
-// |x| < 2^22), and (bits(t) << 23) is n << 23 because the low nine bits of 1.5 * 2^23
-// are zero.  2^f is a cubic fitted to 2^f on [0, 1) for the least maximum relative error
-// (7.5e-5; 1.5e-4 after fp32 rounding), far below the bf16 rounding P gets next.
-// x is clamped to -125: the cubic lies in [0.99, 2), so the exponent field stays normal.
-constexpr float kExpC0 = 0.99992512554644490f;
-constexpr float kExpC1 = 0.69583399210713630f;
-constexpr float kExpC2 = 0.22606707273041300f;
-constexpr float kExpC3 = 0.07802403102605904f;
-__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x) {
-  const float x0 = fmaxf(f2lo(x), -125.f), x1 = fmaxf(f2hi(x), -125.f);
-  const uint64_t xc = f2pack(x0, x1);
-  const uint64_t magic = f2pack(12582912.f, 12582912.f);
-  const uint64_t t = fadd2_rm(xc, magic);
-  const uint64_t n = fadd2(t, f2pack(-12582912.f, -12582912.f));
-  const uint64_t f = fadd2(xc, n ^ 0x8000000080000000ull);  // x - n
-  uint64_t q = ffma2(f, f2pack(kExpC3, kExpC3), f2pack(kExpC2, kExpC2));
-  q = ffma2(f, q, f2pack(kExpC1, kExpC1));
-  q = ffma2(f, q, f2pack(kExpC0, kExpC0));
-  const uint32_t lo = (uint32_t)q + ((uint32_t)t << 23);
-  const uint32_t hi = (uint32_t)(q >> 32) + ((uint32_t)(t >> 32) << 23);
-  return ((uint64_t)hi << 32) | lo;
-}
-
-__device__ __forceinline__ float max3f(float a, float b, float c) {
-  float d;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-  return d;
-}
 
 // Maximum of the raw scores of one softmax warp's 64 columns (eight chains of three-input
 // max); with MASK, columns at or past `valid` are left out.
@@ -231,153 +149,10 @@ template <bool MASK, class Cols>
 __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
                                               float m, uint32_t taddr_p);
 
-// ---------------------------------------------------------------- mbarrier
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Bounded wait for the phase of the given parity.  false = gave up (timeout or abort).
-__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, TcBars* bars,
-                                            PadDevHeader* hdr, int where) {
-  const unsigned long long t0 = globaltimer();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63u) == 0) {
-      if (*reinterpret_cast<volatile int32_t*>(&bars->abort)) return false;
-      if (globaltimer() - t0 > kWaitNs) {
-        pad_set_error(hdr, bars->gen, PAD_ERR_DEVICE_TIMEOUT, (int)blockIdx.x, where, (int)threadIdx.x);
-        *reinterpret_cast<volatile int32_t*>(&bars->abort) = 1;
-        return false;
-      }
-    }
-  }
-}
+// Bounded wait of this kernel: gives up on the CTA's abort flag or after the time limit.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
                                           PadDevHeader* hdr, int where) {
-  if (mbar_try_wait(bar, parity)) return true;
-  return mbar_wait_slow(bar, parity, bars, hdr, where);
-}
-
-// ---------------------------------------------------------------- TMA
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
-                                            int c2, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
-      : "memory");
-}
-
-// ---------------------------------------------------------------- tcgen05
-__device__ __forceinline__ void fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-// Shared-memory matrix descriptor: start address, leading / stride byte offsets,
-// version 1 (bits 46-47), 128-byte swizzle (layout type 2 in bits 61-63).
-__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                       uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
-      : "memory");
-}
-__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                       uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accum)
-      : "memory");
-}
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
-      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
-      "r"(r[29]), "r"(r[30]), "r"(r[31])
-      : "memory");
-}
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15])
-      : "memory");
-}
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-// The registers written by tcgen05.ld are valid only after tcgen05.wait::ld; listing them
-// as operands of the wait makes every later use depend on it in the compiler's view too.
-__device__ __forceinline__ void tmem_wait_ld_dep(uint32_t* r) {
-  asm volatile(
-      "tcgen05.wait::ld.sync.aligned;"
-      : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
-        "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
-        "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]),
-        "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]),
-        "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
-      :
-      : "memory");
-}
-__device__ __forceinline__ void tmem_wait_st() {
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  return mbar_wait_b(bar, parity, &bars->abort, bars->gen, hdr, where);
 }
 
 template <bool MASK, class Cols>
@@ -416,11 +191,6 @@ __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols 
   return f2lo(ls) + f2hi(ls);
 }
 
-__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
-  const unsigned long long t0 = globaltimer();
-  while (!mbar_try_wait(bar, parity) && globaltimer() - t0 < kWaitNs) {
-  }
-}
 
 // Split counters of the fused tail, one per (video, kv-head, 128-row group): bits 15-0
 // count the video's splits that have written their partial rows, bits 31-16 the tasks
@@ -465,44 +235,6 @@ __device__ __forceinline__ bool tail_partials_ready(const KParams& p, const PadV
     }
   }
   return bm::SyncNamed{1}.all(good);
-}
-
-// Once its last K tile is issued (about three tiles before the CTA ends), the K producer
-// warp asks L2 for what the branch/merge kernel after this grid will read first: for the
-// (event, kv-head) task with the CTA's index, if there is one, the branch's stored K/V rows (through the page
-// table, whose entries for those keys no kernel of this step writes), its Q rows and, in the
-// one-call step, its new K/V row.  Those tasks then start on warm lines instead of waiting
-// on HBM behind their page-table reads.  Page ids outside the pool are skipped.
-__device__ __forceinline__ void prefetch_l2(const void* a) {
-  asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
-}
-__device__ __noinline__ void prefetch_branch_tasks(const KParams& p, const __nv_bfloat16* q,
-                                                   const __nv_bfloat16* kpool, const __nv_bfloat16* vpool,
-                                                   int lane) {
-  const int n_tasks = p.n_events * p.h_kv, G = p.group, ps = p.page_size;
-  // one task per CTA at most: a warp that walked many tasks here would hold the CTA (and
-  // the grid the branch/merge kernel waits for) open longer than the prefetch saves.  With
-  // the fused tail, the task this CTA will run itself.
-  const int t0 = p.fused ? plan_tasks(p)[blockIdx.x] : (int)blockIdx.x;
-  for (int t = t0; t >= 0 && t < n_tasks && t < (int)gridDim.x; t += gridDim.x) {
-    const int e = t / p.h_kv, h = t - (t / p.h_kv) * p.h_kv;
-    const int len = plan_events(p)[e].len;
-    const int32_t* ptab = p.page_table + (size_t)e * p.max_pages;
-    for (int k = lane; k < len; k += 32) {
-      const int pg = ptab[k / ps];
-      if (pg < 0 || pg >= p.n_pages) continue;
-      const size_t off = (((size_t)pg * p.h_kv + h) * ps + (k % ps)) * kD;
-      prefetch_l2(kpool + off);
-      prefetch_l2(kpool + off + 64);
-      prefetch_l2(vpool + off);
-      prefetch_l2(vpool + off + 64);
-    }
-    if (lane < 2 * G) prefetch_l2(q + ((size_t)e * p.h_q + h * G + (lane >> 1)) * kD + 64 * (lane & 1));
-    if (p.k_new != nullptr && lane < 4) {
-      const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(lane < 2 ? p.k_new : p.v_new);
-      prefetch_l2(src + ((size_t)e * p.h_kv + h) * kD + 64 * (lane & 1));
-    }
-  }
 }
 
 // Whole-sequence prefill (PREFILL): branch start of token p >= pf_S, from the branch
@@ -1085,8 +817,10 @@ std::mutex g_map_mu;
 MapCacheEntry g_maps[8];
 int g_maps_n = 0, g_maps_next = 0;
 
-bool get_maps(const void* kp, const void* vp, int h_kv, int64_t tokens, int dev, CUtensorMap* mk,
-              CUtensorMap* mv) {
+}  // namespace
+
+bool prefix_tensor_maps(const void* kp, const void* vp, int h_kv, int64_t tokens, int dev, CUtensorMap* mk,
+                        CUtensorMap* mv) {
   std::lock_guard<std::mutex> lk(g_map_mu);
   for (int i = 0; i < g_maps_n; ++i) {
     const MapCacheEntry& e = g_maps[i];
@@ -1111,8 +845,6 @@ bool get_maps(const void* kp, const void* vp, int h_kv, int64_t tokens, int dev,
   return true;
 }
 
-}  // namespace
-
 int prefix_tc_tail_chunk(int branch_rows, int group, int max_splits) {
   int sch = std::min(bm::kMaxChunk, std::max(1, max_splits));
   while (sch > 1 && bm::smem_bytes<kD>(branch_rows, group, sch) > kOffBar) --sch;
@@ -1128,7 +860,7 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   int dev = 0;
   cudaGetDevice(&dev);
   CUtensorMap mk, mv;
-  if (!get_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
+  if (!prefix_tensor_maps(kp, vp, p.h_kv, total_prefix_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
     for (auto fn : {prefix_tc_kernel<false, false, false>, prefix_tc_kernel<true, false, false>,
@@ -1186,7 +918,7 @@ cudaError_t launch_prefill_tc(int32_t n_tokens, int32_t prefix_len, int32_t n_br
   int dev = 0;
   cudaGetDevice(&dev);
   CUtensorMap mk, mv;
-  if (!get_maps(k, v, h_kv, n_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
+  if (!prefix_tensor_maps(k, v, h_kv, n_tokens, dev, &mk, &mv)) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   if (dev >= 0 && dev < 64 && !configured[dev]) {
     cudaError_t e = cudaFuncSetAttribute(prefix_tc_kernel<false, false, true>,

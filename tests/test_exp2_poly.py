@@ -1,5 +1,5 @@
 """Error bound of the FMA-pipe 2^x used for part of the softmax exponentials in the
-tensor-core prefix kernel: the constants are read from the kernel source and the
+tensor-core prefix kernels: the constants are read from the kernels' shared header and the
 instruction sequence (Cody-Waite split, cubic, exponent insertion) is replayed in fp32."""
 import os
 import re
@@ -7,7 +7,7 @@ import re
 import numpy as np
 
 SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
-                   "paper_2607_02963_gb300", "csrc", "pad_prefix_tc.cu")
+                   "paper_2607_02963_gb300", "csrc", "pad_tc_common.cuh")
 
 
 def constants():

@@ -5,6 +5,8 @@ outputs within max-abs <= 1e-2 and relative-L2 <= 2e-3 (bf16 in, fp32
 accumulate); the natural-log LSE within 1e-3 absolute (a log of an fp32 sum of
 positive terms: its error is the relative error of that sum, ~1e-6 here).
 """
+import hashlib
+
 import numpy as np
 import pytest
 import torch
@@ -69,32 +71,32 @@ def check_bookkeeping(db, w, plan):
     assert np.array_equal(gv, np.concatenate(vs)), "V pool contents differ"
 
 
+_ORACLE = {}
+
+
+def oracle_step(w):
+    """fp64 oracle of the whole step (every event, every head), kept per workload so that
+    the kernels compared on one workload share one oracle run."""
+    h = hashlib.sha1()
+    for a in (w.prefix_len, w.prefix_offset, w.event_video, w.event_len, w.q, w.k_prefix, w.v_prefix,
+              w.k_priv, w.v_priv, w.k_new, w.v_new):
+        h.update(np.ascontiguousarray(a).tobytes())
+    key = (h.hexdigest(), w.h_q, w.h_kv, w.head_dim, w.scale)
+    if key not in _ORACLE:
+        _ORACLE.clear()
+        _ORACLE[key] = oracle.decode_step(w)
+    return _ORACLE[key]
+
+
 def run_full(w, flags=0, out_dtype=0, what=""):
     db = DeviceBatch(w, flags=flags, out_dtype=out_dtype)
     plan = db.run_step()
     torch.cuda.synchronize()
     B.pad_device_status(plan)
     check_bookkeeping(db, w, plan)
-    ref_o, ref_lse = oracle.decode_step(w)
+    ref_o, ref_lse = oracle_step(w)
     got = db.out.float().cpu().numpy()
     check_outputs(got, db.lse.cpu().numpy(), ref_o, ref_lse, what or w.name)
-    return db, plan
-
-
-def run_sampled(w, events, heads=None, flags=0, what=""):
-    """Full-size step; the oracle computes the sampled events one by one."""
-    db = DeviceBatch(w, flags=flags)
-    plan = db.run_step()
-    torch.cuda.synchronize()
-    B.pad_device_status(plan)
-    check_bookkeeping(db, w, plan)
-    got_o = db.out.cpu().numpy()
-    got_l = db.lse.cpu().numpy()
-    for e in events:
-        ro, rl = oracle.event_rows(w, int(e), heads)
-        go = got_o[e] if heads is None else got_o[e, heads]
-        gl = got_l[e] if heads is None else got_l[e, heads]
-        check_outputs(go, gl, ro, rl, f"{what or w.name} event {e}")
     return db, plan
 
 
@@ -107,35 +109,28 @@ def test_tiny_full(flags):
     run_full(synth.tiny(), flags=flags)
 
 
-@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_DUAL])
 def test_gqa_8k_full(flags):
     run_full(synth.gqa_8k(), flags=flags)
 
 
-@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
-def test_long_32k_sampled(flags):
-    w = synth.long_32k()
-    rng = np.random.default_rng(0)
-    ev = sorted(set([0, w.n_events - 1] + list(rng.choice(w.n_events, 4, replace=False))))
-    run_sampled(w, ev, flags=flags)
+# The full-size workloads: every output row of every event against the oracle, in the
+# launch configuration the bench times (default flags: the tensor-core kernel), and on the
+# dual tensor-core kernel.
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
+def test_long_32k_full(flags):
+    run_full(synth.long_32k(), flags=flags)
 
 
-@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
-def test_ragged_serving_sampled(flags):
-    w = synth.ragged_serving()
-    ev = []
-    for b in range(w.n_videos):
-        idx = w.events_of_video(b)
-        ev += [int(idx[0]), int(idx[-1])] if b % 3 == 0 else [int(idx[len(idx) // 2])]
-    run_sampled(w, sorted(set(ev)), flags=flags)
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
+def test_ragged_serving_full(flags):
+    run_full(synth.ragged_serving(), flags=flags)
 
 
 @pytest.mark.parametrize("E", synth.SWEEP_E)
-@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_TC])
-def test_event_sweep_sampled(E, flags):
-    w = synth.event_sweep(E)
-    ev = sorted(set([0, E - 1, E // 2]))
-    run_sampled(w, ev, flags=flags)
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
+def test_event_sweep_full(E, flags):
+    run_full(synth.event_sweep(E), flags=flags)
 
 
 # ---------------------------------------------------------------------------
@@ -155,6 +150,24 @@ def test_random_small_tc(seed):
 
 
 @pytest.mark.parametrize("seed", range(6))
+def test_random_small_dual_tile_parity(seed):
+    """<= 128 rows per item: the two softmax groups take alternate tiles of the same rows and
+    their states are merged (odd and even tile counts, one-tile splits)."""
+    run_full(synth.random_small(seed, h_q=8, h_kv=2, max_prefix=900, max_events=7),
+             flags=B.FLAG_PREFIX_DUAL)
+
+
+@pytest.mark.parametrize("E,prefix", [(19, 1000), (32, 130), (36, 100), (37, 1000), (64, 700), (40, 3000)])
+def test_dual_row_groups(E, prefix):
+    """> 128 rows per item (G = 7): two row groups share each tile (19 events: the second
+    group holds 5 rows; 36: 252 rows); more than 256 rows take a second CTA (37 events: 256
+    + 3 rows; 64: 256 + 192; 40: 256 + 24), whose last group may again fall back to tile
+    parities; one- and two-tile splits and a ragged last tile."""
+    lens = [(29 * i + 3) % 97 for i in range(E)]
+    run_full(_w([prefix], [E], lens, seed=90 + E), flags=B.FLAG_PREFIX_DUAL, what=f"dual E {E} prefix {prefix}")
+
+
+@pytest.mark.parametrize("seed", range(6))
 def test_random_small_simt(seed):
     run_full(synth.random_small(seed, h_q=8, h_kv=2, max_prefix=900, max_events=4),
              flags=B.FLAG_PREFIX_SIMT)
@@ -167,7 +180,7 @@ def test_random_small_head_dim_64(seed):
     run_full(w, flags=B.FLAG_PREFIX_SIMT)
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 def test_large_group_and_outlier_channels(flags):
     w = synth.random_small(60, h_q=32, h_kv=2, max_prefix=700, max_events=3, k_scale_sigma=0.5)
     run_full(w, flags=flags)
@@ -183,16 +196,17 @@ def _w(prefix, epv, lens, seed=7, h_q=28, h_kv=4, D=128, sigma=None, page_size=1
                                k_scale_sigma=sigma, page_size=page_size)
 
 
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 @pytest.mark.parametrize("ps", [4, 8, 32, 64])
-def test_page_sizes_many_events(ps):
+def test_page_sizes_many_events(ps, flags):
     """40 events of 7 rows (280 rows: three 128-row groups, two events straddling group
     boundaries) with branch lengths on and around page boundaries, for page sizes other
     than 16, over pools whose unwritten slots hold NaN."""
     lens = [(37 * i) % 131 for i in range(36)] + [ps, ps - 1, 2 * ps + 1, 0]
-    run_full(_w([3000], [40], lens, seed=41 + ps, page_size=ps), flags=B.FLAG_PREFIX_TC, what=f"ps {ps}")
+    run_full(_w([3000], [40], lens, seed=41 + ps, page_size=ps), flags=flags, what=f"ps {ps}")
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_SIMT, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_SIMT, B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 def test_single_event_empty_branch(flags):
     run_full(_w([300], [1], [0]), flags=flags)          # query sees the prefix and itself
 
@@ -202,26 +216,27 @@ def test_page_boundaries(lens):
     run_full(_w([257], [len(lens)], lens))
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 def test_prefix_not_multiple_of_tile_and_tiny_prefix(flags):
     run_full(_w([1, 129, 65], [2, 3, 2], [3, 0, 9, 16, 2, 5, 7]), flags=flags)
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 def test_video_with_empty_prefix_and_video_without_events(flags):
     run_full(_w([0, 500, 200], [2, 0, 3], [4, 1, 0, 16, 2]), flags=flags)
 
 
-@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC])
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_MMA, B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
 def test_sixty_four_events(flags):
     run_full(_w([700], [64], list(np.arange(64) % 40)), flags=flags)
 
 
-def test_long_split_many_tiles_tc():
-    """Few SMs -> long splits: many 64-token tiles per CTA (the 4-stage ring wraps several
-    times, both S buffers alternate, lazy rescaling meets growing maxima)."""
+@pytest.mark.parametrize("flags", [B.FLAG_PREFIX_TC, B.FLAG_PREFIX_DUAL])
+def test_long_split_many_tiles_tc(flags):
+    """Few SMs -> long splits: many tiles per CTA (the stage rings wrap several times, the S
+    buffers alternate, lazy rescaling meets growing maxima)."""
     w = _w([5000, 3001], [5, 9], list(range(0, 70, 5)), sigma=0.5)
-    db = DeviceBatch(w, flags=B.FLAG_PREFIX_TC, num_sms=4)
+    db = DeviceBatch(w, flags=flags, num_sms=4)
     plan = db.run_step()
     torch.cuda.synchronize()
     B.pad_device_status(plan)
@@ -278,8 +293,7 @@ def test_large_batch_reads_descriptors_from_host_image(D, h_q):
     rng = np.random.default_rng(11)
     lens = [int(x) for x in rng.integers(0, 40, size=500)]
     w = _w([96, 40, 0, 130, 64], [100] * 5, lens, seed=11, h_q=h_q, h_kv=2, D=D)
-    ev = [0, 99, 100, 250, 299, 300, 401, 499]
-    db, plan = run_sampled(w, ev)
+    db, plan = run_full(w)
     assert plan.info()["param_descriptor_bytes"] == 0
     o1 = db.out.clone()
     for _ in range(12):  # more than the images kept in flight per device

@@ -101,6 +101,15 @@ def test_workload_sizes_and_kernel_choice(padlib):
     plan = B.pad_plan(prob, cache, [16384], [0], [1], max_pages=4, workspace=None)
     assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_TC
     assert plan.info()["n_work_items"] <= 148
+    # forced: the dual kernel, one 256-row CTA per item
+    prob_d = B.make_problem(28, 4, 128, num_sms=148, flags=B.FLAG_PREFIX_DUAL)
+    info = B.pad_plan(prob_d, cache, [32768], [0] * 32, [1] * 32, max_pages=4, workspace=None).info()
+    assert info["prefix_kernel"] == B.FLAG_PREFIX_DUAL
+    assert 130 <= info["n_work_items"] <= 148
+    # the fused tail asks for the single-group kernel
+    prob_f = B.make_problem(28, 4, 128, num_sms=148, flags=B.FLAG_FUSED_MERGE)
+    info = B.pad_plan(prob_f, cache, [32768], [0] * 32, [1] * 32, max_pages=4, workspace=None).info()
+    assert info["prefix_kernel"] == B.FLAG_PREFIX_TC
     # head_dim 64: warp-level paths, warp-shuffle for <= 8 rows
     prob64 = B.make_problem(16, 4, 64, num_sms=148)
     plan = B.pad_plan(prob64, cache, [4096], [0, 0], [1, 1], max_pages=4, workspace=None)
@@ -109,7 +118,8 @@ def test_workload_sizes_and_kernel_choice(padlib):
     assert plan.info()["prefix_kernel"] == B.FLAG_PREFIX_MMA
 
 
-def test_tc_split_fits_one_wave(padlib):
+@pytest.mark.parametrize("flags,rows_per_cta", [(0, 128), (B.FLAG_PREFIX_DUAL, 256)])
+def test_tc_split_fits_one_wave(padlib, flags, rows_per_cta):
     rng = np.random.default_rng(5)
     for trial in range(50):
         B_ = int(rng.integers(1, 17))
@@ -118,10 +128,10 @@ def test_tc_split_fits_one_wave(padlib):
         ev_video = np.repeat(np.arange(B_, dtype=np.int32), Ev)
         L = np.zeros(ev_video.size, dtype=np.int32)
         sms = int(rng.integers(8, 160))
-        prob = B.make_problem(28, 4, 128, num_sms=sms)
+        prob = B.make_problem(28, 4, 128, num_sms=sms, flags=flags)
         plan = B.pad_plan(prob, B.CacheState(4096), P, ev_video, L, max_pages=2, workspace=None)
         info = plan.info()
-        groups = -(-int(Ev.max()) * 7 // 128)
+        groups = -(-int(Ev.max()) * 7 // rows_per_cta)
         sl = info["split_len"]
         assert sl % 128 == 0
         # one wave unless a single split per (video, kv-head) is already too many
