@@ -40,6 +40,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 constexpr int kDefaultSms = 152;
+constexpr int kPrefixFlags = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC | PAD_FLAG_PREFIX_DUAL;
 
 int query_num_sms() {
   static int cache[64] = {};
@@ -77,9 +78,10 @@ pad_status check_problem(const pad_problem* prob) {
   if (prob->out_dtype != 0 && prob->out_dtype != 1)
     return fail(PAD_ERR_INVALID_ARG, "out_dtype=%d (0 = fp32, 1 = bf16)", prob->out_dtype);
   if (prob->num_sms < 0) return fail(PAD_ERR_INVALID_ARG, "num_sms < 0");
-  const int known = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC | PAD_FLAG_FUSED_MERGE;
+  const int known = PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC | PAD_FLAG_PREFIX_DUAL |
+                    PAD_FLAG_FUSED_MERGE;
   if (prob->flags & ~known) return fail(PAD_ERR_INVALID_ARG, "unknown flags 0x%x", prob->flags);
-  const int f = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
+  const int f = prob->flags & kPrefixFlags;
   if (f && (f & (f - 1))) return fail(PAD_ERR_INVALID_ARG, "at most one PAD_FLAG_PREFIX_* flag");
   return PAD_OK;
 }
@@ -139,7 +141,7 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
 
   // Prefix kernel: forced by a flag, else the tensor-core path for head_dim 128 and the
   // warp-level paths for head_dim 64 (mma.sync above 8 rows, warp-shuffle below).
-  int kern = prob->flags & (PAD_FLAG_PREFIX_SIMT | PAD_FLAG_PREFIX_MMA | PAD_FLAG_PREFIX_TC);
+  int kern = prob->flags & kPrefixFlags;
   if (kern == 0) {
     if (prob->head_dim == 128)
       kern = PAD_FLAG_PREFIX_TC;
@@ -149,7 +151,7 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   if (kern == PAD_FLAG_PREFIX_SIMT && max_rows > 16)
     return fail(PAD_ERR_UNSUPPORTED, "SIMT prefix path takes at most 16 rows per (video, kv-head); got %d",
                 max_rows);
-  if (kern == PAD_FLAG_PREFIX_TC && prob->head_dim != 128)
+  if ((kern == PAD_FLAG_PREFIX_TC || kern == PAD_FLAG_PREFIX_DUAL) && prob->head_dim != 128)
     return fail(PAD_ERR_UNSUPPORTED, "tcgen05 prefix path takes head_dim 128; got %d", prob->head_dim);
   L->prefix_kernel = kern;
 
@@ -157,7 +159,10 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   // (token-heads, times the 128-row groups each item occupies on the tensor-core path)
   // spreads over one wave of SMs.  The tensor-core kernel runs one CTA per SM, so its
   // split is grown until items x row groups fit in a single wave.
-  const int groups = (kern == PAD_FLAG_PREFIX_TC) ? std::max(1, (max_rows + 127) / 128) : 1;
+  // CTAs per item: 128-row groups on the tcgen05 kernel, 256-row groups on the dual one
+  const int groups = (kern == PAD_FLAG_PREFIX_TC)     ? std::max(1, (max_rows + 127) / 128)
+                     : (kern == PAD_FLAG_PREFIX_DUAL) ? std::max(1, (max_rows + 255) / 256)
+                                                      : 1;
   int64_t work = 0;
   for (int b = 0; b < n_videos; ++b)
     if (L->ev_count[b] > 0) work += (int64_t)prefix_len[b] * prob->h_kv * groups;
@@ -170,7 +175,7 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
       if (L->ev_count[b] > 0 && prefix_len[b] > 0) n += (int64_t)prob->h_kv * ((prefix_len[b] + c - 1) / c);
     return n * groups;
   };
-  if (kern == PAD_FLAG_PREFIX_TC) {
+  if (kern == PAD_FLAG_PREFIX_TC || kern == PAD_FLAG_PREFIX_DUAL) {
     int64_t max_prefix = 0;
     for (int b = 0; b < n_videos; ++b)
       if (L->ev_count[b] > 0) max_prefix = std::max<int64_t>(max_prefix, prefix_len[b]);
@@ -795,6 +800,10 @@ pad_status pad_plan_destroy(pad_plan_t* plan) {
   return PAD_OK;
 }
 
+static pad_status static_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new, void* k_pool,
+                                   void* v_pool, cudaStream_t s);
+static pad_status static_status_header(PadDevHeader** out);
+
 static void make_params(const pad_plan_t* plan, KParams& p) {
   const pad_problem& pr = plan->prob;
   p.h_q = pr.h_q;
@@ -852,11 +861,15 @@ pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* 
                          void* k_pool, void* v_pool, pad_stream_t stream) {
   if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
   if (plan->n_events == 0) return PAD_OK;
-  if (!plan->workspace) return fail(PAD_ERR_INVALID_ARG, "plan was built without a workspace");
   if (!k_new || !v_new || !k_pool || !v_pool) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_pool) || !aligned16(v_pool))
     return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // a host-only plan (no workspace): the library's static scratch array stands in for it
+  if (!plan->workspace) {
+    if (!plan->page_table) return fail(PAD_ERR_INVALID_ARG, "plan has no page table");
+    return static_kv_append(plan, k_new, v_new, k_pool, v_pool, s);
+  }
   KParams p;
   make_params(plan, p);
   cudaError_t e = launch_append(p, k_new, v_new, k_pool, v_pool, s);
@@ -907,6 +920,10 @@ static pad_status launch_attention(const pad_plan_t* plan, const void* q, const 
       e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
                            v_pool, out, lse, !timed, s);
       break;
+    case PAD_FLAG_PREFIX_DUAL:
+      e = launch_prefix_dual(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
+                             v_pool, !timed, s);
+      break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }
   if (e != cudaSuccess) return cuda_fail(e, "prefix launch");
@@ -915,7 +932,8 @@ static pad_status launch_attention(const pad_plan_t* plan, const void* q, const 
     g_timing.n++;
   }
   if (!plan->lay.fused) {
-    const bool pdl = !timed && plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC;
+    const bool pdl = !timed && (plan->lay.prefix_kernel == PAD_FLAG_PREFIX_TC ||
+                                plan->lay.prefix_kernel == PAD_FLAG_PREFIX_DUAL);
     e = launch_branch_merge(p, q, k_pool, v_pool, out, lse, pdl, s);
     if (e != cudaSuccess) return cuda_fail(e, "branch/merge launch");
   }
@@ -1139,17 +1157,26 @@ void pad_step_destroy(pad_step_t* step) { delete step; }
 
 pad_status pad_device_status(const pad_plan_t* plan, pad_stream_t stream) {
   if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
-  if (!plan->workspace) return PAD_OK;
+  // a host-only plan reports through the static scratch array's status word (if no call
+  // has used the array on this device, nothing of this plan ran there)
+  const void* word = plan->workspace;
+  if (!word) {
+    PadDevHeader* sh = nullptr;
+    pad_status st = static_status_header(&sh);
+    if (st != PAD_OK) return st;
+    if (!sh) return PAD_OK;
+    word = sh;
+  }
   PadDevHeader h;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = cudaMemcpyAsync(&h, plan->workspace, sizeof(h), cudaMemcpyDeviceToHost, s);
+  cudaError_t e = cudaMemcpyAsync(&h, word, sizeof(h), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "reading device status");
   const int code = (int)(h.word & 0xffull);
   if ((h.word >> 8) == plan->gen && code != PAD_OK) {
     // a failed launch may have left the fused tail's split counters part-way: zero them,
     // so that the next plan on this workspace starts clean
-    if (plan->lay.n_counters > 0) {
+    if (plan->lay.n_counters > 0 && plan->workspace) {
       e = cudaMemsetAsync(static_cast<uint8_t*>(plan->workspace) + plan->lay.off_cnt, 0,
                           (size_t)plan->lay.n_counters * sizeof(unsigned int), s);
       if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -1221,47 +1248,47 @@ static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBy
 std::mutex g_static_mu;
 void* g_static_ptr[64] = {};
 
-}  // namespace
-
-extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q,
-                                                   const void* k_prefix, const void* v_prefix,
-                                                   const void* k_pool, const void* v_pool, void* out,
-                                                   float* lse, pad_stream_t stream) {
-  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
-  if (plan->n_events == 0) return PAD_OK;
-  if (plan->lay.total_bytes > kStaticScratchBytes)
-    return fail(PAD_ERR_WORKSPACE_TOO_SMALL,
-                "plan needs %zu bytes of scratch; the static scratch array holds %zu bytes",
-                plan->lay.total_bytes, kStaticScratchBytes);
-  if (!plan->page_table) return fail(PAD_ERR_INVALID_ARG, "plan has no page table");
-  if (!q || !k_pool || !v_pool || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
-  if (plan->lay.n_items > 0 && (!k_prefix || !v_prefix))
-    return fail(PAD_ERR_INVALID_ARG, "k_prefix / v_prefix is NULL");
-  if (!aligned16(q) || !aligned16(k_prefix) || !aligned16(v_prefix) || !aligned16(k_pool) ||
-      !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
-    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
+// The static array's device address on the current device, looked up on the first call
+// made with that device current and cached (lookup = false: only the cached address, or
+// NULL when no call has used the array on this device yet).
+pad_status static_scratch(bool lookup, uint8_t** out) {
+  *out = nullptr;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(PAD_ERR_UNSUPPORTED, "device index %d", dev);
-  void* scratch = nullptr;
-  {
-    std::lock_guard<std::mutex> lk(g_static_mu);
-    if (!g_static_ptr[dev]) {
-      void* ptr = nullptr;
-      e = cudaGetSymbolAddress(&ptr, g_static_scratch);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
-      g_static_ptr[dev] = ptr;
-    }
-    scratch = g_static_ptr[dev];
+  std::lock_guard<std::mutex> lk(g_static_mu);
+  if (!g_static_ptr[dev] && lookup) {
+    void* ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_static_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(static scratch)");
+    g_static_ptr[dev] = ptr;
   }
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // plan image (header with a zero status word, video and event descriptors, work items);
-  // a copy from the plan's own pageable host buffer, staged by the driver
-  e = cudaMemcpyAsync(scratch, plan->host_image.data(), plan->lay.upload_bytes, cudaMemcpyHostToDevice, s);
-  if (e != cudaSuccess) return cuda_fail(e, "static scratch plan upload");
+  *out = static_cast<uint8_t*>(g_static_ptr[dev]);
+  return PAD_OK;
+}
 
-  KParams p;
+// Launch parameters of a plan whose scratch is the static array.  The plan image (video
+// and event descriptors, work items) is copied into the array on `s`, from the plan's own
+// pageable host buffer: the driver stages that copy, so the call returns once the bytes
+// are staged.  The status word ahead of the image is left as it is: it is tagged with the
+// generation of the plan whose kernels wrote it, so a word from another plan reads as
+// clear, and an error of this plan's append survives until its attention call and
+// pad_device_status read it.
+pad_status static_params(const pad_plan_t* plan, cudaStream_t s, KParams& p, uint8_t** ws_out) {
+  if (plan->lay.total_bytes > kStaticScratchBytes)
+    return fail(PAD_ERR_WORKSPACE_TOO_SMALL,
+                "plan needs %zu bytes of scratch; the static scratch array holds %zu bytes",
+                plan->lay.total_bytes, kStaticScratchBytes);
+  uint8_t* ws = nullptr;
+  pad_status st = static_scratch(true, &ws);
+  if (st != PAD_OK) return st;
+  const size_t hb = sizeof(PadDevHeader);
+  if (plan->lay.upload_bytes > hb) {
+    cudaError_t e = cudaMemcpyAsync(ws + hb, plan->host_image.data() + hb, plan->lay.upload_bytes - hb,
+                                    cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "static scratch plan upload");
+  }
   const pad_problem& pr = plan->prob;
   p.h_q = pr.h_q;
   p.h_kv = pr.h_kv;
@@ -1288,7 +1315,6 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.causal = plan->causal;
   p.fused = plan->lay.fused ? 1 : 0;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
-  auto* ws = static_cast<uint8_t*>(scratch);
   p.tasks = reinterpret_cast<const int32_t*>(ws + plan->lay.off_tasks);
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
   p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;
@@ -1299,7 +1325,57 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
   p.part_ml = reinterpret_cast<float2*>(ws + plan->lay.off_ml);
   p.part_o = reinterpret_cast<float*>(ws + plan->lay.off_o);
   p.page_table = plan->page_table;
+  *ws_out = ws;
+  return PAD_OK;
+}
 
+}  // namespace
+
+// pad_kv_append of a plan built without a workspace: the append kernel reads the plan's
+// event descriptors from the static array and reports into its status word.
+static pad_status static_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new, void* k_pool,
+                                   void* v_pool, cudaStream_t s) {
+  KParams p;
+  uint8_t* ws = nullptr;
+  pad_status st = static_params(plan, s, p, &ws);
+  if (st != PAD_OK) return st;
+  cudaError_t e = launch_append(p, k_new, v_new, k_pool, v_pool, s);
+  if (e != cudaSuccess) return cuda_fail(e, "append launch (static scratch)");
+  return PAD_OK;
+}
+
+// The static array's status header, or NULL when no call has used the array on the
+// current device.
+static pad_status static_status_header(PadDevHeader** out) {
+  uint8_t* ws = nullptr;
+  pad_status st = static_scratch(false, &ws);
+  *out = reinterpret_cast<PadDevHeader*>(ws);
+  return st;
+}
+
+extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const void* q,
+                                                   const void* k_prefix, const void* v_prefix,
+                                                   const void* k_pool, const void* v_pool, void* out,
+                                                   float* lse, pad_stream_t stream) {
+  if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
+  if (plan->n_events == 0) return PAD_OK;
+  if (plan->lay.total_bytes > kStaticScratchBytes)
+    return fail(PAD_ERR_WORKSPACE_TOO_SMALL,
+                "plan needs %zu bytes of scratch; the static scratch array holds %zu bytes",
+                plan->lay.total_bytes, kStaticScratchBytes);
+  if (!plan->page_table) return fail(PAD_ERR_INVALID_ARG, "plan has no page table");
+  if (!q || !k_pool || !v_pool || !out) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
+  if (plan->lay.n_items > 0 && (!k_prefix || !v_prefix))
+    return fail(PAD_ERR_INVALID_ARG, "k_prefix / v_prefix is NULL");
+  if (!aligned16(q) || !aligned16(k_prefix) || !aligned16(v_prefix) || !aligned16(k_pool) ||
+      !aligned16(v_pool) || !aligned16(out) || (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)))
+    return fail(PAD_ERR_INVALID_ARG, "tensors must be 16-byte aligned (lse 4-byte)");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  KParams p;
+  uint8_t* ws = nullptr;
+  pad_status st = static_params(plan, s, p, &ws);
+  if (st != PAD_OK) return st;
+  cudaError_t e = cudaSuccess;
   switch (plan->lay.prefix_kernel) {
     case PAD_FLAG_PREFIX_SIMT: e = launch_prefix_simt(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
     case PAD_FLAG_PREFIX_MMA: e = launch_prefix_mma(p, plan->lay.max_rows, q, k_prefix, v_prefix, s); break;
@@ -1310,6 +1386,10 @@ extern "C" pad_status pad_event_decode_attn_static(const pad_plan_t* plan, const
       }
       e = launch_prefix_tc(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
                            v_pool, out, lse, false, s);
+      break;
+    case PAD_FLAG_PREFIX_DUAL:
+      e = launch_prefix_dual(p, plan->lay.max_rows, q, k_prefix, v_prefix, plan->total_prefix_tokens, k_pool,
+                             v_pool, false, s);
       break;
     default: return fail(PAD_ERR_UNSUPPORTED, "prefix kernel %d", plan->lay.prefix_kernel);
   }

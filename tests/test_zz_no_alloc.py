@@ -69,3 +69,140 @@ def test_static_scratch_matches_workspace_path_twice(padlib, make):
                                        o, lse)
         torch.cuda.synchronize()
         _compare(o, lse, ref_o, ref_l)
+
+
+# ---------------------------------------------------------------------------
+# A whole decode loop with no device scratch: host-only plans for both calls
+# ---------------------------------------------------------------------------
+
+def _next_step(w, seed):
+    """The workload of the following decode step: every branch one token longer (this step's
+    new K/V appended), a fresh q / k_new / v_new, and the page table and free list as the
+    step left them (the oracle's simulation of the append)."""
+    import dataclasses
+    import oracle
+    st, pt, free, _ = oracle.simulate_append(w.page_table, w.free_pages, w.event_len, w.page_size)
+    assert st == oracle.OK
+    rng = np.random.default_rng(seed)
+    kp = [np.concatenate([w.priv_k(e), w.k_new[e:e + 1]]) for e in range(w.n_events)]
+    vp = [np.concatenate([w.priv_v(e), w.v_new[e:e + 1]]) for e in range(w.n_events)]
+    lens = (w.event_len + 1).astype(np.int32)
+    off = np.zeros(w.n_events + 1, np.int64)
+    off[1:] = np.cumsum(lens)
+
+    def draw(shape):
+        return synth.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+
+    return dataclasses.replace(w, event_len=lens, priv_off=off, k_priv=np.concatenate(kp),
+                               v_priv=np.concatenate(vp), q=draw(w.q.shape), k_new=draw(w.k_new.shape),
+                               v_new=draw(w.v_new.shape), page_table=pt, free_pages=free)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
+def test_host_only_plans_run_two_steps_against_the_oracle(padlib, flags):
+    """A caller with no device scratch runs two consecutive steps with pad_kv_append +
+    pad_event_decode_attn_static on plans built without a workspace: branches on page
+    boundaries open pages in the first step and others in the second; the outputs match the
+    fp64 oracle and the page table the simulated bookkeeping, after both steps."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import oracle
+    from paper_2607_02963_gb300.device import bits_to_bf16
+    rng = np.random.default_rng(3)
+    w = synth.make_workload("host_only", 3, 28, 4, 128, [1500, 700], [3, 2], [0, 15, 16, 31, 47], rng=rng)
+    db = DeviceBatch(w)
+    for step in range(2):
+        if step:
+            w = _next_step(w, 40 + step)
+            db.q.copy_(bits_to_bf16(w.q, db.device))
+            db.k_new.copy_(bits_to_bf16(w.k_new, db.device))
+            db.v_new.copy_(bits_to_bf16(w.v_new, db.device))
+        prob = B.make_problem(w.h_q, w.h_kv, w.head_dim, w.page_size, w.scale, flags=flags)
+        plan = B.pad_plan(prob, db.cache, w.prefix_len, w.event_video, w.event_len,
+                          page_table=db.page_table, max_pages=w.max_pages, workspace=None,
+                          prefix_offset=w.prefix_offset)
+        B.pad_kv_append(plan, db.k_new, db.v_new, db.k_pool, db.v_pool)
+        o = torch.full_like(db.out, float("nan"))
+        lse = torch.full_like(db.lse, float("nan"))
+        B.pad_event_decode_attn_static(plan, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool, o, lse)
+        torch.cuda.synchronize()
+        B.pad_device_status(plan)
+        st, pt, _, _ = oracle.simulate_append(w.page_table, w.free_pages, w.event_len, w.page_size)
+        assert st == oracle.OK
+        assert np.array_equal(db.page_table.cpu().numpy(), pt), f"page table after step {step}"
+        ref_o, ref_l = oracle.decode_step(w)
+        _compare(o, lse, torch.from_numpy(ref_o), torch.from_numpy(ref_l))
+
+
+@pytest.mark.gpu
+def test_static_path_reports_device_errors(padlib):
+    """An out-of-pool page id met by the kernels on the static path is reported by
+    pad_device_status for that plan (the status word lives in the static array), and a
+    clean step afterwards on the same array runs and reports nothing."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    w = synth.make_workload("static_bad", 7, 28, 4, 128, [200], [2], [5, 3])
+    db = DeviceBatch(w)
+    good = int(db.page_table[1, 0])
+    db.page_table[1, 0] = w.n_pages + 5
+    plan = B.pad_plan(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                      page_table=db.page_table, max_pages=w.max_pages, workspace=None,
+                      prefix_offset=w.prefix_offset)
+    B.pad_kv_append(plan, db.k_new, db.v_new, db.k_pool, db.v_pool)
+    B.pad_event_decode_attn_static(plan, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool,
+                                   db.out, db.lse)
+    with pytest.raises(B.PadError) as ei:
+        B.pad_device_status(plan)
+    assert ei.value.status == 7
+    plan.release_new_pages(db.cache)
+    db.page_table[1, 0] = good
+    plan2 = B.pad_plan(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                       page_table=db.page_table, max_pages=w.max_pages, workspace=None,
+                       prefix_offset=w.prefix_offset)
+    B.pad_kv_append(plan2, db.k_new, db.v_new, db.k_pool, db.v_pool)
+    B.pad_event_decode_attn_static(plan2, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool,
+                                   db.out, db.lse)
+    torch.cuda.synchronize()
+    B.pad_device_status(plan2)
+    import oracle
+    ref_o, ref_l = oracle.decode_step(w)
+    _compare(db.out, db.lse, torch.from_numpy(ref_o), torch.from_numpy(ref_l))
+
+
+@pytest.mark.gpu
+def test_plan_just_under_the_static_limit(padlib):
+    """A plan whose scratch is just under the array's 16 MiB runs on the static path and
+    matches the workspace path of the same step."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    # videos of 64 events x 7 q-heads per kv-head with short prefixes (one split each): the
+    # partial states grow by ~0.9 MiB per video; take the most videos that still fit
+    prob = B.make_problem(28, 4, 128, num_sms=152)
+    best = None
+    for nv in range(1, 40):
+        ev = np.repeat(np.arange(nv, dtype=np.int32), 64)
+        ws = B.pad_workspace_size(prob, np.full(nv, 300, np.int32), ev)
+        if ws > 16 << 20:
+            break
+        best = (nv, ws)
+    assert best is not None and best[1] > 15 << 20
+    rng = np.random.default_rng(11)
+    w = synth.make_workload("near_limit", 11, 28, 4, 128, [300] * best[0], [64] * best[0],
+                            rng.integers(0, 40, size=64 * best[0]), rng=rng)
+    db = DeviceBatch(w, num_sms=152)
+    plan = db.run_step()
+    torch.cuda.synchronize()
+    B.pad_device_status(plan)
+    assert plan.info()["workspace_bytes"] == best[1]
+    ref_o, ref_l = db.out.clone(), db.lse.clone()
+    db.release_new_pages(plan)
+    hplan = B.pad_plan(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
+                       page_table=db.page_table, max_pages=w.max_pages, workspace=None,
+                       prefix_offset=w.prefix_offset)
+    o = torch.full_like(db.out, float("nan"))
+    lse = torch.full_like(db.lse, float("nan"))
+    B.pad_event_decode_attn_static(hplan, db.q, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool, o, lse)
+    torch.cuda.synchronize()
+    B.pad_device_status(hplan)
+    _compare(o, lse, ref_o, ref_l)
