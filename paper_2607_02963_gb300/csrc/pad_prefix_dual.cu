@@ -581,10 +581,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->phi[wg]);
     }
-    // The slot's O is final once its last P.V has completed; every S and P.V MMA before it
-    // has then completed too, so the K stages (and, after slot 1's, the V stages) are idle
-    // and hold the O rows for the write-out.
+    // The slot's O is final once its last P.V has completed (which, issued by one thread,
+    // implies every earlier P.V: after slot 1's the V stages are idle); the K stages are
+    // idle once the S issuer's last MMA has completed.  They hold the O rows for the
+    // write-out.
     if (ok && n_mine > 0) ok = dwait(&bars->pvdone[wg], (uint32_t)((n_mine - 1) & 1), bars, p.header, 10);
+    // With two row groups, slot 0 stages into the K stages: the S issuer's last MMA
+    // (slot 1's, issued after slot 0's last S, which is all this group has seen complete)
+    // must have finished reading them.
+    if (ok && dual && wg == 0) ok = dwait(&bars->drain_s, 0u, bars, p.header, 14);
     ok = __all_sync(0xffffffffu, ok);
     uint32_t r[32];
     if (dual) {

@@ -347,9 +347,29 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   if (threadIdx.x == 0) {
+    // The first K and V tile go out first (their barriers initialised, then the loads),
+    // before the other barriers, TMEM allocation and the block barrier; the producer warps
+    // issue the rest once that K tile has landed, so that every CTA's first tile is not
+    // queued in DRAM behind the later tiles of all the others.
+    mbar_init(&bars->kfull[0], 1);
+    mbar_init(&bars->vfull[0], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (n_tiles > 0) {
+      mbar_expect_tx(&bars->kfull[0], kTileBytes);
+      tma_load_3d(sbase + kOffK, &tmK, 0, kvh, tile_tok(0), &bars->kfull[0]);
+      tma_load_3d(sbase + kOffK + kHalfBytes, &tmK, 64, kvh, tile_tok(0), &bars->kfull[0]);
+      mbar_expect_tx(&bars->vfull[0], kTileBytes);
+      tma_load_3d(sbase + kOffV, &tmV, 0, kvh, tile_tok(0), &bars->vfull[0]);
+      tma_load_3d(sbase + kOffV + kHalfBytes, &tmV, 64, kvh, tile_tok(0), &bars->vfull[0]);
+    }
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&bars->kfull[s], 1);
-      mbar_init(&bars->vfull[s], 1);
+      if (s > 0) {
+        mbar_init(&bars->kfull[s], 1);
+        mbar_init(&bars->vfull[s], 1);
+      }
       mbar_init(&bars->pvfree[s], 1);
     }
     for (int b = 0; b < kSBuf; ++b) {
@@ -365,19 +385,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     bars->gen = p.gen;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    // The first kStages K and V tiles go out before TMEM allocation and the block
-    // barrier; the producer warps issue the rest.
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
-    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
-    for (int t = 0; t < kStages && t < n_tiles; ++t) {
-      mbar_expect_tx(&bars->kfull[t], kTileBytes);
-      tma_load_3d(sbase + kOffK + t * kTileBytes, &tmK, 0, kvh, tile_tok(t), &bars->kfull[t]);
-      tma_load_3d(sbase + kOffK + t * kTileBytes + kHalfBytes, &tmK, 64, kvh, tile_tok(t), &bars->kfull[t]);
-      mbar_expect_tx(&bars->vfull[t], kTileBytes);
-      tma_load_3d(sbase + kOffV + t * kTileBytes, &tmV, 0, kvh, tile_tok(t), &bars->vfull[t]);
-      tma_load_3d(sbase + kOffV + t * kTileBytes + kHalfBytes, &tmV, 64, kvh, tile_tok(t), &bars->vfull[t]);
-    }
   }
   if (warp == 2) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -403,11 +410,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const bool isK = warp == 0;
       const CUtensorMap* map = isK ? &tmK : &tmV;
-      int issued = min(kStages, n_tiles);  // tiles 0..kStages-1 went out in the prologue
-      bool ok = true;
-      for (int t = kStages; t < n_tiles && ok; ++t) {
+      int issued = min(1, n_tiles);  // tile 0 went out in the prologue
+      // the other stages fill once the first K tile has landed
+      bool ok = n_tiles <= 1 || mbar_wait(&bars->kfull[0], 0u, bars, p.header, isK ? 1 : 2);
+      for (int t = 1; t < n_tiles && ok; ++t) {
         const int s = t % kStages;
-        {
+        if (t >= kStages) {
           // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
           uint64_t* freed = isK ? &bars->sfull[s] : &bars->pvfree[s];
           ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
