@@ -99,6 +99,10 @@ struct Layout {
   // fused tail of the tensor-core path: per prefix CTA its (event * h_kv + kv-head) task or
   // -1, and per (video, kv-head, row group) a split counter
   bool fused = false;
+  // Without the fused tail, the tensor-core kernels take their CTAs from a list of
+  // (work item, row group) pairs, (item << 6) | group, kept in cta_task: a video with fewer
+  // rows than the batch's largest gets no idle CTAs.
+  bool cta_map = false;
   int64_t n_ctas = 0;
   std::vector<int32_t> cta_task, cnt_base;
   int64_t n_counters = 0;
@@ -160,20 +164,27 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   // spreads over one wave of SMs.  The tensor-core kernel runs one CTA per SM, so its
   // split is grown until items x row groups fit in a single wave.
   // CTAs per item: 128-row groups on the tcgen05 kernel, 256-row groups on the dual one
-  const int groups = (kern == PAD_FLAG_PREFIX_TC)     ? std::max(1, (max_rows + 127) / 128)
-                     : (kern == PAD_FLAG_PREFIX_DUAL) ? std::max(1, (max_rows + 255) / 256)
-                                                      : 1;
+  // (per video, as the CTA list gives each item only the groups its video's rows need;
+  // the fused tail keeps one dense grid of the largest count)
+  const int rows_per_cta = (kern == PAD_FLAG_PREFIX_TC) ? 128 : (kern == PAD_FLAG_PREFIX_DUAL) ? 256 : 0;
+  const int groups = rows_per_cta ? std::max(1, (max_rows + rows_per_cta - 1) / rows_per_cta) : 1;
+  const bool want_fused = kern == PAD_FLAG_PREFIX_TC && (prob->flags & PAD_FLAG_FUSED_MERGE);
+  auto groups_of = [&](int b) {
+    if (!rows_per_cta || want_fused) return groups;
+    return std::max(1, (L->ev_count[b] * L->group + rows_per_cta - 1) / rows_per_cta);
+  };
   int64_t work = 0;
   for (int b = 0; b < n_videos; ++b)
-    if (L->ev_count[b] > 0) work += (int64_t)prefix_len[b] * prob->h_kv * groups;
+    if (L->ev_count[b] > 0) work += (int64_t)prefix_len[b] * prob->h_kv * groups_of(b);
   const int64_t target = std::max(1, n_sms);
   int64_t chunk = (work + target - 1) / target;
   chunk = std::max<int64_t>(kSplitGranule, (chunk + kSplitGranule - 1) / kSplitGranule * kSplitGranule);
   auto ctas_for = [&](int64_t c) {
     int64_t n = 0;
     for (int b = 0; b < n_videos; ++b)
-      if (L->ev_count[b] > 0 && prefix_len[b] > 0) n += (int64_t)prob->h_kv * ((prefix_len[b] + c - 1) / c);
-    return n * groups;
+      if (L->ev_count[b] > 0 && prefix_len[b] > 0)
+        n += (int64_t)prob->h_kv * ((prefix_len[b] + c - 1) / c) * groups_of(b);
+    return n;
   };
   if (kern == PAD_FLAG_PREFIX_TC || kern == PAD_FLAG_PREFIX_DUAL) {
     int64_t max_prefix = 0;
@@ -235,6 +246,21 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
       for (int64_t t = 0; t < tasks_n; ++t) L->cta_task[valid[t].second] = (int32_t)t;
       L->fused = true;
     }
+  }
+  L->cta_map = false;
+  if (rows_per_cta && !L->fused && items > 0) {
+    if (items > ((int64_t)1 << 24)) return fail(PAD_ERR_UNSUPPORTED, "batch too large");
+    L->cta_task.clear();
+    int64_t item = 0;
+    for (int b = 0; b < n_videos; ++b) {
+      if (L->ev_count[b] == 0 || L->n_splits[b] == 0) continue;
+      const int gb = groups_of(b);
+      for (int h = 0; h < prob->h_kv; ++h)
+        for (int sp = 0; sp < L->n_splits[b]; ++sp, ++item)
+          for (int g = 0; g < gb; ++g) L->cta_task.push_back((int32_t)((item << 6) | g));
+    }
+    L->n_ctas = (int64_t)L->cta_task.size();
+    L->cta_map = true;
   }
 
   size_t off = sizeof(PadDevHeader);
@@ -836,6 +862,8 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.g_self = plan->g_self;
   p.causal = plan->causal;
   p.fused = plan->lay.fused ? 1 : 0;
+  p.cta_map = plan->lay.cta_map ? 1 : 0;
+  p.n_ctas = (int32_t)plan->lay.n_ctas;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
   p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;
@@ -1314,6 +1342,8 @@ pad_status static_params(const pad_plan_t* plan, cudaStream_t s, KParams& p, uin
   p.g_self = plan->g_self;
   p.causal = plan->causal;
   p.fused = plan->lay.fused ? 1 : 0;
+  p.cta_map = plan->lay.cta_map ? 1 : 0;
+  p.n_ctas = (int32_t)plan->lay.n_ctas;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
   p.tasks = reinterpret_cast<const int32_t*>(ws + plan->lay.off_tasks);
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);

@@ -132,6 +132,9 @@ struct KParams {
   void* pf_out;
   float* pf_lse;
   const int32_t* tasks;           // per prefix CTA: its (event * h_kv + kv-head) task, or -1
+                                  // (fused tail); with cta_map its (work item << 6) | row group
+  int32_t cta_map;                // the tensor-core prefix grid is the n_ctas CTAs of that list
+  int32_t n_ctas;
   // Per (video, kv-head, 128-row group): bits 15-0 how many of the video's prefix splits
   // have written their partials, bits 31-16 how many tasks have taken them.  Zeroed by
   // the append kernel of the step; the last task to take a counter zeroes it again, so a

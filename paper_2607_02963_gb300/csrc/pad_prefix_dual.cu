@@ -200,8 +200,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   // waits for that grid first (the Q loads, the first TMA issue).
   const bool one_call = p.k_new != nullptr;
 
-  const int item = blockIdx.x / n_groups;
-  const int grp = blockIdx.x - item * n_groups;
+  // the CTA's work item and 256-row group: from the plan's CTA list, or the dense grid
+  int item, grp;
+  if (p.cta_map) {
+    const int v = plan_tasks(p)[blockIdx.x];
+    item = v >> 6;
+    grp = v & 63;
+  } else {
+    item = blockIdx.x / n_groups;
+    grp = blockIdx.x - item * n_groups;
+  }
   const PadWorkItem it = plan_items(p)[item];
   const int R = it.n_events * p.group;
   const int row0 = grp * 256;
@@ -708,7 +716,7 @@ cudaError_t launch_prefix_dual(const KParams& p, int max_rows, const void* q, co
   }
   const int n_groups = (max_rows + 255) / 256;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.n_items * n_groups);
+  cfg.gridDim = dim3(p.cta_map ? p.n_ctas : p.n_items * n_groups);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = s;

@@ -279,8 +279,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the grid behind this one.
   const bool one_call = p.k_new != nullptr;
 
-  const int item = blockIdx.x / n_groups;
-  const int group = blockIdx.x - item * n_groups;
+  // the CTA's work item and 128-row group: from the plan's CTA list, or the dense grid
+  int item, group;
+  if (p.cta_map) {
+    const int v = plan_tasks(p)[blockIdx.x];
+    item = v >> 6;
+    group = v & 63;
+  } else {
+    item = blockIdx.x / n_groups;
+    group = blockIdx.x - item * n_groups;
+  }
   PadWorkItem it;
   // PREFILL: the CTA's query tokens [it.first_event, +n_events) of kv-head it.kvh (query
   // tiles in descending order, so that the longest key ranges start first) see the keys
@@ -880,7 +888,7 @@ cudaError_t launch_prefix_tc(const KParams& p, int max_rows, const void* q, cons
   }
   const int n_groups = (max_rows + 127) / 128;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.n_items * n_groups);
+  cfg.gridDim = dim3(p.cta_map ? p.n_ctas : p.n_items * n_groups);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = s;

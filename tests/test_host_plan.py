@@ -131,12 +131,16 @@ def test_tc_split_fits_one_wave(padlib, flags, rows_per_cta):
         prob = B.make_problem(28, 4, 128, num_sms=sms, flags=flags)
         plan = B.pad_plan(prob, B.CacheState(4096), P, ev_video, L, max_pages=2, workspace=None)
         info = plan.info()
-        groups = -(-int(Ev.max()) * 7 // rows_per_cta)
         sl = info["split_len"]
         assert sl % 128 == 0
-        # one wave unless a single split per (video, kv-head) is already too many
+        # each work item gets the row groups its own video needs (a CTA list, not a dense
+        # grid of the largest count): one wave unless a single split per (video, kv-head)
+        # is already too many
+        ctas = sum(4 * -(-int(P[b]) // sl) * -(-int(Ev[b]) * 7 // rows_per_cta) for b in range(B_))
+        items = sum(4 * -(-int(P[b]) // sl) for b in range(B_))
+        assert info["n_work_items"] == items
         if sl < int(P.max()):
-            assert info["n_work_items"] * groups <= sms
+            assert ctas <= sms
 
 
 @pytest.mark.parametrize("case,status", [
