@@ -193,8 +193,56 @@ class ClockSampler:
         for _, rv in self.samples:
             bits |= rv
         reasons = [n for b, n in _REASONS.items() if bits & b]
+        bins = {}
+        for m in mhz:
+            bins[str(m)] = bins.get(str(m), 0) + 1
         return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": self.max_mhz,
-                "sm_mhz_min": min(mhz), "reasons": reasons, "samples": len(mhz), "source": "nvml"}
+                "sm_mhz_min": min(mhz), "reasons": reasons, "samples": len(mhz),
+                "samples_by_sm_mhz": bins, "period_ms": self.period * 1e3, "source": "nvml"}
+
+
+# ---------------------------------------------------------------------------
+# Timed region: blocks of exactly K steps, repeated back to back
+# ---------------------------------------------------------------------------
+
+MIN_REGION_MS = 200.0
+
+
+def timed_blocks(run_step, K, stream, first=0, min_ms=MIN_REGION_MS):
+    """Time blocks of exactly K steps back to back on `stream` until the region covers
+    `min_ms`, with a CUDA event between consecutive blocks.  run_step(i) enqueues step i.
+    Returns (per-block ms, region ms, next step index, host us per step).  The caller
+    brackets the call with its barrier and synchronisation."""
+    import torch
+    # pilot block (not part of the region) sizes the number of blocks
+    p0 = torch.cuda.Event(enable_timing=True)
+    p1 = torch.cuda.Event(enable_timing=True)
+    p0.record(stream)
+    for i in range(K):
+        run_step(first + i)
+    p1.record(stream)
+    torch.cuda.synchronize()
+    i0 = first + K
+    est = max(p0.elapsed_time(p1), 1e-3)
+    n_blocks = max(1, min(100000, int(-(-min_ms // est)) + 1))
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_blocks + 1)]
+    h0 = time.perf_counter()
+    evs[0].record(stream)
+    for b in range(n_blocks):
+        for i in range(K):
+            run_step(i0 + b * K + i)
+        evs[b + 1].record(stream)
+    h1 = time.perf_counter()
+    torch.cuda.synchronize()
+    blocks = [evs[b].elapsed_time(evs[b + 1]) for b in range(n_blocks)]
+    return blocks, evs[0].elapsed_time(evs[-1]), i0 + n_blocks * K, (h1 - h0) * 1e6 / (n_blocks * K)
+
+
+def block_stats(blocks, K):
+    per = sorted(b / K for b in blocks)
+    return {"blocks": len(blocks), "steps_per_block": K,
+            "median_ms_per_step": statistics.median(per), "min_ms_per_step": per[0],
+            "max_ms_per_step": per[-1], "mean_ms_per_step": sum(per) / len(per)}
 
 
 # ---------------------------------------------------------------------------
@@ -303,6 +351,20 @@ def cpu_baseline(w, budget_s=10.0):
 # GPU arm
 # ---------------------------------------------------------------------------
 
+def e2e_breakdown(step, run, n=200):
+    """Where an end-to-end step's time goes: the library's own per-phase profile of
+    pad_step_run_host (CUDA events between the phases on the step's stream, host clock
+    readings beside them), means over n calls in microseconds."""
+    step.profile(True)
+    for i in range(n):
+        run(i)
+    d = step.profile_read()
+    step.profile(False)
+    d["how"] = ("pad_step_profile: events before the input copy, after it, after pad_plan, after "
+                "the launches and after the output copy; host clock beside each; means")
+    return d
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -360,7 +422,8 @@ def run_ours(args):
                             db.page_table, w.max_pages, db.workspace, w.prefix_offset,
                             kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
                             db.k_pool, db.v_pool, db.out, db.lse, stream,
-                            one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal)
+                            one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal,
+                            mapped_host_io=kw.get("mapped", not args.e2e_copy))
 
     one_call = not args.two_call
     api_path = ("pad_step_run (pad_plan + pad_decode_step)" if one_call
@@ -383,26 +446,24 @@ def run_ours(args):
         db.release_new_pages()
     barrier(device)
 
-    # timed loop: the step exactly as a caller runs it (no events between its kernels)
+    # timed region: blocks of exactly K steps, each step exactly as a caller runs it (no
+    # events between its kernels, an event between blocks), repeated to cover >= 200 ms
     sampler = ClockSampler(local)
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
-    sampler.start()
-    h0 = time.perf_counter()
-    ev0.record(stream)
-    for i in range(K):
-        steps[(W + i) % n_rep]()
-    ev1.record(stream)
-    h1 = time.perf_counter()
+    barrier(device)
     torch.cuda.synchronize()
+    sampler.start()
+    blocks, region_ms, nxt, host_us = timed_blocks(lambda i: steps[(W + i) % n_rep](), K, stream)
+    torch.cuda.synchronize()
+    barrier(device)
     clocks = sampler.stop()
-    ms = ev0.elapsed_time(ev1)
+    bstat = block_stats(blocks, K)
+    ms = bstat["median_ms_per_step"] * K
     # the shared-prefix kernel alone: CUDA events around each of its launches (the
     # library records them on the launching stream; overlap with neighbours is off)
-    Kr = min(K, 500)
+    Kr = max(K, 500)
     B.pad_timing_enable(Kr)
     for i in range(Kr):
-        steps[(W + K + i) % n_rep]()
+        steps[(W + nxt + i) % n_rep]()
     torch.cuda.synchronize()
     pre_ms, pre_n = B.pad_timing_read()
     for db in reps:
@@ -430,24 +491,93 @@ def run_ours(args):
     h2d = sum(t.numel() * t.element_size() for t in (hq, hkn, hvn))
     d2h = sum(t.numel() * t.element_size() for t in (hout, hlse))
 
-    def e2e_step(i):
-        # pad_step_run_host: H2D of q / k_new / v_new, the step, D2H of out and lse, and the
-        # wait for the stream, in one call
-        steps[i % n_rep].run_host(hq, hkn, hvn, hout, hlse)
+    def e2e_blocks(run):
+        for i in range(3):
+            run(i)
+        barrier(device)
+        # blocks of Ke steps on the host clock until the region covers >= 200 ms
+        blocks = []
+        t_start = time.perf_counter()
+        i = 0
+        while True:
+            t0 = time.perf_counter()
+            for _ in range(Ke):
+                run(i)
+                i += 1
+            t1 = time.perf_counter()
+            blocks.append((t1 - t0) * 1e3)
+            if (t1 - t_start) * 1e3 >= MIN_REGION_MS:
+                return block_stats(blocks, Ke)
 
-    for i in range(3):
-        e2e_step(i)
-    barrier(device)
-    t0 = time.perf_counter()
-    for i in range(Ke):
-        e2e_step(i)
-    e2e_ms = (time.perf_counter() - t0) * 1e3
-    e_units, e_ms = aggregate(float(w.n_events * Ke), e2e_ms, device)
+    # A second set of page-locked buffers for a second, independent batch (the next replica)
+    h_in2 = torch.empty_like(h_in, pin_memory=True)
+    h_out2 = torch.empty_like(h_out, pin_memory=True)
+    h_in2.copy_(h_in)
+    io = [(hq, hkn, hvn, hout, hlse),
+          (h_in2[:qn].view(hq.shape), h_in2[qn:qn + kn].view(hkn.shape), h_in2[qn + kn:].view(hvn.shape),
+           h_out2[:ob].view(hout.dtype).view(hout.shape), h_out2[ob:].view(torch.float32).view(hlse.shape))]
+    pair = [steps[0], steps[1 % n_rep]]
+
+    def pipelined_block(n):
+        # two batches in flight: batch i % 2 is planned and enqueued (pad_step_enqueue_host)
+        # while the device runs batch (i - 1) % 2, whose outputs the host then waits for
+        pair[0].enqueue_host(*io[0])
+        for i in range(1, n):
+            pair[i % 2].enqueue_host(*io[i % 2])
+            pair[(i - 1) % 2].wait()
+        pair[(n - 1) % 2].wait()
+
+    def e2e_blocks(run_block):
+        run_block(3)
+        barrier(device)
+        # blocks of Ke steps on the host clock until the region covers >= 200 ms
+        blocks = []
+        t_start = time.perf_counter()
+        while True:
+            t0 = time.perf_counter()
+            run_block(Ke)
+            t1 = time.perf_counter()
+            blocks.append((t1 - t0) * 1e3)
+            if (t1 - t_start) * 1e3 >= MIN_REGION_MS:
+                return block_stats(blocks, Ke)
+
+    def serial_block(st):
+        def run(n):
+            for i in range(n):
+                st.run_host(hq, hkn, hvn, hout, hlse)
+        return run
+
+    mapped = not args.e2e_copy
+    io_desc = (("q/k_new/v_new read from pinned mapped host memory by a kernel, " if mapped
+                else "pinned H2D copy of q/k_new/v_new, ")
+               + "pad_plan + " + ("pad_decode_step" if one_call else "pad_kv_append + pad_event_decode_attn")
+               + (", O and LSE written into pinned mapped host memory by the step's kernels" if mapped
+                  else ", D2H copy of O and LSE"))
+    # headline: two independent batches in flight through pad_step_enqueue_host / pad_step_wait
+    e_stat = e2e_blocks(pipelined_block)
+    e_units, e_ms = aggregate(float(w.n_events * Ke), e_stat["median_ms_per_step"] * Ke, device)
     e2e = {"value": e_units / (e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-           "d2h_bytes_per_step": d2h, "steps": Ke,
-           "path": "pad_step_run_host through the C ABI: pinned H2D of q/k_new/v_new, pad_plan + "
-                   + ("pad_decode_step" if one_call else "pad_kv_append + pad_event_decode_attn")
-                   + ", D2H of O and LSE, stream sync, every step"}
+           "d2h_bytes_per_step": d2h, "steps": Ke, "us_per_step": e_stat["median_ms_per_step"] * 1e3,
+           "in_flight": 2,
+           "timing": dict(e_stat, clock="host perf_counter around each block of steps"),
+           "path": "through the C ABI, every step: " + io_desc + "; two independent batches (own "
+                   "executor, own host buffers) in flight: pad_step_enqueue_host of one, then "
+                   "pad_step_wait of the other"}
+    # one batch, each step waited for before the next (pad_step_run_host)
+    s_stat = e2e_blocks(serial_block(steps[0]))
+    e2e["serial"] = {"us_per_step": s_stat["median_ms_per_step"] * 1e3,
+                     "value": w.n_events / s_stat["median_ms_per_step"] * 1e3,
+                     "path": "pad_step_run_host, one batch: " + io_desc + ", stream wait, every step",
+                     "breakdown_us": e2e_breakdown(steps[0], lambda i: steps[0].run_host(hq, hkn, hvn, hout, hlse))}
+    if mapped:
+        # the same serial call on the copy-engine path (cudaMemcpyAsync both ways)
+        alt = launcher(reps[0], mapped=False)
+        a_stat = e2e_blocks(serial_block(alt))
+        e2e["serial_copy_engine"] = {
+            "us_per_step": a_stat["median_ms_per_step"] * 1e3,
+            "value": w.n_events / a_stat["median_ms_per_step"] * 1e3,
+            "breakdown_us": e2e_breakdown(alt, lambda i: alt.run_host(hq, hkn, hvn, hout, hlse))}
+        del alt
 
     if rank != 0:
         return
@@ -475,6 +605,9 @@ def run_ours(args):
         "steps": K,
         "warmup": W,
         "ms_per_step": ms_max / K,
+        "timing": dict(bstat, region_ms=region_ms,
+                       how="CUDA events on the launching stream between back-to-back blocks "
+                           "of exactly K steps; value and ms_per_step from the median block"),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
@@ -521,7 +654,7 @@ def run_ours(args):
             "achieved_gbs": byt["total"] / (step_ms * 1e-3) / 1e9,
             "frac_of_measured_hbm": byt["total"] / (step_ms * 1e-3) / 1e9 / peak,
             "frac_of_nominal_8tbs": byt["total"] / (step_ms * 1e-3) / 1e9 / 8000.0,
-            "host_us_per_step": (h1 - h0) * 1e6 / K,
+            "host_us_per_step": host_us,
         },
         "e2e": e2e,
     }
@@ -805,6 +938,7 @@ def run_sweep(args):
     stream = torch.cuda.current_stream(device)
     l2 = int(getattr(torch.cuda.get_device_properties(device), "L2_cache_size", 0) or (126 << 20))
     flush = torch.empty(3 * l2, dtype=torch.uint8, device=device)
+    peak, peak_kind = hbm_peak()
     for E in (1, 2, 4, 8, 16, 32, 64):
         w = make_workload(f"sweep_e{E}")
         byt_all = w.bytes_algorithmic()
@@ -817,18 +951,26 @@ def run_sweep(args):
                                 db.page_table, w.max_pages, db.workspace, w.prefix_offset, db.q,
                                 db.k_new, db.v_new, db.k_prefix, db.v_prefix, db.k_pool, db.v_pool,
                                 db.out, db.lse, stream) for db in reps]
-        for i in range(max(3, args.warmup)):
+        W = max(3, args.warmup)
+        for i in range(W):
             steps[i % n_rep]()
         torch.cuda.synchronize()
         K = args.steps
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for i in range(K):
-            steps[i % n_rep]()
-        e1.record(stream)
+        sampler = ClockSampler(0)
+        sampler.start()
+        blocks, region_ms, nxt, _ = timed_blocks(lambda i: steps[(W + i) % n_rep](), K, stream)
+        clocks = sampler.stop()
+        bstat = block_stats(blocks, K)
+        ours_us = bstat["median_ms_per_step"] * 1e3
+        B.pad_timing_enable(500)
+        for i in range(500):
+            steps[(W + nxt + i) % n_rep]()
         torch.cuda.synchronize()
-        ours_us = e0.elapsed_time(e1) * 1e3 / K
+        pre_ms, pre_n = B.pad_timing_read()
+        pre_us = pre_ms * 1e3 / max(1, pre_n)
+        for db in reps:
+            B.pad_device_status(db.plan_step(stream))
+            db.release_new_pages()
 
         # naive comparator: per event, its visible keys made contiguous once (outside the
         # timing), then one attention call per event per step; L2 flushed between steps
@@ -861,11 +1003,18 @@ def run_sweep(args):
         naive_us = statistics.median(times)
         ref = torch.stack([o.view(w.h_q, w.head_dim).float() for o in outs])
         diff = float((ref - db.out.float()).abs().max())
-        print(json.dumps({"sweep_E": E, "algorithmic_bytes": byt, "prefix_bytes": byt_all["prefix"],
-                          "branch_bytes": byt_all["branch"], "ours_us_per_step": ours_us,
-                          "ours_gbs": byt / ours_us * 1e-3, "naive_bytes_per_step": naive_bytes,
-                          "naive_us_per_step": naive_us, "naive_gbs": naive_bytes / naive_us * 1e-3,
-                          "max_abs_ours_vs_naive": diff, "replicas": n_rep, "steps": K}), flush=True)
+        gbs = byt / ours_us * 1e-3
+        print(json.dumps({
+            "metric": METRIC, "value": w.n_events / (ours_us * 1e-6), "unit": UNIT,
+            "sweep_E": E, "workload": f"sweep_e{E}", "description": WORKLOADS[f"sweep_e{E}"],
+            "algorithmic_bytes": byt, "prefix_bytes": byt_all["prefix"], "branch_bytes": byt_all["branch"],
+            "ours_us_per_step": ours_us, "ours_min_us_per_step": bstat["min_ms_per_step"] * 1e3,
+            "ours_gbs": gbs, "frac_of_measured_hbm": gbs / peak, "peak_gbs": peak, "peak_kind": peak_kind,
+            "prefix_kernel_us": pre_us, "prefix_kernel_frac": byt_all["prefix"] / pre_us * 1e-3 / peak,
+            "naive_bytes_per_step": naive_bytes, "naive_us_per_step": naive_us,
+            "naive_gbs": naive_bytes / naive_us * 1e-3, "naive_over_ours_time": naive_us / ours_us,
+            "max_abs_ours_vs_naive": diff, "replicas": n_rep,
+            "timing": dict(bstat, region_ms=region_ms), "clocks": clocks}), flush=True)
         del reps, steps, first, db, ks, vs, qs, outs
         torch.cuda.empty_cache()
 
@@ -881,6 +1030,8 @@ def main(argv=None):
     ap.add_argument("--prefix", choices=["auto", "simt", "mma", "tc", "dual"], default="auto",
                     help="shared-prefix kernel (auto = the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=500)
+    ap.add_argument("--e2e-copy", action="store_true",
+                    help="e2e through the copy-engine path of pad_step_run_host (no mapped host I/O)")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused-merge", action="store_true",

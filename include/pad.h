@@ -290,7 +290,8 @@ pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_
  *              workspace and page_table are required
  *   options    PAD_STEP_TWO_CALL: pad_kv_append + pad_event_decode_attn instead of
  *              pad_decode_step; PAD_STEP_RELEASE_PAGES: hand the pages a run took back to
- *              the cache after launching it (to repeat one identical step, e.g. for timing)
+ *              the cache after launching it (to repeat one identical step, e.g. for timing);
+ *              PAD_STEP_MAPPED_HOST_IO: see pad_step_run_host
  *   new_page   [n_events] host, may be NULL: the pages the run took (pad_plan_new_pages)
  * A run that fails before a kernel wrote its new pages into the page table hands them back
  * to the cache and returns the failing call's status.
@@ -299,6 +300,7 @@ pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_
 typedef struct pad_step_t pad_step_t;
 #define PAD_STEP_TWO_CALL 0x1
 #define PAD_STEP_RELEASE_PAGES 0x2
+#define PAD_STEP_MAPPED_HOST_IO 0x4
 pad_status pad_step_create(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
                            const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
                            const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
@@ -316,10 +318,41 @@ pad_status pad_step_run(pad_step_t* step, int32_t* new_page);
  *   or NULL; host memory (page-locked for asynchronous copies).  The call returns after the
  *   stream has finished with them, also when it fails.  Where q, k_new and v_new
  *   follow one another in device memory and their host buffers do too, they go in one copy;
- *   so do out and lse. */
+ *   so do out and lse.
+ *   With PAD_STEP_MAPPED_HOST_IO, and where every host buffer is page-locked, mapped into
+ *   the device's address space (cudaHostAlloc / cudaHostRegister; under unified addressing
+ *   every page-locked allocation is), 16-byte aligned and lies in one such allocation (the
+ *   caller's guarantee; the call checks the first and last byte), no copy engine is used:
+ *   a kernel reads q, k_new and v_new over the host link into the step's device buffers, and
+ *   the step's kernels write O and LSE straight into h_out and h_lse (the step's device out
+ *   and lse are not written).  A buffer that fails the check sends that call down the
+ *   copy path. */
 pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
                              void* h_out, float* h_lse, int32_t* new_page);
+/* pad_step_enqueue_host: pad_step_run_host without the wait.  It returns once the run is on
+ * the stream; the host buffers stay in use until pad_step_wait(step) returns (which waits
+ * for the latest run enqueued on this step) or the stream is synchronised.  A caller with
+ * several independent batches (one step executor and one set of host buffers each) plans
+ * and enqueues the next batch while the device runs the previous one.  A failing enqueue
+ * synchronises the stream before it returns, like pad_step_run_host. */
+pad_status pad_step_enqueue_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
+                                 void* h_out, float* h_lse, int32_t* new_page);
+pad_status pad_step_wait(pad_step_t* step);
 void pad_step_destroy(pad_step_t* step);
+
+/* Measurement aid: where a pad_step_run_host call spends its time.  After
+ * pad_step_profile(step, 1) every pad_step_run_host call on the step records CUDA events on
+ * the step's stream before the input copy, after it, after planning, after the launches and
+ * after the output copy, reads the host clock beside each, and adds the intervals up
+ * (enable 0 stops; either call clears the sums).  pad_step_profile_read writes 12 values
+ * (out must hold n >= 12): out[0] the calls profiled, then means in microseconds:
+ *   host    out[1] input copy call(s)   out[2] pad_plan   out[3] kernel launches
+ *           out[4] output copy call(s)  out[5] stream wait  out[6] whole call
+ *   device  out[7] input copy  out[8] idle until the planned launches  out[9] kernels
+ *           out[10] output copy  out[11] first event to last
+ * The extra event records add a little host time to each profiled call. */
+pad_status pad_step_profile(pad_step_t* step, int32_t enable);
+pad_status pad_step_profile_read(const pad_step_t* step, double* out, int32_t n);
 
 /* Allocation-free variant of pad_event_decode_attn (the paper has no counterpart; this
  * is an interface for callers, not part of the method).  Same arguments and result.  It

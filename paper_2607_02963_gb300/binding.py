@@ -103,6 +103,10 @@ _SIGNATURES = {
     "pad_device_status": (c_int32, [c_void_p, c_void_p]),
     "pad_last_error": (ctypes.c_char_p, []),
     "pad_status_string": (ctypes.c_char_p, [c_int32]),
+    "pad_step_enqueue_host": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, _I32P]),
+    "pad_step_wait": (c_int32, [c_void_p]),
+    "pad_step_profile": (c_int32, [c_void_p, c_int32]),
+    "pad_step_profile_read": (c_int32, [c_void_p, POINTER(ctypes.c_double), c_int32]),
     "pad_timing_enable": (c_int32, [c_int32]),
     "pad_timing_read": (c_int32, [POINTER(c_float), _I32P]),
 }
@@ -384,6 +388,7 @@ def pad_timing_read():
 
 STEP_TWO_CALL = 0x1
 STEP_RELEASE_PAGES = 0x2
+STEP_MAPPED_HOST_IO = 0x4
 
 
 class NativeStep:
@@ -395,7 +400,7 @@ class NativeStep:
     def __init__(self, problem: Problem, cache: CacheState, prefix_len, event_video, event_len,
                  page_table, max_pages, workspace, prefix_offset, q, k_new, v_new, k_prefix,
                  v_prefix, k_pool, v_pool, out, lse, stream, release_pages=True, one_call=True,
-                 rope=None, self_g=None, causal=False):
+                 rope=None, self_g=None, causal=False, mapped_host_io=False):
         self.L = lib()
         self.problem = problem
         self.cache = cache
@@ -407,7 +412,8 @@ class NativeStep:
                               else np.ascontiguousarray(prefix_offset, dtype=np.int64))
         self._keep = [q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse, workspace, page_table]
         self.ne = int(self.event_video.size)
-        opts = (0 if one_call else STEP_TWO_CALL) | (STEP_RELEASE_PAGES if release_pages else 0)
+        opts = ((0 if one_call else STEP_TWO_CALL) | (STEP_RELEASE_PAGES if release_pages else 0)
+                | (STEP_MAPPED_HOST_IO if mapped_host_io else 0))
         h = c_void_p()
         _check(self.L.pad_step_create(
             ctypes.byref(problem), cache.handle, int(self.prefix_len.size), self.prefix_len.ctypes.data_as(_I32P),
@@ -438,9 +444,35 @@ class NativeStep:
         _check(self._run(self.handle, self._np))
 
     def run_host(self, h_q, h_k_new, h_v_new, h_out, h_lse=None):
-        """Host tensors (page-locked): copies in, the step, copies out, stream wait."""
+        """Host tensors (page-locked): copies in, the step, copies out, stream wait (with
+        mapped_host_io, the inputs are read and the outputs written by kernels over the host
+        link where every buffer is page-locked and device-mapped)."""
         _check(self._run_host(self.handle, h_q.data_ptr(), h_k_new.data_ptr(), h_v_new.data_ptr(), h_out.data_ptr(),
                               None if h_lse is None else h_lse.data_ptr(), self._np))
+
+    def enqueue_host(self, h_q, h_k_new, h_v_new, h_out, h_lse=None):
+        """run_host without the wait: the buffers stay in use until wait()."""
+        _check(self.L.pad_step_enqueue_host(self.handle, h_q.data_ptr(), h_k_new.data_ptr(), h_v_new.data_ptr(),
+                                            h_out.data_ptr(), None if h_lse is None else h_lse.data_ptr(),
+                                            self._np))
+
+    def wait(self):
+        _check(self.L.pad_step_wait(self.handle))
+
+    PROFILE_KEYS = ("host_h2d_call", "host_plan", "host_launch", "host_d2h_call", "host_wait",
+                    "host_total", "dev_h2d", "dev_idle_until_launch", "dev_kernels", "dev_d2h",
+                    "dev_span")
+
+    def profile(self, enable=True):
+        """Per-phase timing of run_host (pad_step_profile); read it with profile_read."""
+        _check(self.L.pad_step_profile(self.handle, 1 if enable else 0))
+
+    def profile_read(self):
+        buf = (ctypes.c_double * 12)()
+        _check(self.L.pad_step_profile_read(self.handle, buf, 12))
+        d = dict(zip(self.PROFILE_KEYS, list(buf)[1:]))
+        d["calls"] = int(buf[0])
+        return d
 
     def __del__(self):
         h = getattr(self, "handle", None)

@@ -1011,7 +1011,30 @@ struct pad_step_t {
   const int32_t* g_planning = nullptr;
   const int32_t* g_index = nullptr;
   int32_t branch_mode = PAD_BRANCH_OWN;
+  // pad_step_profile: CUDA events between the phases of pad_step_run_host and host clock
+  // readings around them, summed over the profiled calls
+  struct Profile {
+    bool on = false;
+    cudaEvent_t ev[5] = {};
+    int64_t n = 0;
+    double host[6] = {};  // input copy call, pad_plan, launches, output copy call, wait, total
+    double dev[5] = {};   // input copy, wait for the plan, kernels, output copy, whole span
+  } prof;
+  // pad_step_enqueue_host: recorded behind the latest enqueued run, waited on by pad_step_wait
+  cudaEvent_t done = nullptr;
+  bool pending = false;
+  ~pad_step_t() {
+    for (cudaEvent_t& e : prof.ev)
+      if (e) cudaEventDestroy(e);
+    if (done) cudaEventDestroy(done);
+  }
 };
+
+namespace {
+double host_us() {
+  return std::chrono::duration<double, std::micro>(std::chrono::steady_clock::now().time_since_epoch()).count();
+}
+}  // namespace
 
 pad_status pad_step_create(const pad_problem* prob, pad_cache_state* cache, int32_t n_videos,
                            const int32_t* prefix_len, const int64_t* prefix_offset, int32_t n_events,
@@ -1025,7 +1048,8 @@ pad_status pad_step_create(const pad_problem* prob, pad_cache_state* cache, int3
   pad_status st = check_problem(prob);
   if (st != PAD_OK) return st;
   if (!cache) return fail(PAD_ERR_INVALID_ARG, "cache is NULL");
-  if (options & ~(PAD_STEP_TWO_CALL | PAD_STEP_RELEASE_PAGES)) return fail(PAD_ERR_INVALID_ARG, "unknown options 0x%x", options);
+  if (options & ~(PAD_STEP_TWO_CALL | PAD_STEP_RELEASE_PAGES | PAD_STEP_MAPPED_HOST_IO))
+    return fail(PAD_ERR_INVALID_ARG, "unknown options 0x%x", options);
   if (n_videos < 0 || n_events < 0) return fail(PAD_ERR_INVALID_ARG, "negative batch size");
   if (n_events > 0 && (!event_video || !event_len || !prefix_len)) return fail(PAD_ERR_INVALID_ARG, "NULL host array");
   if (!workspace || !page_table) return fail(PAD_ERR_INVALID_ARG, "workspace / page_table is NULL");
@@ -1088,13 +1112,21 @@ pad_status pad_step_set_branch_visibility(pad_step_t* step, int32_t mode) {
   return PAD_OK;
 }
 
-pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
-  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+namespace {
+// One step: pad_plan, the launches (writing O and LSE to `out` / `lse`), page bookkeeping.
+// With `ht` (profiling) it records event 2 and host time 2 after planning, event 3 and host
+// time 3 after the launches.
+pad_status step_run(pad_step_t* step, int32_t* new_page, double* ht, void* out, float* lse) {
   pad_plan_t* plan = nullptr;
   pad_status st = pad_plan(&step->prob, step->cache, step->n_videos, step->prefix_len, step->prefix_offset,
                            step->n_events, step->event_video, step->event_len, step->page_table, step->max_pages,
                            step->workspace, step->workspace_bytes, step->stream, &plan);
   if (st != PAD_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(step->stream);
+  if (ht) {
+    ht[2] = host_us();
+    cudaEventRecord(step->prof.ev[2], s);
+  }
   if (step->rope_cs) st = pad_plan_set_rope(plan, step->rope_pos, step->rope_cs, step->rope_max);
   if (st == PAD_OK && step->g_mode == PAD_G_SELF)
     st = pad_plan_set_g_visibility(plan, PAD_G_SELF, step->g_planning, step->g_index);
@@ -1106,11 +1138,15 @@ pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
       wrote_pages = st == PAD_OK;
       if (st == PAD_OK)
         st = pad_event_decode_attn(plan, step->q, step->k_prefix, step->v_prefix, step->k_pool, step->v_pool,
-                                   step->out, step->lse, step->stream);
+                                   out, lse, step->stream);
     } else {
       st = pad_decode_step(plan, step->q, step->k_new, step->v_new, step->k_prefix, step->v_prefix, step->k_pool,
-                           step->v_pool, step->out, step->lse, step->stream);
+                           step->v_pool, out, lse, step->stream);
     }
+  }
+  if (ht) {
+    ht[3] = host_us();
+    cudaEventRecord(step->prof.ev[3], s);
   }
   if (st == PAD_OK && new_page) st = pad_plan_new_pages(plan, new_page);
   if ((st != PAD_OK && !wrote_pages) || (step->options & PAD_STEP_RELEASE_PAGES)) {
@@ -1124,9 +1160,69 @@ pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
   pad_plan_destroy(plan);
   return st;
 }
+}  // namespace
 
-pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
-                             void* h_out, float* h_lse, int32_t* new_page) {
+pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  return step_run(step, new_page, nullptr, step->out, step->lse);
+}
+
+pad_status pad_step_profile(pad_step_t* step, int32_t enable) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  auto& pr = step->prof;
+  if (enable) {
+    for (cudaEvent_t& e : pr.ev) {
+      if (e) continue;
+      cudaError_t ce = cudaEventCreate(&e);
+      if (ce != cudaSuccess) return cuda_fail(ce, "cudaEventCreate");
+    }
+  }
+  pr.on = enable != 0;
+  pr.n = 0;
+  for (double& v : pr.host) v = 0.0;
+  for (double& v : pr.dev) v = 0.0;
+  return PAD_OK;
+}
+
+pad_status pad_step_profile_read(const pad_step_t* step, double* out, int32_t n) {
+  if (!step || !out) return fail(PAD_ERR_INVALID_ARG, "NULL argument");
+  if (n < 12) return fail(PAD_ERR_INVALID_ARG, "out needs 12 entries; got %d", n);
+  const auto& pr = step->prof;
+  const double c = pr.n > 0 ? 1.0 / (double)pr.n : 0.0;
+  out[0] = (double)pr.n;
+  for (int i = 0; i < 6; ++i) out[1 + i] = pr.host[i] * c;
+  for (int i = 0; i < 5; ++i) out[7 + i] = pr.dev[i] * c;
+  return PAD_OK;
+}
+
+namespace {
+// Device address of host range [h, h + n) when it is page-locked, device-mapped memory
+// (checked at its first and last byte, which must map n - 1 bytes apart) and aligned to
+// `align` bytes; nullptr otherwise.
+void* mapped_view(const void* h, size_t n, size_t align) {
+  if (!h || n == 0 || (reinterpret_cast<uintptr_t>(h) % align) != 0) return nullptr;
+  cudaPointerAttributes a0{}, a1{};
+  if (cudaPointerGetAttributes(&a0, h) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  const char* last = static_cast<const char*>(h) + (n - 1);
+  if (cudaPointerGetAttributes(&a1, last) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a0.type != cudaMemoryTypeHost || a1.type != cudaMemoryTypeHost || !a0.devicePointer || !a1.devicePointer)
+    return nullptr;
+  if (static_cast<const char*>(a1.devicePointer) - static_cast<const char*>(a0.devicePointer) != (ptrdiff_t)(n - 1))
+    return nullptr;
+  return a0.devicePointer;
+}
+}  // namespace
+
+namespace {
+// pad_step_run_host (wait) and pad_step_enqueue_host (no wait: an event behind the run)
+pad_status host_step(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new, void* h_out,
+                     float* h_lse, int32_t* new_page, bool wait) {
   if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
   if (step->n_events > 0 && (!h_q || !h_k_new || !h_v_new || !h_out))
     return fail(PAD_ERR_INVALID_ARG, "NULL host buffer");
@@ -1141,7 +1237,48 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
     return static_cast<const char*>(a) + n == static_cast<const char*>(b);
   };
   cudaError_t e = cudaSuccess;
-  if (E > 0) {
+  auto& prof = step->prof;
+  double ht[6] = {};
+  double* htp = (prof.on && wait) ? ht : nullptr;
+  if (!wait && !step->done) {
+    e = cudaEventCreateWithFlags(&step->done, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+  }
+  if (htp) {
+    ht[0] = host_us();
+    cudaEventRecord(prof.ev[0], s);
+  }
+  // mapped host I/O: device views of every host buffer, else the copy path
+  void *vq = nullptr, *vk = nullptr, *vv = nullptr, *vo = nullptr, *vl = nullptr;
+  bool mapped = false;
+  if (E > 0 && (step->options & PAD_STEP_MAPPED_HOST_IO)) {
+    vq = mapped_view(h_q, q_bytes, 16);
+    vk = vq ? mapped_view(h_k_new, kv_bytes, 16) : nullptr;
+    vv = vk ? mapped_view(h_v_new, kv_bytes, 16) : nullptr;
+    vo = vv ? mapped_view(h_out, o_bytes, 16) : nullptr;
+    vl = (vo && h_lse) ? mapped_view(h_lse, l_bytes, 4) : nullptr;
+    mapped = vo && (!h_lse || vl) && aligned16(step->q) && aligned16(step->k_new) && aligned16(step->v_new);
+  }
+  if (mapped) {
+    const void* src[3];
+    void* dst[3];
+    size_t nb[3];
+    int n = 0;
+    const bool kq = adjacent(step->q, q_bytes, step->k_new) && adjacent(vq, q_bytes, vk);
+    const bool vk_adj = adjacent(step->k_new, kv_bytes, step->v_new) && adjacent(vk, kv_bytes, vv);
+    if (kq && vk_adj) {
+      src[n] = vq, dst[n] = const_cast<void*>(step->q), nb[n++] = q_bytes + 2 * kv_bytes;
+    } else {
+      src[n] = vq, dst[n] = const_cast<void*>(step->q), nb[n++] = q_bytes;
+      src[n] = vk, dst[n] = const_cast<void*>(step->k_new), nb[n++] = kv_bytes;
+      src[n] = vv, dst[n] = const_cast<void*>(step->v_new), nb[n++] = kv_bytes;
+    }
+    e = launch_host_in(src, dst, nb, n, query_num_sms(), s);
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(s);
+      return cuda_fail(e, "step inputs from mapped host memory");
+    }
+  } else if (E > 0) {
     char* dq = static_cast<char*>(const_cast<void*>(step->q));
     const char* hq = static_cast<const char*>(h_q);
     const bool kq = adjacent(step->q, q_bytes, step->k_new) && adjacent(h_q, q_bytes, h_k_new);
@@ -1158,14 +1295,19 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
       return cuda_fail(e, "step inputs H2D");
     }
   }
-  pad_status st = pad_step_run(step, new_page);
+  if (htp) {
+    ht[1] = host_us();
+    cudaEventRecord(prof.ev[1], s);
+  }
+  pad_status st = mapped ? step_run(step, new_page, htp, vo, static_cast<float*>(vl))
+                         : step_run(step, new_page, htp, step->out, step->lse);
   if (st != PAD_OK) {
     const std::string msg = g_last_error;
     cudaStreamSynchronize(s);
     g_last_error = msg;
     return st;
   }
-  if (E > 0) {
+  if (E > 0 && !mapped) {
     if (h_lse && adjacent(step->out, o_bytes, step->lse) && adjacent(h_out, o_bytes, h_lse)) {
       e = cudaMemcpyAsync(h_out, step->out, o_bytes + l_bytes, cudaMemcpyDeviceToHost, s);
     } else {
@@ -1177,8 +1319,51 @@ pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_
       return cuda_fail(e, "step outputs D2H");
     }
   }
+  if (!wait) {
+    e = cudaEventRecord(step->done, s);
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(s);
+      return cuda_fail(e, "cudaEventRecord");
+    }
+    step->pending = true;
+    return PAD_OK;
+  }
+  if (htp) {
+    ht[4] = host_us();
+    cudaEventRecord(prof.ev[4], s);
+  }
   e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && htp) {
+    ht[5] = host_us();
+    const double hd[6] = {ht[1] - ht[0], ht[2] - ht[1], ht[3] - ht[2], ht[4] - ht[3], ht[5] - ht[4], ht[5] - ht[0]};
+    float dv[5] = {};
+    for (int i = 0; i < 4; ++i) cudaEventElapsedTime(&dv[i], prof.ev[i], prof.ev[i + 1]);
+    cudaEventElapsedTime(&dv[4], prof.ev[0], prof.ev[4]);
+    for (int i = 0; i < 6; ++i) prof.host[i] += hd[i];
+    for (int i = 0; i < 5; ++i) prof.dev[i] += 1e3 * (double)dv[i];
+    ++prof.n;
+  }
+  step->pending = false;
   return e == cudaSuccess ? PAD_OK : cuda_fail(e, "step synchronize");
+}
+}  // namespace
+
+pad_status pad_step_run_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
+                             void* h_out, float* h_lse, int32_t* new_page) {
+  return host_step(step, h_q, h_k_new, h_v_new, h_out, h_lse, new_page, true);
+}
+
+pad_status pad_step_enqueue_host(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new,
+                                 void* h_out, float* h_lse, int32_t* new_page) {
+  return host_step(step, h_q, h_k_new, h_v_new, h_out, h_lse, new_page, false);
+}
+
+pad_status pad_step_wait(pad_step_t* step) {
+  if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
+  if (!step->pending) return PAD_OK;
+  step->pending = false;
+  const cudaError_t e = cudaEventSynchronize(step->done);
+  return e == cudaSuccess ? PAD_OK : cuda_fail(e, "step wait");
 }
 
 void pad_step_destroy(pad_step_t* step) { delete step; }

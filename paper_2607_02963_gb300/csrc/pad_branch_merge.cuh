@@ -22,7 +22,9 @@
 // Staging before griddepcontrol.wait reads nothing the grids ahead write: Q rows, the
 // branch's page ids (key `len`'s page is the one this step took, else the table's entry
 // of an earlier step) and the K/V rows of keys 0..len-1, and key `len` itself when it
-// comes from k_new / v_new.  After it: key `len` when the append kernel wrote it, and the
+// comes from k_new / v_new.  In a one-call step that is all the branch pass reads, so the
+// whole pass (and the merge of its warp states) runs before the wait.  After it: key `len`
+// when the append kernel wrote it (two-call step, the branch pass follows), and the
 // splits' (m, l) pairs and O rows once the caller says they are complete
 // (`partials_ready`: at once for the standalone kernel, whose wait covers the prefix
 // grid; after the split counters for the tensor-core kernel).
@@ -301,26 +303,43 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     stage_keys(0, nv0, 0, nv0_16);
   }
   cp_async_commit();
+  // One-call step: nothing the branch pass reads is written by the grids ahead, so the
+  // whole pass runs before the wait and only the merge of the splits' partials follows it.
+  const bool pre = knew != nullptr;
 
   // ---------------- after the grids ahead (at least the append) completed
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (len_in_first) stage_keys(0, nv0, own, own + 1);
+  if (!pre) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (len_in_first) stage_keys(0, nv0, own, own + 1);
+  }
   cp_async_commit();                          // this round's keys
 
-  // the splits' O rows and (m, l) pairs of chunk [s0, s0 + nch)
+  // the splits' O rows and (m, l) pairs of chunk [s0, s0 + nch): per split, the task's G
+  // rows are one contiguous block of G * D floats, R * D floats after the previous split's
+  // (the flat index is advanced by NT without a division)
   auto stage_chunk = [&](int s0, int nch) {
-    for (int i = tid; i < nch * G * D4; i += NT) {
-      const int sl = i / (G * D4), r = i - sl * (G * D4);
-      cp_async16(spo + (size_t)sl * G * D + (size_t)r * 4,
-                 p.part_o + part_row(vd, kvh, s0 + sl, R, rbase) * D + (size_t)r * 4, true);
+    const int gd4 = G * D4;
+    const float* base = p.part_o + part_row(vd, kvh, s0, R, rbase) * D;
+    const size_t split_stride = (size_t)R * D;
+    int sl = tid / gd4, r = tid - (tid / gd4) * gd4;
+    const int adv_sl = NT / gd4, adv_r = NT - (NT / gd4) * gd4;
+    for (; sl < nch;) {
+      cp_async16(spo + (size_t)sl * G * D + (size_t)r * 4, base + sl * split_stride + (size_t)r * 4, true);
+      sl += adv_sl;
+      r += adv_r;
+      if (r >= gd4) {
+        r -= gd4;
+        ++sl;
+      }
     }
+    const float2* mbase = p.part_ml + part_row(vd, kvh, s0, R, rbase);
     for (int i = tid; i < G * nch; i += NT) {
-      const int g = i / nch, sl = i - g * nch;
-      cp_async8(&sml[g * sch + sl], &p.part_ml[part_row(vd, kvh, s0 + sl, R, rbase + g)]);
+      const int g = i / nch, k = i - g * nch;
+      cp_async8(&sml[g * sch + k], mbase + (size_t)k * R + g);
     }
   };
   bool ok = true;
-  if (early) {
+  if (early && !pre) {
     if (ns > 0) stage_chunk(0, min(sch, ns));
     cp_async_commit();                        // the first chunk, waited for in a5
   }
@@ -341,7 +360,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
       stage_keys(r0, nv, 0, (nv + 15) & ~15);
       cp_async_commit();
       cp_async_wait<0>();
-    } else if (early) {
+    } else if (early && !pre) {
       cp_async_wait<1>();                     // all but the first chunk's group
     } else {
       cp_async_wait<0>();
@@ -470,6 +489,12 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     reinterpret_cast<float4*>(&S.ob[g][0])[d4] = acc;
   }
 
+  if (early && pre) {
+    // ---------------- after the grids ahead (the prefix pass) completed
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (ns > 0) stage_chunk(0, min(sch, ns));
+    cp_async_commit();
+  }
   if (!early && ns > 0) {
     ok = partials_ready();
     if (ok) stage_chunk(0, min(sch, ns));

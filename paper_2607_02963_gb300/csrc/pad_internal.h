@@ -245,6 +245,8 @@ __device__ __forceinline__ float rope_elem(const __nv_bfloat16* row, int D, int 
 #endif
 
 // Launchers (pad_kernels.cu, pad_prefix_tc.cu).  Return the launch error.
+cudaError_t launch_host_in(const void* const* src, void* const* dst, const size_t* bytes, int n, int sms,
+                           cudaStream_t s);
 cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,
                           void* v_pool, cudaStream_t s);
 cudaError_t launch_prefix_simt(const KParams& p, int max_rows, const void* q, const void* kp,

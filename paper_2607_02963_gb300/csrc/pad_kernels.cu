@@ -1,4 +1,5 @@
 // Kernels of one event-factorized decode step (Sec. 3.4, Eq. 3):
+//   host_in_kernel       the step inputs from device-mapped host memory (pad_step_run_host)
 //   append_kernel        a2: scatter each branch's new K/V into its page, write new page-table entries
 //   prefix_simt_kernel   a3 for few rows (R = E_b * G <= 16): warp-shuffle split-KV flash-decode
 //   prefix_mma_kernel    a3 with warp-level mma.sync (m16n8k16, bf16 in, fp32 accumulate)
@@ -10,6 +11,8 @@
 #include <cuda_bf16.h>
 #include <cstddef>
 #include <cstdint>
+
+#include <algorithm>
 
 #include "pad_branch_merge.cuh"
 #include "pad_internal.h"
@@ -532,7 +535,55 @@ __global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __g
                   [] { return true; });
 }
 
+// Step inputs from page-locked, device-mapped host memory into device memory (the
+// mapped-host-I/O form of pad_step_run_host): up to three 16-byte-aligned segments, read
+// by the SMs over the host link.  It releases its dependents at entry, so the step's first
+// kernel is scheduled while it runs and waits for its completion before reading q.
+struct HostInArgs {
+  const uint4* src[3];
+  uint4* dst[3];
+  int64_t n16[3];
+};
+__global__ void __launch_bounds__(256) host_in_kernel(const __grid_constant__ HostInArgs a) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    const int64_t n = a.n16[k];
+    for (int64_t i = t0; i < n; i += 2 * stride) {
+      // two independent loads in flight per thread
+      const bool second = i + stride < n;
+      const uint4 v0 = a.src[k][i];
+      uint4 v1 = make_uint4(0u, 0u, 0u, 0u);
+      if (second) v1 = a.src[k][i + stride];
+      a.dst[k][i] = v0;
+      if (second) a.dst[k][i + stride] = v1;
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_host_in(const void* const* src, void* const* dst, const size_t* bytes, int n, int sms,
+                           cudaStream_t s) {
+  if (n < 0 || n > 3) return cudaErrorInvalidValue;
+  HostInArgs a{};
+  int64_t total = 0;
+  for (int k = 0; k < n; ++k) {
+    if ((bytes[k] & 15u) || (reinterpret_cast<uintptr_t>(src[k]) & 15u) || (reinterpret_cast<uintptr_t>(dst[k]) & 15u))
+      return cudaErrorInvalidValue;
+    a.src[k] = static_cast<const uint4*>(src[k]);
+    a.dst[k] = static_cast<uint4*>(dst[k]);
+    a.n16[k] = (int64_t)(bytes[k] >> 4);
+    total += a.n16[k];
+  }
+  if (total == 0) return cudaSuccess;
+  // about two 16-byte pieces per thread, at most one CTA of 256 per SM
+  const int64_t blocks = std::min<int64_t>(std::max(1, sms), (total + 511) / 512);
+  host_in_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,
                           void* v_pool, cudaStream_t s) {

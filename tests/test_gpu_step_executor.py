@@ -87,6 +87,101 @@ def test_run_host_copies_in_and_out(adjacent):
 
 
 @pytest.mark.parametrize("one_call", [True, False])
+@pytest.mark.parametrize("adjacent", [True, False])
+@pytest.mark.parametrize("make", [synth.gqa_8k, synth.tiny])
+def test_run_host_mapped_io(make, adjacent, one_call):
+    """Mapped host I/O: a kernel reads q / k_new / v_new from the page-locked buffers and the
+    step writes O and LSE straight into them; the results, pools and page table equal the
+    device-buffer run bit for bit, and the step's own device out / lse stay untouched."""
+    w = make()
+    a = DeviceBatch(w)
+    a.run_step(one_call=one_call)
+    torch.cuda.synchronize()
+    b = DeviceBatch(w)
+    if adjacent:
+        h_in = b.io_in.cpu().pin_memory()
+        h_out = torch.full(b.io_out.shape, 0x7f, dtype=torch.uint8).pin_memory()
+        qn, kn = b.q.numel(), b.k_new.numel()
+        hq, hk, hv = h_in[:qn].view(b.q.shape), h_in[qn:qn + kn].view(b.k_new.shape), h_in[qn + kn:].view(b.v_new.shape)
+        ob = b.out.numel() * b.out.element_size()
+        ho = h_out[:ob].view(b.out.dtype).view(b.out.shape)
+        hl = h_out[ob:].view(torch.float32).view(b.lse.shape)
+    else:
+        hq = b.q.cpu().pin_memory()
+        hk = b.k_new.cpu().pin_memory()
+        hv = b.v_new.cpu().pin_memory()
+        ho = torch.full(b.out.shape, float("nan"), dtype=b.out.dtype).pin_memory()
+        hl = torch.full(b.lse.shape, float("nan"), dtype=torch.float32).pin_memory()
+    b.q.zero_()
+    b.k_new.zero_()
+    b.v_new.zero_()
+    b.out.fill_(7.0)
+    b.lse.fill_(7.0)
+    st = _native(b, w, release_pages=False, one_call=one_call, mapped_host_io=True)
+    st.profile(True)
+    st.run_host(hq, hk, hv, ho, hl)
+    prof = st.profile_read()
+    assert prof["calls"] == 1
+    assert torch.equal(ho, a.out.cpu()) and torch.equal(hl, a.lse.cpu())
+    # inputs landed in the device buffers; outputs went to the host only
+    assert torch.equal(b.q.cpu(), a.q.cpu()) and torch.equal(b.k_new.cpu(), a.k_new.cpu())
+    assert torch.equal(b.v_new.cpu(), a.v_new.cpu())
+    assert bool((b.out == 7.0).all()) and bool((b.lse == 7.0).all())
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+    assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
+    assert torch.equal(a.page_table, b.page_table)
+
+
+@pytest.mark.parametrize("mapped", [True, False])
+def test_two_batches_in_flight(mapped):
+    """pad_step_enqueue_host of two independent batches, then pad_step_wait of each: every
+    batch's outputs and state equal its own device-buffer run."""
+    ws = [synth.gqa_8k(), synth.random_small(3)]
+    refs, runs, bufs = [], [], []
+    for w in ws:
+        a = DeviceBatch(w)
+        a.run_step(one_call=True)
+        refs.append(a)
+    torch.cuda.synchronize()
+    for w in ws:
+        b = DeviceBatch(w)
+        hq, hk, hv = b.q.cpu().pin_memory(), b.k_new.cpu().pin_memory(), b.v_new.cpu().pin_memory()
+        ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
+        hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
+        b.q.zero_()
+        runs.append((b, _native(b, w, release_pages=False, mapped_host_io=mapped)))
+        bufs.append((hq, hk, hv, ho, hl))
+    for (b, st), io in zip(runs, bufs):
+        st.enqueue_host(*io)
+    runs[1][1].wait()
+    runs[0][1].wait()
+    runs[0][1].wait()  # nothing pending: returns at once
+    for a, (b, st), io in zip(refs, runs, bufs):
+        assert torch.equal(io[3], a.out.cpu()) and torch.equal(io[4], a.lse.cpu())
+        assert torch.equal(a.page_table, b.page_table)
+        assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+
+
+def test_run_host_mapped_io_falls_back_on_pageable_buffers():
+    """A pageable host buffer fails the mapped check: that call takes the copy path."""
+    w = synth.tiny()
+    a = DeviceBatch(w)
+    a.run_step(one_call=True)
+    torch.cuda.synchronize()
+    b = DeviceBatch(w)
+    hq = b.q.cpu()  # pageable
+    hk = b.k_new.cpu().pin_memory()
+    hv = b.v_new.cpu().pin_memory()
+    ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
+    hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
+    b.q.zero_()
+    st = _native(b, w, release_pages=False, mapped_host_io=True)
+    st.run_host(hq, hk, hv, ho, hl)
+    assert torch.equal(ho, a.out.cpu()) and torch.equal(hl, a.lse.cpu())
+    _same_state(a, b)  # the copy path also writes the step's device out / lse
+
+
+@pytest.mark.parametrize("one_call", [True, False])
 def test_generation_loop_advances_event_len_in_place(one_call):
     """Three steps; each run plans from the executor's event_len as the loop left it."""
     w = synth.make_workload("loop", 61, 28, 4, 128, [2500], [4], [14, 15, 31, 0],

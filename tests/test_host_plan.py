@@ -319,7 +319,7 @@ def test_step_executor_validates_and_returns_pages_of_a_failed_run(padlib):
     fake = 1 << 20  # 16-byte aligned addresses, never dereferenced by the host
     args = [ctypes.byref(prob), cache.handle, 1, pl.ctypes.data_as(B._I32P), None, 3, ev.ctypes.data_as(B._I32P),
             el.ctypes.data_as(B._I32P), fake, 4, fake, 1 << 24] + [fake] * 9 + [None]
-    for bad_opts in (0x4, -1):
+    for bad_opts in (0x8, -1):
         with pytest.raises(B.PadError) as ei:
             B._check(B.lib().pad_step_create(*args, bad_opts, ctypes.byref(h)))
         assert ei.value.status == 1
@@ -328,6 +328,8 @@ def test_step_executor_validates_and_returns_pages_of_a_failed_run(padlib):
     with pytest.raises(B.PadError) as ei:
         B._check(B.lib().pad_step_create(*no_ws, 0, ctypes.byref(h)))
     assert ei.value.status == 1
+    B._check(B.lib().pad_step_create(*args, B.STEP_MAPPED_HOST_IO, ctypes.byref(h)))
+    B.lib().pad_step_destroy(h)
     B._check(B.lib().pad_step_create(*args, 0, ctypes.byref(h)))
     try:
         import torch
