@@ -64,7 +64,7 @@ using namespace tc;
 constexpr int kD = 128;
 constexpr int kBN = 128;       // prefix tokens per K/V tile
 constexpr int kStages = 3;
-constexpr int kSBuf = 3;       // S buffers in TMEM
+constexpr int kPSlots = 2;     // P slots in TMEM
 constexpr int kThreads = 384;
 constexpr uint32_t kHalfBytes = kBN * 128;         // 128 tokens x 64 bf16 = 16 KB
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 32 KB
@@ -74,12 +74,19 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kQTileBytes;
 constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
-constexpr uint32_t kOffX = kOffBar + 256;               // partial row maxima: [2][2][128] fp32
+constexpr uint32_t kOffX = kOffBar + 256;               // the key halves' (m, l): [2][2][128] fp32
 constexpr uint32_t kSmemBytes = kOffX + 2 * 2 * 128 * 4;
 constexpr int kOStage = kD + 4;                       // fp32 row stride of the O staging rows
-static_assert(128 * kOStage * 4 <= kStages * kTileBytes, "O staging fits the K stages");
+static_assert((128 * kOStage + 128) * 4 <= kStages * kTileBytes, "O staging (and 1 / l) fits the K stages");
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 384;
+// TMEM: S of the current tile (fp32, 128 columns), P of two tiles (packed bf16, 64
+// columns each: tokens 0-63, then 64-127) and the P.V accumulators of the two key halves
+// of every tile (tokens 0-63: softmax warps 4-7, 64-127: warps 8-11), which keep separate
+// softmax states and are merged once in the epilogue.
+constexpr uint32_t kColS = 0;
+constexpr uint32_t kColP = 128;
+constexpr uint32_t kColOA = 256;
+constexpr uint32_t kColOB = 384;
 constexpr float kLazyRescale = 8.0f;                  // log2 units
 #ifdef PAD_MUFU_PAIRS
 constexpr int kMufuPairs = PAD_MUFU_PAIRS;
@@ -94,9 +101,11 @@ static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 struct TcBars {
   uint64_t kfull[kStages];
   uint64_t vfull[kStages];
-  uint64_t pvfree[kStages];   // P.V of the tile in this stage / S buffer has completed
-  uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
-  uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (8 warp arrivals)
+  uint64_t kfree[kStages];    // S of the tile in this K stage has completed
+  uint64_t pvfree[kStages];   // P.V of the tile in this V stage has completed
+  uint64_t sfull;             // S of the current tile has completed
+  uint64_t sfree;             // every softmax warp has loaded it (8 warp arrivals)
+  uint64_t pfull[kPSlots];    // P of the tile in this slot is written (8 warp arrivals)
   uint64_t drain_s;           // every S MMA has completed (S issuer)
   uint64_t drain_pv;          // every P.V MMA has completed (P.V issuer)
   uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
@@ -144,7 +153,7 @@ __device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], Cols 
 }
 
 // P = 2^(s * scale_log2 - m) for one softmax warp's 64 columns, written as packed bf16
-// over the S columns already read; returns the fp32 sum of the P values.
+// (two per column) to the 32 TMEM columns at taddr_p; returns the fp32 sum of the P values.
 template <bool MASK, class Cols>
 __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
                                               float m, uint32_t taddr_p);
@@ -378,10 +387,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&bars->kfull[s], 1);
         mbar_init(&bars->vfull[s], 1);
       }
+      mbar_init(&bars->kfree[s], 1);
       mbar_init(&bars->pvfree[s], 1);
     }
-    for (int b = 0; b < kSBuf; ++b) {
-      mbar_init(&bars->sfull[b], 1);
+    mbar_init(&bars->sfull, 1);
+    mbar_init(&bars->sfree, 8);     // one arrival per softmax warp
+    for (int b = 0; b < kPSlots; ++b) {
       mbar_init(&bars->pfull[b], 8);  // one arrival per softmax warp
     }
     mbar_init(&bars->drain_s, 1);
@@ -424,8 +435,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = 1; t < n_tiles && ok; ++t) {
         const int s = t % kStages;
         if (t >= kStages) {
-          // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
-          uint64_t* freed = isK ? &bars->sfull[s] : &bars->pvfree[s];
+          // K stage: S of tile t-3 done (kfree[s], completion t/3 - 1); V stage: its P.V done
+          uint64_t* freed = isK ? &bars->kfree[s] : &bars->pvfree[s];
           ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
           if (!ok) break;
         }
@@ -464,22 +475,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (warp == 1) {
         ok = mbar_wait(&bars->qready, 0u, bars, p.header, 11);
         for (int t = 0; t < n_tiles && ok; ++t) {
-          const uint32_t s = (uint32_t)(t % kStages);
+          const uint32_t s = (uint32_t)(t % kStages);  // K stage
           ok = mbar_wait(&bars->kfull[s], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
           if (!ok) break;
-          // S buffer s holds P of tile t-3 until that P.V completes
-          if (t >= kStages)
-            ok = mbar_wait(&bars->pvfree[s], (uint32_t)((t / kStages - 1) & 1), bars, p.header, 6);
+          // the S buffer holds S of tile t-1 until every softmax warp has loaded it
+          if (t >= 1) ok = mbar_wait(&bars->sfree, (uint32_t)((t - 1) & 1), bars, p.header, 12);
           if (!ok) break;
           fence_after();
-          const uint32_t d = tmem + 128u * s;
+          const uint32_t d = tmem + kColS;
           const uint64_t kb = dK + (s * kTileBytes >> 4);
 #pragma unroll
           for (int kk = 0; kk < kD / 16; ++kk) {
             const uint32_t off = (uint32_t)(kk >> 2) * kQHalfBytes + (uint32_t)(kk & 3) * 32;
             mma_ss(d, dQ + (off >> 4), kb + (off >> 4), kIdescS, kk > 0 ? 1u : 0u);
           }
-          mma_commit(&bars->sfull[s]);
+          mma_commit(&bars->sfull);
+          mma_commit(&bars->kfree[s]);
         }
         mma_commit(&bars->drain_s);
         drain_wait(&bars->drain_s, 0u);
@@ -488,16 +499,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t s = (uint32_t)(j % kStages);
           ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
           if (!ok) break;
-          ok = mbar_wait(&bars->pfull[s], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
+          ok = mbar_wait(&bars->pfull[j % kPSlots], (uint32_t)((j / kPSlots) & 1), bars, p.header, 5);
           if (!ok) break;
           fence_after();
-          const uint32_t a = tmem + 128u * s;
+          const uint32_t a = tmem + kColP + 64u * (uint32_t)(j % kPSlots);
           const uint64_t vb = dV + (s * kTileBytes >> 4);
           const uint32_t acc0 = j > 0 ? 1u : 0u;
+          // tokens 0-63 of the tile into the first key half's O, 64-127 into the second's
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk)
-            mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
-                   kk > 0 ? 1u : acc0);
+            mma_ts(tmem + (kk < 4 ? kColOA : kColOB), a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
+                   (kk & 3) > 0 ? 1u : acc0);
           mma_commit(&bars->pvfree[s]);
         }
         // O is final once every P.V has completed
@@ -572,7 +584,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool warp_active = (row0 + lane_base) < R;  // same for both warps of the quarter
     const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
     const uint32_t col0 = 64u * (uint32_t)half;       // first S column (token) of this warp
-    float* xmax = reinterpret_cast<float*>(smem + kOffX);  // [tile parity][half][row]
+    const uint32_t colO = half ? kColOB : kColOA;     // this key half's P.V accumulator
+    float* xmax = reinterpret_cast<float*>(smem + kOffX);  // [half][m | l][row], epilogue
     uint64_t* xbar = &bars->xchg[quarter];
     const float sl2 = p.scale_log2;
     float m_run = -__builtin_huge_valf(), l_run = 0.f;
@@ -594,18 +607,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     for (int j = 0; j < n_tiles; ++j) {
-      const uint32_t cS = 128u * (uint32_t)(j % kSBuf);
-      ok = mbar_wait(&bars->sfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 8);
+      ok = mbar_wait(&bars->sfull, (uint32_t)(j & 1), bars, p.header, 8);
       ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
       if (!ok) break;
       fence_after();
+      uint32_t sr[2][32];
       if (warp_active) {
-        const int valid = min(kBN, ntok - j * kBN) - (int)col0;  // valid columns of this half
-        uint32_t sr[2][32];
-        tmem_ld32(tl + cS + col0, sr[0]);
-        tmem_ld32(tl + cS + col0 + 32, sr[1]);
+        tmem_ld32(tl + kColS + col0, sr[0]);
+        tmem_ld32(tl + kColS + col0 + 32, sr[1]);
         tmem_wait_ld_dep(sr[0]);
         tmem_wait_ld_dep(sr[1]);
+      }
+      // S is in registers: the S issuer may overwrite the buffer with the next tile's
+      fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->sfree);
+      if (warp_active) {
+        const int valid = min(kBN, ntok - j * kBN) - (int)col0;  // valid columns of this half
         // columns to mask: past the split's end, or (GSELF) hidden planning tokens of this
         // row's event; the path is chosen per warp (tcgen05.st below is warp-collective)
         float pmax;
@@ -636,19 +654,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           masked = valid < 64;
           pmax = masked ? half_row_max<true>(sr, ColsValid{valid}) : half_row_max<false>(sr, ColsValid{valid});
         }
-        // meet the other half: this also orders both warps' S reads before either
-        // writes P over columns the other one read
-        xmax[(j & 1) * 256 + half * 128 + row] = pmax;
-        mbar_arrive(xbar);
-        ok = mbar_wait(xbar, (uint32_t)(j & 1), bars, p.header, 12);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok) break;
-        const float mx = fmaxf(pmax, xmax[(j & 1) * 256 + (1 - half) * 128 + row]) * sl2;
+        // this key half's own running maximum: P is written over columns only this warp
+        // reads, and its P.V goes to this half's own accumulator
+        const float mx = pmax * sl2;
         const float m_new = fmaxf(m_run, mx);
         const bool need = m_new > m_run + kLazyRescale;
         if (__any_sync(0xffffffffu, need && j > 0)) {
-          // O must hold P.V of tile j-1 before it is rescaled (each half rescales its
-          // own 64 head-dim columns; both halves take the same decision per row)
+          // this half's O must hold P.V of tile j-1 before it is rescaled
           ok = mbar_wait(&bars->pvfree[(j - 1) % kStages], (uint32_t)(((j - 1) / kStages) & 1), bars,
                          p.header, 9);
           ok = __all_sync(0xffffffffu, ok);
@@ -656,28 +668,37 @@ __global__ void __launch_bounds__(kThreads, 1)
           fence_after();
           const float alpha = need ? ex2(m_run - m_new) : 1.f;
 #pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            tmem_ld32(tl + kColO + col0 + 32 * c, r);
+          for (int c = 0; c < 4; ++c) {
+            tmem_ld32(tl + colO + 32 * c, r);
             tmem_wait_ld_dep(r);
 #pragma unroll
             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tmem_st32(tl + kColO + col0 + 32 * c, r);
+            tmem_st32(tl + colO + 32 * c, r);
           }
           tmem_wait_st();
           if (need) l_run *= alpha;
         }
         if (need) m_run = m_new;
+        // this key half's P of tile j goes to slot j % 2, which held P of tile j-2 until
+        // that P.V completed
+        const uint32_t taddr_p = tl + kColP + 64u * (uint32_t)(j % kPSlots) + 32u * (uint32_t)half;
+        if (j >= kPSlots) {
+          const int jp = j - kPSlots;
+          ok = mbar_wait(&bars->pvfree[jp % kStages], (uint32_t)((jp / kStages) & 1), bars, p.header, 14);
+          ok = __all_sync(0xffffffffu, ok);
+          if (!ok) break;
+        }
         if (GSELF || PREFILL)
-          l_run += masked ? half_row_exp<true>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2)
-                          : half_row_exp<false>(sr, ColsBits{keep}, sl2, m_run, tl + cS + col0 / 2);
+          l_run += masked ? half_row_exp<true>(sr, ColsBits{keep}, sl2, m_run, taddr_p)
+                          : half_row_exp<false>(sr, ColsBits{keep}, sl2, m_run, taddr_p);
         else
-          l_run += masked ? half_row_exp<true>(sr, ColsValid{valid}, sl2, m_run, tl + cS + col0 / 2)
-                          : half_row_exp<false>(sr, ColsValid{valid}, sl2, m_run, tl + cS + col0 / 2);
+          l_run += masked ? half_row_exp<true>(sr, ColsValid{valid}, sl2, m_run, taddr_p)
+                          : half_row_exp<false>(sr, ColsValid{valid}, sl2, m_run, taddr_p);
         tmem_wait_st();
       }
       fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->pfull[j % kSBuf]);
+      if (lane == 0) mbar_arrive(&bars->pfull[j % kPSlots]);
     }
     // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
     if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
@@ -688,32 +709,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     // consecutive rows fall in distinct banks, then written one 512-byte row per warp
     // instruction.
     float* ostage = reinterpret_cast<float*>(smem + kOffK);
+    float* inv_row = ostage + 128 * kOStage;  // PREFILL: 1 / l of each row for the write-out
     if (ok && warp_active) {
-      fence_after();
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        tmem_ld32(tl + kColO + col0 + 32 * c, r);
-        tmem_wait_ld_dep(r);
-        float4* dst = reinterpret_cast<float4*>(ostage + row * kOStage + col0 + 32 * c);
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-          dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
-                               __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
-      }
-      // row sum = both halves' partial sums (slot n_tiles & 1 was last read two tiles ago)
-      xmax[(n_tiles & 1) * 256 + half * 128 + row] = l_run;
+      // The two key halves meet once: each warp publishes its (m, l), then merges both
+      // halves' accumulators over its 64 head-dim columns by log-sum-exp weights.
+      xmax[half * 256 + row] = m_run;
+      xmax[half * 256 + 128 + row] = l_run;
       mbar_arrive(xbar);
-      ok = mbar_wait(xbar, (uint32_t)(n_tiles & 1), bars, p.header, 13);
-      if (ok && half == 0 && grow < R) {
-        const float l_tot = l_run + xmax[(n_tiles & 1) * 256 + 128 + row];
-        if (PREFILL) {
-          // normalised output: 1 / l for the write-out below (the other slot is free once
-          // both halves met here), the LSE now
-          xmax[((n_tiles + 1) & 1) * 256 + row] = 1.0f / l_tot;
-          const int64_t orow = (int64_t)pf_p * p.h_q + kvh * p.group + grow % p.group;
-          if (p.pf_lse != nullptr) p.pf_lse[orow] = (m_run + log2f(l_tot)) * 0.69314718055994531f;
-        } else {
-          p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_run, l_tot);
+      ok = mbar_wait(xbar, 0u, bars, p.header, 13);
+      ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld below is warp-collective
+      if (ok) {
+        fence_after();
+        const float ma = xmax[row], la = xmax[128 + row];
+        const float mb = xmax[256 + row], lb = xmax[384 + row];
+        const float m_tot = fmaxf(ma, mb);
+        const bool none = m_tot == -__builtin_huge_valf();  // no visible key in the split
+        const float wa = none ? 0.f : ex2(ma - m_tot), wb = none ? 0.f : ex2(mb - m_tot);
+        const float l_tot = wa * la + wb * lb;
+        uint32_t rb[32];
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          tmem_ld32(tl + kColOA + col0 + 32 * c, r);
+          tmem_ld32(tl + kColOB + col0 + 32 * c, rb);
+          tmem_wait_ld_dep(r);
+          tmem_wait_ld_dep(rb);
+          float4* dst = reinterpret_cast<float4*>(ostage + row * kOStage + col0 + 32 * c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(wa * __uint_as_float(r[4 * i]) + wb * __uint_as_float(rb[4 * i]),
+                                 wa * __uint_as_float(r[4 * i + 1]) + wb * __uint_as_float(rb[4 * i + 1]),
+                                 wa * __uint_as_float(r[4 * i + 2]) + wb * __uint_as_float(rb[4 * i + 2]),
+                                 wa * __uint_as_float(r[4 * i + 3]) + wb * __uint_as_float(rb[4 * i + 3]));
+        }
+        if (half == 0 && grow < R) {
+          if (PREFILL) {
+            // normalised output: 1 / l for the write-out below, the LSE now
+            inv_row[row] = 1.0f / l_tot;
+            const int64_t orow = (int64_t)pf_p * p.h_q + kvh * p.group + grow % p.group;
+            if (p.pf_lse != nullptr) p.pf_lse[orow] = (m_tot + log2f(l_tot)) * 0.69314718055994531f;
+          } else {
+            p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_tot, l_tot);
+          }
         }
       }
     }
@@ -727,7 +763,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int rr = warp - 4; rr < nrows; rr += 8) {
       float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
       if (PREFILL) {
-        const float inv = xmax[((n_tiles + 1) & 1) * 256 + rr];
+        const float inv = inv_row[rr];
         v.x *= inv;
         v.y *= inv;
         v.z *= inv;
