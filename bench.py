@@ -260,8 +260,9 @@ def hbm_peak():
 
 
 # The sources that define the dominant kernel of the decode step (the tensor-core prefix
-# kernel, the branch/merge task it can run, and the descriptors both read).
-TRAFFIC_SOURCES = ("pad_internal.h", "pad_branch_merge.cuh", "pad_prefix_tc.cu")
+# kernel, its tcgen05 / TMA helpers, the branch/merge task it can run, and the descriptors
+# both read).
+TRAFFIC_SOURCES = ("pad_internal.h", "pad_tc_common.cuh", "pad_branch_merge.cuh", "pad_prefix_tc.cu")
 
 
 def kernel_source_hash():
@@ -445,6 +446,19 @@ def run_ours(args):
         B.pad_device_status(db.plan_step(stream))
         db.release_new_pages()
     barrier(device)
+    if args.profile_run:
+        # a short run for a profiler: the warm-up above, then exactly this many steps,
+        # no timing loops (launch count = steps x kernels per step)
+        for i in range(args.profile_run):
+            steps[(W + i) % n_rep]()
+        torch.cuda.synchronize()
+        for db in reps:
+            B.pad_device_status(db.plan_step(stream))
+            db.release_new_pages()
+        if rank == 0:
+            print(json.dumps({"profile_run": args.profile_run, "warmup": W, "workload": args.workload,
+                              "kernels_per_step": launches_per_step, "replicas": n_rep}), flush=True)
+        return
 
     # timed region: blocks of exactly K steps, each step exactly as a caller runs it (no
     # events between its kernels, an event between blocks), repeated to cover >= 200 ms
@@ -1050,6 +1064,8 @@ def main(argv=None):
     ap.add_argument("--sweep", action="store_true",
                     help="per-E table of the sweep workload with the naive per-event comparator")
     ap.add_argument("--sweep-naive-steps", type=int, default=20)
+    ap.add_argument("--profile-run", type=int, default=0,
+                    help="run the warm-up and then this many steps only (for ncu), no timing")
     args = ap.parse_args(argv)
     if args.prefill:
         run_prefill(args)
