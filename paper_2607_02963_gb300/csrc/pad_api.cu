@@ -191,6 +191,31 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
     for (int b = 0; b < n_videos; ++b)
       if (L->ev_count[b] > 0) max_prefix = std::max<int64_t>(max_prefix, prefix_len[b]);
     while (ctas_for(chunk) > target && chunk < max_prefix) chunk += kSplitGranule;
+    // The branch/merge CTAs (one per event and kv-head) do their part before the grid wait
+    // (staging, the append and, in a one-call step, the whole branch pass) during the prefix
+    // pass only on SMs the prefix grid leaves free; the others do it after the prefix CTAs
+    // retire.  A split up to two tiles longer is taken when it leaves room for every task and
+    // its extra tiles cost less than that serial part.  Costs measured on GB300: ~0.85 us per
+    // 128-token tile of a CTA in steady state, ~2 us for a task's part before the wait.
+    if (!want_fused) {
+      constexpr double kTileUs = 0.85, kTaskPreWaitUs = 2.0;
+      const int64_t tasks = (int64_t)n_events * prob->h_kv;
+      auto cost = [&](int64_t c) {
+        const int64_t n_free = target - ctas_for(c);
+        return (double)((c + kSplitGranule - 1) / kSplitGranule) * kTileUs + (tasks > n_free ? kTaskPreWaitUs : 0.0);
+      };
+      int64_t best = chunk;
+      double best_cost = cost(chunk);
+      for (int64_t c = chunk + kSplitGranule; c <= std::min<int64_t>(max_prefix, chunk + 2 * kSplitGranule);
+           c += kSplitGranule) {
+        const double v = cost(c);
+        if (v < best_cost) {
+          best = c;
+          best_cost = v;
+        }
+      }
+      chunk = best;
+    }
   }
   if (chunk > (int64_t)1 << 30) return fail(PAD_ERR_UNSUPPORTED, "prefix too long");
   L->split_len = (int)chunk;

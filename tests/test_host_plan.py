@@ -143,6 +143,34 @@ def test_tc_split_fits_one_wave(padlib, flags, rows_per_cta):
             assert ctas <= sms
 
 
+def _split_of(P, E, sms=152, flags=0):
+    prob = B.make_problem(28, 4, 128, num_sms=sms, flags=flags)
+    ev = np.zeros(E, np.int32)
+    plan = B.pad_plan(prob, B.CacheState(4096), np.array([P], np.int32), ev, np.zeros(E, np.int32),
+                      max_pages=2, workspace=None)
+    return plan.info()["split_len"]
+
+
+def test_tc_split_leaves_sms_for_the_branch_tasks(padlib):
+    """The planner takes a split up to two tiles longer than the one-wave minimum when that
+    leaves an SM for every (event, kv-head) branch task and the extra tiles cost less than
+    running the tasks' pre-wait part after the prefix pass (0.85 us per tile, 2 us)."""
+    # 16384-token prefix, 4 kv-heads, one row group: 128 one-wave CTAs of 4 tiles
+    assert _split_of(16384, 4) == 512        # 16 tasks fit the 24 free SMs already
+    assert _split_of(16384, 8) == 640        # 32 tasks: 104 CTAs of 5 tiles leave 48 SMs
+    assert _split_of(16384, 16) == 768       # 64 tasks: 88 CTAs of 6 tiles leave 64 SMs
+    assert _split_of(8192, 8) == 384         # gqa_8k: 88 CTAs of 3 tiles
+    # 128 tasks never fit beside a one-wave grid: the minimum split stays
+    assert _split_of(32768, 32) == 1792
+    # the fused tail plans its own grid
+    assert _split_of(16384, 8, flags=B.FLAG_FUSED_MERGE) == 512
+    # every candidate stays within one wave
+    for E in (1, 3, 8, 12, 20):
+        sl = _split_of(16384, E, sms=100)
+        groups = -(-E * 7 // 128)
+        assert 4 * -(-16384 // sl) * groups <= 100
+
+
 @pytest.mark.parametrize("case,status", [
     (dict(event_video=[1, 0]), 1),                       # not sorted by video
     (dict(event_video=[0, 2]), 1),                       # video out of range
