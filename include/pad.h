@@ -273,7 +273,13 @@ pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const vo
  * (pools, page table, out and lse all end up identical), with one kernel launch fewer.
  * The shared-prefix pass starts the step; each (event, kv-head) branch task reads its
  * newest key from k_new / v_new, writes it into the pools (and the page table) itself,
- * and attends to it.  Arguments as in those two calls; k_pool and v_pool are written. */
+ * and attends to it.  Arguments as in those two calls; k_pool and v_pool are written.
+ * The step's first kernel uses programmatic dependent launch: it may start while the grid
+ * before it on the stream is still running, if that grid releases its dependents early
+ * (griddepcontrol.launch_dependents; the library's own kernels do), and it reads the first
+ * tile of k_prefix / v_prefix before it waits for that grid.  Everything else it reads only
+ * after that grid has completed.  So k_prefix and v_prefix must not be written by a grid
+ * that releases its dependents before those writes. */
 pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_new, const void* v_new,
                            const void* k_prefix, const void* v_prefix, void* k_pool, void* v_pool,
                            void* out, float* lse, pad_stream_t stream);

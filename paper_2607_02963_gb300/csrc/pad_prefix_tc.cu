@@ -367,13 +367,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The first K and V tile go out first (their barriers initialised, then the loads),
     // before the other barriers, TMEM allocation and the block barrier; the producer warps
     // issue the rest once that K tile has landed, so that every CTA's first tile is not
-    // queued in DRAM behind the later tiles of all the others.
+    // queued in DRAM behind the later tiles of all the others.  The prefix K/V is written by
+    // no grid of the library's own that may run ahead of this one (and, by the call's
+    // contract, by no grid that releases its dependents before its writes), so that tile is
+    // requested even before the wait for the grid ahead; nothing else is.
     mbar_init(&bars->kfull[0], 1);
     mbar_init(&bars->vfull[0], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
-    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
     if (n_tiles > 0) {
       mbar_expect_tx(&bars->kfull[0], kTileBytes);
       tma_load_3d(sbase + kOffK, &tmK, 0, kvh, tile_tok(0), &bars->kfull[0]);
@@ -382,6 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_load_3d(sbase + kOffV, &tmV, 0, kvh, tile_tok(0), &bars->vfull[0]);
       tma_load_3d(sbase + kOffV + kHalfBytes, &tmV, 64, kvh, tile_tok(0), &bars->vfull[0]);
     }
+    if (one_call) asm volatile("griddepcontrol.wait;" ::: "memory");
     for (int s = 0; s < kStages; ++s) {
       if (s > 0) {
         mbar_init(&bars->kfull[s], 1);
