@@ -537,29 +537,39 @@ __global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __g
 
 // Step inputs from page-locked, device-mapped host memory into device memory (the
 // mapped-host-I/O form of pad_step_run_host): up to three 16-byte-aligned segments, read
-// by the SMs over the host link.  It releases its dependents at entry, so the step's first
-// kernel is scheduled while it runs and waits for its completion before reading q.
+// by the SMs over the host link.  It is launched so that it may start while the grid ahead
+// still runs: each thread first loads up to kHeld pieces of every segment from host memory
+// (the slow part), then waits for the grid ahead (which may still read these device
+// buffers) before it stores anything.  It releases its dependents at entry; the step's first
+// kernel waits for its completion before reading q.
 struct HostInArgs {
   const uint4* src[3];
   uint4* dst[3];
   int64_t n16[3];
 };
+constexpr int kHostInHeld = 4;
 __global__ void __launch_bounds__(256) host_in_kernel(const __grid_constant__ HostInArgs a) {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  uint4 v[3][kHostInHeld];
+#pragma unroll
+  for (int k = 0; k < 3; ++k)
+#pragma unroll
+    for (int j = 0; j < kHostInHeld; ++j) {
+      const int64_t i = t0 + j * stride;
+      if (i < a.n16[k]) v[k][j] = a.src[k][i];
+    }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 #pragma unroll
   for (int k = 0; k < 3; ++k) {
-    const int64_t n = a.n16[k];
-    for (int64_t i = t0; i < n; i += 2 * stride) {
-      // two independent loads in flight per thread
-      const bool second = i + stride < n;
-      const uint4 v0 = a.src[k][i];
-      uint4 v1 = make_uint4(0u, 0u, 0u, 0u);
-      if (second) v1 = a.src[k][i + stride];
-      a.dst[k][i] = v0;
-      if (second) a.dst[k][i + stride] = v1;
+#pragma unroll
+    for (int j = 0; j < kHostInHeld; ++j) {
+      const int64_t i = t0 + j * stride;
+      if (i < a.n16[k]) a.dst[k][i] = v[k][j];
     }
+    // pieces past what a thread holds (inputs larger than the grid x kHostInHeld pieces)
+    for (int64_t i = t0 + kHostInHeld * stride; i < a.n16[k]; i += stride) a.dst[k][i] = a.src[k][i];
   }
 }
 
@@ -569,20 +579,30 @@ cudaError_t launch_host_in(const void* const* src, void* const* dst, const size_
                            cudaStream_t s) {
   if (n < 0 || n > 3) return cudaErrorInvalidValue;
   HostInArgs a{};
-  int64_t total = 0;
+  int64_t largest = 0;
   for (int k = 0; k < n; ++k) {
     if ((bytes[k] & 15u) || (reinterpret_cast<uintptr_t>(src[k]) & 15u) || (reinterpret_cast<uintptr_t>(dst[k]) & 15u))
       return cudaErrorInvalidValue;
     a.src[k] = static_cast<const uint4*>(src[k]);
     a.dst[k] = static_cast<uint4*>(dst[k]);
     a.n16[k] = (int64_t)(bytes[k] >> 4);
-    total += a.n16[k];
+    largest = std::max(largest, a.n16[k]);
   }
-  if (total == 0) return cudaSuccess;
-  // about two 16-byte pieces per thread, at most one CTA of 256 per SM
-  const int64_t blocks = std::min<int64_t>(std::max(1, sms), (total + 511) / 512);
-  host_in_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  if (largest == 0) return cudaSuccess;
+  // enough threads that each holds at most kHostInHeld pieces of the largest segment,
+  // at most one CTA of 256 per SM
+  const int64_t per_cta = 256 * kHostInHeld;
+  const int64_t blocks = std::min<int64_t>(std::max(1, sms), (largest + per_cta - 1) / per_cta);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, host_in_kernel, a);
 }
 
 cudaError_t launch_append(const KParams& p, const void* k_new, const void* v_new, void* k_pool,
