@@ -224,7 +224,8 @@ def timed_blocks(run_step, K, stream, first=0, min_ms=MIN_REGION_MS):
     torch.cuda.synchronize()
     i0 = first + K
     est = max(p0.elapsed_time(p1), 1e-3)
-    n_blocks = max(1, min(100000, int(-(-min_ms // est)) + 1))
+    # a quarter more blocks than the pilot suggests (a warm block is shorter than the pilot)
+    n_blocks = max(1, min(100000, int(-(-1.25 * min_ms // est)) + 1))
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_blocks + 1)]
     h0 = time.perf_counter()
     evs[0].record(stream)

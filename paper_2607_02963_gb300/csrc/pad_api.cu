@@ -13,11 +13,22 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "pad_internal.h"
 
 using namespace pad;
 
 namespace {
+// A named NVTX range around each call of the C ABI that does device work or plans it, so
+// that a profiler's timeline shows plan / append / attention / step (no cost without one).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 
 thread_local std::string g_last_error;
 
@@ -563,6 +574,7 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
                     const int32_t* event_video, const int32_t* event_len, int32_t* page_table,
                     int32_t max_pages, void* workspace, size_t workspace_bytes,
                     pad_stream_t stream, pad_plan_t** plan_out) {
+  NvtxRange nvtx_range("pad_plan");
   if (!plan_out) return fail(PAD_ERR_INVALID_ARG, "plan_out is NULL");
   *plan_out = nullptr;
   pad_status st = check_problem(prob);
@@ -912,6 +924,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
 
 pad_status pad_kv_append(const pad_plan_t* plan, const void* k_new, const void* v_new,
                          void* k_pool, void* v_pool, pad_stream_t stream) {
+  NvtxRange nvtx_range("pad_kv_append");
   if (!plan) return fail(PAD_ERR_INVALID_ARG, "plan is NULL");
   if (plan->n_events == 0) return PAD_OK;
   if (!k_new || !v_new || !k_pool || !v_pool) return fail(PAD_ERR_INVALID_ARG, "NULL tensor");
@@ -1001,12 +1014,14 @@ static pad_status launch_attention(const pad_plan_t* plan, const void* q, const 
 pad_status pad_event_decode_attn(const pad_plan_t* plan, const void* q, const void* k_prefix,
                                  const void* v_prefix, const void* k_pool, const void* v_pool,
                                  void* out, float* lse, pad_stream_t stream) {
+  NvtxRange nvtx_range("pad_event_decode_attn");
   return launch_attention(plan, q, nullptr, nullptr, k_prefix, v_prefix, k_pool, v_pool, out, lse, stream);
 }
 
 pad_status pad_decode_step(const pad_plan_t* plan, const void* q, const void* k_new, const void* v_new,
                            const void* k_prefix, const void* v_prefix, void* k_pool, void* v_pool,
                            void* out, float* lse, pad_stream_t stream) {
+  NvtxRange nvtx_range("pad_decode_step");
   if (plan && plan->n_events > 0 && (!k_new || !v_new)) return fail(PAD_ERR_INVALID_ARG, "NULL k_new / v_new");
   return launch_attention(plan, q, k_new, v_new, k_prefix, v_prefix, k_pool, v_pool, out, lse, stream);
 }
@@ -1188,6 +1203,7 @@ pad_status step_run(pad_step_t* step, int32_t* new_page, double* ht, void* out, 
 }  // namespace
 
 pad_status pad_step_run(pad_step_t* step, int32_t* new_page) {
+  NvtxRange nvtx_range("pad_step_run");
   if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
   return step_run(step, new_page, nullptr, step->out, step->lse);
 }
@@ -1248,6 +1264,7 @@ namespace {
 // pad_step_run_host (wait) and pad_step_enqueue_host (no wait: an event behind the run)
 pad_status host_step(pad_step_t* step, const void* h_q, const void* h_k_new, const void* h_v_new, void* h_out,
                      float* h_lse, int32_t* new_page, bool wait) {
+  NvtxRange nvtx_range(wait ? "pad_step_run_host" : "pad_step_enqueue_host");
   if (!step) return fail(PAD_ERR_INVALID_ARG, "step is NULL");
   if (step->n_events > 0 && (!h_q || !h_k_new || !h_v_new || !h_out))
     return fail(PAD_ERR_INVALID_ARG, "NULL host buffer");
