@@ -234,7 +234,8 @@ typedef struct {
   int32_t n_videos;
   int32_t n_events;
   int32_t n_work_items;     /* (video, kv-head, split) items of the prefix pass */
-  int32_t split_len;        /* prefix tokens per split (last split of a video may be shorter) */
+  int32_t split_len;        /* prefix tokens of the longest split (each video has its own split
+                               length; a video's last split may be shorter) */
   int32_t prefix_kernel;    /* PAD_FLAG_PREFIX_* of the implementation that will run */
   int32_t n_new_pages;
   int64_t partial_rows;     /* rows of (m, l, O) partial softmax states in the workspace */
@@ -243,6 +244,8 @@ typedef struct {
                                      0 = the kernels read them from the plan's page-locked image */
   int32_t fused_tail;       /* 1: the branch pass and the merge run inside the prefix kernel */
   uint64_t generation;      /* the number tagging this plan's device status word and counters */
+  int32_t prefix_ctas;      /* CTAs of the prefix pass (a batch of videos may take several waves) */
+  int32_t max_split_tiles;  /* 128-token tiles of the longest split */
 } pad_plan_info;
 pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info);
 pad_status pad_plan_destroy(pad_plan_t* plan);

@@ -9,6 +9,7 @@
 #include <chrono>
 #include <deque>
 #include <mutex>
+#include <queue>
 #include <random>
 #include <string>
 #include <vector>
@@ -105,6 +106,8 @@ struct Layout {
   int max_rows = 0;
   int prefix_kernel = 0;
   std::vector<int32_t> ev_first, ev_count, n_splits, part_base;
+  std::vector<int64_t> vsplit;  // prefix tokens per split, per video
+  bool longest_first = false;   // CTA list ordered by descending split length
   int64_t n_items = 0;
   int64_t partial_rows = 0;
   // fused tail of the tensor-core path: per prefix CTA its (event * h_kv + kv-head) task or
@@ -229,11 +232,115 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
     }
   }
   if (chunk > (int64_t)1 << 30) return fail(PAD_ERR_UNSUPPORTED, "prefix too long");
-  L->split_len = (int)chunk;
+  // Per-video splits for a batch of videos on the tensor-core kernels.  One split length for
+  // all, sized to one wave, gives the longest video's CTAs the most tiles while a short
+  // video's single CTA idles, and one wave leaves the splits coarse.  So the planner sizes
+  // each video's splits for a grid of 1, 2 or 3 waves: every video starts with one split per
+  // (kv-head, row group), and the video whose CTAs hold the most tiles takes one more split
+  // while the grid has room.  Each candidate is costed by list-scheduling its CTAs, longest
+  // first, onto the SMs (a CTA costs kCtaUs of set-up and drain plus kTileUs per tile,
+  // measured on GB300), and the cheapest is kept; the CTA list is then ordered longest first.
+  // The decision depends only on the batch's shape, so the last one is reused.
+  L->vsplit.assign(n_videos, chunk);
+  L->longest_first = false;
+  if ((kern == PAD_FLAG_PREFIX_TC || kern == PAD_FLAG_PREFIX_DUAL) && !want_fused && n_videos > 1) {
+    constexpr double kTileUs = 0.85, kCtaUs = 4.0;
+    std::vector<int64_t> tiles(n_videos, 0), units(n_videos, 0);
+    int64_t base_ctas = 0;
+    for (int b = 0; b < n_videos; ++b) {
+      if (L->ev_count[b] == 0 || prefix_len[b] == 0) continue;
+      tiles[b] = (prefix_len[b] + kSplitGranule - 1) / kSplitGranule;
+      units[b] = (int64_t)prob->h_kv * groups_of(b);
+      base_ctas += units[b];
+    }
+    thread_local std::vector<int64_t> memo_key, memo_split;
+    std::vector<int64_t> key;
+    key.reserve(2 * (size_t)n_videos + 3);
+    key.push_back(target);
+    key.push_back(chunk);
+    key.push_back(prob->flags);
+    for (int b = 0; b < n_videos; ++b) {
+      key.push_back(tiles[b]);
+      key.push_back(units[b]);
+    }
+    if (key == memo_key) {
+      L->vsplit = memo_split;
+    } else if (base_ctas <= 3 * target) {
+      auto split_for = [&](int64_t budget, std::vector<int64_t>& ns) {
+        ns.assign(n_videos, 0);
+        std::priority_queue<std::pair<int64_t, int>> pq;  // (tiles per CTA, video)
+        for (int b = 0; b < n_videos; ++b)
+          if (tiles[b] > 0) {
+            ns[b] = 1;
+            pq.push({tiles[b], b});
+          }
+        budget -= base_ctas;
+        while (!pq.empty()) {
+          const int top = pq.top().second;
+          if (tiles[top] <= ns[top] || units[top] > budget) break;
+          pq.pop();
+          ++ns[top];
+          budget -= units[top];
+          pq.push({(tiles[top] + ns[top] - 1) / ns[top], top});
+        }
+      };
+      auto makespan = [&](const std::vector<int64_t>& ns) {
+        std::vector<std::pair<int64_t, int64_t>> durs;  // (tiles, CTA count), longest first
+        for (int b = 0; b < n_videos; ++b) {
+          if (ns[b] == 0) continue;
+          const int64_t per = (tiles[b] + ns[b] - 1) / ns[b], n = (tiles[b] + per - 1) / per;
+          durs.push_back({per, units[b] * (n - 1)});
+          durs.push_back({tiles[b] - per * (n - 1), units[b]});
+        }
+        std::sort(durs.begin(), durs.end(),
+                  [](const std::pair<int64_t, int64_t>& x, const std::pair<int64_t, int64_t>& y) {
+                    return x.first > y.first;
+                  });
+        std::priority_queue<double, std::vector<double>, std::greater<double>> sm;
+        for (int64_t i = 0; i < target; ++i) sm.push(0.0);
+        double end = 0.0;
+        for (const auto& d : durs)
+          for (int64_t k = 0; k < d.second; ++k) {
+            const double t = sm.top() + kCtaUs + kTileUs * (double)d.first;
+            sm.pop();
+            sm.push(t);
+            end = std::max(end, t);
+          }
+        return end;
+      };
+      // the one-split-length plan as the baseline
+      std::vector<int64_t> ns_global(n_videos, 0);
+      const int64_t chunk_tiles = chunk / kSplitGranule;
+      for (int b = 0; b < n_videos; ++b)
+        if (tiles[b] > 0) ns_global[b] = (tiles[b] + chunk_tiles - 1) / chunk_tiles;
+      double best = makespan(ns_global);
+      std::vector<int64_t> ns, best_ns;
+      for (int waves = 1; waves <= 3; ++waves) {
+        if (base_ctas > waves * target) continue;
+        split_for(waves * target, ns);
+        const double v = makespan(ns);
+        if (v < best) {
+          best = v;
+          best_ns = ns;
+        }
+      }
+      if (!best_ns.empty())
+        for (int b = 0; b < n_videos; ++b)
+          if (best_ns[b] > 0) L->vsplit[b] = (tiles[b] + best_ns[b] - 1) / best_ns[b] * kSplitGranule;
+      memo_key = key;
+      memo_split = L->vsplit;
+    }
+    L->longest_first = true;
+  }
+  int64_t longest = 0;
+  for (int b = 0; b < n_videos; ++b)
+    if (L->ev_count[b] > 0 && prefix_len[b] > 0) longest = std::max(longest, L->vsplit[b]);
+  L->split_len = (int)(longest > 0 ? longest : chunk);
   int64_t items = 0, rows = 0;
   for (int b = 0; b < n_videos; ++b) {
     if (L->ev_count[b] == 0 || prefix_len[b] == 0) continue;
-    const int ns = (int)((prefix_len[b] + chunk - 1) / chunk);
+    const int64_t vs = L->vsplit[b];
+    const int ns = (int)((prefix_len[b] + vs - 1) / vs);
     if (ns > 32767) return fail(PAD_ERR_UNSUPPORTED, "too many splits for video %d", b);
     L->n_splits[b] = ns;
     if (rows > INT32_MAX) return fail(PAD_ERR_UNSUPPORTED, "partial rows exceed int32");
@@ -287,14 +394,26 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
   if (rows_per_cta && !L->fused && items > 0) {
     if (items > ((int64_t)1 << 24)) return fail(PAD_ERR_UNSUPPORTED, "batch too large");
     L->cta_task.clear();
+    std::vector<std::pair<int64_t, int32_t>> order;  // (split tokens, CTA entry)
     int64_t item = 0;
     for (int b = 0; b < n_videos; ++b) {
       if (L->ev_count[b] == 0 || L->n_splits[b] == 0) continue;
       const int gb = groups_of(b);
+      const int64_t vs = L->vsplit[b];
       for (int h = 0; h < prob->h_kv; ++h)
-        for (int sp = 0; sp < L->n_splits[b]; ++sp, ++item)
-          for (int g = 0; g < gb; ++g) L->cta_task.push_back((int32_t)((item << 6) | g));
+        for (int sp = 0; sp < L->n_splits[b]; ++sp, ++item) {
+          const int64_t tok = std::min<int64_t>(prefix_len[b], (sp + 1) * vs) - sp * vs;
+          for (int g = 0; g < gb; ++g) order.push_back({tok, (int32_t)((item << 6) | g)});
+        }
     }
+    // a batch of videos: the longest splits start first
+    if (L->longest_first)
+      std::stable_sort(order.begin(), order.end(),
+                       [](const std::pair<int64_t, int32_t>& x, const std::pair<int64_t, int32_t>& y) {
+                         return x.first > y.first;
+                       });
+    L->cta_task.reserve(order.size());
+    for (const auto& o : order) L->cta_task.push_back(o.second);
     L->n_ctas = (int64_t)L->cta_task.size();
     L->cta_map = true;
   }
@@ -651,8 +770,9 @@ pad_status pad_plan(const pad_problem* prob, pad_cache_state* cache, int32_t n_v
     for (int h = 0; h < prob->h_kv; ++h) {
       for (int s = 0; s < L.n_splits[b]; ++s) {
         PadWorkItem it;
-        it.tok_begin = s * L.split_len;
-        it.tok_end = std::min(prefix_len[b], (s + 1) * L.split_len);
+        const int32_t vs = (int32_t)L.vsplit[b];
+        it.tok_begin = s * vs;
+        it.tok_end = std::min(prefix_len[b], (s + 1) * vs);
         it.tok0 = vids[b].prefix_off + it.tok_begin;
         it.first_event = L.ev_first[b];
         it.n_events = L.ev_count[b];
@@ -855,6 +975,8 @@ pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
   info->param_descriptor_bytes = (int32_t)plan->param_image.size();
   info->fused_tail = plan->lay.fused ? 1 : 0;
   info->generation = plan->gen;
+  info->prefix_ctas = (int32_t)(plan->lay.n_ctas > 0 ? plan->lay.n_ctas : plan->lay.n_items);
+  info->max_split_tiles = (plan->lay.split_len + kSplitGranule - 1) / kSplitGranule;
   return PAD_OK;
 }
 

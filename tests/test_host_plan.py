@@ -136,11 +136,21 @@ def test_tc_split_fits_one_wave(padlib, flags, rows_per_cta):
         # each work item gets the row groups its own video needs (a CTA list, not a dense
         # grid of the largest count): one wave unless a single split per (video, kv-head)
         # is already too many
-        ctas = sum(4 * -(-int(P[b]) // sl) * -(-int(Ev[b]) * 7 // rows_per_cta) for b in range(B_))
-        items = sum(4 * -(-int(P[b]) // sl) for b in range(B_))
-        assert info["n_work_items"] == items
-        if sl < int(P.max()):
-            assert ctas <= sms
+        groups = [-(-int(Ev[b]) * 7 // rows_per_cta) for b in range(B_)]
+        if B_ == 1:
+            ctas = sum(4 * -(-int(P[b]) // sl) * groups[b] for b in range(B_))
+            items = sum(4 * -(-int(P[b]) // sl) for b in range(B_))
+            assert info["n_work_items"] == items
+            assert info["prefix_ctas"] == ctas
+            if sl < int(P.max()):
+                assert ctas <= sms
+        else:
+            # a batch of videos: per-video splits, a grid of at most three waves unless one
+            # split per (video, kv-head, row group) is already more
+            base = sum(4 * g for g in groups)
+            assert base <= info["prefix_ctas"] <= max(base, 3 * sms)
+            assert info["max_split_tiles"] == sl // 128
+            assert 4 * B_ <= info["n_work_items"] <= info["prefix_ctas"]
 
 
 def _split_of(P, E, sms=152, flags=0):
@@ -169,6 +179,26 @@ def test_tc_split_leaves_sms_for_the_branch_tasks(padlib):
         sl = _split_of(16384, E, sms=100)
         groups = -(-E * 7 // 128)
         assert 4 * -(-16384 // sl) * groups <= 100
+
+
+def test_batch_of_videos_takes_balanced_splits_over_several_waves(padlib):
+    """16 videos of 4k-16k prefix tokens (the ragged serving batch): one split length sized
+    to one wave leaves CTAs of 82 tiles beside CTAs of 32; per-video splits over two waves,
+    longest first, bring the longest CTA to 32 tiles."""
+    w = synth.ragged_serving()
+    prob = B.make_problem(w.h_q, w.h_kv, w.head_dim, w.page_size, num_sms=152)
+    cache = B.CacheState(w.n_pages, used_pages=w.page_table[w.page_table >= 0])
+    plan = B.pad_plan(prob, cache, w.prefix_len, w.event_video, w.event_len, max_pages=w.max_pages,
+                      workspace=None)
+    info = plan.info()
+    plan.release_new_pages(cache)
+    assert 152 < info["prefix_ctas"] <= 2 * 152
+    assert info["max_split_tiles"] <= 32
+    # the same batch forced to one split length per video when there is a single video
+    w1 = synth.make_workload("one", 3, 28, 4, 128, [16000], [20], [5] * 20, rng=np.random.default_rng(3))
+    p1 = B.pad_plan(prob, B.CacheState(w1.n_pages, used_pages=w1.page_table[w1.page_table >= 0]),
+                    w1.prefix_len, w1.event_video, w1.event_len, max_pages=w1.max_pages, workspace=None)
+    assert p1.info()["prefix_ctas"] <= 152
 
 
 @pytest.mark.parametrize("case,status", [

@@ -176,25 +176,27 @@ def test_plan_just_under_the_static_limit(padlib):
     matches the workspace path of the same step."""
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
-    # videos of 64 events x 7 q-heads per kv-head with short prefixes (one split each): the
-    # partial states grow by ~0.9 MiB per video; take the most videos that still fit
+    # videos of E events x 7 q-heads per kv-head with short prefixes: the partial states grow
+    # with the videos, the events and the splits the planner gives them; take the largest
+    # scratch that still fits
     prob = B.make_problem(28, 4, 128, num_sms=152)
     best = None
-    for nv in range(1, 40):
-        ev = np.repeat(np.arange(nv, dtype=np.int32), 64)
-        ws = B.pad_workspace_size(prob, np.full(nv, 300, np.int32), ev)
-        if ws > 16 << 20:
-            break
-        best = (nv, ws)
-    assert best is not None and best[1] > 15 << 20
+    for nv in range(1, 24):
+        for E in (64, 56, 48, 40, 32):
+            ev = np.repeat(np.arange(nv, dtype=np.int32), E)
+            ws = B.pad_workspace_size(prob, np.full(nv, 300, np.int32), ev)
+            if ws <= 16 << 20 and (best is None or ws > best[2]):
+                best = (nv, E, ws)
+    assert best is not None and best[2] > 15 << 20
+    nv, E = best[0], best[1]
     rng = np.random.default_rng(11)
-    w = synth.make_workload("near_limit", 11, 28, 4, 128, [300] * best[0], [64] * best[0],
-                            rng.integers(0, 40, size=64 * best[0]), rng=rng)
+    w = synth.make_workload("near_limit", 11, 28, 4, 128, [300] * nv, [E] * nv,
+                            rng.integers(0, 40, size=E * nv), rng=rng)
     db = DeviceBatch(w, num_sms=152)
     plan = db.run_step()
     torch.cuda.synchronize()
     B.pad_device_status(plan)
-    assert plan.info()["workspace_bytes"] == best[1]
+    assert plan.info()["workspace_bytes"] == best[2]
     ref_o, ref_l = db.out.clone(), db.lse.clone()
     db.release_new_pages(plan)
     hplan = B.pad_plan(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
