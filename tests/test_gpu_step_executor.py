@@ -162,6 +162,48 @@ def test_two_batches_in_flight(mapped):
         assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
 
 
+@pytest.mark.parametrize("mapped", [True, False])
+def test_two_steps_of_one_executor_in_flight(mapped):
+    """Two consecutive steps of one generation loop enqueued back to back on one executor
+    (their own host buffers, no wait in between): the second step's inputs reach the device
+    only after the first step's kernels have read theirs, so both steps' outputs, the pools
+    and the page table equal the same two steps run one after the other."""
+    w = synth.make_workload("two", 21, 28, 4, 128, [3000], [6], [15, 16, 31, 0, 47, 8],
+                            rng=np.random.default_rng(21))
+    rng = np.random.default_rng(5)
+    ins = [[torch.from_numpy(rng.standard_normal(t.shape).astype(np.float32)).to(torch.bfloat16)
+            for t in (w.q, w.k_new, w.v_new)] for _ in range(2)]
+    # reference: two serial steps
+    a = DeviceBatch(w)
+    sa = _native(a, w, release_pages=False, mapped_host_io=mapped)
+    ref = []
+    for k in range(2):
+        hq, hk, hv = (x.pin_memory() for x in ins[k])
+        ho = torch.empty(a.out.shape, dtype=a.out.dtype).pin_memory()
+        hl = torch.empty(a.lse.shape, dtype=torch.float32).pin_memory()
+        sa.run_host(hq, hk, hv, ho, hl)
+        ref.append((ho.clone(), hl.clone()))
+        sa.event_len += 1
+    # the same two steps in flight
+    b = DeviceBatch(w)
+    sb = _native(b, w, release_pages=False, mapped_host_io=mapped)
+    outs = []
+    for k in range(2):
+        hq, hk, hv = (x.pin_memory() for x in ins[k])
+        ho = torch.full(b.out.shape, float("nan"), dtype=b.out.dtype).pin_memory()
+        hl = torch.full(b.lse.shape, float("nan"), dtype=torch.float32).pin_memory()
+        sb.enqueue_host(hq, hk, hv, ho, hl)
+        outs.append((hq, hk, hv, ho, hl))
+        sb.event_len += 1
+    sb.wait()
+    torch.cuda.synchronize()
+    for k in range(2):
+        assert torch.equal(outs[k][3], ref[k][0]) and torch.equal(outs[k][4], ref[k][1])
+    assert torch.equal(a.k_pool.view(torch.int16), b.k_pool.view(torch.int16))
+    assert torch.equal(a.v_pool.view(torch.int16), b.v_pool.view(torch.int16))
+    assert torch.equal(a.page_table, b.page_table)
+
+
 def test_run_host_mapped_io_falls_back_on_pageable_buffers():
     """A pageable host buffer fails the mapped check: that call takes the copy path."""
     w = synth.tiny()
