@@ -39,9 +39,9 @@
 namespace pad {
 namespace bm {
 
-constexpr int kThreads = 256;                 // threads of one task
+constexpr int kThreads = 256;                 // threads of one task (the default of 8 warps)
 constexpr int kWarps = kThreads / 32;
-constexpr int kKeys = 16 * kWarps;            // branch keys staged per round
+constexpr int kKeys = 16 * kWarps;            // branch keys staged per round, at most
 constexpr int kMaxChunk = 64;                 // prefix splits merged per staged chunk
 constexpr float kNegInf = -__builtin_huge_valf();
 
@@ -64,13 +64,17 @@ struct Head {
   alignas(16) float ob[16][D];                // merged numerator (read as float4)
   float M[16], L[16], a[16];
 };
-template <int D>
-__host__ __device__ constexpr size_t kv_bytes(int nkr, int G) {
-  return align16(max_sz((size_t)2 * nkr * Head<D>::LD * 2, (size_t)kWarps * G * D * 4));
+// Keys staged per round by a task of NW warps (16 per warp), for a launch's branch_rows.
+__host__ __device__ constexpr int round_keys(int branch_rows, int NW) {
+  return branch_rows < 16 * NW ? branch_rows : 16 * NW;
 }
-template <int D>
-__host__ __device__ constexpr size_t smem_bytes(int nkr, int G, int sch) {
-  return align16(sizeof(Head<D>)) + kv_bytes<D>(nkr, G) + align16((size_t)G * sch * 8) +
+template <int D, int NW = kWarps>
+__host__ __device__ constexpr size_t kv_bytes(int nkr, int G) {
+  return align16(max_sz((size_t)2 * nkr * Head<D>::LD * 2, (size_t)NW * G * D * 4));
+}
+template <int D, int NW = kWarps>
+__host__ __device__ constexpr size_t smem_bytes(int branch_rows, int G, int sch) {
+  return align16(sizeof(Head<D>)) + kv_bytes<D, NW>(round_keys(branch_rows, NW), G) + align16((size_t)G * sch * 8) +
          (size_t)sch * G * D * 4;
 }
 
@@ -159,14 +163,15 @@ struct SyncNamed {
 // partials cannot be read (then only the status word is written).
 // CAUSAL: 0 = the method's own-branch keys, 1 = the causal-attention key list, 2 = read
 // KParams::causal at run time (separate instantiations keep the common one lean).
-template <int D, bool ROPE, int CAUSAL, class Sync, class Ready>
+template <int D, bool ROPE, int CAUSAL, int NW = kWarps, class Sync, class Ready>
 __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* __restrict__ q,
                                          const __nv_bfloat16* __restrict__ kpool,
                                          const __nv_bfloat16* __restrict__ vpool, void* __restrict__ out,
                                          float* __restrict__ lse, int e, int kvh, int tid,
                                          unsigned char* smem, int sch, const Sync& sy, bool early,
                                          Ready partials_ready) {
-  constexpr int NT = kThreads;
+  static_assert(NW >= 1 && NW <= kWarps, "warps per task");
+  constexpr int NT = 32 * NW;
   constexpr int CH = D / 8;                   // 16-byte pieces of a bf16 row
   constexpr int KS = D / 16;                  // k-steps of S = Q K^T
   constexpr int OT = D / 8;                   // n8 tiles of O
@@ -174,12 +179,12 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   constexpr int LD = Head<D>::LD;
   Head<D>& S = *reinterpret_cast<Head<D>*>(smem);
   const int G = p.group;
-  const int nkr = p.branch_rows;              // keys per round (multiple of 16, <= kKeys)
+  const int nkr = round_keys(p.branch_rows, NW);  // keys per round (multiple of 16, <= 16 NW)
   unsigned char* kv_raw = smem + align16(sizeof(Head<D>));
   __nv_bfloat16 (*sK)[LD] = reinterpret_cast<__nv_bfloat16 (*)[LD]>(kv_raw);
   __nv_bfloat16 (*sV)[LD] = reinterpret_cast<__nv_bfloat16 (*)[LD]>(kv_raw + (size_t)nkr * LD * 2);
   float* wo = reinterpret_cast<float*>(kv_raw);  // [warp][G][d] after the branch pass
-  float2* sml = reinterpret_cast<float2*>(kv_raw + kv_bytes<D>(nkr, G));
+  float2* sml = reinterpret_cast<float2*>(kv_raw + kv_bytes<D, NW>(nkr, G));
   float* spo = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sml) + align16((size_t)G * sch * 8));
 
   const int warp = tid >> 5, lane = tid & 31;
@@ -461,13 +466,13 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   sy.sync();
 
   // ---------------- a5: the warp states, then the prefix splits in chunks of `sch`
-  for (int g = warp; g < G; g += kWarps) {
-    const float mw = lane < kWarps ? S.wm[lane][g] : kNegInf;
+  for (int g = warp; g < G; g += NW) {
+    const float mw = lane < NW ? S.wm[lane][g] : kNegInf;
     float mx = warp_max(mw);
     if (mx == kNegInf) mx = 0.f;              // no key of the branch passed its bounds check
-    const float wgt = lane < kWarps ? ex2(mw - mx) : 0.f;
-    const float sum = warp_sum(lane < kWarps ? S.wl[lane][g] * wgt : 0.f);
-    if (lane < kWarps) S.sc[g][lane] = wgt;
+    const float wgt = lane < NW ? ex2(mw - mx) : 0.f;
+    const float sum = warp_sum(lane < NW ? S.wl[lane][g] * wgt : 0.f);
+    if (lane < NW) S.sc[g][lane] = wgt;
     if (lane == 0) {
       S.M[g] = mx;
       S.L[g] = sum;
@@ -478,7 +483,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     const int g = i / D4, d4 = i - g * D4;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NW; ++w) {
       const float c = S.sc[g][w];
       const float4 v = reinterpret_cast<const float4*>(wo)[(w * G + g) * D4 + d4];
       acc.x = fmaf(c, v.x, acc.x);
@@ -510,7 +515,7 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
     cp_async_wait<0>();
     sy.sync();
     // row statistics, one warp per row, lanes over splits
-    for (int g = warp; g < G; g += kWarps) {
+    for (int g = warp; g < G; g += NW) {
       float mx = kNegInf;
       for (int sl = lane; sl < nch; sl += 32) mx = fmaxf(mx, sml[g * sch + sl].x);
       mx = warp_max(mx);

@@ -516,8 +516,10 @@ __global__ void __launch_bounds__(128) prefix_mma_kernel(const __grid_constant__
 // programmatic dependent launch: its griddepcontrol.wait covers the prefix grid, so the
 // split partials are complete once it returns.
 // ---------------------------------------------------------------------------
-template <int D, bool ROPE, int CAUSAL>
-__global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __grid_constant__ KParams p,
+// NW warps per task: 8 (two CTAs per SM) by default, 4 (three per SM) when the step has more
+// than two waves of tasks, so that more of its latency-bound tasks are in flight at once.
+template <int D, bool ROPE, int CAUSAL, int NW>
+__global__ void __launch_bounds__(32 * NW, NW == bm::kWarps ? 2 : 3) branch_merge_kernel(const __grid_constant__ KParams p,
                                                                     const __nv_bfloat16* __restrict__ q,
                                                                     const __nv_bfloat16* __restrict__ kpool,
                                                                     const __nv_bfloat16* __restrict__ vpool,
@@ -531,8 +533,8 @@ __global__ void __launch_bounds__(bm::kThreads, 2) branch_merge_kernel(const __g
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int e = blockIdx.x / p.h_kv;
   const int kvh = blockIdx.x - e * p.h_kv;
-  bm::run_task<D, ROPE, CAUSAL>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch, bm::SyncCta{}, true,
-                  [] { return true; });
+  bm::run_task<D, ROPE, CAUSAL, NW>(p, q, kpool, vpool, out, lse, e, kvh, (int)threadIdx.x, bm_raw, sch,
+                                     bm::SyncCta{}, true, [] { return true; });
 }
 
 // Step inputs from page-locked, device-mapped host memory into device memory (the
@@ -667,36 +669,40 @@ cudaError_t launch_prefix_mma(const KParams& p, int max_rows, const void* q, con
 
 // Split partials merged per staged chunk: as many as a shared-memory budget allows next to
 // the branch staging.
-template <int D>
+template <int D, int NW = bm::kWarps>
 int bm_chunk(const KParams& p, size_t budget) {
   const int G = p.group;
-  const size_t fixed = bm::align16(sizeof(bm::Head<D>)) + bm::kv_bytes<D>(p.branch_rows, G) + 16;
+  const size_t fixed =
+      bm::align16(sizeof(bm::Head<D>)) + bm::kv_bytes<D, NW>(bm::round_keys(p.branch_rows, NW), G) + 16;
   const size_t per_split = (size_t)G * D * sizeof(float) + sizeof(float2);
   int sch = fixed + per_split <= budget ? (int)((budget - fixed) / per_split) : 1;
   if (p.max_splits > 0 && sch > p.max_splits) sch = p.max_splits;
   return sch < 1 ? 1 : (sch > bm::kMaxChunk ? bm::kMaxChunk : sch);
 }
-// The standalone kernel: a grid of more CTAs than SMs keeps two per SM.
+// The standalone kernel: a grid of more CTAs than SMs keeps two per SM (8 warps each), one
+// of more than two waves three (4 warps each).
+inline bool bm_narrow(const KParams& p) { return (int64_t)p.n_events * p.h_kv > 2 * (int64_t)p.n_sms; }
 inline size_t n_cta_budget(const KParams& p) {
+  if (bm_narrow(p)) return 74 * 1024;
   return p.n_events * p.h_kv > p.n_sms ? 110 * 1024 : 200 * 1024;
 }
 
-template <int D>
-static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
-                             void* out, float* lse, bool pdl, cudaStream_t s) {
+template <int D, int NW>
+static cudaError_t launch_bm_nw(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
+                                void* out, float* lse, bool pdl, cudaStream_t s) {
   const int G = p.group;
   const int nkr = p.branch_rows;
   if (nkr <= 0 || nkr > bm::kKeys || nkr % 16 != 0) return cudaErrorInvalidValue;
-  const int sch = bm_chunk<D>(p, n_cta_budget(p));
-  const size_t smem = bm::smem_bytes<D>(nkr, G, sch);
+  const int sch = bm_chunk<D, NW>(p, n_cta_budget(p));
+  const size_t smem = bm::smem_bytes<D, NW>(nkr, G, sch);
   constexpr int kMaxSmem = 227 * 1024;
   if (smem > (size_t)kMaxSmem) return cudaErrorInvalidValue;
   static bool configured[64] = {};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !configured[dev]) {
-    for (auto fn : {branch_merge_kernel<D, false, 0>, branch_merge_kernel<D, true, 0>, branch_merge_kernel<D, false, 1>,
-                    branch_merge_kernel<D, true, 1>}) {
+    for (auto fn : {branch_merge_kernel<D, false, 0, NW>, branch_merge_kernel<D, true, 0, NW>,
+                    branch_merge_kernel<D, false, 1, NW>, branch_merge_kernel<D, true, 1, NW>}) {
       cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
       if (e != cudaSuccess) return e;
     }
@@ -704,7 +710,7 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_events * p.h_kv);
-  cfg.blockDim = dim3(bm::kThreads);
+  cfg.blockDim = dim3(32 * NW);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -712,11 +718,17 @@ static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool
   attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  auto fn = p.causal ? (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 1> : branch_merge_kernel<D, false, 1>)
-                     : (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 0> : branch_merge_kernel<D, false, 0>);
+  auto fn = p.causal ? (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 1, NW> : branch_merge_kernel<D, false, 1, NW>)
+                     : (p.rope_cs != nullptr ? branch_merge_kernel<D, true, 0, NW> : branch_merge_kernel<D, false, 0, NW>);
   return cudaLaunchKernelEx(&cfg, fn, p, static_cast<const __nv_bfloat16*>(q),
                             static_cast<const __nv_bfloat16*>(k_pool), static_cast<const __nv_bfloat16*>(v_pool),
                             out, lse, sch);
+}
+template <int D>
+static cudaError_t launch_bm(const KParams& p, const void* q, const void* k_pool, const void* v_pool,
+                             void* out, float* lse, bool pdl, cudaStream_t s) {
+  return bm_narrow(p) ? launch_bm_nw<D, 4>(p, q, k_pool, v_pool, out, lse, pdl, s)
+                      : launch_bm_nw<D, bm::kWarps>(p, q, k_pool, v_pool, out, lse, pdl, s);
 }
 
 cudaError_t launch_branch_merge(const KParams& p, const void* q, const void* k_pool,
