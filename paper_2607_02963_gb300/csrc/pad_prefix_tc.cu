@@ -16,12 +16,14 @@
 //   warp 2      TMEM allocator (512 columns) and deallocator; its lane 0 issues
 //               O += P V with P read back from TMEM
 //   warp 3      TMA producer of V tiles (refilled once the P.V of the tile completed)
-//   warps 4-11  softmax: two warps per 32-row lane quarter, each taking 64 of the
-//               tile's 128 columns for one query row per thread; they meet once per
-//               tile to combine their partial row maxima (an mbarrier, so the wait is
-//               bounded); online max and sum in base 2, P written as packed bf16 over
-//               the S columns already read, lazy rescaling of O (only when a row
-//               maximum grows by more than 2^8)
+//   warps 4-11  softmax: two warps per 32-row lane quarter.  Decode: each warp takes 16
+//               of the quarter's rows and all 128 columns of a tile (two rows per
+//               thread, a row shared by a quad of lanes), so the warps never meet.
+//               Whole-sequence prefill: each takes 64 of the columns for one row per
+//               thread, and the two meet once per tile to combine their partial row
+//               maxima (an mbarrier, so the wait is bounded).  Online max and sum in
+//               base 2, P written as packed bf16 over the S columns already read, lazy
+//               rescaling of O (only when a row maximum grows by more than 2^8)
 //
 // Every MMA has N = 128 (S: 128 tokens; P.V: 128 head-dim columns), the size at
 // which one tcgen05.mma carries as much tensor work as it costs to issue.
@@ -64,7 +66,7 @@ using namespace tc;
 constexpr int kD = 128;
 constexpr int kBN = 128;       // prefix tokens per K/V tile
 constexpr int kStages = 3;
-constexpr int kPSlots = 2;     // P slots in TMEM
+constexpr int kSBuf = 3;       // S buffers in TMEM
 constexpr int kThreads = 384;
 constexpr uint32_t kHalfBytes = kBN * 128;         // 128 tokens x 64 bf16 = 16 KB
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;    // one K (or V) tile: 32 KB
@@ -74,43 +76,26 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kQTileBytes;
 constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStages * kTileBytes;
-constexpr uint32_t kOffX = kOffBar + 256;               // the key halves' (m, l): [2][2][128] fp32
+constexpr uint32_t kOffX = kOffBar + 256;               // prefill: partial row maxima [2][2][128] fp32
 constexpr uint32_t kSmemBytes = kOffX + 2 * 2 * 128 * 4;
 constexpr int kOStage = kD + 4;                       // fp32 row stride of the O staging rows
 static_assert((128 * kOStage + 128) * 4 <= kStages * kTileBytes, "O staging (and 1 / l) fits the K stages");
 constexpr uint32_t kTmemCols = 512;
-// TMEM: S of the current tile (fp32, 128 columns), P of two tiles (packed bf16, 64
-// columns each: tokens 0-63, then 64-127) and the P.V accumulators of the two key halves
-// of every tile (tokens 0-63: softmax warps 4-7, 64-127: warps 8-11), which keep separate
-// softmax states and are merged once in the epilogue.
-constexpr uint32_t kColS = 0;
-constexpr uint32_t kColP = 128;
-constexpr uint32_t kColOA = 256;
-constexpr uint32_t kColOB = 384;
+constexpr uint32_t kColO = 384;
 constexpr float kLazyRescale = 8.0f;                  // log2 units
-#ifdef PAD_MUFU_PAIRS
-constexpr int kMufuPairs = PAD_MUFU_PAIRS;
-#else
-// Exponential pairs (of every 16) on the MUFU unit; the rest use exp2_poly2 on the FMA
-// pipe.  Measured on GB300, the softmax here is latency-bound rather than MUFU-bound, so
-// the extra polynomial instructions cost more than they save: all 16 go to MUFU.
-constexpr int kMufuPairs = 16;
-#endif
 static_assert(kSmemBytes <= 232448, "fits the 227 KB opt-in shared memory");
 
 struct TcBars {
   uint64_t kfull[kStages];
   uint64_t vfull[kStages];
-  uint64_t kfree[kStages];    // S of the tile in this K stage has completed
-  uint64_t pvfree[kStages];   // P.V of the tile in this V stage has completed
-  uint64_t sfull;             // S of the current tile has completed
-  uint64_t sfree;             // every softmax warp has loaded it (8 warp arrivals)
-  uint64_t pfull[kPSlots];    // P of the tile in this slot is written (8 warp arrivals)
+  uint64_t pvfree[kStages];   // P.V of the tile in this stage / S buffer has completed
+  uint64_t sfull[kSBuf];      // S of the tile in this buffer has completed (also frees its K stage)
+  uint64_t pfull[kSBuf];      // P of the tile in this buffer is written (8 warp arrivals)
   uint64_t drain_s;           // every S MMA has completed (S issuer)
   uint64_t drain_pv;          // every P.V MMA has completed (P.V issuer)
   uint64_t qready;            // Q staged in shared memory (8 warp arrivals)
   uint64_t tdone;             // the softmax warps are done with TMEM (8 warp arrivals)
-  uint64_t xchg[4];           // the two softmax warps of a lane quarter met (64 thread arrivals)
+  uint64_t xchg[4];           // prefill: the two softmax warps of a lane quarter met (64 arrivals)
   uint64_t gen;               // the plan's generation, for the status word
   uint32_t tmem_base;
   int32_t abort;
@@ -120,18 +105,17 @@ static_assert(sizeof(TcBars) <= 256, "barrier block fits its slot");
 constexpr uint32_t kIdescS = make_idesc(128, kBN, false);   // S = Q K^T: B = K tile, K-major
 constexpr uint32_t kIdescPV = make_idesc(128, kD, true);    // O += P V: B = V tile, N(=d)-major
 
-// Maximum of the raw scores of one softmax warp's 64 columns (eight chains of three-input
-// max); with MASK, columns at or past `valid` are left out.
-// Visible columns of a warp's 64 (used on the MASK path only): the first `valid` ones (the
-// split's end), or the set bits of `keep` (also the self G-token mask).
-struct ColsValid {
-  int valid;
-  __device__ bool vis(int c) const { return c < valid; }
-};
-struct ColsBits {
+// The prefill path splits a 128-row group by columns: the two warps of a lane quarter take
+// 64 columns each of its 32 rows (one row per thread) and meet on every tile to share their
+// row maxima; one causal mask per thread keeps it below the register limit, where two rows'
+// masks per thread spilled.
+// Visible columns of a warp's 64 (used on the MASK path only): the set bits of `keep`.
+struct HalfBits {
   uint64_t keep;
   __device__ bool vis(int c) const { return (keep >> c) & 1ull; }
 };
+// Maximum of the raw scores of one softmax warp's 64 columns (eight chains of three-input
+// max); with MASK, columns the row does not see are left out.
 template <bool MASK, class Cols>
 __device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], Cols cols) {
   float mxa[8];
@@ -153,16 +137,10 @@ __device__ __forceinline__ float half_row_max(const uint32_t (&sr)[2][32], Cols 
 }
 
 // P = 2^(s * scale_log2 - m) for one softmax warp's 64 columns, written as packed bf16
-// (two per column) to the 32 TMEM columns at taddr_p; returns the fp32 sum of the P values.
+// over the S columns already read; returns the fp32 sum of the P values.
 template <bool MASK, class Cols>
 __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
                                               float m, uint32_t taddr_p);
-
-// Bounded wait of this kernel: gives up on the CTA's abort flag or after the time limit.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
-                                          PadDevHeader* hdr, int where) {
-  return mbar_wait_b(bar, parity, &bars->abort, bars->gen, hdr, where);
-}
 
 template <bool MASK, class Cols>
 __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols cols, float sl2,
@@ -177,15 +155,7 @@ __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols 
       const int col = 32 * c + 2 * i;
       const uint64_t x =
           ffma2(f2pack(__uint_as_float(sr[c][2 * i]), __uint_as_float(sr[c][2 * i + 1])), sc2, nm2);
-      float p0, p1;
-      if (i < kMufuPairs) {
-        p0 = ex2(f2lo(x));
-        p1 = ex2(f2hi(x));
-      } else {
-        const uint64_t e = exp2_poly2(x);
-        p0 = f2lo(e);
-        p1 = f2hi(e);
-      }
+      float p0 = ex2(f2lo(x)), p1 = ex2(f2hi(x));
       if (MASK) {
         if (!cols.vis(col)) p0 = 0.f;
         if (!cols.vis(col + 1)) p1 = 0.f;
@@ -198,6 +168,104 @@ __device__ __forceinline__ float half_row_exp(const uint32_t (&sr)[2][32], Cols 
   }
   const uint64_t ls = fadd2(fadd2(lacc[0], lacc[1]), fadd2(lacc[2], lacc[3]));
   return f2lo(ls) + f2hi(ls);
+}
+
+
+// The softmax warps split a 128-row group by rows: warp w of lane quarter q takes the 16
+// rows 32q + 16h .. +15 (h = (w-4)/4) and every column of a tile, through the 16-lane TMEM
+// shapes, so no row is shared by two warps and they never have to meet.  Thread t holds rows
+// a = t/4 and a + 8 of the warp's 16 and, in each 8-column chunk, columns 2(t%4) and
+// 2(t%4) + 1: s[x][4k..4k+3] = (a, c), (a, c+1), (a+8, c), (a+8, c+1) with
+// c = 64x + 8k + 2(t%4).  A row's maximum and sum are shared by the four threads of its
+// quad (lanes 4(t/4) .. +3).
+// Visible columns of one row: the first `valid`, or the set bits of a 128-column mask.
+struct ColsValid {
+  int valid;
+  __device__ bool vis(int c) const { return c < valid; }
+};
+struct ColsBits {
+  uint64_t lo, hi;  // columns 0-63, 64-127
+  __device__ bool vis(int c) const { return ((c < 64 ? lo >> c : hi >> (c - 64)) & 1ull) != 0; }
+};
+__device__ __forceinline__ float quad_max(float v) {
+  v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+  return fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+}
+__device__ __forceinline__ float quad_sum(float v) {
+  v += __shfl_xor_sync(0xffffffffu, v, 1);
+  return v + __shfl_xor_sync(0xffffffffu, v, 2);
+}
+
+// Maxima of the raw scores of this thread's two rows over all 128 columns (with MASK,
+// columns a row does not see are left out), reduced over the quad.
+template <bool MASK, class CA, class CB>
+__device__ __forceinline__ void rows_max(const uint32_t (&s)[2][32], int cq, CA ca, CB cb, float& ma, float& mb) {
+  float xa[4], xb[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) xa[u] = xb[u] = -__builtin_huge_valf();
+#pragma unroll
+  for (int x = 0; x < 2; ++x)
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int c = 64 * x + 8 * k + cq;
+      float a0 = __uint_as_float(s[x][4 * k]), a1 = __uint_as_float(s[x][4 * k + 1]);
+      float b0 = __uint_as_float(s[x][4 * k + 2]), b1 = __uint_as_float(s[x][4 * k + 3]);
+      if (MASK) {
+        if (!ca.vis(c)) a0 = -__builtin_huge_valf();
+        if (!ca.vis(c + 1)) a1 = -__builtin_huge_valf();
+        if (!cb.vis(c)) b0 = -__builtin_huge_valf();
+        if (!cb.vis(c + 1)) b1 = -__builtin_huge_valf();
+      }
+      xa[k & 3] = max3f(xa[k & 3], a0, a1);
+      xb[k & 3] = max3f(xb[k & 3], b0, b1);
+    }
+  ma = quad_max(fmaxf(fmaxf(xa[0], xa[1]), fmaxf(xa[2], xa[3])));
+  mb = quad_max(fmaxf(fmaxf(xb[0], xb[1]), fmaxf(xb[2], xb[3])));
+}
+
+// P = 2^(s * scale_log2 - m) of this thread's two rows, written as packed bf16 (two tokens
+// per column: column 4k + t%4 of chunk k holds tokens 8k + 2(t%4) and + 1, the layout the
+// P.V MMA reads) to the 64 TMEM columns at taddr_p; adds this thread's share of each row's
+// sum of P to la / lb.
+template <bool MASK, class CA, class CB>
+__device__ __forceinline__ void rows_exp(const uint32_t (&s)[2][32], int cq, CA ca, CB cb, float sl2, float ma,
+                                         float mb, uint32_t taddr_p, float& la, float& lb) {
+  const uint64_t sc2 = f2pack(sl2, sl2), na = f2pack(-ma, -ma), nb = f2pack(-mb, -mb);
+  uint64_t acc_a[2] = {0ull, 0ull}, acc_b[2] = {0ull, 0ull};
+#pragma unroll
+  for (int x = 0; x < 2; ++x) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int c = 64 * x + 8 * k + cq;
+      const uint64_t ya =
+          ffma2(f2pack(__uint_as_float(s[x][4 * k]), __uint_as_float(s[x][4 * k + 1])), sc2, na);
+      const uint64_t yb =
+          ffma2(f2pack(__uint_as_float(s[x][4 * k + 2]), __uint_as_float(s[x][4 * k + 3])), sc2, nb);
+      float a0 = ex2(f2lo(ya)), a1 = ex2(f2hi(ya)), b0 = ex2(f2lo(yb)), b1 = ex2(f2hi(yb));
+      if (MASK) {
+        if (!ca.vis(c)) a0 = 0.f;
+        if (!ca.vis(c + 1)) a1 = 0.f;
+        if (!cb.vis(c)) b0 = 0.f;
+        if (!cb.vis(c + 1)) b1 = 0.f;
+      }
+      acc_a[k & 1] = fadd2(acc_a[k & 1], f2pack(a0, a1));
+      acc_b[k & 1] = fadd2(acc_b[k & 1], f2pack(b0, b1));
+      pk[2 * k] = pack_bf16(a0, a1);
+      pk[2 * k + 1] = pack_bf16(b0, b1);
+    }
+    // P columns 32x + 4k + t%4 (tokens 64x + 8k + 2(t%4), + 1)
+    tmem_st16x128_x8(taddr_p + 32 * x, pk);
+  }
+  const uint64_t sa = fadd2(acc_a[0], acc_a[1]), sb = fadd2(acc_b[0], acc_b[1]);
+  la += f2lo(sa) + f2hi(sa);
+  lb += f2lo(sb) + f2hi(sb);
+}
+
+// Bounded wait of this kernel: gives up on the CTA's abort flag or after the time limit.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, TcBars* bars,
+                                          PadDevHeader* hdr, int where) {
+  return mbar_wait_b(bar, parity, &bars->abort, bars->gen, hdr, where);
 }
 
 
@@ -390,12 +458,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&bars->kfull[s], 1);
         mbar_init(&bars->vfull[s], 1);
       }
-      mbar_init(&bars->kfree[s], 1);
       mbar_init(&bars->pvfree[s], 1);
     }
-    mbar_init(&bars->sfull, 1);
-    mbar_init(&bars->sfree, 8);     // one arrival per softmax warp
-    for (int b = 0; b < kPSlots; ++b) {
+    for (int b = 0; b < kSBuf; ++b) {
+      mbar_init(&bars->sfull[b], 1);
       mbar_init(&bars->pfull[b], 8);  // one arrival per softmax warp
     }
     mbar_init(&bars->drain_s, 1);
@@ -438,8 +504,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = 1; t < n_tiles && ok; ++t) {
         const int s = t % kStages;
         if (t >= kStages) {
-          // K stage: S of tile t-3 done (kfree[s], completion t/3 - 1); V stage: its P.V done
-          uint64_t* freed = isK ? &bars->kfree[s] : &bars->pvfree[s];
+          // K stage: S of tile t-3 done (sfull[s], completion t/3 - 1); V stage: its P.V done
+          uint64_t* freed = isK ? &bars->sfull[s] : &bars->pvfree[s];
           ok = mbar_wait(freed, (uint32_t)((t / kStages - 1) & 1), bars, p.header, isK ? 1 : 2);
           if (!ok) break;
         }
@@ -478,22 +544,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (warp == 1) {
         ok = mbar_wait(&bars->qready, 0u, bars, p.header, 11);
         for (int t = 0; t < n_tiles && ok; ++t) {
-          const uint32_t s = (uint32_t)(t % kStages);  // K stage
+          const uint32_t s = (uint32_t)(t % kStages);
           ok = mbar_wait(&bars->kfull[s], (uint32_t)((t / kStages) & 1), bars, p.header, 3);
           if (!ok) break;
-          // the S buffer holds S of tile t-1 until every softmax warp has loaded it
-          if (t >= 1) ok = mbar_wait(&bars->sfree, (uint32_t)((t - 1) & 1), bars, p.header, 12);
+          // S buffer s holds P of tile t-3 until that P.V completes
+          if (t >= kStages)
+            ok = mbar_wait(&bars->pvfree[s], (uint32_t)((t / kStages - 1) & 1), bars, p.header, 6);
           if (!ok) break;
           fence_after();
-          const uint32_t d = tmem + kColS;
+          const uint32_t d = tmem + 128u * s;
           const uint64_t kb = dK + (s * kTileBytes >> 4);
 #pragma unroll
           for (int kk = 0; kk < kD / 16; ++kk) {
             const uint32_t off = (uint32_t)(kk >> 2) * kQHalfBytes + (uint32_t)(kk & 3) * 32;
             mma_ss(d, dQ + (off >> 4), kb + (off >> 4), kIdescS, kk > 0 ? 1u : 0u);
           }
-          mma_commit(&bars->sfull);
-          mma_commit(&bars->kfree[s]);
+          mma_commit(&bars->sfull[s]);
         }
         mma_commit(&bars->drain_s);
         drain_wait(&bars->drain_s, 0u);
@@ -502,17 +568,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t s = (uint32_t)(j % kStages);
           ok = mbar_wait(&bars->vfull[s], (uint32_t)((j / kStages) & 1), bars, p.header, 4);
           if (!ok) break;
-          ok = mbar_wait(&bars->pfull[j % kPSlots], (uint32_t)((j / kPSlots) & 1), bars, p.header, 5);
+          ok = mbar_wait(&bars->pfull[s], (uint32_t)((j / kSBuf) & 1), bars, p.header, 5);
           if (!ok) break;
           fence_after();
-          const uint32_t a = tmem + kColP + 64u * (uint32_t)(j % kPSlots);
+          const uint32_t a = tmem + 128u * s;
           const uint64_t vb = dV + (s * kTileBytes >> 4);
           const uint32_t acc0 = j > 0 ? 1u : 0u;
-          // tokens 0-63 of the tile into the first key half's O, 64-127 into the second's
 #pragma unroll
           for (int kk = 0; kk < kBN / 16; ++kk)
-            mma_ts(tmem + (kk < 4 ? kColOA : kColOB), a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
-                   (kk & 3) > 0 ? 1u : acc0);
+            mma_ts(tmem + kColO, a + kk * 8, vb + ((uint32_t)kk * 2048 >> 4), kIdescPV,
+                   kk > 0 ? 1u : acc0);
           mma_commit(&bars->pvfree[s]);
         }
         // O is final once every P.V has completed
@@ -523,7 +588,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= 4) {
     // ------------------------------------------------------------ softmax
     const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31 (query rows)
-    const int half = (warp - 4) >> 2;          // columns 64*half .. +63 of every tile
+    const int half = (warp - 4) >> 2;          // rows 16*half .. +15 of the quarter
     const int lane_base = 32 * quarter;
     // Q rows (loaded in the prologue) into the 128-byte-swizzled K-major layout the
     // MMA reads: row r, 16-byte chunk cc of half h at h*16K + r*128 + ((cc ^ (r & 7)) << 4).
@@ -582,177 +647,235 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncwarp();
     if (lane == 0) mbar_arrive(&bars->qready);
-    const int row = lane_base + lane;
-    const int grow = row0 + row;
-    const bool warp_active = (row0 + lane_base) < R;  // same for both warps of the quarter
-    const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
-    const uint32_t col0 = 64u * (uint32_t)half;       // first S column (token) of this warp
-    const uint32_t colO = half ? kColOB : kColOA;     // this key half's P.V accumulator
-    float* xmax = reinterpret_cast<float*>(smem + kOffX);  // [half][m | l][row], epilogue
-    uint64_t* xbar = &bars->xchg[quarter];
     const float sl2 = p.scale_log2;
-    float m_run = -__builtin_huge_valf(), l_run = 0.f;
     bool ok = true;
-    uint32_t r[32];
-    // self G-token mask: the video's planning tokens G^1..G^K (prefix-relative [g_lo, g_hi))
-    // PREFILL: this row's token and the first token of its branch (-1 in the prefix)
-    int pf_p = 0, pf_bs = -1;
-    if (PREFILL && grow < R) {
-      pf_p = it.first_event + grow / p.group;
-      pf_bs = pf_p >= p.pf_S ? pf_branch_start(p, pf_p) : -1;
-    }
-    int g_lo = 0, g_hi = 0;
-    if (GSELF) {
-      const PadVideoDesc vdg = plan_videos(p)[plan_events(p)[it.first_event].video];
-      if (vdg.n_planning > 0) {
-        g_lo = vdg.prefix_len - 1 - vdg.n_planning;
-        g_hi = vdg.prefix_len - 1;
+    // O leaves through shared memory: rows are staged in the K stages (idle once every MMA
+    // has completed) at a padded stride, then written one 512-byte row per warp instruction.
+    float* ostage = reinterpret_cast<float*>(smem + kOffK);
+    float* inv_row = ostage + 128 * kOStage;  // PREFILL: 1 / l of each row for the write-out
+    if constexpr (PREFILL) {
+      // columns 64*half .. +63 of every tile, one query row per thread
+      const int row = lane_base + lane;
+      const int grow = row0 + row;
+      const bool warp_active = (row0 + lane_base) < R;  // same for both warps of the quarter
+      const uint32_t tl = tmem + ((uint32_t)lane_base << 16);
+      const uint32_t col0 = 64u * (uint32_t)half;
+      float* xmax = reinterpret_cast<float*>(smem + kOffX);  // [tile parity][half][row]
+      uint64_t* xbar = &bars->xchg[quarter];
+      float m_run = -__builtin_huge_valf(), l_run = 0.f;
+      uint32_t r[32];
+      // this row's token and the first token of its branch (-1 in the prefix)
+      int pf_p = 0, pf_bs = -1;
+      if (grow < R) {
+        pf_p = it.first_event + grow / p.group;
+        pf_bs = pf_p >= p.pf_S ? pf_branch_start(p, pf_p) : -1;
       }
-    }
-    for (int j = 0; j < n_tiles; ++j) {
-      ok = mbar_wait(&bars->sfull, (uint32_t)(j & 1), bars, p.header, 8);
-      ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
-      if (!ok) break;
-      fence_after();
-      uint32_t sr[2][32];
-      if (warp_active) {
-        tmem_ld32(tl + kColS + col0, sr[0]);
-        tmem_ld32(tl + kColS + col0 + 32, sr[1]);
-        tmem_wait_ld_dep(sr[0]);
-        tmem_wait_ld_dep(sr[1]);
-      }
-      // S is in registers: the S issuer may overwrite the buffer with the next tile's
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->sfree);
-      if (warp_active) {
-        const int valid = min(kBN, ntok - j * kBN) - (int)col0;  // valid columns of this half
-        // columns to mask: past the split's end, or (GSELF) hidden planning tokens of this
-        // row's event; the path is chosen per warp (tcgen05.st below is warp-collective)
-        float pmax;
-        bool masked;
-        uint64_t keep = ~0ull;
-        if (PREFILL) {
+      for (int j = 0; j < n_tiles; ++j) {
+        const uint32_t cS = 128u * (uint32_t)(j % kSBuf);
+        ok = mbar_wait(&bars->sfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 8);
+        ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
+        if (!ok) break;
+        fence_after();
+        if (warp_active) {
+          uint32_t sr[2][32];
+          tmem_ld32(tl + cS + col0, sr[0]);
+          tmem_ld32(tl + cS + col0 + 32, sr[1]);
+          tmem_wait_ld_dep(sr[0]);
+          tmem_wait_ld_dep(sr[1]);
           // the tile's range end, then this row's rule: a prefix token sees keys up to
           // itself, a branch token the prefix and its own branch up to itself
           const int tb = tile_tok(j);
           const int t0 = tb + (int)col0;
-          keep = range_bits(0, min(kBN, (j < pf_a_tiles ? pf_a_end : pf_last + 1) - tb) - (int)col0);
+          uint64_t keep = range_bits(0, min(kBN, (j < pf_a_tiles ? pf_a_end : pf_last + 1) - tb) - (int)col0);
           if (grow < R)
             keep &= pf_bs < 0 ? range_bits(0, pf_p - t0 + 1)
                               : (range_bits(0, p.pf_S - t0) | range_bits(pf_bs - t0, pf_p - t0 + 1));
-          masked = __any_sync(0xffffffffu, keep != ~0ull);
-          pmax = masked ? half_row_max<true>(sr, ColsBits{keep}) : half_row_max<false>(sr, ColsBits{keep});
-        } else if (GSELF) {
-          const int t0 = it.tok_begin + j * kBN + (int)col0;
-          if (valid < 64 || (t0 < g_hi && t0 + 64 > g_lo)) {
-            GMask gm{0, 0, -1};
-            if (g_lo < g_hi && grow < R)
-              gm = GMask{g_lo, g_hi, g_lo + plan_events(p)[it.first_event + grow / p.group].gidx};
-            keep = keep_bits(valid, gm, t0);
-          }
-          masked = __any_sync(0xffffffffu, keep != ~0ull);
-          pmax = masked ? half_row_max<true>(sr, ColsBits{keep}) : half_row_max<false>(sr, ColsBits{keep});
-        } else {
-          masked = valid < 64;
-          pmax = masked ? half_row_max<true>(sr, ColsValid{valid}) : half_row_max<false>(sr, ColsValid{valid});
-        }
-        // this key half's own running maximum: P is written over columns only this warp
-        // reads, and its P.V goes to this half's own accumulator
-        const float mx = pmax * sl2;
-        const float m_new = fmaxf(m_run, mx);
-        const bool need = m_new > m_run + kLazyRescale;
-        if (__any_sync(0xffffffffu, need && j > 0)) {
-          // this half's O must hold P.V of tile j-1 before it is rescaled
-          ok = mbar_wait(&bars->pvfree[(j - 1) % kStages], (uint32_t)(((j - 1) / kStages) & 1), bars,
-                         p.header, 9);
+          const bool masked = __any_sync(0xffffffffu, keep != ~0ull);
+          const float pmax = masked ? half_row_max<true>(sr, HalfBits{keep}) : half_row_max<false>(sr, HalfBits{keep});
+          // meet the other half: this also orders both warps' S reads before either
+          // writes P over columns the other one read
+          xmax[(j & 1) * 256 + half * 128 + row] = pmax;
+          mbar_arrive(xbar);
+          ok = mbar_wait(xbar, (uint32_t)(j & 1), bars, p.header, 12);
           ok = __all_sync(0xffffffffu, ok);
           if (!ok) break;
-          fence_after();
-          const float alpha = need ? ex2(m_run - m_new) : 1.f;
+          const float mx = fmaxf(pmax, xmax[(j & 1) * 256 + (1 - half) * 128 + row]) * sl2;
+          const float m_new = fmaxf(m_run, mx);
+          const bool need = m_new > m_run + kLazyRescale;
+          if (__any_sync(0xffffffffu, need && j > 0)) {
+            // O must hold P.V of tile j-1 before it is rescaled (each half rescales its
+            // own 64 head-dim columns; both halves take the same decision per row)
+            ok = mbar_wait(&bars->pvfree[(j - 1) % kStages], (uint32_t)(((j - 1) / kStages) & 1), bars,
+                           p.header, 9);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            fence_after();
+            const float alpha = need ? ex2(m_run - m_new) : 1.f;
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            tmem_ld32(tl + colO + 32 * c, r);
-            tmem_wait_ld_dep(r);
+            for (int c = 0; c < 2; ++c) {
+              tmem_ld32(tl + kColO + col0 + 32 * c, r);
+              tmem_wait_ld_dep(r);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tmem_st32(tl + colO + 32 * c, r);
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+              tmem_st32(tl + kColO + col0 + 32 * c, r);
+            }
+            tmem_wait_st();
+            if (need) l_run *= alpha;
           }
+          if (need) m_run = m_new;
+          l_run += masked ? half_row_exp<true>(sr, HalfBits{keep}, sl2, m_run, tl + cS + col0 / 2)
+                          : half_row_exp<false>(sr, HalfBits{keep}, sl2, m_run, tl + cS + col0 / 2);
           tmem_wait_st();
-          if (need) l_run *= alpha;
         }
-        if (need) m_run = m_new;
-        // this key half's P of tile j goes to slot j % 2, which held P of tile j-2 until
-        // that P.V completed
-        const uint32_t taddr_p = tl + kColP + 64u * (uint32_t)(j % kPSlots) + 32u * (uint32_t)half;
-        if (j >= kPSlots) {
-          const int jp = j - kPSlots;
-          ok = mbar_wait(&bars->pvfree[jp % kStages], (uint32_t)((jp / kStages) & 1), bars, p.header, 14);
-          ok = __all_sync(0xffffffffu, ok);
-          if (!ok) break;
-        }
-        if (GSELF || PREFILL)
-          l_run += masked ? half_row_exp<true>(sr, ColsBits{keep}, sl2, m_run, taddr_p)
-                          : half_row_exp<false>(sr, ColsBits{keep}, sl2, m_run, taddr_p);
-        else
-          l_run += masked ? half_row_exp<true>(sr, ColsValid{valid}, sl2, m_run, taddr_p)
-                          : half_row_exp<false>(sr, ColsValid{valid}, sl2, m_run, taddr_p);
-        tmem_wait_st();
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->pfull[j % kSBuf]);
       }
-      fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->pfull[j % kPSlots]);
-    }
-    // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
-    if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
-    ok = __all_sync(0xffffffffu, ok);
-    // O leaves through shared memory: TMEM gives one row per thread, which stored straight
-    // to global memory would touch 32 lines per instruction.  Rows are staged in the K
-    // stages (idle once every MMA has completed) at a padded stride, so that eight
-    // consecutive rows fall in distinct banks, then written one 512-byte row per warp
-    // instruction.
-    float* ostage = reinterpret_cast<float*>(smem + kOffK);
-    float* inv_row = ostage + 128 * kOStage;  // PREFILL: 1 / l of each row for the write-out
-    if (ok && warp_active) {
-      // The two key halves meet once: each warp publishes its (m, l), then merges both
-      // halves' accumulators over its 64 head-dim columns by log-sum-exp weights.
-      xmax[half * 256 + row] = m_run;
-      xmax[half * 256 + 128 + row] = l_run;
-      mbar_arrive(xbar);
-      ok = mbar_wait(xbar, 0u, bars, p.header, 13);
-      ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld below is warp-collective
-      if (ok) {
+      // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
+      if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok && warp_active) {
         fence_after();
-        const float ma = xmax[row], la = xmax[128 + row];
-        const float mb = xmax[256 + row], lb = xmax[384 + row];
-        const float m_tot = fmaxf(ma, mb);
-        const bool none = m_tot == -__builtin_huge_valf();  // no visible key in the split
-        const float wa = none ? 0.f : ex2(ma - m_tot), wb = none ? 0.f : ex2(mb - m_tot);
-        const float l_tot = wa * la + wb * lb;
-        uint32_t rb[32];
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
-          tmem_ld32(tl + kColOA + col0 + 32 * c, r);
-          tmem_ld32(tl + kColOB + col0 + 32 * c, rb);
+          tmem_ld32(tl + kColO + col0 + 32 * c, r);
           tmem_wait_ld_dep(r);
-          tmem_wait_ld_dep(rb);
           float4* dst = reinterpret_cast<float4*>(ostage + row * kOStage + col0 + 32 * c);
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            dst[i] = make_float4(wa * __uint_as_float(r[4 * i]) + wb * __uint_as_float(rb[4 * i]),
-                                 wa * __uint_as_float(r[4 * i + 1]) + wb * __uint_as_float(rb[4 * i + 1]),
-                                 wa * __uint_as_float(r[4 * i + 2]) + wb * __uint_as_float(rb[4 * i + 2]),
-                                 wa * __uint_as_float(r[4 * i + 3]) + wb * __uint_as_float(rb[4 * i + 3]));
+            dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                 __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
         }
-        if (half == 0 && grow < R) {
-          if (PREFILL) {
-            // normalised output: 1 / l for the write-out below, the LSE now
-            inv_row[row] = 1.0f / l_tot;
-            const int64_t orow = (int64_t)pf_p * p.h_q + kvh * p.group + grow % p.group;
-            if (p.pf_lse != nullptr) p.pf_lse[orow] = (m_tot + log2f(l_tot)) * 0.69314718055994531f;
+        // row sum = both halves' partial sums (slot n_tiles & 1 was last read two tiles ago)
+        xmax[(n_tiles & 1) * 256 + half * 128 + row] = l_run;
+        mbar_arrive(xbar);
+        ok = mbar_wait(xbar, (uint32_t)(n_tiles & 1), bars, p.header, 13);
+        if (ok && half == 0 && grow < R) {
+          // normalised output: 1 / l for the write-out below, the LSE now
+          const float l_tot = l_run + xmax[(n_tiles & 1) * 256 + 128 + row];
+          inv_row[row] = 1.0f / l_tot;
+          const int64_t orow = (int64_t)pf_p * p.h_q + kvh * p.group + grow % p.group;
+          if (p.pf_lse != nullptr) p.pf_lse[orow] = (m_run + log2f(l_tot)) * 0.69314718055994531f;
+        }
+      }
+    } else {
+      // this warp's 16 rows (TMEM lanes), this thread's two of them and its first column of
+      // every 8-column chunk
+      const int wrow = lane_base + 16 * half;
+      const int ra = wrow + (lane >> 2), rb = ra + 8;
+      const int ga = row0 + ra, gb = row0 + rb;
+      const int cq = 2 * (lane & 3);
+      const bool warp_active = (row0 + wrow) < R;
+      const uint32_t tl = tmem + ((uint32_t)wrow << 16);
+      float m_a = -__builtin_huge_valf(), m_b = -__builtin_huge_valf(), l_a = 0.f, l_b = 0.f;
+      // self G-token mask: the video's planning tokens G^1..G^K (prefix-relative [g_lo, g_hi))
+      // and each row's own one
+      int g_lo = 0, g_hi = 0, g_oa = -1, g_ob = -1;
+      if (GSELF) {
+        const PadVideoDesc vdg = plan_videos(p)[plan_events(p)[it.first_event].video];
+        if (vdg.n_planning > 0) {
+          g_lo = vdg.prefix_len - 1 - vdg.n_planning;
+          g_hi = vdg.prefix_len - 1;
+          if (ga < R) g_oa = g_lo + plan_events(p)[it.first_event + ga / p.group].gidx;
+          if (gb < R) g_ob = g_lo + plan_events(p)[it.first_event + gb / p.group].gidx;
+        }
+      }
+      uint32_t sr[2][32];
+      for (int j = 0; j < n_tiles; ++j) {
+        const uint32_t cS = 128u * (uint32_t)(j % kSBuf);
+        ok = mbar_wait(&bars->sfull[j % kSBuf], (uint32_t)((j / kSBuf) & 1), bars, p.header, 8);
+        ok = __all_sync(0xffffffffu, ok);  // tcgen05.ld/st below are warp-collective
+        if (!ok) break;
+        fence_after();
+        if (warp_active) {
+          const int valid = min(kBN, ntok - j * kBN);  // valid columns of the tile
+          tmem_ld16x256_x8(tl + cS, sr[0]);
+          tmem_ld16x256_x8(tl + cS + 64, sr[1]);
+          tmem_wait_ld_dep(sr[0]);
+          tmem_wait_ld_dep(sr[1]);
+          // columns to mask: past the split's end, or (GSELF) hidden planning tokens of the
+          // row's event; the path is chosen per warp (tcgen05.st below is warp-collective)
+          float mxa, mxb;
+          bool masked;
+          ColsBits ka{~0ull, ~0ull}, kb{~0ull, ~0ull};
+          if (GSELF) {
+            const int t0 = it.tok_begin + j * kBN;
+            if (valid < kBN || (t0 < g_hi && t0 + kBN > g_lo)) {
+              const GMask gma{g_lo, g_hi, g_oa}, gmb{g_lo, g_hi, g_ob};
+              ka = ColsBits{keep_bits(valid, gma, t0), keep_bits(valid - 64, gma, t0 + 64)};
+              kb = ColsBits{keep_bits(valid, gmb, t0), keep_bits(valid - 64, gmb, t0 + 64)};
+            }
+            masked = __any_sync(0xffffffffu, (ka.lo & ka.hi & kb.lo & kb.hi) != ~0ull);
+            if (masked) rows_max<true>(sr, cq, ka, kb, mxa, mxb);
+            else rows_max<false>(sr, cq, ka, kb, mxa, mxb);
           } else {
-            p.part_ml[(int64_t)it.part_row0 + grow] = make_float2(m_tot, l_tot);
+            masked = valid < kBN;
+            if (masked) rows_max<true>(sr, cq, ColsValid{valid}, ColsValid{valid}, mxa, mxb);
+            else rows_max<false>(sr, cq, ColsValid{valid}, ColsValid{valid}, mxa, mxb);
           }
+          const float na = fmaxf(m_a, mxa * sl2), nb = fmaxf(m_b, mxb * sl2);
+          const bool need_a = na > m_a + kLazyRescale, need_b = nb > m_b + kLazyRescale;
+          if (__any_sync(0xffffffffu, (need_a || need_b) && j > 0)) {
+            // O must hold P.V of tile j-1 before its rows are rescaled
+            ok = mbar_wait(&bars->pvfree[(j - 1) % kStages], (uint32_t)(((j - 1) / kStages) & 1), bars,
+                           p.header, 9);
+            ok = __all_sync(0xffffffffu, ok);
+            if (!ok) break;
+            fence_after();
+            const float al_a = need_a ? ex2(m_a - na) : 1.f, al_b = need_b ? ex2(m_b - nb) : 1.f;
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+              uint32_t o[32];
+              tmem_ld16x256_x8(tl + kColO + 64 * x, o);
+              tmem_wait_ld_dep(o);
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                o[i] = __float_as_uint(__uint_as_float(o[i]) * ((i & 2) ? al_b : al_a));
+              tmem_st16x256_x8(tl + kColO + 64 * x, o);
+            }
+            tmem_wait_st();
+            l_a *= al_a;
+            l_b *= al_b;
+          }
+          if (need_a) m_a = na;
+          if (need_b) m_b = nb;
+          // P of the tile over the first 64 columns of its S buffer, in this warp's own rows
+          if (GSELF) {
+            if (masked) rows_exp<true>(sr, cq, ka, kb, sl2, m_a, m_b, tl + cS, l_a, l_b);
+            else rows_exp<false>(sr, cq, ka, kb, sl2, m_a, m_b, tl + cS, l_a, l_b);
+          } else {
+            if (masked) rows_exp<true>(sr, cq, ColsValid{valid}, ColsValid{valid}, sl2, m_a, m_b, tl + cS, l_a, l_b);
+            else rows_exp<false>(sr, cq, ColsValid{valid}, ColsValid{valid}, sl2, m_a, m_b, tl + cS, l_a, l_b);
+          }
+          tmem_wait_st();
+        }
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->pfull[j % kSBuf]);
+      }
+      // the P.V issuer commits `drain_pv` after its last MMA: O is final once it lands
+      if (ok) ok = mbar_wait(&bars->drain_pv, 0u, bars, p.header, 10);
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok && warp_active) {
+        fence_after();
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+          uint32_t o[32];
+          tmem_ld16x256_x8(tl + kColO + 64 * x, o);
+          tmem_wait_ld_dep(o);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const int c = 64 * x + 8 * k + cq;
+            *reinterpret_cast<float2*>(ostage + ra * kOStage + c) =
+                make_float2(__uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]));
+            *reinterpret_cast<float2*>(ostage + rb * kOStage + c) =
+                make_float2(__uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
+          }
+        }
+        const float la = quad_sum(l_a), lb = quad_sum(l_b);
+        if ((lane & 3) == 0) {
+          if (ga < R) p.part_ml[(int64_t)it.part_row0 + ga] = make_float2(m_a, la);
+          if (gb < R) p.part_ml[(int64_t)it.part_row0 + gb] = make_float2(m_b, lb);
         }
       }
     }

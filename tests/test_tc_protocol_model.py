@@ -2,23 +2,23 @@
 
 The kernel (csrc/pad_prefix_tc.cu) runs a K producer, a V producer, an S issuer, a P.V
 issuer and eight softmax warps that hand 128-token tiles to each other through
-mbarriers waited on by phase parity: 3 K/V stages ("K tile loaded", "V tile loaded",
-"S of the tile in this K stage done", "P.V of the tile in this V stage done"), one TMEM
-S buffer ("S done", "S loaded by every softmax warp") and two TMEM P slots ("P written").
-The two key halves of a tile (tokens 0-63: softmax warps 0-3 here, 64-127: warps 4-7)
-keep their own softmax state and P.V accumulator: the first four P.V MMAs of a tile add
-into O_A, the last four into O_B, and a warp rescales only its own half's O.  A
-tcgen05.commit arrives when every MMA issued *by the committing thread* so far has
-completed, so each issuer has its own completion barriers.
+mbarriers waited on by phase parity: 3 K/V stages whose index is also the TMEM S buffer,
+per-stage barriers for "K tile loaded", "V tile loaded", "S done", "P written" and "P.V
+done".  A tcgen05.commit arrives when every MMA issued *by the committing thread* so far
+has completed, so each issuer has its own completion barriers.  In decode, each softmax
+warp owns 16 rows of the tile outright (all 128 columns), so it writes P over S columns
+that no other warp reads: the warps never meet inside the loop.  In whole-sequence
+prefill the two warps of a lane quarter split the columns and meet on a barrier of their
+own between the row maximum and the P store; that meeting is a step inside the softmax
+here (it involves no other role, and its parity alternates with the tile, like the S
+buffers').
 
 This model mirrors that schedule with asynchronous loads and MMAs that complete after
-random delays and in any order, and checks under many random interleavings that no stage,
-buffer or slot is reused while something still reads it, that an O accumulator is
-rescaled only when no P.V into it is in flight, and that nothing deadlocks.  Schedules
-with a plausible mistake fail it: one that shares one P-ready barrier and one P.V barrier
-across tiles, one that issues the next S before every softmax warp has loaded the current
-one, and one that writes P into a slot before the P.V of two tiles back has read it.  TMEM
-is freed only after all eight softmax warps have arrived on their own completion barrier.
+random delays and in any order, and checks under many random interleavings that no stage
+or buffer is reused while something still reads it, that O is rescaled only when no P.V
+is in flight, and that nothing deadlocks.  A schedule that shares one P-ready barrier and
+one P.V barrier across tiles (so that a waiter can miss a phase) fails it.  TMEM is
+freed only after all eight softmax warps have arrived on their own completion barrier.
 """
 import random
 
@@ -41,35 +41,34 @@ class Bar:
         return (s.done % 2) != parity
 
 
-ST = 3  # K/V stages
-PS = 2  # TMEM P slots
-N_SOFTMAX = 8  # warps 0-3: key half A, 4-7: key half B
+ST = 3  # K/V stages = S buffers
 
 
-def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_slot_unchecked=False):
+def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=False):
+    """prefetch: the softmax warps load tile j + 1's S during tile j (after the two halves
+    meet, before P(j) is released), as a softmax that hides the load behind the
+    exponentials would."""
     rnd = random.Random(seed)
     kfull = [Bar(1) for _ in range(ST)]
     vfull = [Bar(1) for _ in range(ST)]
-    kfree = [Bar(1) for _ in range(ST)]
+    sfull = [Bar(1) for _ in range(ST)]
+    pfull = [Bar(n_softmax) for _ in range(ST)]
     pvfree = [Bar(1) for _ in range(ST)]
-    sfull = Bar(1)
-    sfree = Bar(N_SOFTMAX)
-    pfull = [Bar(N_SOFTMAX) for _ in range(PS)]
     drain_s, drain_pv = Bar(1), Bar(1)
-    tdone = Bar(N_SOFTMAX)
-    xchg = Bar(N_SOFTMAX)
-    tmem_users = [True] * N_SOFTMAX
+    tdone = Bar(n_softmax)
+    tmem_users = [True] * n_softmax
     if single_barriers:
-        pfull = [pfull[0]] * PS
+        pfull = [pfull[0]] * ST
         pvfree = [pvfree[0]] * ST
+
+    def wpar(tile, per_stage=True):
+        # phase parity of the completion belonging to `tile` on its barrier
+        return ((tile // ST) & 1) if per_stage else (tile & 1)
 
     kst = [None] * ST
     vst = [None] * ST
-    S_done, PV_done = set(), set()
-    P_written = {}                 # tile -> halves whose P is written
-    PV_issued = set()
-    pv_inflight = {0: 0, 1: 0}     # P.V MMAs into O_A / O_B not yet complete
-    holding = [set() for _ in range(N_SOFTMAX)]  # tiles whose S a softmax warp still reads
+    S_done, PV_done, P_written, PV_issued = set(), set(), set(), set()
+    holding = [set() for _ in range(n_softmax)]  # tiles whose S a softmax warp has loaded, unconsumed
     inflight = []
     commits = []
     issued = {"S": [], "PV": []}  # per-issuer MMA ops (a commit tracks only its own)
@@ -95,37 +94,30 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_
             done()
         async_op(fin)
 
-    pv_half_done = {}
-
     def issue_S(t):
         def chk():
             assert kst[t % ST] == t, f"S({t}) reads a K stage not holding tile {t}"
+            for j in PV_issued:
+                if j % ST == t % ST and j not in PV_done:
+                    raise AssertionError(f"S({t}) overwrites P({j}) still read by its P.V")
+            if t >= ST:
+                assert (t - ST) in PV_done, f"S({t}) before P.V({t - ST}) done"
             for h in holding:
-                for j in h:
-                    if j != t:
-                        raise AssertionError(f"S({t}) overwrites S({j}) that a softmax warp still loads")
+                assert (t - ST) not in h, f"S({t}) overwrites S({t - ST}) that a softmax warp still holds"
         mma("S", chk, lambda: S_done.add(t))
 
-    def issue_PV(j, half):
-        # the four MMAs of one key half, into that half's accumulator
+    def issue_PV(j):
         def chk():
-            assert half in P_written.get(j, set()), f"P.V({j}) half {half} before its P"
+            assert j in P_written, f"P.V({j}) before P({j})"
             assert vst[j % ST] == j, f"P.V({j}) reads a V stage not holding tile {j}"
             PV_issued.add(j)
-            pv_inflight[half] += 1
-
-        def done():
-            pv_inflight[half] -= 1
-            pv_half_done[j] = pv_half_done.get(j, 0) + 1
-            if pv_half_done[j] == 2:
-                PV_done.add(j)
-        mma("PV", chk, done)
+        mma("PV", chk, lambda: PV_done.add(j))
 
     def kprod():
         for t in range(n):
             s = t % ST
             if t >= ST:
-                yield (kfree[s], ((t // ST) - 1) & 1)
+                yield (sfull[s], ((t // ST) - 1) & 1)
                 assert (t - ST) in S_done, f"K stage reused before S({t - ST}) done"
             kst[s] = None
 
@@ -134,17 +126,11 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_
                 kfull[s].arrive()
             async_op(ld)
 
-    def pv_wait(tile):
-        # the completion of P.V(tile) on its V stage's barrier
-        if single_barriers:
-            return (pvfree[0], tile & 1)
-        return (pvfree[tile % ST], (tile // ST) & 1)
-
     def vprod():
         for t in range(n):
             s = t % ST
             if t >= ST:
-                yield pv_wait(t - ST)
+                yield (pvfree[s], ((t // ST) - 1) & 1) if not single_barriers else (pvfree[s], (t - ST) & 1)
                 assert (t - ST) in PV_done, f"V stage reused before P.V({t - ST}) done"
             vst[s] = None
 
@@ -157,11 +143,10 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_
         for t in range(n):
             s = t % ST
             yield (kfull[s], (t // ST) & 1)
-            if t >= 1 and not s_before_loaded:
-                yield (sfree, (t - 1) & 1)  # every softmax warp has loaded S(t - 1)
+            if t >= ST:
+                yield (pvfree[s], ((t // ST) - 1) & 1) if not single_barriers else (pvfree[s], (t - ST) & 1)
             issue_S(t)
-            commit("S", sfull)
-            commit("S", kfree[s])
+            commit("S", sfull[s])
         commit("S", drain_s)
         yield (drain_s, 0)
 
@@ -169,49 +154,45 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_
         for j in range(n):
             s = j % ST
             yield (vfull[s], (j // ST) & 1)
-            yield (pfull[0], j & 1) if single_barriers else (pfull[j % PS], (j // PS) & 1)
-            issue_PV(j, 0)
-            issue_PV(j, 1)
+            yield (pfull[s], wpar(j, not single_barriers))
+            issue_PV(j)
             commit("PV", pvfree[s])
         commit("PV", drain_pv)
         yield (drain_pv, 0)
 
-    p_count = {}
-
     def softmax(w):
-        half = w // (N_SOFTMAX // 2)
+        if prefetch and n > 0:
+            yield (sfull[0], 0)
+            assert 0 in S_done, "softmax loads S(0) before it is done"
+            holding[w].add(0)
         for j in range(n):
-            yield (sfull, j & 1)
-            assert j in S_done, f"softmax reads S({j}) before it is done"
-            holding[w].add(j)
-            for _ in range(rnd.randint(0, 2)):  # S load
+            if prefetch:
+                assert j in holding[w], f"softmax uses S({j}) it has not loaded"
+            else:
+                yield (sfull[j % ST], (j // ST) & 1)
+                assert j in S_done, f"softmax reads S({j}) before it is done"
+                holding[w].add(j)
+            for _ in range(rnd.randint(0, 2)):  # the row maximum, the halves meeting
                 yield None
-            holding[w].discard(j)
-            sfree.arrive()
-            for _ in range(rnd.randint(0, 2)):  # row maximum
-                yield None
+            if prefetch and j + 1 < n:
+                yield (sfull[(j + 1) % ST], ((j + 1) // ST) & 1)
+                assert (j + 1) in S_done, f"softmax loads S({j + 1}) before it is done"
+                holding[w].add(j + 1)
             if j > 0 and rnd.random() < lazy_prob:
-                yield pv_wait(j - 1)
+                yield ((pvfree[(j - 1) % ST], ((j - 1) // ST) & 1) if not single_barriers
+                       else (pvfree[0], (j - 1) & 1))
                 assert (j - 1) in PV_done, f"O rescaled before P.V({j - 1}) done"
-                assert pv_inflight[half] == 0, "O rescaled while a P.V into it is in flight"
-            if j >= PS and not p_slot_unchecked:
-                yield pv_wait(j - PS)  # P slot j % 2 held P(j - 2) until its P.V completed
-            for jj in PV_issued:
-                if jj % PS == j % PS and jj != j and jj not in PV_done:
-                    raise AssertionError(f"P({j}) overwrites P({jj}) still read by its P.V")
-            for _ in range(rnd.randint(0, 3)):  # exponentials
+                for jj in PV_issued:
+                    assert jj in PV_done or jj >= j, "O rescaled while a P.V is in flight"
+            for _ in range(rnd.randint(0, 3)):
                 yield None
-            key = (j, half)
-            p_count[key] = p_count.get(key, 0) + 1
-            if p_count[key] == N_SOFTMAX // 2:
-                P_written.setdefault(j, set()).add(half)
-            pfull[j % PS].arrive()
+            if w == 0:
+                P_written.add(j)
+            holding[w].discard(j)
+            pfull[j % ST].arrive()
         yield (drain_pv, 0)
         assert len(PV_done) == n, "epilogue before every P.V completed"
-        # the two halves meet once, then each merges both accumulators
-        xchg.arrive()
-        yield (xchg, 0)
-        for _ in range(rnd.randint(0, 3)):  # reads O_A and O_B out of TMEM
+        for _ in range(rnd.randint(0, 3)):  # reads O out of TMEM
             yield None
         tmem_users[w] = False
         tdone.arrive()
@@ -221,7 +202,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, s_before_loaded=False, p_
         yield (tdone, 0)
         assert not any(tmem_users), "TMEM freed while a softmax warp still reads it"
 
-    actors = [kprod(), vprod(), s_issuer(), pv_issuer(), dealloc()] + [softmax(w) for w in range(N_SOFTMAX)]
+    actors = [kprod(), vprod(), s_issuer(), pv_issuer(), dealloc()] + [softmax(w) for w in range(n_softmax)]
     waiting = [None] * len(actors)
     alive = [True] * len(actors)
     steps = 0
@@ -272,24 +253,20 @@ def test_tc_kernel_barrier_protocol(n):
         assert run(n, seed * 131 + n)
 
 
-def _fails(**kw):
-    fails = 0
-    for n in range(3, 13):
-        for seed in range(40):
-            try:
-                run(n, seed * 7 + n, **kw)
-            except AssertionError:
-                fails += 1
-    return fails
+@pytest.mark.parametrize("n", range(1, 13))
+def test_prefetching_softmax_keeps_the_protocol(n):
+    """Loading tile j + 1's S during tile j (waiting for its S-done barrier before releasing
+    P(j)) neither deadlocks nor lets an S MMA overwrite a buffer a softmax warp still holds."""
+    for seed in range(120):
+        assert run(n, seed * 173 + n, prefetch=True)
 
 
 def test_model_detects_phase_aliasing():
-    assert _fails(single_barriers=True) > 0
-
-
-def test_model_detects_s_issued_before_every_warp_loaded_the_last():
-    assert _fails(s_before_loaded=True) > 0
-
-
-def test_model_detects_p_slot_reuse_before_its_pv():
-    assert _fails(p_slot_unchecked=True) > 0
+    fails = 0
+    for n in range(4, 13):
+        for seed in range(40):
+            try:
+                run(n, seed * 7 + n, single_barriers=True)
+            except AssertionError:
+                fails += 1
+    assert fails > 0
