@@ -44,10 +44,20 @@ class Bar:
 ST = 3  # K/V stages = S buffers
 
 
-def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=False):
-    """prefetch: the softmax warps load tile j + 1's S during tile j (after the two halves
-    meet, before P(j) is released), as a softmax that hides the load behind the
-    exponentials would."""
+MISTAKES = ("s_skips_pvfree", "k_refill_early", "v_refill_early", "rescale_without_wait",
+            "dealloc_without_tdone", "one_xchg_slot")
+
+
+def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=False, meet=False,
+        mistake=None):
+    """prefetch: the softmax warps load tile j + 1's S during tile j (after the row maximum,
+    before P(j) is released), as a softmax that hides the load behind the exponentials would.
+    meet: the prefill softmax, where warps w and w + 4 (the two column halves of a lane
+    quarter) exchange their partial row maxima through two shared-memory slots (tile parity)
+    and a per-quarter barrier on every tile, and their row sums once more after the loop.
+    mistake: one of MISTAKES, a plausible slip planted in the schedule (a wait left out, or
+    one exchange slot instead of two)."""
+    assert mistake is None or mistake in MISTAKES
     rnd = random.Random(seed)
     kfull = [Bar(1) for _ in range(ST)]
     vfull = [Bar(1) for _ in range(ST)]
@@ -56,6 +66,8 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
     pvfree = [Bar(1) for _ in range(ST)]
     drain_s, drain_pv = Bar(1), Bar(1)
     tdone = Bar(n_softmax)
+    xbar = [Bar(2) for _ in range(n_softmax // 2)]
+    xslot = {}  # (slot, half, quarter) -> what the warp last wrote there
     tmem_users = [True] * n_softmax
     if single_barriers:
         pfull = [pfull[0]] * ST
@@ -116,8 +128,9 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
     def kprod():
         for t in range(n):
             s = t % ST
-            if t >= ST:
+            if t >= ST and mistake != "k_refill_early":
                 yield (sfull[s], ((t // ST) - 1) & 1)
+            if t >= ST:
                 assert (t - ST) in S_done, f"K stage reused before S({t - ST}) done"
             kst[s] = None
 
@@ -129,8 +142,9 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
     def vprod():
         for t in range(n):
             s = t % ST
-            if t >= ST:
+            if t >= ST and mistake != "v_refill_early":
                 yield (pvfree[s], ((t // ST) - 1) & 1) if not single_barriers else (pvfree[s], (t - ST) & 1)
+            if t >= ST:
                 assert (t - ST) in PV_done, f"V stage reused before P.V({t - ST}) done"
             vst[s] = None
 
@@ -143,7 +157,7 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
         for t in range(n):
             s = t % ST
             yield (kfull[s], (t // ST) & 1)
-            if t >= ST:
+            if t >= ST and mistake != "s_skips_pvfree":
                 yield (pvfree[s], ((t // ST) - 1) & 1) if not single_barriers else (pvfree[s], (t - ST) & 1)
             issue_S(t)
             commit("S", sfull[s])
@@ -172,15 +186,18 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
                 yield (sfull[j % ST], (j // ST) & 1)
                 assert j in S_done, f"softmax reads S({j}) before it is done"
                 holding[w].add(j)
-            for _ in range(rnd.randint(0, 2)):  # the row maximum, the halves meeting
+            for _ in range(rnd.randint(0, 2)):  # the row maximum
                 yield None
+            if meet:
+                yield from exchange(w, j, ("m", j))
             if prefetch and j + 1 < n:
                 yield (sfull[(j + 1) % ST], ((j + 1) // ST) & 1)
                 assert (j + 1) in S_done, f"softmax loads S({j + 1}) before it is done"
                 holding[w].add(j + 1)
             if j > 0 and rnd.random() < lazy_prob:
-                yield ((pvfree[(j - 1) % ST], ((j - 1) // ST) & 1) if not single_barriers
-                       else (pvfree[0], (j - 1) & 1))
+                if mistake != "rescale_without_wait":
+                    yield ((pvfree[(j - 1) % ST], ((j - 1) // ST) & 1) if not single_barriers
+                           else (pvfree[0], (j - 1) & 1))
                 assert (j - 1) in PV_done, f"O rescaled before P.V({j - 1}) done"
                 for jj in PV_issued:
                     assert jj in PV_done or jj >= j, "O rescaled while a P.V is in flight"
@@ -194,12 +211,30 @@ def run(n, seed, lazy_prob=0.3, single_barriers=False, n_softmax=8, prefetch=Fal
         assert len(PV_done) == n, "epilogue before every P.V completed"
         for _ in range(rnd.randint(0, 3)):  # reads O out of TMEM
             yield None
+        if meet:
+            yield from exchange(w, n, ("l", n))
         tmem_users[w] = False
         tdone.arrive()
 
+    def exchange(w, k, tag):
+        # write this half's value into slot k & 1, meet the other half (completion k of the
+        # quarter's barrier), read the other half's value of the same round
+        quarter, half = w % (n_softmax // 2), w // (n_softmax // 2)
+        slot = 0 if mistake == "one_xchg_slot" else k & 1
+        xslot[(slot, half, quarter)] = tag
+        xbar[quarter].arrive()
+        yield (xbar[quarter], k & 1)
+        for _ in range(rnd.randint(0, 2)):
+            yield None
+        assert xslot.get((slot, 1 - half, quarter)) == tag, \
+            f"warp {w} reads the other half's {xslot.get((slot, 1 - half, quarter))} for {tag}"
+
     def dealloc():
         # warp 2 frees TMEM once every softmax warp has arrived on tdone
-        yield (tdone, 0)
+        if mistake != "dealloc_without_tdone":
+            yield (tdone, 0)
+        else:
+            yield (drain_pv, 0)
         assert not any(tmem_users), "TMEM freed while a softmax warp still reads it"
 
     actors = [kprod(), vprod(), s_issuer(), pv_issuer(), dealloc()] + [softmax(w) for w in range(n_softmax)]
@@ -259,6 +294,29 @@ def test_prefetching_softmax_keeps_the_protocol(n):
     P(j)) neither deadlocks nor lets an S MMA overwrite a buffer a softmax warp still holds."""
     for seed in range(120):
         assert run(n, seed * 173 + n, prefetch=True)
+
+
+@pytest.mark.parametrize("n", range(1, 13))
+def test_prefill_softmax_exchange_keeps_the_protocol(n):
+    """The prefill softmax's per-tile meeting of the two column halves (two slots by tile
+    parity, one barrier per lane quarter) reads the other half's value of the same tile,
+    and neither deadlocks nor disturbs the MMA schedule."""
+    for seed in range(120):
+        assert run(n, seed * 191 + n, meet=True)
+
+
+@pytest.mark.parametrize("mistake", MISTAKES)
+def test_model_detects_planted_mistakes(mistake):
+    """Each plausible slip in the schedule (a wait dropped, or one exchange slot for both
+    tile parities) fails the model under some interleaving."""
+    fails = 0
+    for n in range(2, 10):
+        for seed in range(40):
+            try:
+                run(n, seed * 11 + n, lazy_prob=0.6, meet=True, mistake=mistake)
+            except AssertionError:
+                fails += 1
+    assert fails > 0, mistake
 
 
 def test_model_detects_phase_aliasing():
