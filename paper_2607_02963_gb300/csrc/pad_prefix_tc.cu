@@ -649,8 +649,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) mbar_arrive(&bars->qready);
     const float sl2 = p.scale_log2;
     bool ok = true;
-    // O leaves through shared memory: rows are staged in the K stages (idle once every MMA
-    // has completed) at a padded stride, then written one 512-byte row per warp instruction.
+    // Prefill: O leaves through shared memory, its rows staged in the K stages (idle once
+    // every MMA has completed) at a padded stride, then normalised and written one 512-byte
+    // row per warp instruction.  (One row per thread stored straight to global memory would
+    // touch 32 lines per instruction; the decode layout stores straight, eight rows of 32
+    // contiguous bytes per instruction.)
     float* ostage = reinterpret_cast<float*>(smem + kOffK);
     float* inv_row = ostage + 128 * kOStage;  // PREFILL: 1 / l of each row for the write-out
     if constexpr (PREFILL) {
@@ -858,6 +861,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xffffffffu, ok);
       if (ok && warp_active) {
         fence_after();
+        // O rows straight from the 16-lane layout: a quad writes 32 contiguous bytes of a
+        // row, a warp instruction eight such segments
+        float* po_a = p.part_o + ((int64_t)it.part_row0 + ga) * kD;
+        float* po_b = po_a + 8 * kD;
 #pragma unroll
         for (int x = 0; x < 2; ++x) {
           uint32_t o[32];
@@ -866,10 +873,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const int c = 64 * x + 8 * k + cq;
-            *reinterpret_cast<float2*>(ostage + ra * kOStage + c) =
-                make_float2(__uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]));
-            *reinterpret_cast<float2*>(ostage + rb * kOStage + c) =
-                make_float2(__uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
+            if (ga < R)
+              *reinterpret_cast<float2*>(po_a + c) = make_float2(__uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]));
+            if (gb < R)
+              *reinterpret_cast<float2*>(po_b + c) =
+                  make_float2(__uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
           }
         }
         const float la = quad_sum(l_a), lb = quad_sum(l_b);
@@ -883,27 +891,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&bars->tdone);
-    // every softmax warp reaches this barrier exactly once (the loop above only breaks)
-    asm volatile("bar.sync 1, 256;" ::: "memory");
-    const int nrows = min(128, R - row0);
+    // every softmax warp reaches this barrier exactly once (the loop above only breaks);
+    // it orders the staged rows (prefill) and the partial rows before the fused tail
+    if (PREFILL || p.fused) asm volatile("bar.sync 1, 256;" ::: "memory");
+    const int nrows = PREFILL ? min(128, R - row0) : 0;  // prefill: normalised rows out
     for (int rr = warp - 4; rr < nrows; rr += 8) {
       float4 v = *reinterpret_cast<const float4*>(ostage + rr * kOStage + 4 * lane);
-      if (PREFILL) {
-        const float inv = inv_row[rr];
-        v.x *= inv;
-        v.y *= inv;
-        v.z *= inv;
-        v.w *= inv;
-        const int gr = row0 + rr;
-        const size_t oi = ((size_t)(it.first_event + gr / p.group) * p.h_q + kvh * p.group + gr % p.group) * kD + 4 * lane;
-        if (p.out_bf16)
-          *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.pf_out) + oi) =
-              make_uint2(bm::pack_bf16(v.x, v.y), bm::pack_bf16(v.z, v.w));
-        else
-          *reinterpret_cast<float4*>(static_cast<float*>(p.pf_out) + oi) = v;
-      } else {
-        *reinterpret_cast<float4*>(p.part_o + ((int64_t)it.part_row0 + row0 + rr) * kD + 4 * lane) = v;
-      }
+      const float inv = inv_row[rr];
+      v.x *= inv;
+      v.y *= inv;
+      v.z *= inv;
+      v.w *= inv;
+      const int gr = row0 + rr;
+      const size_t oi = ((size_t)(it.first_event + gr / p.group) * p.h_q + kvh * p.group + gr % p.group) * kD + 4 * lane;
+      if (p.out_bf16)
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.pf_out) + oi) =
+            make_uint2(bm::pack_bf16(v.x, v.y), bm::pack_bf16(v.z, v.w));
+      else
+        *reinterpret_cast<float4*>(static_cast<float*>(p.pf_out) + oi) = v;
     }
     if (!PREFILL && p.fused) {
       // ---------------------------------------------------------- fused a4 + a5
