@@ -246,6 +246,9 @@ typedef struct {
   uint64_t generation;      /* the number tagging this plan's device status word and counters */
   int32_t prefix_ctas;      /* CTAs of the prefix pass (a batch of videos may take several waves) */
   int32_t max_split_tiles;  /* 128-token tiles of the longest split */
+  int32_t merge_first;      /* 1: in a one-call step the branch tasks wait for the prefix pass
+                               before their branch pass (too few SMs are left beside it for
+                               them to run there), staging the split partials meanwhile */
 } pad_plan_info;
 pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info);
 pad_status pad_plan_destroy(pad_plan_t* plan);

@@ -49,7 +49,8 @@ class PlanInfo(ctypes.Structure):
                 ("split_len", c_int32), ("prefix_kernel", c_int32), ("n_new_pages", c_int32),
                 ("partial_rows", c_int64), ("workspace_bytes", c_int64),
                 ("param_descriptor_bytes", c_int32), ("fused_tail", c_int32),
-                ("generation", ctypes.c_uint64), ("prefix_ctas", c_int32), ("max_split_tiles", c_int32)]
+                ("generation", ctypes.c_uint64), ("prefix_ctas", c_int32), ("max_split_tiles", c_int32),
+                ("merge_first", c_int32)]
 
 
 _I32P = POINTER(c_int32)

@@ -118,6 +118,9 @@ struct Layout {
   // rows than the batch's largest gets no idle CTAs.
   bool cta_map = false;
   int64_t n_ctas = 0;
+  // The branch/merge CTAs of a one-call step wait for the prefix grid before their branch
+  // pass (see KParams::merge_first).
+  bool merge_first = false;
   std::vector<int32_t> cta_task, cnt_base;
   int64_t n_counters = 0;
   size_t off_videos = 0, off_events = 0, off_items = 0, off_tasks = 0, upload_bytes = 0;
@@ -416,6 +419,17 @@ pad_status compute_layout(const pad_problem* prob, int32_t n_videos, const int32
     for (const auto& o : order) L->cta_task.push_back(o.second);
     L->n_ctas = (int64_t)L->cta_task.size();
     L->cta_map = true;
+  }
+  // A branch/merge CTA that starts beside the prefix grid runs its branch pass there, then
+  // holds its slot until that grid completes; with a one-wave tensor-core grid, the slots
+  // beside it are those of the SMs it leaves free (two CTAs each).  When some (event,
+  // kv-head) task gets none, it starts only once the prefix CTAs leave, and the whole step
+  // then waits for its branch pass and merge in series: there every task waits for the
+  // prefix grid first and stages the split partials while its branch pass runs.
+  L->merge_first = false;
+  if (kern == PAD_FLAG_PREFIX_TC && !L->fused && L->n_ctas > 0 && L->n_ctas <= n_sms) {
+    const int64_t free_slots = 2 * ((int64_t)n_sms - L->n_ctas);
+    L->merge_first = (int64_t)n_events * prob->h_kv > free_slots;
   }
 
   size_t off = sizeof(PadDevHeader);
@@ -977,6 +991,7 @@ pad_status pad_plan_get_info(const pad_plan_t* plan, pad_plan_info* info) {
   info->generation = plan->gen;
   info->prefix_ctas = (int32_t)(plan->lay.n_ctas > 0 ? plan->lay.n_ctas : plan->lay.n_items);
   info->max_split_tiles = (plan->lay.split_len + kSplitGranule - 1) / kSplitGranule;
+  info->merge_first = plan->lay.merge_first ? 1 : 0;
   return PAD_OK;
 }
 
@@ -1024,6 +1039,7 @@ static void make_params(const pad_plan_t* plan, KParams& p) {
   p.cta_map = plan->lay.cta_map ? 1 : 0;
   p.n_ctas = (int32_t)plan->lay.n_ctas;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
+  p.merge_first = plan->lay.merge_first ? 1 : 0;
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
   p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;
   if (p.img_n > 0) {
@@ -1694,6 +1710,7 @@ pad_status static_params(const pad_plan_t* plan, cudaStream_t s, KParams& p, uin
   p.cta_map = plan->lay.cta_map ? 1 : 0;
   p.n_ctas = (int32_t)plan->lay.n_ctas;
   p.tail_chunk = p.fused ? prefix_tc_tail_chunk(p.branch_rows, p.group, p.max_splits) : 0;
+  p.merge_first = plan->lay.merge_first ? 1 : 0;
   p.tasks = reinterpret_cast<const int32_t*>(ws + plan->lay.off_tasks);
   p.counters = reinterpret_cast<unsigned int*>(ws + plan->lay.off_cnt);
   p.n_counters = p.fused ? (int32_t)plan->lay.n_counters : 0;

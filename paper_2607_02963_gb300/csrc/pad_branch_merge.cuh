@@ -309,8 +309,10 @@ __device__ __forceinline__ void run_task(const KParams& p, const __nv_bfloat16* 
   }
   cp_async_commit();
   // One-call step: nothing the branch pass reads is written by the grids ahead, so the
-  // whole pass runs before the wait and only the merge of the splits' partials follows it.
-  const bool pre = knew != nullptr;
+  // whole pass runs before the wait and only the merge of the splits' partials follows it;
+  // unless the plan says this CTA cannot start before the prefix grid completes anyway
+  // (merge_first), where waiting first lets the partials load during the branch pass.
+  const bool pre = knew != nullptr && !p.merge_first;
 
   // ---------------- after the grids ahead (at least the append) completed
   if (!pre) {

@@ -104,6 +104,10 @@ struct KParams {
   int32_t fused;                  // the tensor-core prefix kernel runs a4 + a5 itself (one
                                   // (event, kv-head) task per CTA after its split)
   int32_t tail_chunk;             // split partials merged per staged chunk in that tail
+  int32_t merge_first;            // one-call step whose prefix grid leaves too few SMs for
+                                  // the branch/merge CTAs to run beside it: each of them
+                                  // waits for it first, then stages the split partials
+                                  // while its branch pass runs
   float scale_log2;               // scale * log2(e)
   uint64_t gen;                   // generation of the plan (tags errors in the status word)
   PadDevHeader* header;

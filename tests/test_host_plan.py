@@ -181,6 +181,41 @@ def test_tc_split_leaves_sms_for_the_branch_tasks(padlib):
         assert 4 * -(-16384 // sl) * groups <= 100
 
 
+def _info_of(P, E, sms=152, flags=0):
+    prob = B.make_problem(28, 4, 128, num_sms=sms, flags=flags)
+    ev = np.zeros(E, np.int32)
+    plan = B.pad_plan(prob, B.CacheState(4096), np.array([P], np.int32), ev, np.zeros(E, np.int32),
+                      max_pages=2, workspace=None)
+    return plan.info()
+
+
+def test_branch_tasks_wait_first_only_when_no_slot_is_left_beside_the_prefix_grid(padlib):
+    """merge_first: the branch tasks wait for the prefix pass before their branch pass when
+    some (event, kv-head) task cannot get one of the two slots of each SM that the one-wave
+    tensor-core grid leaves free; otherwise they run their branch pass beside it."""
+    # 32 events x 4 kv-heads = 128 tasks beside a 152-CTA grid: no free SM
+    info = _info_of(32768, 32)
+    assert info["prefix_ctas"] == 152 and info["merge_first"] == 1
+    # 64 tasks beside 88 CTAs: 128 free slots
+    info = _info_of(16384, 16)
+    assert info["prefix_ctas"] == 88 and info["merge_first"] == 0
+    # one event: 4 tasks, 24 free SMs
+    assert _info_of(16384, 1)["merge_first"] == 0
+    # a smaller GPU: the split grows to keep one wave, still with no SM free
+    assert _info_of(32768, 32, sms=64)["merge_first"] == 1
+    # a second wave (4 row groups x 4 kv-heads on 8 SMs) keeps the branch pass before the wait
+    info = _info_of(16384, 64, sms=8)
+    assert info["prefix_ctas"] > 8 and info["merge_first"] == 0
+    # the fused tail runs its tasks in the prefix kernel
+    assert _info_of(16384, 8, flags=B.FLAG_FUSED_MERGE)["merge_first"] == 0
+    # every rule in one place: tasks > 2 x free SMs of a one-wave grid
+    for P, E in ((16384, 32), (16384, 64), (8192, 8), (65536, 4), (4096, 40)):
+        info = _info_of(P, E)
+        free = 152 - info["prefix_ctas"]
+        want = int(info["prefix_ctas"] <= 152 and E * 4 > 2 * free)
+        assert info["merge_first"] == want, (P, E, info)
+
+
 def test_batch_of_videos_takes_balanced_splits_over_several_waves(padlib):
     """16 videos of 4k-16k prefix tokens (the ragged serving batch): one split length sized
     to one wave leaves CTAs of 82 tiles beside CTAs of 32; per-video splits over two waves,
