@@ -88,9 +88,9 @@ def oracle_step(w):
     return _ORACLE[key]
 
 
-def run_full(w, flags=0, out_dtype=0, what=""):
+def run_full(w, flags=0, out_dtype=0, what="", one_call=False):
     db = DeviceBatch(w, flags=flags, out_dtype=out_dtype)
-    plan = db.run_step()
+    plan = db.run_step(one_call=one_call)
     torch.cuda.synchronize()
     B.pad_device_status(plan)
     check_bookkeeping(db, w, plan)
@@ -115,22 +115,39 @@ def test_gqa_8k_full(flags):
 
 
 # The full-size workloads: every output row of every event against the oracle, in the
-# launch configuration the bench times (default flags: the tensor-core kernel), and on the
-# dual tensor-core kernel.
+# launch configuration the bench times (default flags: the tensor-core kernel; the one-call
+# step, pad_decode_step), through the two-call step, and on the dual tensor-core kernel.
+# In the one-call step on the tensor-core kernel, long_32k and the E = 32, 64 sweep points
+# leave no SM free beside the prefix grid, so their branch tasks wait for it first
+# (merge_first); the others run their branch pass beside it.
+_MERGE_FIRST = {"long_32k": 1, "ragged_serving": 0, 1: 0, 2: 0, 4: 0, 8: 0, 16: 0, 32: 1, 64: 1}
+
+
+def _check_merge_first(plan, key, flags):
+    assert plan.info()["merge_first"] == (_MERGE_FIRST[key] if flags == 0 else 0)
+
+
+@pytest.mark.parametrize("one_call", [True, False])
 @pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
-def test_long_32k_full(flags):
-    run_full(synth.long_32k(), flags=flags)
+def test_long_32k_full(flags, one_call):
+    _, plan = run_full(synth.long_32k(), flags=flags, one_call=one_call)
+    _check_merge_first(plan, "long_32k", flags)
 
 
+@pytest.mark.parametrize("one_call", [True, False])
 @pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
-def test_ragged_serving_full(flags):
-    run_full(synth.ragged_serving(), flags=flags)
+def test_ragged_serving_full(flags, one_call):
+    _, plan = run_full(synth.ragged_serving(), flags=flags, one_call=one_call)
+    _check_merge_first(plan, "ragged_serving", flags)
 
 
+# (E outermost, so that the cases of one workload share its oracle run)
+@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
+@pytest.mark.parametrize("one_call", [True, False])
 @pytest.mark.parametrize("E", synth.SWEEP_E)
-@pytest.mark.parametrize("flags", [0, B.FLAG_PREFIX_DUAL])
-def test_event_sweep_full(E, flags):
-    run_full(synth.event_sweep(E), flags=flags)
+def test_event_sweep_full(E, flags, one_call):
+    _, plan = run_full(synth.event_sweep(E), flags=flags, one_call=one_call)
+    _check_merge_first(plan, E, flags)
 
 
 # ---------------------------------------------------------------------------

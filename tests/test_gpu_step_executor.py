@@ -38,8 +38,11 @@ def _same_state(a, b):
 
 
 @pytest.mark.parametrize("one_call", [True, False])
-@pytest.mark.parametrize("make", [synth.gqa_8k, lambda: synth.random_small(5), synth.tiny])
+@pytest.mark.parametrize("make", [synth.gqa_8k, lambda: synth.random_small(5), synth.tiny, synth.long_32k])
 def test_run_matches_the_step_calls(make, one_call):
+    """The executor (pad_step_run, the call the bench times) against pad_plan plus the step
+    calls: the same outputs, pools and page table, and the oracle's outputs (long_32k: the
+    plan whose branch tasks wait for the prefix grid first)."""
     w = make()
     a = DeviceBatch(w)
     pa = a.run_step(one_call=one_call)
