@@ -423,7 +423,7 @@ def run_ours(args):
         return B.NativeStep(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len,
                             db.page_table, w.max_pages, db.workspace, w.prefix_offset,
                             kw.get("q", db.q), db.k_new, db.v_new, db.k_prefix, db.v_prefix,
-                            db.k_pool, db.v_pool, db.out, db.lse, stream,
+                            db.k_pool, db.v_pool, db.out, db.lse, kw.get("stream", stream),
                             one_call=not args.two_call, rope=rope, self_g=self_g, causal=args.causal,
                             mapped_host_io=kw.get("mapped", not args.e2e_copy))
 
@@ -531,7 +531,10 @@ def run_ours(args):
     io = [(hq, hkn, hvn, hout, hlse),
           (h_in2[:qn].view(hq.shape), h_in2[qn:qn + kn].view(hkn.shape), h_in2[qn + kn:].view(hvn.shape),
            h_out2[:ob].view(hout.dtype).view(hout.shape), h_out2[ob:].view(torch.float32).view(hlse.shape))]
-    pair = [steps[0], steps[1 % n_rep]]
+    # the second batch on a stream of its own (--e2e-streams 2), so that one batch's host
+    # reads and writes and its merge tail can overlap the other batch's kernels
+    stream2 = torch.cuda.Stream(device) if args.e2e_streams > 1 else stream
+    pair = [steps[0], launcher(reps[1 % n_rep], stream=stream2) if args.e2e_streams > 1 else steps[1 % n_rep]]
 
     def pipelined_block(n):
         # two batches in flight: batch i % 2 is planned and enqueued (pad_step_enqueue_host)
@@ -576,8 +579,8 @@ def run_ours(args):
            "in_flight": 2,
            "timing": dict(e_stat, clock="host perf_counter around each block of steps"),
            "path": "through the C ABI, every step: " + io_desc + "; two independent batches (own "
-                   "executor, own host buffers) in flight: pad_step_enqueue_host of one, then "
-                   "pad_step_wait of the other"}
+                   "executor, own host buffers" + (", own stream" if args.e2e_streams > 1 else ", one stream")
+                   + ") in flight: pad_step_enqueue_host of one, then pad_step_wait of the other"}
     # one batch, each step waited for before the next (pad_step_run_host)
     s_stat = e2e_blocks(serial_block(steps[0]))
     e2e["serial"] = {"us_per_step": s_stat["median_ms_per_step"] * 1e3,
@@ -1045,6 +1048,8 @@ def main(argv=None):
     ap.add_argument("--prefix", choices=["auto", "simt", "mma", "tc", "dual"], default="auto",
                     help="shared-prefix kernel (auto = the library's choice)")
     ap.add_argument("--e2e-steps", type=int, default=500)
+    ap.add_argument("--e2e-streams", type=int, default=2, choices=(1, 2),
+                    help="streams of the two batches in flight in the headline e2e measurement")
     ap.add_argument("--e2e-copy", action="store_true",
                     help="e2e through the copy-engine path of pad_step_run_host (no mapped host I/O)")
     ap.add_argument("--cpu-budget", type=float, default=10.0, help="seconds of oracle work")

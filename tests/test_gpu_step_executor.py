@@ -24,10 +24,11 @@ def _cuda(padlib):
     torch.cuda.init()
 
 
-def _native(db, w, **kw):
+def _native(db, w, stream=None, **kw):
     return B.NativeStep(db.problem, db.cache, w.prefix_len, w.event_video, w.event_len, db.page_table,
                         w.max_pages, db.workspace, w.prefix_offset, db.q, db.k_new, db.v_new, db.k_prefix,
-                        db.v_prefix, db.k_pool, db.v_pool, db.out, db.lse, torch.cuda.current_stream(), **kw)
+                        db.v_prefix, db.k_pool, db.v_pool, db.out, db.lse,
+                        stream if stream is not None else torch.cuda.current_stream(), **kw)
 
 
 def _same_state(a, b):
@@ -135,11 +136,14 @@ def test_run_host_mapped_io(make, adjacent, one_call):
     assert torch.equal(a.page_table, b.page_table)
 
 
+@pytest.mark.parametrize("own_stream", [False, True])
 @pytest.mark.parametrize("mapped", [True, False])
-def test_two_batches_in_flight(mapped):
+def test_two_batches_in_flight(mapped, own_stream):
     """pad_step_enqueue_host of two independent batches, then pad_step_wait of each: every
-    batch's outputs and state equal its own device-buffer run."""
-    ws = [synth.gqa_8k(), synth.random_small(3)]
+    batch's outputs and state equal its own device-buffer run.  With own_stream the second
+    batch's executor runs on a stream of its own (how the bench keeps two batches in flight),
+    so the two batches' kernels and host reads and writes may overlap."""
+    ws = [synth.long_32k() if own_stream else synth.gqa_8k(), synth.random_small(3)]
     refs, runs, bufs = [], [], []
     for w in ws:
         a = DeviceBatch(w)
@@ -152,7 +156,8 @@ def test_two_batches_in_flight(mapped):
         ho = torch.empty(b.out.shape, dtype=b.out.dtype).pin_memory()
         hl = torch.empty(b.lse.shape, dtype=torch.float32).pin_memory()
         b.q.zero_()
-        runs.append((b, _native(b, w, release_pages=False, mapped_host_io=mapped)))
+        stream = torch.cuda.Stream() if own_stream and len(runs) == 1 else None
+        runs.append((b, _native(b, w, stream=stream, release_pages=False, mapped_host_io=mapped)))
         bufs.append((hq, hk, hv, ho, hl))
     for (b, st), io in zip(runs, bufs):
         st.enqueue_host(*io)
